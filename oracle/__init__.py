@@ -1,0 +1,178 @@
+"""CPU oracle for the FQ-ViT integer inference path (test infrastructure).
+
+This package is the checker, not the product.  Only ``tests/``, the smoke
+check in ``__graft_entry__`` and the CPU-baseline leg of ``bench.py`` may
+import it.  It wraps ``fqvit_oracle.c`` (plain C, fp32/fp64 IEEE arithmetic,
+int64 integers) through ctypes and takes / returns numpy arrays.  It shares
+no code with the CUDA library.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+from pathlib import Path
+
+import numpy as np
+
+_HERE = Path(__file__).resolve().parent
+_SRC = _HERE / "fqvit_oracle.c"
+_LIB = _HERE / "liboracle.so"
+_CFLAGS = ["-O2", "-ffp-contract=off", "-fno-fast-math", "-fopenmp", "-fPIC",
+           "-shared", "-Wall", "-Wextra"]
+
+_lib = None
+
+
+def build(force: bool = False) -> Path:
+    """Compile the oracle shared object next to its source."""
+    if force or not _LIB.exists() or _LIB.stat().st_mtime < _SRC.stat().st_mtime:
+        tmp = _LIB.with_suffix(f".so.{os.getpid()}")
+        subprocess.run(["gcc", *_CFLAGS, "-o", str(tmp), str(_SRC), "-lm"], check=True)
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    if _lib is not None:
+        return _lib
+    build()
+    lib = ctypes.CDLL(str(_LIB))
+    P = ctypes.c_void_p
+    i64, i32, f32 = ctypes.c_int64, ctypes.c_int32, ctypes.c_float
+    lib.or_calibrate_ptf.argtypes = [P, i64, i32, i64, i32, P, P, P, P]
+    lib.or_calibrate_ptf.restype = ctypes.c_int
+    lib.or_ptf_quantize.argtypes = [P, i64, i32, i64, f32, i32, P, P, i64]
+    lib.or_ptf_quantize.restype = ctypes.c_int
+    lib.or_ptf_layernorm.argtypes = [P, i64, i32, i64, i32, P, P, P, f32, i32, P, i64, P, P]
+    lib.or_ptf_layernorm.restype = ctypes.c_int
+    lib.or_iexp_consts.argtypes = [f32, P, P, P]
+    lib.or_iexp_consts.restype = None
+    lib.or_iexp.argtypes = [i64, i32, i64, i64, i64]
+    lib.or_iexp.restype = ctypes.c_uint64
+    lib.or_ilog2.argtypes = [ctypes.c_uint64]
+    lib.or_ilog2.restype = i32
+    lib.or_lis_softmax.argtypes = [P, i64, i32, i64, f32, i32, P, i32, i32, P, i64, P]
+    lib.or_lis_softmax.restype = ctypes.c_int
+    lib.or_lis_attn_v.argtypes = [P, i64, P, i64, i32, i64, i32, i32, P, i64]
+    lib.or_lis_attn_v.restype = ctypes.c_int
+    lib.or_num_threads.argtypes = []
+    lib.or_num_threads.restype = ctypes.c_int
+    lib.or_set_num_threads.argtypes = [ctypes.c_int]
+    lib.or_set_num_threads.restype = None
+    _lib = lib
+    return lib
+
+
+def _ptr(a: np.ndarray | None):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    a = np.asarray(a)
+    if a.dtype != dtype:
+        raise TypeError(f"expected {dtype}, got {a.dtype}")
+    if not a.flags.c_contiguous:
+        a = np.ascontiguousarray(a)
+    return a
+
+
+def num_threads() -> int:
+    return int(_load().or_num_threads())
+
+
+def set_num_threads(n: int) -> None:
+    _load().or_set_num_threads(int(n))
+
+
+def calibrate_ptf(x: np.ndarray, K: int = 3):
+    """Eqs. 8-10: returns (s, zp, alpha[C] uint8, sse[C, K+1] float64)."""
+    x = _c(x, np.float32)
+    rows, C = x.shape
+    s = np.zeros(1, np.float32)
+    zp = np.zeros(1, np.int32)
+    alpha = np.zeros(C, np.uint8)
+    sse = np.zeros((C, K + 1), np.float64)
+    rc = _load().or_calibrate_ptf(_ptr(x), rows, C, C, K, _ptr(s), _ptr(zp), _ptr(alpha), _ptr(sse))
+    if rc:
+        raise ValueError("or_calibrate_ptf rejected its arguments")
+    return float(s[0]), int(zp[0]), alpha, sse
+
+
+def ptf_quantize(x: np.ndarray, s: float, zp: int, alpha: np.ndarray) -> np.ndarray:
+    """Eq. 7: fp32 [rows, C] -> uint8 codes."""
+    x = _c(x, np.float32)
+    alpha = _c(alpha, np.uint8)
+    rows, C = x.shape
+    out = np.zeros((rows, C), np.uint8)
+    rc = _load().or_ptf_quantize(_ptr(x), rows, C, C, np.float32(s), zp, _ptr(alpha), _ptr(out), C)
+    if rc:
+        raise ValueError("or_ptf_quantize rejected its arguments")
+    return out
+
+
+def ptf_layernorm(xq, zp_in, alpha, gamma, beta, s_out, zp_out):
+    """Supplement LayerNorm: returns (Y_Q uint8 [rows, C], M1 int64, M2 int64)."""
+    xq = _c(xq, np.uint8)
+    alpha = _c(alpha, np.uint8)
+    gamma = _c(gamma, np.float32)
+    beta = _c(beta, np.float32)
+    rows, C = xq.shape
+    y = np.zeros((rows, C), np.uint8)
+    m1 = np.zeros(rows, np.int64)
+    m2 = np.zeros(rows, np.int64)
+    rc = _load().or_ptf_layernorm(_ptr(xq), rows, C, C, zp_in, _ptr(alpha), _ptr(gamma), _ptr(beta),
+                                  np.float32(s_out), zp_out, _ptr(y), C, _ptr(m1), _ptr(m2))
+    if rc:
+        raise ValueError("or_ptf_layernorm rejected its arguments")
+    return y, m1, m2
+
+
+def iexp_consts(s: float):
+    a, b, c = ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64()
+    _load().or_iexp_consts(np.float32(s), ctypes.byref(a), ctypes.byref(b), ctypes.byref(c))
+    return a.value, b.value, c.value
+
+
+def iexp(q: int, s: float, n: int = 15) -> int:
+    """Algorithm 1 on one non-positive integer q."""
+    a, b, c = iexp_consts(s)
+    return int(_load().or_iexp(int(q), n, a, b, c))
+
+
+def ilog2(x: int) -> int:
+    """Algorithm 2's I-Log2."""
+    return int(_load().or_ilog2(int(x)))
+
+
+def lis_softmax(logits: np.ndarray, L: int, s: float, n: int = 15, bias=None, heads: int = 1,
+                window: int = 7):
+    """Algorithm 2 over rows of int8 logits [n_rows, >=L].
+
+    Returns (codes uint8 [n_rows, L], rowsum uint64 [n_rows])."""
+    logits = _c(logits, np.int8)
+    n_rows, ld = logits.shape
+    codes = np.zeros((n_rows, L), np.uint8)
+    rowsum = np.zeros(n_rows, np.uint64)
+    b = None if bias is None else _c(bias, np.int8)
+    rc = _load().or_lis_softmax(_ptr(logits), n_rows, L, ld, np.float32(s), n, _ptr(b),
+                                heads, window, _ptr(codes), L, _ptr(rowsum))
+    if rc:
+        raise ValueError("or_lis_softmax rejected its arguments")
+    return codes, rowsum
+
+
+def lis_attn_v(codes: np.ndarray, v: np.ndarray, zp_v: int = 0):
+    """Eq. 15: codes uint8 [BH*L, L], v int8 [BH, L, d] -> int32 [BH, L, d].
+
+    Returns (acc, overflowed)."""
+    codes = _c(codes, np.uint8)
+    v = _c(v, np.int8)
+    BH, L, d = v.shape
+    assert codes.shape[0] == BH * L and codes.shape[1] >= L
+    acc = np.zeros((BH, L, d), np.int32)
+    rc = _load().or_lis_attn_v(_ptr(codes), codes.shape[1], _ptr(v), d, zp_v, BH, L, d, _ptr(acc), d)
+    if rc not in (0, 3):
+        raise ValueError("or_lis_attn_v rejected its arguments")
+    return acc, rc == 3

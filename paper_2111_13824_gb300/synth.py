@@ -1,0 +1,184 @@
+"""Seeded synthetic workloads shaped like the paper's DeiT / ViT / Swin layers.
+
+This module only draws inputs; it holds none of the integer path's arithmetic
+(no PTF quantizer, no integer LayerNorm, no i-exp, no log2 code, no
+BitShift).  Both the CUDA path and the CPU oracle consume what it returns.
+
+Recipe (per layer l of a config with seed S, generator seeded with
+S * 1000 + l, draws in this fixed order):
+
+* LayerNorm input (fp32, ``[rows, C]``): per-channel range r_c drawn
+  log-normal(0, 1), then stretched in the log domain so that
+  max(r) / median(r) = 40 (the inter-channel variation reported for vision
+  transformers, Sec. 3.2).  ``outliers`` channels are then forced to
+  U(40, 60) x median.  Channel centre m_c ~ N(0, (r_c / 4)^2); values
+  m_c + (r_c / 6) N(0, 1).
+* Calibration batch: 32 images' worth of rows (``32 * tokens``) from the
+  same channel model.
+* gamma ~ N(1, 0.1^2), beta ~ N(0, 0.1^2).
+* Output quantizer of the LayerNorm: the min / max of a textbook fp64
+  LayerNorm of the calibration batch mapped to 0..255 (MinMax, as the paper
+  uses for activations).
+* Q, K ~ N(0, sigma^2) fp32 ``[BH, L, d]``, rounded symmetrically to int8;
+  the exact integer Q K^T times s_q s_k / sqrt(d) is mapped onto the full
+  int8 range by its min / max (``s_logit``).  sigma = 1 is the literal
+  config, sigma = 2 the "peaked" variant whose rows put most mass on a few
+  keys (Sec. 3.3: 98.8 % of ViT-L attention values are below 1/16).
+* V: int8 uniform in [-128, 127], zero point 0.
+* Swin relative-position bias: int8 ``[H, (2w-1)^2]`` uniform in [-16, 16].
+
+Rows of logits are padded to a multiple of 16 bytes (``ld_logit``).
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+
+import torch
+
+
+@dataclass(frozen=True)
+class Stage:
+    """One attention / LayerNorm shape inside a config."""
+    rows: int          # LayerNorm rows (tokens in the batch)
+    C: int             # channels
+    BH: int            # attention problems (batch x windows x heads)
+    H: int             # heads
+    L: int             # tokens per attention row
+    d: int             # head dimension
+    layers: int        # how many layers of this shape
+    calib_rows: int    # calibration rows (32 images)
+    window: int = 0    # Swin window side (0 = no relative-position bias)
+
+
+@dataclass(frozen=True)
+class Config:
+    name: str
+    seed: int
+    stages: tuple
+    K: int = 3
+    outliers: int = 0
+    first_tokens: int = 0   # tokens of the first layer per image x batch
+    note: str = ""
+
+    @property
+    def layers(self) -> int:
+        return sum(s.layers for s in self.stages)
+
+
+def _vit(name, seed, B, L, C, H, d, layers, outliers=0, note=""):
+    st = Stage(rows=B * L, C=C, BH=B * H, H=H, L=L, d=d, layers=layers, calib_rows=32 * L)
+    return Config(name=name, seed=seed, stages=(st,), outliers=outliers, first_tokens=B * L, note=note)
+
+
+def _swin():
+    B, w = 64, 7
+    stages = []
+    for C, H, depth, side in ((96, 3, 2, 56), (192, 6, 2, 28), (384, 12, 18, 14), (768, 24, 2, 7)):
+        tokens = side * side
+        nwin = (side // w) ** 2
+        stages.append(Stage(rows=B * tokens, C=C, BH=B * nwin * H, H=H, L=w * w, d=32,
+                            layers=depth, calib_rows=32 * tokens, window=w))
+    return Config(name="swin_s", seed=4, stages=tuple(stages), first_tokens=B * 56 * 56,
+                  note="Swin-S, 7x7 windows, relative-position bias")
+
+
+CONFIGS = {
+    "deit_t": _vit("deit_t", 0, 1, 197, 192, 3, 64, 1, note="DeiT-T block, batch 1"),
+    "deit_s": _vit("deit_s", 1, 64, 197, 384, 6, 64, 12, note="DeiT-S stack, batch 64"),
+    "vit_b": _vit("vit_b", 2, 64, 197, 768, 12, 64, 12, outliers=8, note="ViT-B/16 stack, batch 64"),
+    "vit_l384": _vit("vit_l384", 3, 32, 577, 1024, 16, 64, 24, note="ViT-L/16 at 384 px, batch 32"),
+    "swin_s": _swin(),
+}
+
+
+def ld_pad(n: int, align: int = 16) -> int:
+    return (n + align - 1) // align * align
+
+
+def layer_stage(cfg: Config, layer: int) -> Stage:
+    for st in cfg.stages:
+        if layer < st.layers:
+            return st
+        layer -= st.layers
+    raise IndexError("layer out of range")
+
+
+def _gen(seed: int, device) -> torch.Generator:
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    return g
+
+
+def _channel_model(g, C, outliers, device):
+    r = torch.exp(torch.randn(C, generator=g, device=device, dtype=torch.float64))
+    med = torch.median(r)
+    lmax, lmed = torch.log(r.max()), torch.log(med)
+    if float(lmax - lmed) > 0:
+        r = torch.exp(lmed + (torch.log(r) - lmed) * (math.log(40.0) / (lmax - lmed)))
+    if outliers:
+        idx = torch.randperm(C, generator=g, device=device)[:outliers]
+        r[idx] = med * (40.0 + 20.0 * torch.rand(outliers, generator=g, device=device, dtype=torch.float64))
+    m = 0.25 * r * torch.randn(C, generator=g, device=device, dtype=torch.float64)
+    return r, m
+
+
+def _channel_values(g, rows, r, m):
+    z = torch.randn(rows, r.numel(), generator=g, device=r.device, dtype=torch.float64)
+    return (m + (r / 6.0) * z).to(torch.float32)
+
+
+def ln_inputs(cfg: Config, layer: int, device="cpu", rows: int | None = None):
+    """LayerNorm-side inputs of one layer: x, calibration x, gamma, beta, s_out, zp_out."""
+    st = layer_stage(cfg, layer)
+    g = _gen(cfg.seed * 1000 + layer, device)
+    r, m = _channel_model(g, st.C, cfg.outliers, device)
+    n = st.rows if rows is None else rows
+    x = _channel_values(g, n, r, m)
+    xc = _channel_values(g, st.calib_rows, r, m)
+    gamma = (1.0 + 0.1 * torch.randn(st.C, generator=g, device=device)).to(torch.float32)
+    beta = (0.1 * torch.randn(st.C, generator=g, device=device)).to(torch.float32)
+    # output quantizer: MinMax of a textbook fp64 LayerNorm of the calibration batch
+    xd = xc.double()
+    mu = xd.mean(dim=1, keepdim=True)
+    var = xd.var(dim=1, unbiased=False, keepdim=True)
+    yf = (xd - mu) / torch.sqrt(var + 1e-6) * gamma.double() + beta.double()
+    lo, hi = float(yf.min()), float(yf.max())
+    s_out = (hi - lo) / 255.0
+    zp_out = int(min(255, max(0, round(-lo / s_out))))
+    return dict(x=x, x_calib=xc, gamma=gamma, beta=beta, s_out=float(torch.tensor(s_out, dtype=torch.float32)),
+                zp_out=zp_out, C=st.C, rows=n)
+
+
+def attn_inputs(cfg: Config, layer: int, device="cpu", sigma: float = 1.0, bh: int | None = None):
+    """Attention-side inputs of one layer: int8 logits [BH*L, ld], s_logit, int8 V [BH, L, d], bias."""
+    st = layer_stage(cfg, layer)
+    g = _gen(cfg.seed * 1000 + layer, device)
+    # skip the LayerNorm draws so that the attention draws follow them in the fixed order
+    r, m = _channel_model(g, st.C, cfg.outliers, device)
+    _ = torch.randn(st.rows + st.calib_rows, st.C, generator=g, device=device, dtype=torch.float64)
+    _ = torch.randn(2 * st.C, generator=g, device=device)
+    BH = st.BH if bh is None else bh
+    L, d = st.L, st.d
+    q = sigma * torch.randn(BH, L, d, generator=g, device=device)
+    k = sigma * torch.randn(BH, L, d, generator=g, device=device)
+    v = torch.randint(-128, 128, (BH, L, d), generator=g, device=device, dtype=torch.int16).to(torch.int8)
+    bias = None
+    if st.window:
+        nb = (2 * st.window - 1) ** 2
+        bias = torch.randint(-16, 17, (st.H, nb), generator=g, device=device, dtype=torch.int16).to(torch.int8)
+    sq = float(q.abs().max()) / 127.0
+    sk = float(k.abs().max()) / 127.0
+    qi = torch.clamp(torch.round(q / sq), -127, 127)
+    ki = torch.clamp(torch.round(k / sk), -127, 127)
+    prod = torch.bmm(qi, ki.transpose(1, 2))  # exact integers (|sum| < 2^24 in fp32)
+    real = prod * (sq * sk / math.sqrt(d))
+    lo, hi = float(real.min()), float(real.max())
+    s_logit = max(hi - lo, 1e-6) / 255.0
+    s_logit = float(torch.tensor(s_logit, dtype=torch.float32))
+    qq = torch.clamp(torch.round((real - lo) / s_logit), 0, 255) - 128
+    ld = ld_pad(L)
+    logits = torch.zeros(BH * L, ld, dtype=torch.int8, device=device)
+    logits[:, :L] = qq.reshape(BH * L, L).to(torch.int8)
+    return dict(logits=logits, ld_logit=ld, s_logit=s_logit, v=v.contiguous(), bias=bias,
+                heads=st.H, window=st.window, BH=BH, L=L, d=d)
