@@ -174,10 +174,11 @@ OR_EXPORT int or_ptf_quantize(const float *x, int64_t rows, int32_t C, int64_t l
  *   D  = C*M2 - M1^2, so sigma ~ (s/C) sqrt(D), mu = (s/C) M1.
  * The affine terms with s_in = s cancel:
  *   A = gamma * C / (s_out sqrt(D)),  B = beta/s_out - (gamma/s_out) M1/sqrt(D).
- * Evaluation order (fixed, no fused multiply-add):
- *   sd = sqrt((double)D); r = (float)(C/sd); t = (float)(M1/sd)
- *   gs = (float)(gamma/s_out); bs = (float)(beta/s_out)     (fp64 divisions)
- *   A = gs*r;  B = bs - gs*t                                  (fp32)
+ * Evaluation order (fixed, no fused multiply-add, every operation fp32 and
+ * correctly rounded; the paper does not fix the precision of these terms):
+ *   sd = sqrtf((float)D); r = C / sd; t = (float)M1 / sd
+ *   gs = gamma / s_out; bs = beta / s_out
+ *   A = gs*r;  B = bs - gs*t
  * Readings where the paper is silent:
  *   - epsilon is dropped by the paper; for D == 0 (constant row) X - mu is
  *     exactly zero, so r = t = 0 (the epsilon -> 0 limit: output = beta).
@@ -208,17 +209,16 @@ OR_EXPORT int or_ptf_layernorm(const uint8_t *xq, int64_t rows, int32_t C, int64
         if (m1_out) m1_out[r] = M1;
         if (m2_out) m2_out[r] = M2;
         int64_t D = (int64_t)C * M2 - M1 * M1;
-        double rd = 0.0, td = 0.0;
+        float rf = 0.0f, tf = 0.0f;
         if (D != 0) {
-            double sd = sqrt((double)D);
-            rd = (double)C / sd;
-            td = (double)M1 / sd;
+            float sd = sqrtf((float)D);
+            rf = (float)C / sd;
+            tf = (float)M1 / sd;
         }
-        float rf = (float)rd, tf = (float)td;
         for (int32_t c = 0; c < C; ++c) {
             int64_t xh = ((int64_t)xr[c] - zp_in) * ((int64_t)1 << alpha[c]);
-            float gs = (float)((double)gamma[c] / (double)s_out);
-            float bs = (float)((double)beta[c] / (double)s_out);
+            float gs = gamma[c] / s_out;
+            float bs = beta[c] / s_out;
             float A = gs * rf;
             float gt = gs * tf;
             float B = bs - gt;
