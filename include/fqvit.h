@@ -1,0 +1,216 @@
+/*
+ * fqvit.h -- C ABI of libfqvit.so: the integer inference hot path of
+ * FQ-ViT ("Post-Training Quantization for Fully Quantized Vision
+ * Transformer", IJCAI 2022) on one GB300 GPU (sm_103a).
+ *
+ * Conventions for every entry point
+ *   - Pointers are DEVICE pointers owned by the caller unless stated
+ *     otherwise.  Nothing is retained after the call returns; the library
+ *     allocates no device memory.
+ *   - Every call is asynchronous on `stream` (a cudaStream_t passed as
+ *     void*; NULL is the legacy default stream).  Results are ready when
+ *     the stream reaches the call.
+ *   - Matrices are row-major.  ld_* are row strides in ELEMENTS of the
+ *     matrix's type (bytes for 8-bit data).
+ *   - Return value: FQVIT_OK or one of the error codes below.  Arguments
+ *     are validated on the host before anything is launched; on error
+ *     nothing is launched and fqvit_last_error() describes the problem.
+ *   - Scalars that the paper computes offline after calibration (s, zp,
+ *     s_out, zp_out, s_logit) are passed by value.
+ */
+#ifndef FQVIT_H
+#define FQVIT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define FQVIT_API __attribute__((visibility("default")))
+#else
+#define FQVIT_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define FQVIT_OK 0
+#define FQVIT_ERR_INVALID_ARG 1 /* NULL, bad size, stride or alignment            */
+#define FQVIT_ERR_UNSUPPORTED 2 /* valid in the paper, not handled by this build  */
+#define FQVIT_ERR_RANGE 3       /* reserved: a value outside an exactness bound   */
+#define FQVIT_ERR_CUDA 4        /* a CUDA launch or runtime call failed           */
+
+/* Library version, (major << 16) | minor. */
+FQVIT_API int fqvit_version(void);
+
+/* Thread-local description of the last non-OK status returned on this
+ * thread (empty string if none).  Valid until the next call on the thread. */
+FQVIT_API const char *fqvit_last_error(void);
+
+/* ------------------------------------------------------------------ */
+/* Power-of-Two Factor calibration (Sec. 3.2, Eqs. 8-10)              */
+/* ------------------------------------------------------------------ */
+
+/* Bytes of device workspace fqvit_calibrate_ptf needs (a few KB). */
+FQVIT_API size_t fqvit_calibrate_workspace_size(int64_t rows, int32_t C, int32_t K);
+
+/*
+ * Layer-wise scale s and zero point zp (Eqs. 8-9) and per-channel factors
+ * alpha_c in {0..K} (Eq. 10) from a calibration batch x [rows, C] fp32.
+ *   s0 = (max x - min x) / (2^bits - 1) in fp32 (a zero range counts as 1),
+ *   s  = s0 / 2^K,  zp = clip(rint(-min x / s0), 0, 2^bits - 1).
+ *   err_c(a) = sum over rows, in ascending row order, in fp64, of
+ *     (x - clip(rint(x / (2^a s)), -zp, 255 - zp) * 2^a s)^2,
+ *   the quotient, rint, product and difference being fp32; alpha_c is the
+ *   smallest a with the least error.
+ * Outputs (device): s[1], zp[1], alpha[C]; sse_opt[C][K+1] if not NULL.
+ * workspace: device buffer of fqvit_calibrate_workspace_size() bytes,
+ *   8-byte aligned; its contents on entry do not matter.
+ * Supported: bits == 8, 0 <= K <= 7, 1 <= C <= 8192, ld_x >= C, rows >= 1.
+ * x must be finite.
+ */
+FQVIT_API int fqvit_calibrate_ptf(const float *x, int64_t rows, int32_t C, int64_t ld_x,
+                        int32_t bits, int32_t K, float *s, int32_t *zp, uint8_t *alpha,
+                        double *sse_opt, void *workspace, size_t ws_bytes, void *stream);
+
+/*
+ * PTF quantizer (Eq. 7): xq[r][c] = clip(rint(x[r][c] / (2^alpha_c s)) + zp, 0, 255),
+ * fp32 quotient, ties to even.  x [rows, C] fp32, alpha [C] (device),
+ * xq [rows, C] uint8 with stride ld_q.
+ */
+FQVIT_API int fqvit_ptf_quantize(const float *x, int64_t rows, int32_t C, int64_t ld_x, float s,
+                       int32_t zp, const uint8_t *alpha, uint8_t *xq, int64_t ld_q,
+                       void *stream);
+
+/* ------------------------------------------------------------------ */
+/* Integer LayerNorm on PTF-quantized input (supplement, "Quantized    */
+/* Inference of LayerNorm", Eqs. 11-13 and the dyadic requantization)  */
+/* ------------------------------------------------------------------ */
+
+/*
+ * Per row of xq [rows, C] (uint8, stride ld_in):
+ *   Xh_c = (xq_c - zp_in) * 2^alpha_c;  M1 = sum Xh;  M2 = sum Xh^2 (int64);
+ *   D = C M2 - M1^2;  sd = sqrtf((float)D);  r = C / sd;  t = (float)M1 / sd
+ *   (fp32, correctly rounded; r = t = 0 when D == 0, i.e. a constant row);
+ *   gs_c = gamma_c / s_out, bs_c = beta_c / s_out (fp32);
+ *   A = gs_c r, B = bs_c - gs_c t (fp32, no fused multiply-add);
+ *   N1 = min(7 - floor(log2 |A|), 31), N2 = floor(|A| 2^N1) (A == 0: 0, 0);
+ *   Bq = rint(B 2^N1);  Y = clip(round_half_up((sign(A) N2 Xh + Bq) / 2^N1)
+ *                              + zp_out, 0, 255)   (N1 < 0 multiplies).
+ * The input scale s cancels (A and B are independent of it) and is not an
+ * argument.  Output yq [rows, C] uint8, stride ld_out.  m1_opt / m2_opt
+ * (int64 [rows]) receive M1 / M2 when not NULL.
+ * Supported: 1 <= C <= 8192, alpha_c <= 7, s_out > 0 and finite.
+ */
+FQVIT_API int fqvit_ptf_layernorm(const uint8_t *xq, int64_t rows, int32_t C, int64_t ld_in,
+                        int32_t zp_in, const uint8_t *alpha, const float *gamma,
+                        const float *beta, float s_out, int32_t zp_out, uint8_t *yq,
+                        int64_t ld_out, int64_t *m1_opt, int64_t *m2_opt, void *stream);
+
+/* ------------------------------------------------------------------ */
+/* Log-Int-Softmax (Sec. 3.3, Eqs. 16-17; supplement Algorithms 1-2)  */
+/* ------------------------------------------------------------------ */
+
+/* Relative-position bias for windowed (Swin) attention, not in the paper:
+ * table [heads][(2 window - 1)^2] int8 (device), same scale as the
+ * logits; the entry for query i, key j of a window is at
+ * (y_i - y_j + window - 1)(2 window - 1) + (x_i - x_j + window - 1)
+ * with y = index / window, x = index % window. */
+typedef struct fqvit_relpos_bias {
+    const int8_t *table;
+    int32_t heads;
+    int32_t window;
+} fqvit_relpos_bias;
+
+/*
+ * Log-Int-Softmax of n_rows rows of int8 logits (stride ld_logit bytes,
+ * L keys per row; rows ordered [batch][head][query]):
+ *   q~ = q (+ bias) - max;  e = i-exp(q~) with q_ln2 = floor(-ln2/s),
+ *   q_b = floor(1.353/s), q_c = floor(0.344/(0.3585 s^2)) in fp64, the
+ *   clamp q~ >= n q_ln2, z = q~ / q_ln2, q_p = q~ - z q_ln2,
+ *   e = ((q_p + q_b)^2 + q_c) << (n - z)   (Algorithm 1);
+ *   S = sum e;  q_rev = floor((2S + e) / (2e))  (round half up);
+ *   code = min(I-Log2(q_rev), 15)  (Algorithm 2, Eq. 33; I-Log2(x) = M + bit
+ *   M-1 of x, M the index of the leading one).
+ * The code is Attn_Q (4 bits); the LIS output of Eq. 17 is 15 - code with
+ * scale 1/2^15.  codes: packed nibbles, code of key j in byte j/2 of the
+ * row (low nibble for even j), row stride ld_codes >= ceil(L/2) bytes; a
+ * pad nibble of odd L is written as 0.  rowsum_opt (uint64 [n_rows])
+ * receives S when not NULL.
+ * Supported: n_shift == 15 (the exponent headroom n of Algorithm 1), 1 <= L
+ * <= 1024, s_logit in [2^-7, 0.5] (the range where every i-exp value fits 31
+ * bits), ld_logit a multiple of 4 and >= L.  With bias_opt: window^2 == L,
+ * heads >= 1, n_rows a multiple of heads * L.
+ */
+FQVIT_API int fqvit_lis_softmax(const int8_t *logits, int64_t n_rows, int32_t L, int64_t ld_logit,
+                      float s_logit, int32_t n_shift, const fqvit_relpos_bias *bias_opt,
+                      uint8_t *codes, int64_t ld_codes, uint64_t *rowsum_opt, void *stream);
+
+/*
+ * BitShift attention times values (Eq. 15; supplement Attn.V):
+ *   acc[bh][i][t] = sum_j (v[bh][j][t] - zp_v) << (15 - code[bh][i][j])
+ * (a left shift of a negative value is a multiplication by 2^(15 - code));
+ * the real result is acc * s_V / 2^15.
+ * codes: packed nibbles as written by fqvit_lis_softmax, [BH * L] rows of
+ * ld_codes bytes.  v: int8 [BH][L][ld_v] (head stride L * ld_v).  acc: int32
+ * [BH][L][ld_acc] (head stride L * ld_acc).  range_flag_opt (device int32)
+ * is set to 1 if some row's sum could leave int32 (arbitrary codes only;
+ * never for codes made by fqvit_lis_softmax); it is not cleared.
+ * Supported: d in {32, 64}, 1 <= L <= 1024, |zp_v| <= 255.
+ */
+FQVIT_API int fqvit_lis_attn_v(const uint8_t *codes, int64_t ld_codes, const int8_t *v, int64_t ld_v,
+                     int32_t zp_v, int64_t BH, int32_t L, int32_t d, int32_t *acc,
+                     int64_t ld_acc, int32_t *range_flag_opt, void *stream);
+
+/*
+ * Fused Log-Int-Softmax and BitShift attention times values: the same
+ * result as fqvit_lis_softmax followed by fqvit_lis_attn_v, without the
+ * codes leaving the chip unless codes_opt is not NULL (then they are also
+ * written, packed as above).  logits [BH * L] rows of ld_logit bytes, v and
+ * acc as in fqvit_lis_attn_v.
+ * Supported: as fqvit_lis_softmax and fqvit_lis_attn_v.
+ */
+FQVIT_API int fqvit_lis_attention(const int8_t *logits, int64_t ld_logit, float s_logit,
+                        int32_t n_shift, const fqvit_relpos_bias *bias_opt, const int8_t *v,
+                        int64_t ld_v, int32_t zp_v, int64_t BH, int32_t L, int32_t d,
+                        int32_t *acc, int64_t ld_acc, uint8_t *codes_opt, int64_t ld_codes,
+                        void *stream);
+
+/* ------------------------------------------------------------------ */
+/* One layer: norm1 LayerNorm and the attention core (Fig. 4 dataflow) */
+/* ------------------------------------------------------------------ */
+
+typedef struct fqvit_block_desc {
+    /* PTF LayerNorm (see fqvit_ptf_layernorm), contiguous rows */
+    const uint8_t *xq;
+    int64_t rows;
+    int32_t C;
+    int32_t zp_in;
+    const uint8_t *alpha;
+    const float *gamma;
+    const float *beta;
+    float s_out;
+    int32_t zp_out;
+    uint8_t *yq;
+    /* attention core (see fqvit_lis_attention); logits rows padded to ld_logit */
+    const int8_t *logits;
+    int64_t ld_logit;
+    float s_logit;
+    const int8_t *v;   /* [BH][L][d] contiguous */
+    int32_t zp_v;
+    int64_t BH;
+    int32_t L;
+    int32_t d;
+    const fqvit_relpos_bias *bias; /* NULL = none */
+    int32_t *acc;      /* [BH][L][d] contiguous */
+} fqvit_block_desc;
+
+/* Runs the LayerNorm and the fused attention of one layer on `stream`
+ * (two launches, in that order).  Supported: as the two calls. */
+FQVIT_API int fqvit_block_int(const fqvit_block_desc *desc, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FQVIT_H */

@@ -1,0 +1,217 @@
+// api.cu -- extern "C" entry points of libfqvit.so (declared in
+// include/fqvit.h): host-side validation, then launches on the caller's
+// stream.  Nothing is allocated and nothing is retained.
+#include "fqvit.h"
+#include "fqvit_internal.cuh"
+
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+int fail(int code, const char *fmt, ...)
+{
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int ok()
+{
+    g_err[0] = '\0';
+    return FQVIT_OK;
+}
+
+int cuda_status(cudaError_t e, const char *what)
+{
+    if (e != cudaSuccess) return fail(FQVIT_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+    return ok();
+}
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+cudaStream_t as_stream(void *s) { return reinterpret_cast<cudaStream_t>(s); }
+
+// s_logit range in which every i-exp value fits 31 bits (see lis.cu)
+bool logit_scale_ok(float s) { return s >= 0.0078125f && s <= 0.5f; }
+
+}  // namespace
+
+namespace fqvit {
+
+int sm_count()
+{
+    static int cached[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+    if (cached[dev] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+        cached[dev] = n;
+    }
+    return cached[dev];
+}
+
+}  // namespace fqvit
+
+extern "C" {
+
+int fqvit_version(void) { return (0 << 16) | 1; }
+
+const char *fqvit_last_error(void) { return g_err; }
+
+size_t fqvit_calibrate_workspace_size(int64_t rows, int32_t C, int32_t K)
+{
+    if (C < 1 || K < 0 || K > 7) return 0;
+    return fqvit::calibrate_workspace_bytes(rows, C, K);
+}
+
+int fqvit_calibrate_ptf(const float *x, int64_t rows, int32_t C, int64_t ld_x, int32_t bits,
+                        int32_t K, float *s, int32_t *zp, uint8_t *alpha, double *sse_opt,
+                        void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!x || !s || !zp || !alpha || !workspace) return fail(FQVIT_ERR_INVALID_ARG, "calibrate_ptf: NULL pointer");
+    if (rows < 1 || C < 1 || C > 8192 || ld_x < C)
+        return fail(FQVIT_ERR_INVALID_ARG, "calibrate_ptf: bad shape rows=%lld C=%d ld_x=%lld",
+                    (long long)rows, C, (long long)ld_x);
+    if (bits != 8) return fail(FQVIT_ERR_UNSUPPORTED, "calibrate_ptf: bits=%d (only 8)", bits);
+    if (K < 0 || K > 7) return fail(FQVIT_ERR_UNSUPPORTED, "calibrate_ptf: K=%d (0..7)", K);
+    if (!aligned(x, 4) || !aligned(s, 4) || !aligned(zp, 4) || !aligned(workspace, 8) ||
+        (sse_opt && !aligned(sse_opt, 8)))
+        return fail(FQVIT_ERR_INVALID_ARG, "calibrate_ptf: misaligned pointer");
+    size_t need = fqvit::calibrate_workspace_bytes(rows, C, K);
+    if (ws_bytes < need)
+        return fail(FQVIT_ERR_INVALID_ARG, "calibrate_ptf: workspace %zu bytes, need %zu", ws_bytes, need);
+    return cuda_status(fqvit::launch_calibrate(x, rows, C, ld_x, K, s, zp, alpha, sse_opt, workspace,
+                                               as_stream(stream)),
+                       "calibrate_ptf");
+}
+
+int fqvit_ptf_quantize(const float *x, int64_t rows, int32_t C, int64_t ld_x, float s, int32_t zp,
+                       const uint8_t *alpha, uint8_t *xq, int64_t ld_q, void *stream)
+{
+    if (!x || !alpha || !xq) return fail(FQVIT_ERR_INVALID_ARG, "ptf_quantize: NULL pointer");
+    if (rows < 1 || C < 1 || C > 8192 || ld_x < C || ld_q < C)
+        return fail(FQVIT_ERR_INVALID_ARG, "ptf_quantize: bad shape");
+    if (!(s > 0.0f) || !(s < 3.0e38f)) return fail(FQVIT_ERR_INVALID_ARG, "ptf_quantize: s must be positive and finite");
+    if (zp < 0 || zp > 255) return fail(FQVIT_ERR_INVALID_ARG, "ptf_quantize: zp=%d", zp);
+    if (!aligned(x, 4)) return fail(FQVIT_ERR_INVALID_ARG, "ptf_quantize: misaligned x");
+    return cuda_status(fqvit::launch_quantize(x, rows, C, ld_x, s, zp, alpha, xq, ld_q, as_stream(stream)),
+                       "ptf_quantize");
+}
+
+int fqvit_ptf_layernorm(const uint8_t *xq, int64_t rows, int32_t C, int64_t ld_in, int32_t zp_in,
+                        const uint8_t *alpha, const float *gamma, const float *beta, float s_out,
+                        int32_t zp_out, uint8_t *yq, int64_t ld_out, int64_t *m1_opt, int64_t *m2_opt,
+                        void *stream)
+{
+    if (!xq || !alpha || !gamma || !beta || !yq) return fail(FQVIT_ERR_INVALID_ARG, "ptf_layernorm: NULL pointer");
+    if (rows < 1 || C < 1 || C > 8192 || ld_in < C || ld_out < C)
+        return fail(FQVIT_ERR_INVALID_ARG, "ptf_layernorm: bad shape rows=%lld C=%d", (long long)rows, C);
+    if (zp_in < 0 || zp_in > 255 || zp_out < 0 || zp_out > 255)
+        return fail(FQVIT_ERR_INVALID_ARG, "ptf_layernorm: zero point outside 0..255");
+    if (!(s_out > 0.0f) || !(s_out < 3.0e38f))
+        return fail(FQVIT_ERR_INVALID_ARG, "ptf_layernorm: s_out must be positive and finite");
+    if (!aligned(gamma, 4) || !aligned(beta, 4) || (m1_opt && !aligned(m1_opt, 8)) || (m2_opt && !aligned(m2_opt, 8)))
+        return fail(FQVIT_ERR_INVALID_ARG, "ptf_layernorm: misaligned pointer");
+    fqvit::LnArgs a{xq, rows, C, ld_in, zp_in, alpha, gamma, beta, s_out, zp_out, yq, ld_out, m1_opt, m2_opt};
+    return cuda_status(fqvit::launch_layernorm(a, as_stream(stream)), "ptf_layernorm");
+}
+
+static int check_lis(const int8_t *logits, int64_t n_rows, int32_t L, int64_t ld_logit, float s_logit,
+                     int32_t n_shift, const fqvit_relpos_bias *bias, const char *who)
+{
+    if (!logits) return fail(FQVIT_ERR_INVALID_ARG, "%s: NULL logits", who);
+    if (n_rows < 1 || L < 1 || ld_logit < L) return fail(FQVIT_ERR_INVALID_ARG, "%s: bad shape", who);
+    if (L > 1024) return fail(FQVIT_ERR_UNSUPPORTED, "%s: L=%d (at most 1024)", who, L);
+    if (ld_logit % 4 != 0 || !aligned(logits, 4))
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: logits rows must be 4-byte aligned (ld %% 4 == 0)", who);
+    if (n_shift != 15) return fail(FQVIT_ERR_UNSUPPORTED, "%s: n_shift=%d (only 15)", who, n_shift);
+    if (!logit_scale_ok(s_logit))
+        return fail(FQVIT_ERR_UNSUPPORTED, "%s: s_logit=%g outside [2^-7, 0.5]", who, (double)s_logit);
+    if (bias) {
+        if (!bias->table || bias->heads < 1 || bias->window < 1)
+            return fail(FQVIT_ERR_INVALID_ARG, "%s: bad relative-position bias", who);
+        if (bias->window * bias->window != L)
+            return fail(FQVIT_ERR_INVALID_ARG, "%s: window^2 != L", who);
+        if (n_rows % ((int64_t)bias->heads * L) != 0)
+            return fail(FQVIT_ERR_INVALID_ARG, "%s: rows not a multiple of heads*L", who);
+        if ((int64_t)bias->heads * (2 * bias->window - 1) * (2 * bias->window - 1) > 64 * 1024)
+            return fail(FQVIT_ERR_UNSUPPORTED, "%s: bias table too large", who);
+    }
+    return FQVIT_OK;
+}
+
+int fqvit_lis_softmax(const int8_t *logits, int64_t n_rows, int32_t L, int64_t ld_logit, float s_logit,
+                      int32_t n_shift, const fqvit_relpos_bias *bias_opt, uint8_t *codes, int64_t ld_codes,
+                      uint64_t *rowsum_opt, void *stream)
+{
+    int rc = check_lis(logits, n_rows, L, ld_logit, s_logit, n_shift, bias_opt, "lis_softmax");
+    if (rc) return rc;
+    if (!codes) return fail(FQVIT_ERR_INVALID_ARG, "lis_softmax: NULL codes");
+    if (ld_codes < (L + 1) / 2) return fail(FQVIT_ERR_INVALID_ARG, "lis_softmax: ld_codes < ceil(L/2)");
+    if (rowsum_opt && !aligned(rowsum_opt, 8)) return fail(FQVIT_ERR_INVALID_ARG, "lis_softmax: misaligned rowsum");
+    fqvit::LisArgs a{logits, n_rows, L, ld_logit, s_logit,
+                     bias_opt ? bias_opt->table : nullptr, bias_opt ? bias_opt->heads : 1,
+                     bias_opt ? bias_opt->window : 0, codes, ld_codes,
+                     reinterpret_cast<uint64_t *>(rowsum_opt)};
+    return cuda_status(fqvit::launch_lis_softmax(a, as_stream(stream)), "lis_softmax");
+}
+
+static int check_attnv(const int8_t *v, int64_t ld_v, int32_t zp_v, int64_t BH, int32_t L, int32_t d,
+                       const int32_t *acc, int64_t ld_acc, const char *who)
+{
+    if (!v || !acc) return fail(FQVIT_ERR_INVALID_ARG, "%s: NULL pointer", who);
+    if (BH < 1 || L < 1 || BH > 65535) return fail(FQVIT_ERR_INVALID_ARG, "%s: bad shape BH=%lld L=%d", who, (long long)BH, L);
+    if (L > 1024) return fail(FQVIT_ERR_UNSUPPORTED, "%s: L=%d (at most 1024)", who, L);
+    if (d != 32 && d != 64) return fail(FQVIT_ERR_UNSUPPORTED, "%s: d=%d (32 or 64)", who, d);
+    if (ld_v < d || ld_acc < d) return fail(FQVIT_ERR_INVALID_ARG, "%s: stride below d", who);
+    if (zp_v < -255 || zp_v > 255) return fail(FQVIT_ERR_UNSUPPORTED, "%s: |zp_v| > 255", who);
+    if (!aligned(acc, 4)) return fail(FQVIT_ERR_INVALID_ARG, "%s: misaligned acc", who);
+    return FQVIT_OK;
+}
+
+int fqvit_lis_attn_v(const uint8_t *codes, int64_t ld_codes, const int8_t *v, int64_t ld_v, int32_t zp_v,
+                     int64_t BH, int32_t L, int32_t d, int32_t *acc, int64_t ld_acc, int32_t *range_flag_opt,
+                     void *stream)
+{
+    int rc = check_attnv(v, ld_v, zp_v, BH, L, d, acc, ld_acc, "lis_attn_v");
+    if (rc) return rc;
+    if (!codes || ld_codes < (L + 1) / 2) return fail(FQVIT_ERR_INVALID_ARG, "lis_attn_v: bad codes");
+    fqvit::AttnVArgs a{codes, ld_codes, v, ld_v, zp_v, BH, L, d, acc, ld_acc, range_flag_opt};
+    return cuda_status(fqvit::launch_lis_attn_v(a, as_stream(stream)), "lis_attn_v");
+}
+
+int fqvit_lis_attention(const int8_t *logits, int64_t ld_logit, float s_logit, int32_t n_shift,
+                        const fqvit_relpos_bias *bias_opt, const int8_t *v, int64_t ld_v, int32_t zp_v,
+                        int64_t BH, int32_t L, int32_t d, int32_t *acc, int64_t ld_acc, uint8_t *codes_opt,
+                        int64_t ld_codes, void *stream)
+{
+    int rc = check_attnv(v, ld_v, zp_v, BH, L, d, acc, ld_acc, "lis_attention");
+    if (rc) return rc;
+    rc = check_lis(logits, BH * L, L, ld_logit, s_logit, n_shift, bias_opt, "lis_attention");
+    if (rc) return rc;
+    if (codes_opt && ld_codes < (L + 1) / 2) return fail(FQVIT_ERR_INVALID_ARG, "lis_attention: ld_codes < ceil(L/2)");
+    fqvit::LisArgs la{logits, BH * L, L, ld_logit, s_logit,
+                      bias_opt ? bias_opt->table : nullptr, bias_opt ? bias_opt->heads : 1,
+                      bias_opt ? bias_opt->window : 0, codes_opt, ld_codes, nullptr};
+    fqvit::AttnVArgs a{nullptr, 0, v, ld_v, zp_v, BH, L, d, acc, ld_acc, nullptr};
+    return cuda_status(fqvit::launch_lis_attention(la, a, as_stream(stream)), "lis_attention");
+}
+
+int fqvit_block_int(const fqvit_block_desc *b, void *stream)
+{
+    if (!b) return fail(FQVIT_ERR_INVALID_ARG, "block_int: NULL descriptor");
+    int rc = fqvit_ptf_layernorm(b->xq, b->rows, b->C, b->C, b->zp_in, b->alpha, b->gamma, b->beta, b->s_out,
+                                 b->zp_out, b->yq, b->C, nullptr, nullptr, stream);
+    if (rc) return rc;
+    return fqvit_lis_attention(b->logits, b->ld_logit, b->s_logit, 15, b->bias, b->v, b->d, b->zp_v, b->BH,
+                               b->L, b->d, b->acc, b->d, nullptr, 0, stream);
+}
+
+}  // extern "C"

@@ -1,0 +1,75 @@
+// fqvit_internal.cuh -- declarations shared by the host entry points
+// (api.cu) and the kernel files.  Nothing here is part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace fqvit {
+
+// Number of SMs of the current device (cached per device).
+int sm_count();
+
+// ---- PTF calibration / quantizer (ptf.cu) ---------------------------------
+size_t calibrate_workspace_bytes(int64_t rows, int C, int K);
+cudaError_t launch_calibrate(const float *x, int64_t rows, int C, int64_t ld_x, int K, float *s,
+                             int32_t *zp, uint8_t *alpha, double *sse, void *ws,
+                             cudaStream_t st);
+cudaError_t launch_quantize(const float *x, int64_t rows, int C, int64_t ld_x, float s,
+                            int32_t zp, const uint8_t *alpha, uint8_t *xq, int64_t ld_q,
+                            cudaStream_t st);
+
+// ---- integer LayerNorm (layernorm.cu) -------------------------------------
+struct LnArgs {
+    const uint8_t *xq;
+    int64_t rows;
+    int C;
+    int64_t ld_in;
+    int zp_in;
+    const uint8_t *alpha;
+    const float *gamma;
+    const float *beta;
+    float s_out;
+    int zp_out;
+    uint8_t *yq;
+    int64_t ld_out;
+    int64_t *m1;
+    int64_t *m2;
+};
+cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st);
+
+// ---- Log-Int-Softmax and BitShift attention (lis.cu) -----------------------
+struct LisArgs {
+    const int8_t *logits;
+    int64_t n_rows;  // BH * L
+    int L;
+    int64_t ld_logit;
+    float s_logit;
+    const int8_t *bias;  // [heads][(2w-1)^2] or nullptr
+    int heads;
+    int window;
+    uint8_t *codes;  // packed nibbles or nullptr
+    int64_t ld_codes;
+    uint64_t *rowsum;  // or nullptr
+};
+cudaError_t launch_lis_softmax(const LisArgs &a, cudaStream_t st);
+
+struct AttnVArgs {
+    const uint8_t *codes;
+    int64_t ld_codes;
+    const int8_t *v;
+    int64_t ld_v;
+    int zp_v;
+    int64_t BH;
+    int L;
+    int d;
+    int32_t *acc;
+    int64_t ld_acc;
+    int32_t *range_flag;
+};
+cudaError_t launch_lis_attn_v(const AttnVArgs &a, cudaStream_t st);
+
+// fused softmax + attn.V; codes written only when a.codes != nullptr
+cudaError_t launch_lis_attention(const LisArgs &a, const AttnVArgs &b, cudaStream_t st);
+
+}  // namespace fqvit

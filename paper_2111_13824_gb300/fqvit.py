@@ -1,0 +1,211 @@
+"""Thin Python binding of libfqvit.so (include/fqvit.h).
+
+Argument marshalling only: every function passes torch tensors' device
+pointers and the current CUDA stream to the C ABI of the same name and
+raises ``FqvitError`` on a non-OK status.  There is no fallback: if the
+library is missing or was not built, loading fails loudly.
+"""
+from __future__ import annotations
+
+import ctypes
+from pathlib import Path
+
+import torch
+
+_LIB_PATH = Path(__file__).resolve().parent / "libfqvit.so"
+_lib = None
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_RANGE, ERR_CUDA = 0, 1, 2, 3, 4
+
+
+class FqvitError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"fqvit error {code}: {msg}")
+        self.code = code
+
+
+class RelposBias(ctypes.Structure):
+    _fields_ = [("table", ctypes.c_void_p), ("heads", ctypes.c_int32), ("window", ctypes.c_int32)]
+
+
+class BlockDesc(ctypes.Structure):
+    _fields_ = [
+        ("xq", ctypes.c_void_p), ("rows", ctypes.c_int64), ("C", ctypes.c_int32), ("zp_in", ctypes.c_int32),
+        ("alpha", ctypes.c_void_p), ("gamma", ctypes.c_void_p), ("beta", ctypes.c_void_p),
+        ("s_out", ctypes.c_float), ("zp_out", ctypes.c_int32), ("yq", ctypes.c_void_p),
+        ("logits", ctypes.c_void_p), ("ld_logit", ctypes.c_int64), ("s_logit", ctypes.c_float),
+        ("v", ctypes.c_void_p), ("zp_v", ctypes.c_int32), ("BH", ctypes.c_int64), ("L", ctypes.c_int32),
+        ("d", ctypes.c_int32), ("bias", ctypes.c_void_p), ("acc", ctypes.c_void_p),
+    ]
+
+
+EXPORTS = (
+    "fqvit_version", "fqvit_last_error", "fqvit_calibrate_workspace_size", "fqvit_calibrate_ptf",
+    "fqvit_ptf_quantize", "fqvit_ptf_layernorm", "fqvit_lis_softmax", "fqvit_lis_attn_v",
+    "fqvit_lis_attention", "fqvit_block_int",
+)
+
+
+def library_path() -> Path:
+    return _LIB_PATH
+
+
+def load(path: str | Path | None = None):
+    """Load libfqvit.so and declare its signatures (raises if it is missing)."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = Path(path) if path else _LIB_PATH
+    if not p.exists():
+        raise FileNotFoundError(f"{p} is missing: build it with paper_2111_13824_gb300.build.build()")
+    lib = ctypes.CDLL(str(p))
+    P, i64, i32, f32, sz = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_float, ctypes.c_size_t
+    sig = {
+        "fqvit_version": ([], ctypes.c_int),
+        "fqvit_last_error": ([], ctypes.c_char_p),
+        "fqvit_calibrate_workspace_size": ([i64, i32, i32], sz),
+        "fqvit_calibrate_ptf": ([P, i64, i32, i64, i32, i32, P, P, P, P, P, sz, P], ctypes.c_int),
+        "fqvit_ptf_quantize": ([P, i64, i32, i64, f32, i32, P, P, i64, P], ctypes.c_int),
+        "fqvit_ptf_layernorm": ([P, i64, i32, i64, i32, P, P, P, f32, i32, P, i64, P, P, P], ctypes.c_int),
+        "fqvit_lis_softmax": ([P, i64, i32, i64, f32, i32, P, P, i64, P, P], ctypes.c_int),
+        "fqvit_lis_attn_v": ([P, i64, P, i64, i32, i64, i32, i32, P, i64, P, P], ctypes.c_int),
+        "fqvit_lis_attention": ([P, i64, f32, i32, P, P, i64, i32, i64, i32, i32, P, i64, P, i64, P],
+                                ctypes.c_int),
+        "fqvit_block_int": ([P, P], ctypes.c_int),
+    }
+    for name, (args, res) in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = res
+    if path is None:
+        _lib = lib
+    return lib
+
+
+def _check(rc: int):
+    if rc != OK:
+        raise FqvitError(rc, load().fqvit_last_error().decode())
+
+
+def _p(t):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("expected a torch.Tensor")
+    if not t.is_cuda:
+        raise ValueError("libfqvit takes device tensors (got a CPU tensor)")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _ld(t: torch.Tensor) -> int:
+    return t.stride(0) if t.dim() >= 2 else t.shape[-1]
+
+
+def _bias(bias, heads, window):
+    if bias is None:
+        return None
+    b = RelposBias(ctypes.c_void_p(bias.data_ptr()), heads, window)
+    return b
+
+
+def version() -> int:
+    return int(load().fqvit_version())
+
+
+def calibrate_workspace_size(rows: int, C: int, K: int) -> int:
+    return int(load().fqvit_calibrate_workspace_size(rows, C, K))
+
+
+def calibrate_ptf(x: torch.Tensor, K: int = 3, bits: int = 8, sse: torch.Tensor | None = None,
+                  workspace: torch.Tensor | None = None, stream=None):
+    """Eqs. 8-10 on the device; returns device tensors (s[1] f32, zp[1] i32, alpha[C] u8)."""
+    rows, C = x.shape
+    dev = x.device
+    s = torch.empty(1, dtype=torch.float32, device=dev)
+    zp = torch.empty(1, dtype=torch.int32, device=dev)
+    alpha = torch.empty(C, dtype=torch.uint8, device=dev)
+    nbytes = calibrate_workspace_size(rows, C, K)
+    if workspace is None:
+        workspace = torch.empty(max(nbytes, 8) // 8 + 1, dtype=torch.float64, device=dev)
+    _check(load().fqvit_calibrate_ptf(_p(x), rows, C, _ld(x), bits, K, _p(s), _p(zp), _p(alpha), _p(sse),
+                                      _p(workspace), workspace.numel() * workspace.element_size(),
+                                      _stream(stream)))
+    return s, zp, alpha
+
+
+def ptf_quantize(x: torch.Tensor, s: float, zp: int, alpha: torch.Tensor, out: torch.Tensor | None = None,
+                 stream=None) -> torch.Tensor:
+    rows, C = x.shape
+    if out is None:
+        out = torch.empty(rows, C, dtype=torch.uint8, device=x.device)
+    _check(load().fqvit_ptf_quantize(_p(x), rows, C, _ld(x), float(s), int(zp), _p(alpha), _p(out), _ld(out),
+                                     _stream(stream)))
+    return out
+
+
+def ptf_layernorm(xq: torch.Tensor, zp_in: int, alpha, gamma, beta, s_out: float, zp_out: int,
+                  out: torch.Tensor | None = None, m1: torch.Tensor | None = None, m2: torch.Tensor | None = None,
+                  stream=None) -> torch.Tensor:
+    rows, C = xq.shape
+    if out is None:
+        out = torch.empty(rows, C, dtype=torch.uint8, device=xq.device)
+    _check(load().fqvit_ptf_layernorm(_p(xq), rows, C, _ld(xq), int(zp_in), _p(alpha), _p(gamma), _p(beta),
+                                      float(s_out), int(zp_out), _p(out), _ld(out), _p(m1), _p(m2),
+                                      _stream(stream)))
+    return out
+
+
+def lis_softmax(logits: torch.Tensor, L: int, s_logit: float, codes: torch.Tensor | None = None,
+                rowsum: torch.Tensor | None = None, bias: torch.Tensor | None = None, heads: int = 1,
+                window: int = 0, n_shift: int = 15, stream=None) -> torch.Tensor:
+    n_rows = logits.shape[0]
+    if codes is None:
+        codes = torch.empty(n_rows, (L + 1) // 2, dtype=torch.uint8, device=logits.device)
+    b = _bias(bias, heads, window)
+    _check(load().fqvit_lis_softmax(_p(logits), n_rows, L, _ld(logits), float(s_logit), n_shift,
+                                    ctypes.byref(b) if b is not None else None, _p(codes), _ld(codes),
+                                    _p(rowsum), _stream(stream)))
+    return codes
+
+
+def lis_attn_v(codes: torch.Tensor, v: torch.Tensor, zp_v: int = 0, acc: torch.Tensor | None = None,
+               range_flag: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    BH, L, d = v.shape
+    if acc is None:
+        acc = torch.empty(BH, L, d, dtype=torch.int32, device=v.device)
+    _check(load().fqvit_lis_attn_v(_p(codes), _ld(codes), _p(v), v.stride(1), int(zp_v), BH, L, d, _p(acc),
+                                   acc.stride(1), _p(range_flag), _stream(stream)))
+    return acc
+
+
+def lis_attention(logits: torch.Tensor, s_logit: float, v: torch.Tensor, zp_v: int = 0,
+                  acc: torch.Tensor | None = None, codes: torch.Tensor | None = None,
+                  bias: torch.Tensor | None = None, heads: int = 1, window: int = 0, n_shift: int = 15,
+                  stream=None) -> torch.Tensor:
+    BH, L, d = v.shape
+    if acc is None:
+        acc = torch.empty(BH, L, d, dtype=torch.int32, device=v.device)
+    b = _bias(bias, heads, window)
+    _check(load().fqvit_lis_attention(_p(logits), _ld(logits), float(s_logit), n_shift,
+                                      ctypes.byref(b) if b is not None else None, _p(v), v.stride(1), int(zp_v),
+                                      BH, L, d, _p(acc), acc.stride(1), _p(codes),
+                                      _ld(codes) if codes is not None else 0, _stream(stream)))
+    return acc
+
+
+def block_int(xq, zp_in, alpha, gamma, beta, s_out, zp_out, yq, logits, ld_logit, s_logit, v, zp_v, acc,
+              bias=None, heads=1, window=0, stream=None):
+    """One layer: LayerNorm then fused LIS attention (fqvit_block_int)."""
+    BH, L, d = v.shape
+    b = _bias(bias, heads, window)
+    desc = BlockDesc(xq.data_ptr(), xq.shape[0], xq.shape[1], int(zp_in), alpha.data_ptr(), gamma.data_ptr(),
+                     beta.data_ptr(), float(s_out), int(zp_out), yq.data_ptr(), logits.data_ptr(), int(ld_logit),
+                     float(s_logit), v.data_ptr(), int(zp_v), BH, L, d,
+                     ctypes.cast(ctypes.pointer(b), ctypes.c_void_p) if b is not None else None, acc.data_ptr())
+    _check(load().fqvit_block_int(ctypes.byref(desc), _stream(stream)))
+    return yq, acc

@@ -1,0 +1,78 @@
+"""The C-ABI library loads, exports every symbol include/fqvit.h declares, and
+rejects bad arguments on the host before launching anything (no GPU needed)."""
+import ctypes
+import re
+from pathlib import Path
+
+import pytest
+
+from paper_2111_13824_gb300 import build as fbuild
+from paper_2111_13824_gb300 import fqvit
+
+HEADER = Path(__file__).resolve().parents[1] / "include" / "fqvit.h"
+
+
+@pytest.fixture(scope="module")
+def lib():
+    fbuild.build()
+    return fqvit.load()
+
+
+def declared_functions():
+    text = HEADER.read_text()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(fqvit_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_path():
+    names = declared_functions()
+    for n in ("fqvit_calibrate_ptf", "fqvit_ptf_layernorm", "fqvit_lis_softmax", "fqvit_lis_attn_v",
+              "fqvit_block_int", "fqvit_lis_attention", "fqvit_ptf_quantize"):
+        assert n in names
+
+
+def test_exports_every_declared_symbol(lib):
+    raw = ctypes.CDLL(str(fqvit.library_path()))
+    for name in declared_functions():
+        assert hasattr(raw, name), name
+    assert set(fqvit.EXPORTS) == set(declared_functions())
+
+
+def test_version(lib):
+    assert lib.fqvit_version() >= 1
+
+
+def _err(lib):
+    return lib.fqvit_last_error().decode()
+
+
+def test_null_and_shape_checks(lib):
+    P = ctypes.c_void_p
+    fake = P(4096)  # never dereferenced: validation fails first
+    assert lib.fqvit_ptf_layernorm(None, 10, 64, 64, 0, fake, fake, fake, 0.1, 0, fake, 64, None, None, None) == 1
+    assert "NULL" in _err(lib)
+    assert lib.fqvit_ptf_layernorm(fake, 10, 64, 32, 0, fake, fake, fake, 0.1, 0, fake, 64, None, None, None) == 1
+    assert lib.fqvit_ptf_layernorm(fake, 10, 64, 64, 300, fake, fake, fake, 0.1, 0, fake, 64, None, None, None) == 1
+    assert lib.fqvit_ptf_layernorm(fake, 10, 64, 64, 0, fake, fake, fake, -1.0, 0, fake, 64, None, None, None) == 1
+    assert lib.fqvit_lis_softmax(fake, 10, 2000, 2048, 0.05, 15, None, fake, 1024, None, None) == 2
+    assert lib.fqvit_lis_softmax(fake, 10, 197, 197, 0.05, 15, None, fake, 100, None, None) == 1
+    assert "aligned" in _err(lib)
+    assert lib.fqvit_lis_softmax(fake, 10, 197, 208, 0.05, 14, None, fake, 100, None, None) == 2
+    assert lib.fqvit_lis_softmax(fake, 10, 197, 208, 0.001, 15, None, fake, 100, None, None) == 2
+    assert lib.fqvit_lis_softmax(fake, 10, 197, 208, 0.05, 15, None, fake, 50, None, None) == 1
+    assert lib.fqvit_lis_attn_v(fake, 25, fake, 48, 0, 2, 49, 48, fake, 48, None, None) == 2
+    assert lib.fqvit_lis_attn_v(fake, 25, fake, 64, 300, 2, 49, 64, fake, 64, None, None) == 2
+    assert lib.fqvit_calibrate_ptf(fake, 10, 64, 64, 4, 3, fake, fake, fake, None, fake, 1 << 20, None) == 2
+    assert lib.fqvit_calibrate_ptf(fake, 10, 64, 64, 8, 9, fake, fake, fake, None, fake, 1 << 20, None) == 2
+    assert lib.fqvit_calibrate_ptf(fake, 10, 64, 64, 8, 3, fake, fake, fake, None, fake, 16, None) == 1
+    assert "workspace" in _err(lib)
+    assert lib.fqvit_block_int(None, None) == 1
+
+
+def test_relpos_bias_checks(lib):
+    fake = ctypes.c_void_p(4096)
+    # only invalid descriptors here: a valid one would launch on the fake pointers
+    bad = fqvit.RelposBias(fake, 3, 6)
+    assert lib.fqvit_lis_softmax(fake, 3 * 49, 49, 64, 0.05, 15, ctypes.byref(bad), fake, 25, None, None) == 1
+    b2 = fqvit.RelposBias(fake, 4, 7)
+    assert lib.fqvit_lis_softmax(fake, 3 * 49, 49, 64, 0.05, 15, ctypes.byref(b2), fake, 25, None, None) == 1
