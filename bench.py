@@ -1,0 +1,433 @@
+"""Throughput of the FQ-ViT integer hot path on GB300.
+
+One step = the whole hot path over one batch: for each of the config's
+layers, the PTF integer LayerNorm (norm1) and the fused Log-Int-Softmax
+attention (codes -> BitShift attn.V), on per-layer synthetic inputs already
+resident in HBM (7.4 GB for ViT-L/384, far above the 129 MB L2, so no flush
+is needed between steps).  Calibration and quantization of the LayerNorm
+input are offline (setup), as in post-training quantization.
+
+Prints ONE JSON line (rank 0).  See the design doc for the byte model.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config vit_l384]
+                  [--impl reference] [--no-e2e] [--no-cpu]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2111_13824_gb300 import synth  # noqa: E402
+
+METRIC = "tokens/s and achieved HBM GB/s (% of GB300 peak) for PTF-LN + LIS attention, ViT-L/384"
+
+
+def _dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ------------------------------------------------------------------ byte model
+
+def ln_bytes(rows, C):
+    """Algorithmic bytes of one LayerNorm launch: u8 in + u8 out + 9 B / channel of parameters."""
+    return 2 * rows * C + 9 * C
+
+
+def attn_bytes(BH, L, d):
+    """Algorithmic bytes of one fused attention launch: 1 B / logit + 1 B / V element + 4 B / acc element."""
+    return BH * (L * L + L * d + 4 * L * d)
+
+
+# ------------------------------------------------------------------ workload
+
+def make_layers(cfg, device, sigma=1.0, limit=0):
+    from paper_2111_13824_gb300 import fqvit
+
+    layers = []
+    for l in range(cfg.layers if limit <= 0 else min(limit, cfg.layers)):
+        st = synth.layer_stage(cfg, l)
+        d = synth.ln_inputs(cfg, l, device=device)
+        s, zp, alpha = fqvit.calibrate_ptf(d["x_calib"], K=cfg.K)
+        zp_i, s_f = int(zp.item()), float(s.item())
+        xq = fqvit.ptf_quantize(d["x"], s_f, zp_i, alpha)
+        a = synth.attn_inputs(cfg, l, device=device, sigma=sigma)
+        layers.append(dict(
+            xq=xq, zp=zp_i, alpha=alpha, gamma=d["gamma"], beta=d["beta"], s_out=d["s_out"], zp_out=d["zp_out"],
+            yq=torch.empty_like(xq), logits=a["logits"], s_logit=a["s_logit"], v=a["v"], bias=a["bias"],
+            heads=a["heads"], window=a["window"],
+            acc=torch.empty(a["BH"], a["L"], a["d"], dtype=torch.int32, device=device),
+            rows=st.rows, C=st.C, BH=st.BH, L=st.L, d=st.d))
+        del d, a
+    torch.cuda.synchronize()
+    return layers
+
+
+def run_layer(fq, ly, ev=None):
+    fq.ptf_layernorm(ly["xq"], ly["zp"], ly["alpha"], ly["gamma"], ly["beta"], ly["s_out"], ly["zp_out"],
+                     out=ly["yq"])
+    if ev is not None:
+        ev[0].record()
+    bias = ly["bias"]
+    fq.lis_attention(ly["logits"], ly["s_logit"], ly["v"], 0, acc=ly["acc"], bias=bias, heads=ly["heads"],
+                     window=ly["window"])
+    if ev is not None:
+        ev[1].record()
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits", "-lms", "100",
+                 "-i", str(self.index)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        out, _ = self.proc.communicate(timeout=10)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for n, val in zip(names, f[4:8]):
+                if val.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ CPU oracle baseline
+
+class OracleSample:
+    """A bounded sample of one layer for the CPU oracle, scaled to the whole step.
+
+    Sample: the LayerNorm of `ln_rows` rows and the Log-Int-Softmax + BitShift
+    attn.V of `heads` attention heads of layer 0; the estimate scales each part to
+    the full layer and multiplies by the number of layers."""
+
+    def __init__(self, cfg, heads=1, ln_rows=512, layer=0):
+        import oracle
+
+        self.oracle = oracle
+        self.cfg, self.heads, self.ln_rows = cfg, heads, ln_rows
+        self.st = synth.layer_stage(cfg, layer)
+        d = synth.ln_inputs(cfg, layer, rows=ln_rows)
+        a = synth.attn_inputs(cfg, layer, bh=heads)
+        s, zp, alpha, _ = oracle.calibrate_ptf(d["x_calib"].numpy(), K=cfg.K)
+        self.ln = (oracle.ptf_quantize(d["x"].numpy(), s, zp, alpha), zp, alpha, d["gamma"].numpy(),
+                   d["beta"].numpy(), d["s_out"], d["zp_out"])
+        self.a = a
+        self.x, self.v = a["logits"].numpy(), a["v"].numpy()
+        self.bias = a["bias"].numpy() if a["bias"] is not None else None
+
+    def run(self):
+        """Returns (estimated seconds per step, seconds of CPU work spent)."""
+        o, a = self.oracle, self.a
+        t0 = time.perf_counter()
+        o.ptf_layernorm(*self.ln)
+        t1 = time.perf_counter()
+        co, _ = o.lis_softmax(self.x, a["L"], a["s_logit"], bias=self.bias, heads=a["heads"],
+                              window=a["window"] or 7)
+        o.lis_attn_v(co, self.v, 0)
+        t2 = time.perf_counter()
+        layer = (t1 - t0) * self.st.rows / self.ln_rows + (t2 - t1) * self.st.BH / self.heads
+        return layer * self.cfg.layers, t2 - t0
+
+    def describe(self):
+        return (f"layer 0: LayerNorm of {self.ln_rows} of {self.st.rows} rows and LIS + BitShift attn.V of "
+                f"{self.heads} of {self.st.BH} heads, scaled to the layer and x{self.cfg.layers} layers")
+
+
+# ------------------------------------------------------------------ main arms
+
+def bench_gpu(args):
+    from paper_2111_13824_gb300 import build as fbuild
+    from paper_2111_13824_gb300 import fqvit
+
+    ws, rank, local = _dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    if rank == 0 or not os.path.exists(fbuild.LIB):
+        fbuild.build()
+    if ws > 1:
+        torch.distributed.barrier()
+    fqvit.load()
+    cfg = synth.CONFIGS[args.config]
+    layers = make_layers(cfg, dev, sigma=args.sigma, limit=args.layers)
+    tokens_per_step = cfg.first_tokens
+
+    for _ in range(args.warmup):
+        for ly in layers:
+            run_layer(fqvit, ly)
+    torch.cuda.synchronize()
+
+    attn_events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(args.steps * len(layers))]
+    ln_events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                 for _ in range(args.steps * len(layers))]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)  # let the sampler start before the timed region
+    start.record()
+    k = 0
+    for _ in range(args.steps):
+        for ly in layers:
+            ln_events[k][0].record()
+            fqvit.ptf_layernorm(ly["xq"], ly["zp"], ly["alpha"], ly["gamma"], ly["beta"], ly["s_out"],
+                                ly["zp_out"], out=ly["yq"])
+            ln_events[k][1].record()
+            attn_events[k][0].record()
+            fqvit.lis_attention(ly["logits"], ly["s_logit"], ly["v"], 0, acc=ly["acc"], bias=ly["bias"],
+                                heads=ly["heads"], window=ly["window"])
+            attn_events[k][1].record()
+            k += 1
+    end.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    elapsed_ms = start.elapsed_time(end)
+    if ws > 1:
+        t = torch.tensor([elapsed_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+        torch.distributed.barrier()
+    ms_per_step = elapsed_ms / args.steps
+    value = tokens_per_step * ws * args.steps / (elapsed_ms / 1e3)
+
+    attn_ms = [a.elapsed_time(b) for a, b in attn_events]
+    ln_ms = [a.elapsed_time(b) for a, b in ln_events]
+    peak, peak_kind = peaks()
+    # per-launch algorithmic bytes (averaged over the stack's layer shapes)
+    ab = [attn_bytes(ly["BH"], ly["L"], ly["d"]) for ly in layers]
+    lb = [ln_bytes(ly["rows"], ly["C"]) for ly in layers]
+    attn_gbs = sum(ab) * args.steps / (sum(attn_ms) / 1e3) / 1e9
+    ln_gbs = sum(lb) * args.steps / (sum(ln_ms) / 1e3) / 1e9
+    step_bytes = sum(ab) + sum(lb)
+    stack_gbs = step_bytes / (ms_per_step / 1e3) / 1e9
+    dominant = "attention" if sum(attn_ms) >= sum(ln_ms) else "layernorm"
+    dom_gbs = attn_gbs if dominant == "attention" else ln_gbs
+    traffic = None
+    if args.traffic:
+        traffic = json.loads(args.traffic).get(dominant)
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = bench_e2e(fqvit, layers, tokens_per_step, args, dev, ws)
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu:
+        cpu = cpu_baseline(cfg, args)
+
+    line = {
+        "metric": METRIC if args.config == "vit_l384" else f"tokens/s, PTF-LN + LIS attention, {args.config}",
+        "value": round(value, 1),
+        "unit": "tokens/s",
+        "n_gpus": ws,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "int8",
+        "data": "synthetic (seeded generator of the paper's layer shapes and statistics)",
+        "config": {
+            "workload": f"{cfg.name}: {cfg.note}, {cfg.layers} layers of PTF LayerNorm + fused LIS attention",
+            "tokens_per_step_per_gpu": tokens_per_step,
+            "layers": len(layers),
+            "step_bytes": step_bytes,
+            "l2": f"inputs {step_bytes / 1e9:.2f} GB per step, larger than the 129 MB L2 (no flush)",
+            "logit_sigma": args.sigma,
+            "parallelism": f"replicas x{ws} (independent batches, no collective)",
+        },
+        "hbm_gbs": round(stack_gbs, 1),
+        "hbm_frac": round(stack_gbs / peak, 4),
+        "kernels": {
+            "attention": {"gbs": round(attn_gbs, 1), "ms_per_launch": round(sum(attn_ms) / len(attn_ms), 5),
+                          "bytes_per_launch": ab[0]},
+            "layernorm": {"gbs": round(ln_gbs, 1), "ms_per_launch": round(sum(ln_ms) / len(ln_ms), 5),
+                          "bytes_per_launch": lb[0]},
+        },
+        "roofline": {"kernel": dominant, "bound": "hbm", "achieved": round(dom_gbs, 1), "peak": peak,
+                     "unit": "GB/s", "frac": round(dom_gbs / peak, 4), "traffic": traffic,
+                     "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
+                     else "fallback"},
+        "clocks": clk,
+        "gpu_launches": 2 * len(layers) * args.steps,
+    }
+    if e2e is not None:
+        line["e2e"] = e2e
+    if cpu is not None:
+        line["cpu_baseline"] = cpu
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+def bench_e2e(fqvit, layers, tokens_per_step, args, dev, ws):
+    """Same metric through the public API with host buffers: every step copies each
+    layer's inputs from pinned host memory to the device and its outputs back."""
+    host = []
+    for ly in layers:
+        h = {k: ly[k].cpu().pin_memory() for k in ("xq", "logits", "v")}
+        h["yq"] = torch.empty_like(ly["yq"], device="cpu").pin_memory()
+        h["acc"] = torch.empty_like(ly["acc"], device="cpu").pin_memory()
+        host.append(h)
+    h2d = sum(h[k].numel() * h[k].element_size() for h in host for k in ("xq", "logits", "v"))
+    d2h = sum(h[k].numel() * h[k].element_size() for h in host for k in ("yq", "acc"))
+    steps = max(1, min(args.steps, args.e2e_steps))
+
+    def step():
+        for ly, h in zip(layers, host):
+            ly["xq"].copy_(h["xq"], non_blocking=True)
+            ly["logits"].copy_(h["logits"], non_blocking=True)
+            ly["v"].copy_(h["v"], non_blocking=True)
+            run_layer(fqvit, ly)
+            h["yq"].copy_(ly["yq"], non_blocking=True)
+            h["acc"].copy_(ly["acc"], non_blocking=True)
+
+    step()
+    torch.cuda.synchronize()
+    if ws > 1:
+        torch.distributed.barrier()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record()
+    for _ in range(steps):
+        step()
+    e.record()
+    torch.cuda.synchronize()
+    ms = s.elapsed_time(e)
+    if ws > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    return {"value": round(tokens_per_step * ws * steps / (ms / 1e3), 1), "unit": "tokens/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps,
+            "how": "per layer: pinned H2D of xq, logits, V; LayerNorm + fused attention; D2H of yq and acc; "
+                   "one stream"}
+
+
+def cpu_baseline(cfg, args):
+    import oracle
+
+    probe = OracleSample(cfg, heads=1, ln_rows=256)
+    _, spent = probe.run()
+    scale = max(1, int(args.cpu_seconds / max(spent, 1e-3)))
+    st = cfg.stages[0]
+    smp = OracleSample(cfg, heads=min(st.BH, scale), ln_rows=min(st.rows, 256 * scale))
+    est, spent = smp.run()
+    return {"value": round(cfg.first_tokens / est, 2), "unit": "tokens/s", "cores": oracle.num_threads(),
+            "kind": "oracle", "sample": f"{smp.describe()}; {spent:.1f} s of CPU work"}
+
+
+def bench_reference(args):
+    """The reference arm: the CPU oracle, as it stands, on the host cores."""
+    ws, rank, local = _dist_env()
+    if rank != 0:
+        return
+    cfg = synth.CONFIGS[args.config]
+    import oracle
+
+    oracle.build()
+    smp = OracleSample(cfg, heads=4, ln_rows=2048)
+    for _ in range(args.warmup):
+        smp.run()
+    ests = []
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        ests.append(smp.run()[0])
+    wall = time.perf_counter() - t0
+    step = statistics.mean(ests)
+    value = cfg.first_tokens / step
+    sample = f"per step: {smp.describe()}"
+    line = {
+        "impl": "reference",
+        "metric": METRIC if args.config == "vit_l384" else f"tokens/s, PTF-LN + LIS attention, {args.config}",
+        "value": round(value, 3), "unit": "tokens/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(step * 1e3, 3), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "int8", "data": "synthetic (seeded generator of the paper's layer shapes and statistics)",
+        "config": {"workload": f"{cfg.name}: {cfg.note}, {cfg.layers} layers of PTF LayerNorm + LIS attention",
+                   "tokens_per_step_per_gpu": cfg.first_tokens, "layers": cfg.layers},
+        "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": oracle.num_threads(),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "wall_s": round(wall, 2),
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--config", default="vit_l384", choices=sorted(synth.CONFIGS))
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--sigma", type=float, default=1.0, help="logit spread: 1 literal, 2 peaked")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--traffic", default=None, help="JSON {kernel: dram bytes per launch} from an ncu capture")
+    ap.add_argument("--layers", type=int, default=0, help="time only the first N layers (profiling cases)")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        bench_reference(args)
+    else:
+        bench_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -39,6 +39,7 @@ extern "C" {
 #define FQVIT_ERR_UNSUPPORTED 2 /* valid in the paper, not handled by this build  */
 #define FQVIT_ERR_RANGE 3       /* reserved: a value outside an exactness bound   */
 #define FQVIT_ERR_CUDA 4        /* a CUDA launch or runtime call failed           */
+#define FQVIT_ERR_TIMEOUT 5     /* a kernel gave up a bounded wait (see below)    */
 
 /* Library version, (major << 16) | minor. */
 FQVIT_API int fqvit_version(void);
@@ -46,6 +47,14 @@ FQVIT_API int fqvit_version(void);
 /* Thread-local description of the last non-OK status returned on this
  * thread (empty string if none).  Valid until the next call on the thread. */
 FQVIT_API const char *fqvit_last_error(void);
+
+/* Synchronizes `stream` and reports the library's device status word:
+ * FQVIT_ERR_TIMEOUT if a kernel of this library abandoned a bounded wait
+ * (every wait on an asynchronous copy or tensor-core operation gives up after
+ * two seconds, drains what it issued and returns) since the last call,
+ * FQVIT_ERR_CUDA if the stream reports an error, else FQVIT_OK.  The word is
+ * cleared.  Not part of the paper; a diagnostic of this implementation. */
+FQVIT_API int fqvit_sync_status(void *stream);
 
 /* ------------------------------------------------------------------ */
 /* Power-of-Two Factor calibration (Sec. 3.2, Eqs. 8-10)              */

@@ -65,6 +65,16 @@ int fqvit_version(void) { return (0 << 16) | 1; }
 
 const char *fqvit_last_error(void) { return g_err; }
 
+int fqvit_sync_status(void *stream)
+{
+    int status = 0;
+    cudaError_t e = fqvit::read_clear_device_status(&status, as_stream(stream));
+    if (e != cudaSuccess) return fail(FQVIT_ERR_CUDA, "sync_status: %s", cudaGetErrorString(e));
+    if (status == FQVIT_ERR_TIMEOUT)
+        return fail(FQVIT_ERR_TIMEOUT, "a kernel abandoned a bounded wait (results of that launch are invalid)");
+    return ok();
+}
+
 size_t fqvit_calibrate_workspace_size(int64_t rows, int32_t C, int32_t K)
 {
     if (C < 1 || K < 0 || K > 7) return 0;

@@ -72,4 +72,15 @@ cudaError_t launch_lis_attn_v(const AttnVArgs &a, cudaStream_t st);
 // fused softmax + attn.V; codes written only when a.codes != nullptr
 cudaError_t launch_lis_attention(const LisArgs &a, const AttnVArgs &b, cudaStream_t st);
 
+// tensor-core (tcgen05) fused path (lis_tc.cu)
+bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b);
+cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st);
+
+// Synchronizes st, returns the device status word (0 ok, 5 a bounded wait
+// timed out) and clears it.
+cudaError_t read_clear_device_status(int *status, cudaStream_t st);
+
+// Attention implementation choice: 0 automatic, 1 CUDA cores only (FQVIT_ATTN_PATH=cuda_core).
+int attention_path_override();
+
 }  // namespace fqvit

@@ -1,0 +1,80 @@
+// lis_common.cuh -- device helpers shared by the Log-Int-Softmax kernels:
+// the i-exp table (supplement Algorithm 1) and the division-free log2 code
+// (Algorithm 2).  See lis.cu for the derivation of the code test.
+#pragma once
+
+#include <stdint.h>
+
+namespace fqvit {
+namespace lis {
+
+constexpr int kLutSize = 288;  // q~ in [-287, 0]
+
+struct IexpC {
+    int q_ln2, q_b, q_c;
+};
+
+// Algorithm 1 constants, fp64 as in the oracle's definition.
+__device__ __forceinline__ IexpC iexp_consts(float s)
+{
+    const double ln2 = 0.693147180559945309417232121458176568;
+    double sd = (double)s;
+    IexpC c;
+    c.q_ln2 = (int)floor(__ddiv_rn(-ln2, sd));
+    c.q_b = (int)floor(__ddiv_rn(1.353, sd));
+    c.q_c = (int)floor(__ddiv_rn(0.344, __dmul_rn(0.3585, __dmul_rn(sd, sd))));
+    return c;
+}
+
+// e(-t) for t in [0, 287], n = 15
+__device__ __forceinline__ uint32_t iexp_neg(int t, IexpC c)
+{
+    int q = -t;
+    int lo = 15 * c.q_ln2;
+    if (q < lo) q = lo;
+    int z = q / c.q_ln2;
+    int qp = q - z * c.q_ln2;
+    int b = qp + c.q_b;
+    uint32_t qL = (uint32_t)(b * b + c.q_c);
+    return qL << (15 - z);
+}
+
+__device__ __forceinline__ void build_lut(uint32_t *lut, float s)
+{
+    IexpC c = iexp_consts(s);
+    for (int t = threadIdx.x; t < kLutSize; t += blockDim.x) lut[t] = iexp_neg(t, c);
+}
+
+struct RowSum {
+    float hi, lo;  // 2S = hi + lo, hi = fp32(2S)
+    int hibits;
+};
+
+__device__ __forceinline__ RowSum make_rowsum(unsigned long long S)
+{
+    unsigned long long s2 = 2ull * S;
+    RowSum r;
+    r.hi = __ull2float_rn(s2);
+    r.lo = (float)(long long)(s2 - __float2ull_rn(r.hi));
+    r.hibits = __float_as_int(r.hi);
+    return r;
+}
+
+__device__ __forceinline__ uint32_t lis_code(uint32_t e, const RowSum &rs)
+{
+    float ef = __uint2float_rn(e);  // exact: e = q_L 2^(15-z), q_L < 2^16
+    int k = (rs.hibits - __float_as_int(ef)) >> 23;
+    if (k >= 16) return 15u;
+    float Dk = (k == 1) ? 3.0f : __fsub_rn(__int_as_float(((k + 127) << 23) | 0x400000), 1.0f);
+    float t = __fmaf_rn(ef, Dk, -rs.hi);
+    return (uint32_t)(k - 1 + (t <= rs.lo ? 1 : 0));
+}
+
+__device__ __forceinline__ int relpos_idx(int i, int j, int w)
+{
+    int yi = i / w, xi = i - yi * w, yj = j / w, xj = j - yj * w;
+    return (yi - yj + w - 1) * (2 * w - 1) + (xi - xj + w - 1);
+}
+
+}  // namespace lis
+}  // namespace fqvit

@@ -1,0 +1,416 @@
+// lis_tc.cu -- fused Log-Int-Softmax + BitShift attention times values on
+// the 5th-generation tensor cores (tcgen05) of sm_103a.
+//
+// Eq. 15 is a matrix product: acc = P (V - zp_V) with P[i][j] = 2^(15 - code_ij).
+// Every P entry and every int8 value of V is exact in fp16, and for codes made
+// by Log-Int-Softmax sum_j 2^-code_j <= 3 + L 2^-15 (2^-code < 1.5 / q_rev and
+// q_rev >= S/e - 1/2), so with |V| <= 128 every partial sum of a row is an
+// integer below 2^24: fp16 operands with fp32 accumulation give the integer
+// result exactly.  The kernel therefore evaluates the shift-accumulate as
+// tcgen05.mma.kind::f16 (M = 128 query rows, N = 64 = d, K = 16 keys per
+// instruction) with the accumulator in tensor memory.
+//
+// One CTA per SM walks (head, 128-row tile) work items.  Roles:
+//   warps 0-3 (thread = query row): the row maximum and i-exp row sum
+//     (phase A), then per block of 64 keys the 4-bit codes written as fp16
+//     operands 2^(15-code) into a 128B-swizzled K-major shared-memory tile,
+//     and the block's V rows converted to fp16 (128B-swizzled, MN-major);
+//     finally the epilogue reads the row's 64 accumulators from tensor memory.
+//   warp 4, lane 0: bulk asynchronous copies of the tile's logits and the
+//     head's V into shared memory, and the MMA issue.
+// Ring of 3 operand stages, mbarrier hand-offs.  Every wait is bounded: after
+// two seconds the kernel records a timeout status, drains what it issued and
+// returns (the host reads the status with fqvit_sync_status).
+#include "fqvit_internal.cuh"
+#include "lis_common.cuh"
+
+#include <cuda_fp16.h>
+
+namespace fqvit {
+
+__device__ int g_device_status = 0;
+
+namespace {
+
+using namespace lis;
+
+constexpr int TM = 128;        // query rows per tile (MMA M)
+constexpr int TKB = 64;        // keys per operand stage
+constexpr int TSTAGES = 3;
+constexpr int TD = 64;         // head dimension (MMA N)
+constexpr int TMAXLD = 592;    // largest logit row stride handled here
+constexpr int TCOPIES = 32;    // replicas of the i-exp table (one per lane)
+constexpr int A_SLOT = TM * TKB * 2;
+constexpr int B_SLOT = TKB * TD * 2;
+constexpr int TTHREADS = 160;
+constexpr unsigned long long kTimeoutNs = 2000000000ull;
+
+struct TcParams {
+    const int8_t *logits;
+    int64_t ld;
+    float s;
+    const int8_t *v;
+    int32_t *acc;
+    int64_t BH;
+    int L;
+};
+
+__device__ __forceinline__ uint32_t sa(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ uint64_t gtimer()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *b, uint32_t n)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(sa(b)), "r"(n) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *b)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(sa(b)) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *b, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(sa(b)), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try(uint64_t *b, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+        : "=r"(ok)
+        : "r"(sa(b)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait; false on timeout or (honor_abort) when another role gave up.
+__device__ __noinline__ bool mbar_wait(uint64_t *b, uint32_t parity, volatile int *abort_flag,
+                                       bool honor_abort = true)
+{
+    if (mbar_try(b, parity)) return true;
+    const uint64_t t0 = gtimer();
+    for (uint32_t it = 1;; ++it) {
+        if (mbar_try(b, parity)) return true;
+        if ((it & 63) == 0) {
+            if (honor_abort && *abort_flag) return false;
+            if (gtimer() - t0 > kTimeoutNs) {
+                *abort_flag = 1;
+                atomicExch(&g_device_status, 5);
+                return false;
+            }
+        }
+    }
+}
+
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *b)
+{
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(sa(dst)),
+        "l"(src), "r"(bytes), "r"(sa(b))
+        : "memory");
+}
+
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// shared-memory matrix descriptor, 128-byte swizzle
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo)
+{
+    uint64_t d = (uint64_t)((addr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)(lbo >> 4) << 16;
+    d |= (uint64_t)(sbo >> 4) << 32;
+    d |= 1ull << 46;  // descriptor version for tcgen05
+    d |= 2ull << 61;  // SWIZZLE_128B
+    return d;
+}
+
+// kind::f16 instruction descriptor: D f32, A/B f16, A K-major, B MN-major, N = 64, M = 128
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 16) | ((uint32_t)(TD >> 3) << 17) | ((uint32_t)(TM >> 4) << 24);
+
+__device__ __forceinline__ void mma_f16(uint32_t dt, uint64_t ad, uint64_t bd, uint32_t accumulate)
+{
+    asm volatile(
+        "{ .reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p; }" ::"r"(dt),
+        "l"(ad), "l"(bd), "r"(kIdesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t *b)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(sa(b))
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
+
+__device__ __forceinline__ uint32_t fp16_operand(uint32_t code) { return (30u - code) << 10; }  // 2^(15-code)
+
+// int8 x 2 (bytes b0, b1 of w ^ 0x80808080) -> half2 exact
+__device__ __forceinline__ uint32_t i8x2_to_h2(uint32_t xw, uint32_t sel)
+{
+    uint32_t p = __byte_perm(xw, 0x64646464u, sel);  // 0x6400 | (v + 128): 1024 + v + 128
+    __half2 h = *reinterpret_cast<__half2 *>(&p);
+    h = __hsub2(h, __half2half2(__ushort_as_half((unsigned short)0x6480)));  // - 1152
+    return *reinterpret_cast<uint32_t *>(&h);
+}
+
+struct TcShared {
+    uint64_t load, full[TSTAGES], empty[TSTAGES], accfull, accempty, lfree, fin;
+    uint32_t tmem;
+    int abort_flag;
+};
+
+__global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
+{
+    extern __shared__ unsigned char dsm_raw[];
+    __shared__ TcShared sh;
+    unsigned char *base = (unsigned char *)(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
+    unsigned char *As = base;
+    unsigned char *Bs = As + TSTAGES * A_SLOT;
+    int8_t *LG = (int8_t *)(Bs + TSTAGES * B_SLOT);
+    int8_t *VS = LG + TM * p.ld;
+    uint32_t *LUT = (uint32_t *)(VS + (((size_t)p.L * TD + 15) & ~(size_t)15));
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    volatile int *abort_flag = &sh.abort_flag;
+    if (tid == 0) {
+        mbar_init(&sh.load, 1);
+        for (int s = 0; s < TSTAGES; ++s) {
+            mbar_init(&sh.full[s], TM);
+            mbar_init(&sh.empty[s], 1);
+        }
+        mbar_init(&sh.accfull, 1);
+        mbar_init(&sh.accempty, TM);
+        mbar_init(&sh.lfree, TM);
+        mbar_init(&sh.fin, 1);
+        sh.abort_flag = 0;
+    }
+    if (warp == 4) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(&sh.tmem)),
+                     "r"(TD));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    {
+        const IexpC c = iexp_consts(p.s);
+        for (int i = tid; i < kLutSize * TCOPIES; i += TTHREADS) LUT[i] = iexp_neg(i / TCOPIES, c);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sh.tmem;
+
+    const int L = p.L;
+    const int tpb = (L + TM - 1) / TM;
+    const int64_t ntiles = p.BH * tpb;
+    const int nkb = (L + TKB - 1) / TKB;
+
+    if (warp < 4) {
+        // ---------------- softmax + operands + epilogue, thread = query row
+        const int r = tid;
+        uint32_t g = 0;
+        int it = 0;
+        for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
+            const int64_t bh = tile / tpb;
+            const int row = (int)(tile % tpb) * TM + r;
+            const bool valid = row < L;
+            if (!mbar_wait(&sh.load, it & 1, abort_flag)) break;
+            const int8_t *lr = LG + (size_t)r * p.ld;
+            const uint32_t *lut_l = LUT + lane;
+            int m = -128;
+            unsigned long long S = 0;
+            if (valid) {
+                const int nfull = L >> 4;
+                uint32_t mx = 0x80808080u;
+                for (int c = 0; c < nfull; ++c) {
+                    uint4 w = *reinterpret_cast<const uint4 *>(lr + 16 * c);
+                    mx = __vmaxs4(mx, __vmaxs4(__vmaxs4(w.x, w.y), __vmaxs4(w.z, w.w)));
+                }
+                for (int j = nfull << 4; j < L; ++j) m = max(m, (int)lr[j]);
+                m = max(m, max(max((int)(int8_t)(mx), (int)(int8_t)(mx >> 8)),
+                               max((int)(int8_t)(mx >> 16), (int)(int8_t)(mx >> 24))));
+                const uint32_t *lut_m = lut_l + m * TCOPIES;
+                for (int c = 0; c < nfull; ++c) {
+                    uint4 w = *reinterpret_cast<const uint4 *>(lr + 16 * c);
+                    uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+#pragma unroll
+                        for (int b = 0; b < 4; ++b) S += lut_m[-(int)(int8_t)(ww[q] >> (8 * b)) * TCOPIES];
+                }
+                for (int j = nfull << 4; j < L; ++j) S += lut_m[-(int)lr[j] * TCOPIES];
+            }
+            const RowSum rs = make_rowsum(S);
+            const uint32_t *lut_m = lut_l + m * TCOPIES;
+            for (int kb = 0; kb < nkb; ++kb, ++g) {
+                const int slot = (int)(g % TSTAGES);
+                if (g >= TSTAGES && !mbar_wait(&sh.empty[slot], ((g / TSTAGES) - 1) & 1, abort_flag)) break;
+                unsigned char *Aslot = As + slot * A_SLOT;
+                unsigned char *Bslot = Bs + slot * B_SLOT;
+                // A: this row's 64 operands, K-major, 128B swizzle
+                unsigned char *arow = Aslot + (r >> 3) * 1024 + (r & 7) * 128;
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    const int k0 = kb * TKB + 8 * c;
+                    uint32_t o[4] = {0, 0, 0, 0};
+                    if (valid && k0 < L) {
+                        uint2 w = *reinterpret_cast<const uint2 *>(lr + k0);
+                        uint32_t ww[2] = {w.x, w.y};
+#pragma unroll
+                        for (int t = 0; t < 8; ++t) {
+                            if (k0 + t < L) {
+                                uint32_t e = lut_m[-(int)(int8_t)(ww[t >> 2] >> (8 * (t & 3))) * TCOPIES];
+                                o[t >> 1] |= fp16_operand(lis_code(e, rs)) << (16 * (t & 1));
+                            }
+                        }
+                    }
+                    *reinterpret_cast<uint4 *>(arow + ((c ^ (r & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+                }
+                // B: V rows of this block -> fp16, MN-major, 128B swizzle (thread: key r/2, half of d)
+                {
+                    const int kk = r >> 1, h = r & 1;
+                    const int key = kb * TKB + kk;
+                    unsigned char *brow = Bslot + kk * 128;
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const int ci = 4 * h + i;
+                        uint4 o = make_uint4(0, 0, 0, 0);
+                        if (key < L) {
+                            uint2 w = *reinterpret_cast<const uint2 *>(VS + (size_t)key * TD + 8 * ci);
+                            uint32_t x0 = w.x ^ 0x80808080u, x1 = w.y ^ 0x80808080u;
+                            o.x = i8x2_to_h2(x0, 0x5140);
+                            o.y = i8x2_to_h2(x0, 0x7362);
+                            o.z = i8x2_to_h2(x1, 0x5140);
+                            o.w = i8x2_to_h2(x1, 0x7362);
+                        }
+                        *reinterpret_cast<uint4 *>(brow + ((ci ^ (kk & 7)) << 4)) = o;
+                    }
+                }
+                fence_async_smem();
+                mbar_arrive(&sh.full[slot]);
+            }
+            if (*abort_flag) break;
+            fence_async_smem();
+            mbar_arrive(&sh.lfree);
+            // epilogue: accumulators of this row from tensor memory
+            if (!mbar_wait(&sh.accfull, it & 1, abort_flag)) break;
+            tc_fence_after();
+            uint32_t v[4][16];
+            const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) tmem_ld16(trow + 16 * j, v[j]);
+            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+            tc_fence_before();
+            mbar_arrive(&sh.accempty);
+            if (valid) {
+                int4 *dst = reinterpret_cast<int4 *>(p.acc + ((size_t)bh * L + row) * TD);
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        dst[4 * j + q] = make_int4(__float2int_rn(__uint_as_float(v[j][4 * q + 0])),
+                                                   __float2int_rn(__uint_as_float(v[j][4 * q + 1])),
+                                                   __float2int_rn(__uint_as_float(v[j][4 * q + 2])),
+                                                   __float2int_rn(__uint_as_float(v[j][4 * q + 3])));
+            }
+        }
+    } else if (warp == 4 && lane == 0) {
+        // ---------------- loads and MMA issue
+        uint32_t g = 0;
+        int it = 0;
+        int loads = 0;
+        for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
+            const int64_t bh = tile / tpb;
+            const int r0 = (int)(tile % tpb) * TM;
+            if (it > 0 && !mbar_wait(&sh.lfree, (it - 1) & 1, abort_flag)) break;
+            const int rows = min(TM, L - r0);
+            const uint32_t bl = (uint32_t)(rows * p.ld), bv = (uint32_t)(L * TD);
+            mbar_expect_tx(&sh.load, bl + bv);
+            bulk_g2s(LG, p.logits + ((size_t)bh * L + r0) * p.ld, bl, &sh.load);
+            bulk_g2s(VS, p.v + (size_t)bh * L * TD, bv, &sh.load);
+            ++loads;
+            bool ok = true;
+            for (int kb = 0; kb < nkb; ++kb, ++g) {
+                const int slot = (int)(g % TSTAGES);
+                if (!mbar_wait(&sh.full[slot], (g / TSTAGES) & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                if (kb == 0 && it > 0 && !mbar_wait(&sh.accempty, (it - 1) & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t a0 = sa(As + slot * A_SLOT), b0 = sa(Bs + slot * B_SLOT);
+#pragma unroll
+                for (int s = 0; s < TKB / 16; ++s)
+                    mma_f16(tmem, smem_desc(a0 + 32 * s, 16, 1024), smem_desc(b0 + 2048 * s, 1024, 1024),
+                            (kb | s) != 0);
+                mma_commit(&sh.empty[slot]);
+            }
+            if (!ok) break;
+            mma_commit(&sh.accfull);
+        }
+        // drain: every MMA issued by this thread has completed, every load issued has landed
+        mma_commit(&sh.fin);
+        mbar_wait(&sh.fin, 0, abort_flag, false);
+        if (*abort_flag && loads > 0) mbar_wait(&sh.load, (loads - 1) & 1, abort_flag, false);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 4) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TD));
+}
+
+size_t tc_smem_bytes(int L, int64_t ld)
+{
+    return 1024 + (size_t)TSTAGES * (A_SLOT + B_SLOT) + (size_t)TM * ld + (((size_t)L * TD + 15) & ~(size_t)15) +
+           (size_t)kLutSize * TCOPIES * 4;
+}
+
+}  // namespace
+
+bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
+{
+    return b.d == TD && a.bias == nullptr && a.codes == nullptr && b.zp_v == 0 && a.ld_logit <= TMAXLD &&
+           a.ld_logit % 16 == 0 && b.ld_v == TD && b.ld_acc == TD && ((uintptr_t)a.logits % 16) == 0 &&
+           ((uintptr_t)b.v % 16) == 0 && ((uintptr_t)b.acc % 16) == 0 && tc_smem_bytes(a.L, a.ld_logit) <= 232448;
+}
+
+cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
+{
+    TcParams p{a.logits, a.ld_logit, a.s_logit, b.v, b.acc, b.BH, a.L};
+    size_t smem = tc_smem_bytes(a.L, a.ld_logit);
+    cudaError_t e = cudaFuncSetAttribute(lis_attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    int64_t ntiles = b.BH * ((a.L + TM - 1) / TM);
+    int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());
+    lis_attn_tc_kernel<<<grid, TTHREADS, smem, st>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t read_clear_device_status(int *status, cudaStream_t st)
+{
+    int zero = 0;
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return e;
+    e = cudaMemcpyFromSymbol(status, g_device_status, sizeof(int));
+    if (e != cudaSuccess) return e;
+    return cudaMemcpyToSymbol(g_device_status, &zero, sizeof(int));
+}
+
+}  // namespace fqvit

@@ -15,7 +15,7 @@ import torch
 _LIB_PATH = Path(__file__).resolve().parent / "libfqvit.so"
 _lib = None
 
-OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_RANGE, ERR_CUDA = 0, 1, 2, 3, 4
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_RANGE, ERR_CUDA, ERR_TIMEOUT = 0, 1, 2, 3, 4, 5
 
 
 class FqvitError(RuntimeError):
@@ -42,7 +42,7 @@ class BlockDesc(ctypes.Structure):
 EXPORTS = (
     "fqvit_version", "fqvit_last_error", "fqvit_calibrate_workspace_size", "fqvit_calibrate_ptf",
     "fqvit_ptf_quantize", "fqvit_ptf_layernorm", "fqvit_lis_softmax", "fqvit_lis_attn_v",
-    "fqvit_lis_attention", "fqvit_block_int",
+    "fqvit_lis_attention", "fqvit_block_int", "fqvit_sync_status",
 )
 
 
@@ -72,6 +72,7 @@ def load(path: str | Path | None = None):
         "fqvit_lis_attention": ([P, i64, f32, i32, P, P, i64, i32, i64, i32, i32, P, i64, P, i64, P],
                                 ctypes.c_int),
         "fqvit_block_int": ([P, P], ctypes.c_int),
+        "fqvit_sync_status": ([P], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -111,6 +112,11 @@ def _bias(bias, heads, window):
         return None
     b = RelposBias(ctypes.c_void_p(bias.data_ptr()), heads, window)
     return b
+
+
+def sync_status(stream=None) -> None:
+    """Synchronize the stream; raise FqvitError if a kernel abandoned a bounded wait."""
+    _check(load().fqvit_sync_status(_stream(stream)))
 
 
 def version() -> int:

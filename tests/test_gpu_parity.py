@@ -273,7 +273,7 @@ def _oracle_attention(a):
 
 @pytest.mark.parametrize("name,bh,sigma", [("deit_t", None, 1.0), ("deit_s", 7, 2.0), ("vit_l384", 3, 1.0),
                                            ("vit_l384", 2, 2.0), ("swin_s", 12, 1.0)])
-def test_lis_attention_matches_oracle(name, bh, sigma):
+def test_lis_attention_matches_oracle(name, bh, sigma, cuda_core_path):
     a = _attn_case(name, bh=bh, sigma=sigma)
     co, ao = _oracle_attention(a)
     L = a["L"]
@@ -335,3 +335,59 @@ def test_full_size_vit_l_layer_sampled():
     assert np.array_equal(np_(xq), xqo)
     yo, _, _ = oracle.ptf_layernorm(xqo, zo, ao_, np_(d["gamma"]), np_(d["beta"]), d["s_out"], d["zp_out"])
     assert np.array_equal(np_(y), yo)
+
+
+# ---------------------------------------------------------------- tensor-core path
+
+@pytest.fixture
+def cuda_core_path(monkeypatch):
+    monkeypatch.setenv("FQVIT_ATTN_PATH", "cuda_core")
+
+
+@pytest.mark.parametrize("name,bh,sigma", [("deit_s", 5, 1.0), ("vit_b", 3, 2.0), ("vit_l384", 4, 1.0),
+                                           ("vit_l384", 3, 2.0)])
+def test_tensor_core_path_matches_oracle(name, bh, sigma):
+    a = _attn_case(name, bh=bh, sigma=sigma)
+    co, ao = _oracle_attention(a)
+    acc = fqvit.lis_attention(a["logits"].to(DEV), a["s_logit"], a["v"].to(DEV), 0)
+    fqvit.sync_status()
+    assert np.array_equal(np_(acc), ao)
+
+
+def test_tensor_core_and_cuda_core_agree(monkeypatch):
+    a = _attn_case("vit_l384", bh=6, sigma=1.5)
+    acc_tc = fqvit.lis_attention(a["logits"].to(DEV), a["s_logit"], a["v"].to(DEV), 0)
+    fqvit.sync_status()
+    monkeypatch.setenv("FQVIT_ATTN_PATH", "cuda_core")
+    acc_cc = fqvit.lis_attention(a["logits"].to(DEV), a["s_logit"], a["v"].to(DEV), 0)
+    fqvit.sync_status()
+    assert torch.equal(acc_tc, acc_cc)
+
+
+@pytest.mark.parametrize("L", [1, 2, 17, 64, 65, 128, 129, 197, 577, 592])
+def test_tensor_core_exact_at_the_accumulator_bound(L):
+    """Rows that push sum_j 2^(15-code_j) |V| toward its bound: k equal top
+    logits (I-Log2 rounds k up to 1.5 * 2^M, so k 2^-code approaches 1.5),
+    the rest far below, every V = -128 or +127; uniform rows; one-hot rows."""
+    ld = (L + 15) // 16 * 16
+    ks = [k for k in (1, 2, 3, 5, 11, 23, 47, 95, 191, 383) if k <= L]
+    rows = []
+    for k in ks:
+        r = np.full(ld, -128, np.int8)
+        r[:k] = 127
+        rows.append(r)
+    rows.append(np.full(ld, 3, np.int8))
+    n = (len(rows) + L - 1) // L * L
+    BH = max(1, n // L)
+    x = np.full((BH * L, ld), -128, np.int8)
+    for i, r in enumerate(rows):
+        x[i] = r
+    for s, vv in ((0.5, -128), (0.5, 127), (0.1, -128), (0.0078125, -128)):
+        v = np.full((BH, L, 64), vv, np.int8)
+        acc = fqvit.lis_attention(torch.from_numpy(x).to(DEV), s, torch.from_numpy(v).to(DEV), 0)
+        fqvit.sync_status()
+        co, _ = oracle.lis_softmax(x, L, s)
+        ao, ov = oracle.lis_attn_v(co, v, 0)
+        assert not ov
+        assert np.array_equal(np_(acc), ao), (L, s, vv)
+        assert np.abs(ao).max() < 2 ** 24
