@@ -42,7 +42,6 @@ constexpr int TMAXLD = 592;    // largest logit row stride handled here
 constexpr int TCOPIES = 32;    // replicas of the i-exp table (one per lane)
 constexpr int A_SLOT = TM * TKB * 2;
 constexpr int B_SLOT = TKB * TD * 2;
-constexpr int TTHREADS = 160;
 constexpr unsigned long long kTimeoutNs = 2000000000ull;
 
 struct TcParams {
@@ -175,7 +174,23 @@ struct TcShared {
     int abort_flag;
 };
 
-__global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
+constexpr int TPARTS = 4;                      // threads per query row
+constexpr int TSOFT = TM * TPARTS;             // softmax threads (16 warps)
+constexpr int TPRODUCER_WARP = TSOFT / 32;     // warp 16: loads + MMA issue
+
+// fp16 exponent field of the operand 2^(15-code) for an i-exp value e of a
+// row with 2S = hi + lo (G = bits of hi); see the file comment of lis.cu.
+__device__ __forceinline__ uint32_t operand_exp(uint32_t e, int G, float hi, float lo)
+{
+    const float ef = __uint2float_rn(e);
+    const int k = min((G - __float_as_int(ef)) >> 23, 16);
+    const float Dk = fmaxf(__fsub_rn(__int_as_float((k << 23) + 0x3FC00000), 1.0f), 3.0f);
+    const float t = __fmaf_rn(ef, Dk, -hi);
+    const int code = k - 1 + (t <= lo ? 1 : 0);
+    return (uint32_t)(30 - min(code, 15));
+}
+
+__global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
 {
     extern __shared__ unsigned char dsm_raw[];
     __shared__ TcShared sh;
@@ -191,23 +206,23 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     if (tid == 0) {
         mbar_init(&sh.load, 1);
         for (int s = 0; s < TSTAGES; ++s) {
-            mbar_init(&sh.full[s], TM);
+            mbar_init(&sh.full[s], TSOFT);
             mbar_init(&sh.empty[s], 1);
         }
         mbar_init(&sh.accfull, 1);
         mbar_init(&sh.accempty, TM);
-        mbar_init(&sh.lfree, TM);
+        mbar_init(&sh.lfree, TSOFT);
         mbar_init(&sh.fin, 1);
         sh.abort_flag = 0;
     }
-    if (warp == 4) {
+    if (warp == TPRODUCER_WARP) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(&sh.tmem)),
                      "r"(TD));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     {
         const IexpC c = iexp_consts(p.s);
-        for (int i = tid; i < kLutSize * TCOPIES; i += TTHREADS) LUT[i] = iexp_neg(i / TCOPIES, c);
+        for (int i = tid; i < kLutSize * TCOPIES; i += blockDim.x) LUT[i] = iexp_neg(i / TCOPIES, c);
     }
     tc_fence_before();
     __syncthreads();
@@ -219,9 +234,10 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     const int64_t ntiles = p.BH * tpb;
     const int nkb = (L + TKB - 1) / TKB;
 
-    if (warp < 4) {
-        // ---------------- softmax + operands + epilogue, thread = query row
-        const int r = tid;
+    if (tid < TSOFT) {
+        // ---------------- softmax: thread = (query row r, quarter q of every 64-key block)
+        const int r = tid >> 2, q = tid & 3;
+        const uint32_t *lut_l = LUT + lane;
         uint32_t g = 0;
         int it = 0;
         for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
@@ -229,76 +245,97 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
             const int row = (int)(tile % tpb) * TM + r;
             const bool valid = row < L;
             if (!mbar_wait(&sh.load, it & 1, abort_flag)) break;
-            const int8_t *lr = LG + (size_t)r * p.ld;
-            const uint32_t *lut_l = LUT + lane;
+            const int8_t *lr = LG + (size_t)r * p.ld + 16 * q;
+            // phase A: row maximum, then the i-exp row sum (4 threads per row)
             int m = -128;
-            unsigned long long S = 0;
             if (valid) {
-                const int nfull = L >> 4;
                 uint32_t mx = 0x80808080u;
-                for (int c = 0; c < nfull; ++c) {
-                    uint4 w = *reinterpret_cast<const uint4 *>(lr + 16 * c);
+                for (int kb = 0; kb < nkb; ++kb) {
+                    const int k0 = kb * TKB + 16 * q;
+                    if (k0 >= L) break;
+                    uint4 w = *reinterpret_cast<const uint4 *>(lr + kb * TKB);
+                    if (k0 + 16 > L) {  // keys at or past L do not count
+                        const int n = L - k0;
+                        uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                        for (int b = 0; b < 4; ++b) {
+                            const int keep = n - 4 * b;  // bytes of this word below L
+                            if (keep <= 0)
+                                ww[b] = 0x80808080u;
+                            else if (keep < 4)
+                                ww[b] = (ww[b] & (0xFFFFFFFFu >> (32 - 8 * keep))) |
+                                        (0x80808080u & ~(0xFFFFFFFFu >> (32 - 8 * keep)));
+                        }
+                        w = make_uint4(ww[0], ww[1], ww[2], ww[3]);
+                    }
                     mx = __vmaxs4(mx, __vmaxs4(__vmaxs4(w.x, w.y), __vmaxs4(w.z, w.w)));
                 }
-                for (int j = nfull << 4; j < L; ++j) m = max(m, (int)lr[j]);
-                m = max(m, max(max((int)(int8_t)(mx), (int)(int8_t)(mx >> 8)),
-                               max((int)(int8_t)(mx >> 16), (int)(int8_t)(mx >> 24))));
-                const uint32_t *lut_m = lut_l + m * TCOPIES;
-                for (int c = 0; c < nfull; ++c) {
-                    uint4 w = *reinterpret_cast<const uint4 *>(lr + 16 * c);
-                    uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-                    for (int q = 0; q < 4; ++q)
-#pragma unroll
-                        for (int b = 0; b < 4; ++b) S += lut_m[-(int)(int8_t)(ww[q] >> (8 * b)) * TCOPIES];
-                }
-                for (int j = nfull << 4; j < L; ++j) S += lut_m[-(int)lr[j] * TCOPIES];
+                m = max(max((int)(int8_t)(mx), (int)(int8_t)(mx >> 8)),
+                        max((int)(int8_t)(mx >> 16), (int)(int8_t)(mx >> 24)));
             }
-            const RowSum rs = make_rowsum(S);
+            m = max(m, __shfl_xor_sync(0xffffffffu, m, 1));
+            m = max(m, __shfl_xor_sync(0xffffffffu, m, 2));
             const uint32_t *lut_m = lut_l + m * TCOPIES;
+            unsigned long long S = 0;
+            if (valid) {
+                for (int kb = 0; kb < nkb; ++kb) {
+                    const int k0 = kb * TKB + 16 * q;
+                    if (k0 >= L) break;
+                    const uint4 w = *reinterpret_cast<const uint4 *>(lr + kb * TKB);
+                    const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+                    const int n = min(16, L - k0);
+                    if (n == 16) {
+#pragma unroll
+                        for (int b = 0; b < 8; ++b) {
+                            const uint32_t e0 = lut_m[-(int)(int8_t)(ww[b >> 1] >> (16 * (b & 1))) * TCOPIES];
+                            const uint32_t e1 = lut_m[-(int)(int8_t)(ww[b >> 1] >> (16 * (b & 1) + 8)) * TCOPIES];
+                            S += (unsigned long long)(e0 + e1);  // each e < 2^31
+                        }
+                    } else {
+                        for (int b = 0; b < n; ++b) S += lut_m[-(int)(int8_t)(ww[b >> 2] >> (8 * (b & 3))) * TCOPIES];
+                    }
+                }
+            }
+            S += __shfl_xor_sync(0xffffffffu, S, 1);
+            S += __shfl_xor_sync(0xffffffffu, S, 2);
+            const RowSum rs = make_rowsum(S);
+            // phase B: fp16 operands of this row's 16 keys of every block, V of the block
+            const int kk = tid >> 3, ci = tid & 7;  // V conversion: key kk of the block, 8 values ci
             for (int kb = 0; kb < nkb; ++kb, ++g) {
                 const int slot = (int)(g % TSTAGES);
                 if (g >= TSTAGES && !mbar_wait(&sh.empty[slot], ((g / TSTAGES) - 1) & 1, abort_flag)) break;
-                unsigned char *Aslot = As + slot * A_SLOT;
-                unsigned char *Bslot = Bs + slot * B_SLOT;
-                // A: this row's 64 operands, K-major, 128B swizzle
-                unsigned char *arow = Aslot + (r >> 3) * 1024 + (r & 7) * 128;
+                unsigned char *arow = As + slot * A_SLOT + (r >> 3) * 1024 + (r & 7) * 128;
+                const int k0 = kb * TKB + 16 * q;
+                uint32_t o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                if (valid && k0 < L) {
+                    const uint4 w = *reinterpret_cast<const uint4 *>(lr + kb * TKB);
+                    const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+                    const int n = min(16, L - k0);
 #pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    const int k0 = kb * TKB + 8 * c;
-                    uint32_t o[4] = {0, 0, 0, 0};
-                    if (valid && k0 < L) {
-                        uint2 w = *reinterpret_cast<const uint2 *>(lr + k0);
-                        uint32_t ww[2] = {w.x, w.y};
-#pragma unroll
-                        for (int t = 0; t < 8; ++t) {
-                            if (k0 + t < L) {
-                                uint32_t e = lut_m[-(int)(int8_t)(ww[t >> 2] >> (8 * (t & 3))) * TCOPIES];
-                                o[t >> 1] |= fp16_operand(lis_code(e, rs)) << (16 * (t & 1));
-                            }
-                        }
+                    for (int b = 0; b < 8; ++b) {
+                        const int j0 = 2 * b, j1 = 2 * b + 1;
+                        uint32_t x0 = 0, x1 = 0;
+                        if (j0 < n) x0 = operand_exp(lut_m[-(int)(int8_t)(ww[j0 >> 2] >> (8 * (j0 & 3))) * TCOPIES],
+                                                     rs.hibits, rs.hi, rs.lo);
+                        if (j1 < n) x1 = operand_exp(lut_m[-(int)(int8_t)(ww[j1 >> 2] >> (8 * (j1 & 3))) * TCOPIES],
+                                                     rs.hibits, rs.hi, rs.lo);
+                        o[b] = (__byte_perm(x0, x1, 0x5410) << 10);
                     }
-                    *reinterpret_cast<uint4 *>(arow + ((c ^ (r & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
                 }
-                // B: V rows of this block -> fp16, MN-major, 128B swizzle (thread: key r/2, half of d)
+                *reinterpret_cast<uint4 *>(arow + (((2 * q) ^ (r & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+                *reinterpret_cast<uint4 *>(arow + (((2 * q + 1) ^ (r & 7)) << 4)) = make_uint4(o[4], o[5], o[6], o[7]);
                 {
-                    const int kk = r >> 1, h = r & 1;
                     const int key = kb * TKB + kk;
-                    unsigned char *brow = Bslot + kk * 128;
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const int ci = 4 * h + i;
-                        uint4 o = make_uint4(0, 0, 0, 0);
-                        if (key < L) {
-                            uint2 w = *reinterpret_cast<const uint2 *>(VS + (size_t)key * TD + 8 * ci);
-                            uint32_t x0 = w.x ^ 0x80808080u, x1 = w.y ^ 0x80808080u;
-                            o.x = i8x2_to_h2(x0, 0x5140);
-                            o.y = i8x2_to_h2(x0, 0x7362);
-                            o.z = i8x2_to_h2(x1, 0x5140);
-                            o.w = i8x2_to_h2(x1, 0x7362);
-                        }
-                        *reinterpret_cast<uint4 *>(brow + ((ci ^ (kk & 7)) << 4)) = o;
+                    uint4 v4 = make_uint4(0, 0, 0, 0);
+                    if (key < L) {
+                        const uint2 w = *reinterpret_cast<const uint2 *>(VS + (size_t)key * TD + 8 * ci);
+                        const uint32_t x0 = w.x ^ 0x80808080u, x1 = w.y ^ 0x80808080u;
+                        v4.x = i8x2_to_h2(x0, 0x5140);
+                        v4.y = i8x2_to_h2(x0, 0x7362);
+                        v4.z = i8x2_to_h2(x1, 0x5140);
+                        v4.w = i8x2_to_h2(x1, 0x7362);
                     }
+                    *reinterpret_cast<uint4 *>(Bs + slot * B_SLOT + kk * 128 + ((ci ^ (kk & 7)) << 4)) = v4;
                 }
                 fence_async_smem();
                 mbar_arrive(&sh.full[slot]);
@@ -306,29 +343,32 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
             if (*abort_flag) break;
             fence_async_smem();
             mbar_arrive(&sh.lfree);
-            // epilogue: accumulators of this row from tensor memory
-            if (!mbar_wait(&sh.accfull, it & 1, abort_flag)) break;
-            tc_fence_after();
-            uint32_t v[4][16];
-            const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+            if (warp < 4) {
+                // epilogue: warp w reads tensor-memory lanes 32w..32w+31 = rows of the tile
+                if (!mbar_wait(&sh.accfull, it & 1, abort_flag)) break;
+                tc_fence_after();
+                uint32_t v[4][16];
+                const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
 #pragma unroll
-            for (int j = 0; j < 4; ++j) tmem_ld16(trow + 16 * j, v[j]);
-            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-            tc_fence_before();
-            mbar_arrive(&sh.accempty);
-            if (valid) {
-                int4 *dst = reinterpret_cast<int4 *>(p.acc + ((size_t)bh * L + row) * TD);
+                for (int j = 0; j < 4; ++j) tmem_ld16(trow + 16 * j, v[j]);
+                asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+                tc_fence_before();
+                mbar_arrive(&sh.accempty);
+                const int erow = (int)(tile % tpb) * TM + tid;
+                if (erow < L) {
+                    int4 *dst = reinterpret_cast<int4 *>(p.acc + ((size_t)bh * L + erow) * TD);
 #pragma unroll
-                for (int j = 0; j < 4; ++j)
+                    for (int j = 0; j < 4; ++j)
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        dst[4 * j + q] = make_int4(__float2int_rn(__uint_as_float(v[j][4 * q + 0])),
-                                                   __float2int_rn(__uint_as_float(v[j][4 * q + 1])),
-                                                   __float2int_rn(__uint_as_float(v[j][4 * q + 2])),
-                                                   __float2int_rn(__uint_as_float(v[j][4 * q + 3])));
+                        for (int c = 0; c < 4; ++c)
+                            dst[4 * j + c] = make_int4(__float2int_rn(__uint_as_float(v[j][4 * c + 0])),
+                                                       __float2int_rn(__uint_as_float(v[j][4 * c + 1])),
+                                                       __float2int_rn(__uint_as_float(v[j][4 * c + 2])),
+                                                       __float2int_rn(__uint_as_float(v[j][4 * c + 3])));
+                }
             }
         }
-    } else if (warp == 4 && lane == 0) {
+    } else if (warp == TPRODUCER_WARP && lane == 0) {
         // ---------------- loads and MMA issue
         uint32_t g = 0;
         int it = 0;
@@ -373,7 +413,8 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 4) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TD));
+    if (warp == TPRODUCER_WARP)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TD));
 }
 
 size_t tc_smem_bytes(int L, int64_t ld)
@@ -399,7 +440,7 @@ cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaSt
     if (e != cudaSuccess) return e;
     int64_t ntiles = b.BH * ((a.L + TM - 1) / TM);
     int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());
-    lis_attn_tc_kernel<<<grid, TTHREADS, smem, st>>>(p);
+    lis_attn_tc_kernel<<<grid, TSOFT + 32, smem, st>>>(p);
     return cudaGetLastError();
 }
 
