@@ -97,6 +97,7 @@ __device__ __noinline__ bool mbar_wait(uint64_t *b, uint32_t parity, volatile in
     const uint64_t t0 = gtimer();
     for (uint32_t it = 1;; ++it) {
         if (mbar_try(b, parity)) return true;
+        if (it > 4) __nanosleep(64);
         if ((it & 63) == 0) {
             if (honor_abort && *abort_flag) return false;
             if (gtimer() - t0 > kTimeoutNs) {
@@ -178,23 +179,32 @@ constexpr int TPARTS = 4;                      // threads per query row
 constexpr int TSOFT = TM * TPARTS;             // softmax threads (16 warps)
 constexpr int TPRODUCER_WARP = TSOFT / 32;     // warp 16: loads + MMA issue
 
-// fp16 exponent field of the operand 2^(15-code) for an i-exp value e of a
-// row with 2S = hi + lo (G = bits of hi); see the file comment of lis.cu.
+// fp16 exponent field (30 - code) of the operand 2^(15-code) for an i-exp
+// value e of a row with 2S = hi + lo (G = bits of hi); see the file comment
+// of lis.cu.  k = floor(log2(2S/e)) >= 1; codes above 15 clip to 15.
 __device__ __forceinline__ uint32_t operand_exp(uint32_t e, int G, float hi, float lo)
 {
     const float ef = __uint2float_rn(e);
-    const int k = min((G - __float_as_int(ef)) >> 23, 16);
+    const int k = (G - __float_as_int(ef)) >> 23;
     const float Dk = fmaxf(__fsub_rn(__int_as_float((k << 23) + 0x3FC00000), 1.0f), 3.0f);
     const float t = __fmaf_rn(ef, Dk, -hi);
-    const int code = k - 1 + (t <= lo ? 1 : 0);
-    return (uint32_t)(30 - min(code, 15));
+    uint32_t le;  // 0xFFFFFFFF when e D_k <= 2S
+    asm("set.le.u32.f32 %0, %1, %2;" : "=r"(le) : "f"(t), "f"(lo));
+    return (uint32_t)max(31 - k + (int)le, 15);
+}
+
+__device__ __forceinline__ uint32_t lds32(uint32_t a)
+{
+    uint32_t v;
+    asm("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
 }
 
 __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
 {
     extern __shared__ unsigned char dsm_raw[];
     __shared__ TcShared sh;
-    unsigned char *base = (unsigned char *)(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
+    unsigned char *base = dsm_raw + ((1024u - (sa(dsm_raw) & 1023u)) & 1023u);
     unsigned char *As = base;
     unsigned char *Bs = As + TSTAGES * A_SLOT;
     int8_t *LG = (int8_t *)(Bs + TSTAGES * B_SLOT);
@@ -237,7 +247,6 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
     if (tid < TSOFT) {
         // ---------------- softmax: thread = (query row r, quarter q of every 64-key block)
         const int r = tid >> 2, q = tid & 3;
-        const uint32_t *lut_l = LUT + lane;
         uint32_t g = 0;
         int it = 0;
         for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
@@ -275,7 +284,8 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
             }
             m = max(m, __shfl_xor_sync(0xffffffffu, m, 1));
             m = max(m, __shfl_xor_sync(0xffffffffu, m, 2));
-            const uint32_t *lut_m = lut_l + m * TCOPIES;
+            // i-exp table entry of logit q for this lane: lutq - 128 q  (entry m - q)
+            const uint32_t lutq = sa(LUT) + 4u * (uint32_t)lane + (uint32_t)(m * TCOPIES * 4);
             unsigned long long S = 0;
             if (valid) {
                 for (int kb = 0; kb < nkb; ++kb) {
@@ -283,16 +293,22 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
                     if (k0 >= L) break;
                     const uint4 w = *reinterpret_cast<const uint4 *>(lr + kb * TKB);
                     const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-                    const int n = min(16, L - k0);
-                    if (n == 16) {
+                    if (k0 + 16 <= L) {
+                        uint32_t part = 0;
 #pragma unroll
-                        for (int b = 0; b < 8; ++b) {
-                            const uint32_t e0 = lut_m[-(int)(int8_t)(ww[b >> 1] >> (16 * (b & 1))) * TCOPIES];
-                            const uint32_t e1 = lut_m[-(int)(int8_t)(ww[b >> 1] >> (16 * (b & 1) + 8)) * TCOPIES];
-                            S += (unsigned long long)(e0 + e1);  // each e < 2^31
+                        for (int j = 0; j < 16; ++j) {
+                            const uint32_t e = lds32(lutq - 128u * (uint32_t)(int)(int8_t)(ww[j >> 2] >> (8 * (j & 3))));
+                            if (j & 1) {
+                                S += (unsigned long long)(part + e);  // two values < 2^31 each
+                            } else {
+                                part = e;
+                            }
                         }
                     } else {
-                        for (int b = 0; b < n; ++b) S += lut_m[-(int)(int8_t)(ww[b >> 2] >> (8 * (b & 3))) * TCOPIES];
+                        const int n = L - k0;
+#pragma unroll
+                        for (int j = 0; j < 16; ++j)
+                            if (j < n) S += lds32(lutq - 128u * (uint32_t)(int)(int8_t)(ww[j >> 2] >> (8 * (j & 3))));
                     }
                 }
             }
@@ -310,17 +326,19 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
                 if (valid && k0 < L) {
                     const uint4 w = *reinterpret_cast<const uint4 *>(lr + kb * TKB);
                     const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-                    const int n = min(16, L - k0);
+                    uint32_t x[16];
 #pragma unroll
-                    for (int b = 0; b < 8; ++b) {
-                        const int j0 = 2 * b, j1 = 2 * b + 1;
-                        uint32_t x0 = 0, x1 = 0;
-                        if (j0 < n) x0 = operand_exp(lut_m[-(int)(int8_t)(ww[j0 >> 2] >> (8 * (j0 & 3))) * TCOPIES],
-                                                     rs.hibits, rs.hi, rs.lo);
-                        if (j1 < n) x1 = operand_exp(lut_m[-(int)(int8_t)(ww[j1 >> 2] >> (8 * (j1 & 3))) * TCOPIES],
-                                                     rs.hibits, rs.hi, rs.lo);
-                        o[b] = (__byte_perm(x0, x1, 0x5410) << 10);
+                    for (int j = 0; j < 16; ++j)
+                        x[j] = operand_exp(lds32(lutq - 128u * (uint32_t)(int)(int8_t)(ww[j >> 2] >> (8 * (j & 3)))),
+                                           rs.hibits, rs.hi, rs.lo);
+                    if (k0 + 16 > L) {  // keys at or past L get a zero operand
+                        const int n = L - k0;
+#pragma unroll
+                        for (int j = 0; j < 16; ++j)
+                            if (j >= n) x[j] = 0;
                     }
+#pragma unroll
+                    for (int b = 0; b < 8; ++b) o[b] = __byte_perm(x[2 * b], x[2 * b + 1], 0x5410) << 10;
                 }
                 *reinterpret_cast<uint4 *>(arow + (((2 * q) ^ (r & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
                 *reinterpret_cast<uint4 *>(arow + (((2 * q + 1) ^ (r & 7)) << 4)) = make_uint4(o[4], o[5], o[6], o[7]);
