@@ -89,24 +89,30 @@ __device__ __forceinline__ bool mbar_try(uint64_t *b, uint32_t parity)
     return ok != 0;
 }
 
-// Bounded wait; false on timeout or (honor_abort) when another role gave up.
+// Bounded wait with exponential back-off (sleeping warps leave the issue slots
+// to working ones); false on timeout or (honor_abort) when another role gave up.
 __device__ __noinline__ bool mbar_wait(uint64_t *b, uint32_t parity, volatile int *abort_flag,
                                        bool honor_abort = true)
 {
     if (mbar_try(b, parity)) return true;
     const uint64_t t0 = gtimer();
-    for (uint32_t it = 1;; ++it) {
+    uint32_t ns = 32;
+    for (;;) {
+        __nanosleep(ns);
         if (mbar_try(b, parity)) return true;
-        if (it > 4) __nanosleep(64);
-        if ((it & 63) == 0) {
-            if (honor_abort && *abort_flag) return false;
-            if (gtimer() - t0 > kTimeoutNs) {
-                *abort_flag = 1;
-                atomicExch(&g_device_status, 5);
-                return false;
-            }
+        if (ns < 1024) ns <<= 1;
+        if (honor_abort && *abort_flag) return false;
+        if (gtimer() - t0 > kTimeoutNs) {
+            *abort_flag = 1;
+            atomicExch(&g_device_status, 5);
+            return false;
         }
     }
+}
+
+__device__ __forceinline__ void prefetch_l2(const void *src, uint32_t bytes)
+{
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
 }
 
 __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *b)
@@ -170,7 +176,7 @@ __device__ __forceinline__ uint32_t i8x2_to_h2(uint32_t xw, uint32_t sel)
 }
 
 struct TcShared {
-    uint64_t load, full[TSTAGES], empty[TSTAGES], accfull, accempty, lfree, fin;
+    uint64_t lload, vload, full[TSTAGES], empty[TSTAGES], accfull, accempty, lfree, vfree, fin;
     uint32_t tmem;
     int abort_flag;
 };
@@ -178,6 +184,7 @@ struct TcShared {
 constexpr int TPARTS = 4;                      // threads per query row
 constexpr int TSOFT = TM * TPARTS;             // softmax threads (16 warps)
 constexpr int TPRODUCER_WARP = TSOFT / 32;     // warp 16: loads + MMA issue
+constexpr int TMAXKB = TMAXLD / TKB + 1;       // key blocks of the longest row
 
 // fp16 exponent field (30 - code) of the operand 2^(15-code) for an i-exp
 // value e of a row with 2S = hi + lo (G = bits of hi); see the file comment
@@ -200,6 +207,23 @@ __device__ __forceinline__ uint32_t lds32(uint32_t a)
     return v;
 }
 
+// byte j of w, sign-extended
+template <int J>
+__device__ __forceinline__ int sbyte(uint32_t w)
+{
+    uint32_t y;
+    asm("prmt.b32 %0, %1, 0, %2;" : "=r"(y) : "r"(w), "n"(J | ((J | 8) << 4) | ((J | 8) << 8) | ((J | 8) << 12)));
+    return (int)y;
+}
+
+// i-exp value of byte J of w: table entry m - q of this lane
+template <int J>
+__device__ __forceinline__ uint32_t iexp_at(uint32_t lutq, uint32_t w)
+{
+    return lds32(lutq - 128u * (uint32_t)sbyte<J>(w));
+}
+
+template <int NKB>
 __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
 {
     extern __shared__ unsigned char dsm_raw[];
@@ -208,13 +232,15 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
     unsigned char *As = base;
     unsigned char *Bs = As + TSTAGES * A_SLOT;
     int8_t *LG = (int8_t *)(Bs + TSTAGES * B_SLOT);
-    int8_t *VS = LG + TM * p.ld;
+    int8_t *VS = LG + (size_t)TM * p.ld;
     uint32_t *LUT = (uint32_t *)(VS + (((size_t)p.L * TD + 15) & ~(size_t)15));
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile int *abort_flag = &sh.abort_flag;
     if (tid == 0) {
-        mbar_init(&sh.load, 1);
+        mbar_init(&sh.lload, 1);
+        mbar_init(&sh.vload, 1);
+        mbar_init(&sh.vfree, TSOFT);
         for (int s = 0; s < TSTAGES; ++s) {
             mbar_init(&sh.full[s], TSOFT);
             mbar_init(&sh.empty[s], 1);
@@ -242,95 +268,103 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
     const int L = p.L;
     const int tpb = (L + TM - 1) / TM;
     const int64_t ntiles = p.BH * tpb;
-    const int nkb = (L + TKB - 1) / TKB;
 
     if (tid < TSOFT) {
-        // ---------------- softmax: thread = (query row r, quarter q of every 64-key block)
+        // ---------------- softmax: thread = (query row r, 16-key quarter q of every 64-key block)
         const int r = tid >> 2, q = tid & 3;
+        const int kk = tid >> 3, ci = tid & 7;  // V conversion: key kk of a block, values 8ci..8ci+7
+        const uint32_t lut_lane = sa(LUT) + 4u * (uint32_t)lane;
         uint32_t g = 0;
         int it = 0;
         for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
             const int64_t bh = tile / tpb;
             const int row = (int)(tile % tpb) * TM + r;
             const bool valid = row < L;
-            if (!mbar_wait(&sh.load, it & 1, abort_flag)) break;
+            if (!mbar_wait(&sh.lload, it & 1, abort_flag)) break;
+            // the row's keys 64 kb + 16 q .. +15 of every block, from the staged tile
             const int8_t *lr = LG + (size_t)r * p.ld + 16 * q;
-            // phase A: row maximum, then the i-exp row sum (4 threads per row)
-            int m = -128;
-            if (valid) {
-                uint32_t mx = 0x80808080u;
-                for (int kb = 0; kb < nkb; ++kb) {
-                    const int k0 = kb * TKB + 16 * q;
-                    if (k0 >= L) break;
-                    uint4 w = *reinterpret_cast<const uint4 *>(lr + kb * TKB);
-                    if (k0 + 16 > L) {  // keys at or past L do not count
-                        const int n = L - k0;
-                        uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+            uint4 w[NKB];
 #pragma unroll
-                        for (int b = 0; b < 4; ++b) {
-                            const int keep = n - 4 * b;  // bytes of this word below L
-                            if (keep <= 0)
-                                ww[b] = 0x80808080u;
-                            else if (keep < 4)
-                                ww[b] = (ww[b] & (0xFFFFFFFFu >> (32 - 8 * keep))) |
-                                        (0x80808080u & ~(0xFFFFFFFFu >> (32 - 8 * keep)));
-                        }
-                        w = make_uint4(ww[0], ww[1], ww[2], ww[3]);
+            for (int kb = 0; kb < NKB; ++kb) {
+                const int k0 = kb * TKB + 16 * q;
+                w[kb] = (valid && k0 < L) ? *reinterpret_cast<const uint4 *>(lr + kb * TKB)
+                                          : make_uint4(0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u);
+                if (k0 < L && k0 + 16 > L) {  // keys at or past L: -128 (no effect on the max)
+                    const int n = L - k0;
+                    uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
+#pragma unroll
+                    for (int b = 0; b < 4; ++b) {
+                        const int keep = n - 4 * b;
+                        if (keep <= 0)
+                            ww[b] = 0x80808080u;
+                        else if (keep < 4)
+                            ww[b] = (ww[b] & (0xFFFFFFFFu >> (32 - 8 * keep))) |
+                                    (0x80808080u & ~(0xFFFFFFFFu >> (32 - 8 * keep)));
                     }
-                    mx = __vmaxs4(mx, __vmaxs4(__vmaxs4(w.x, w.y), __vmaxs4(w.z, w.w)));
+                    w[kb] = make_uint4(ww[0], ww[1], ww[2], ww[3]);
                 }
-                m = max(max((int)(int8_t)(mx), (int)(int8_t)(mx >> 8)),
-                        max((int)(int8_t)(mx >> 16), (int)(int8_t)(mx >> 24)));
             }
+            fence_async_smem();
+            mbar_arrive(&sh.lfree);  // the staged logits are in registers now: the next tile may load
+            // phase A: row maximum and i-exp row sum
+            uint32_t mx = 0x80808080u;
+#pragma unroll
+            for (int kb = 0; kb < NKB; ++kb)
+                mx = __vmaxs4(mx, __vmaxs4(__vmaxs4(w[kb].x, w[kb].y), __vmaxs4(w[kb].z, w[kb].w)));
+            int m = max(max(sbyte<0>(mx), sbyte<1>(mx)), max(sbyte<2>(mx), sbyte<3>(mx)));
             m = max(m, __shfl_xor_sync(0xffffffffu, m, 1));
             m = max(m, __shfl_xor_sync(0xffffffffu, m, 2));
-            // i-exp table entry of logit q for this lane: lutq - 128 q  (entry m - q)
-            const uint32_t lutq = sa(LUT) + 4u * (uint32_t)lane + (uint32_t)(m * TCOPIES * 4);
+            const uint32_t lutq = lut_lane + (uint32_t)(m * TCOPIES * 4);
             unsigned long long S = 0;
             if (valid) {
-                for (int kb = 0; kb < nkb; ++kb) {
-                    const int k0 = kb * TKB + 16 * q;
-                    if (k0 >= L) break;
-                    const uint4 w = *reinterpret_cast<const uint4 *>(lr + kb * TKB);
-                    const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-                    if (k0 + 16 <= L) {
-                        uint32_t part = 0;
 #pragma unroll
-                        for (int j = 0; j < 16; ++j) {
-                            const uint32_t e = lds32(lutq - 128u * (uint32_t)(int)(int8_t)(ww[j >> 2] >> (8 * (j & 3))));
-                            if (j & 1) {
-                                S += (unsigned long long)(part + e);  // two values < 2^31 each
-                            } else {
-                                part = e;
-                            }
+                for (int kb = 0; kb < NKB; ++kb) {
+                    const int k0 = kb * TKB + 16 * q;
+                    const uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
+                    if (k0 + 16 <= L) {
+#pragma unroll
+                        for (int b = 0; b < 4; ++b) {
+                            const uint32_t e0 = iexp_at<0>(lutq, ww[b]), e1 = iexp_at<1>(lutq, ww[b]);
+                            const uint32_t e2 = iexp_at<2>(lutq, ww[b]), e3 = iexp_at<3>(lutq, ww[b]);
+                            S += (unsigned long long)(e0 + e1) + (unsigned long long)(e2 + e3);  // each e < 2^31
                         }
-                    } else {
+                    } else if (k0 < L) {
                         const int n = L - k0;
 #pragma unroll
-                        for (int j = 0; j < 16; ++j)
-                            if (j < n) S += lds32(lutq - 128u * (uint32_t)(int)(int8_t)(ww[j >> 2] >> (8 * (j & 3))));
+                        for (int b = 0; b < 4; ++b) {
+                            if (4 * b + 0 < n) S += iexp_at<0>(lutq, ww[b]);
+                            if (4 * b + 1 < n) S += iexp_at<1>(lutq, ww[b]);
+                            if (4 * b + 2 < n) S += iexp_at<2>(lutq, ww[b]);
+                            if (4 * b + 3 < n) S += iexp_at<3>(lutq, ww[b]);
+                        }
                     }
                 }
             }
             S += __shfl_xor_sync(0xffffffffu, S, 1);
             S += __shfl_xor_sync(0xffffffffu, S, 2);
             const RowSum rs = make_rowsum(S);
-            // phase B: fp16 operands of this row's 16 keys of every block, V of the block
-            const int kk = tid >> 3, ci = tid & 7;  // V conversion: key kk of the block, 8 values ci
-            for (int kb = 0; kb < nkb; ++kb, ++g) {
+            // phase B: the row's operands and the block's V, per 64-key block
+            if (!mbar_wait(&sh.vload, it & 1, abort_flag)) break;
+            bool stop = false;
+#pragma unroll
+            for (int kb = 0; kb < NKB; ++kb) {
                 const int slot = (int)(g % TSTAGES);
-                if (g >= TSTAGES && !mbar_wait(&sh.empty[slot], ((g / TSTAGES) - 1) & 1, abort_flag)) break;
-                unsigned char *arow = As + slot * A_SLOT + (r >> 3) * 1024 + (r & 7) * 128;
+                if (g >= TSTAGES && !mbar_wait(&sh.empty[slot], ((g / TSTAGES) - 1) & 1, abort_flag)) {
+                    stop = true;
+                    break;
+                }
                 const int k0 = kb * TKB + 16 * q;
                 uint32_t o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
                 if (valid && k0 < L) {
-                    const uint4 w = *reinterpret_cast<const uint4 *>(lr + kb * TKB);
-                    const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+                    const uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
                     uint32_t x[16];
 #pragma unroll
-                    for (int j = 0; j < 16; ++j)
-                        x[j] = operand_exp(lds32(lutq - 128u * (uint32_t)(int)(int8_t)(ww[j >> 2] >> (8 * (j & 3)))),
-                                           rs.hibits, rs.hi, rs.lo);
+                    for (int b = 0; b < 4; ++b) {
+                        x[4 * b + 0] = operand_exp(iexp_at<0>(lutq, ww[b]), rs.hibits, rs.hi, rs.lo);
+                        x[4 * b + 1] = operand_exp(iexp_at<1>(lutq, ww[b]), rs.hibits, rs.hi, rs.lo);
+                        x[4 * b + 2] = operand_exp(iexp_at<2>(lutq, ww[b]), rs.hibits, rs.hi, rs.lo);
+                        x[4 * b + 3] = operand_exp(iexp_at<3>(lutq, ww[b]), rs.hibits, rs.hi, rs.lo);
+                    }
                     if (k0 + 16 > L) {  // keys at or past L get a zero operand
                         const int n = L - k0;
 #pragma unroll
@@ -340,14 +374,15 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
 #pragma unroll
                     for (int b = 0; b < 8; ++b) o[b] = __byte_perm(x[2 * b], x[2 * b + 1], 0x5410) << 10;
                 }
+                unsigned char *arow = As + slot * A_SLOT + (r >> 3) * 1024 + (r & 7) * 128;
                 *reinterpret_cast<uint4 *>(arow + (((2 * q) ^ (r & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
                 *reinterpret_cast<uint4 *>(arow + (((2 * q + 1) ^ (r & 7)) << 4)) = make_uint4(o[4], o[5], o[6], o[7]);
                 {
                     const int key = kb * TKB + kk;
                     uint4 v4 = make_uint4(0, 0, 0, 0);
                     if (key < L) {
-                        const uint2 w = *reinterpret_cast<const uint2 *>(VS + (size_t)key * TD + 8 * ci);
-                        const uint32_t x0 = w.x ^ 0x80808080u, x1 = w.y ^ 0x80808080u;
+                        const uint2 vw = *reinterpret_cast<const uint2 *>(VS + (size_t)key * TD + 8 * ci);
+                        const uint32_t x0 = vw.x ^ 0x80808080u, x1 = vw.y ^ 0x80808080u;
                         v4.x = i8x2_to_h2(x0, 0x5140);
                         v4.y = i8x2_to_h2(x0, 0x7362);
                         v4.z = i8x2_to_h2(x1, 0x5140);
@@ -357,12 +392,14 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
                 }
                 fence_async_smem();
                 mbar_arrive(&sh.full[slot]);
+                ++g;
             }
-            if (*abort_flag) break;
+            if (stop || *abort_flag) break;
             fence_async_smem();
-            mbar_arrive(&sh.lfree);
+            mbar_arrive(&sh.vfree);  // the staged V of this tile is no longer read
             if (warp < 4) {
-                // epilogue: warp w reads tensor-memory lanes 32w..32w+31 = rows of the tile
+                // epilogue by warps 0-3 (tensor-memory lanes 32w..32w+31 = rows); the
+                // other warps go on to the next tile meanwhile
                 if (!mbar_wait(&sh.accfull, it & 1, abort_flag)) break;
                 tc_fence_after();
                 uint32_t v[4][16];
@@ -387,20 +424,32 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
             }
         }
     } else if (warp == TPRODUCER_WARP && lane == 0) {
-        // ---------------- loads and MMA issue
+        // ---------------- staged loads (logits as soon as the previous tile's are in registers,
+        // V once its previous copy is converted), L2 prefetch of the next tile, MMA issue
         uint32_t g = 0;
         int it = 0;
-        int loads = 0;
+        int lloads = 0, vloads = 0;
+        const int nkb = (L + TKB - 1) / TKB;
+        const uint32_t bv = (uint32_t)(L * TD);
         for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
             const int64_t bh = tile / tpb;
             const int r0 = (int)(tile % tpb) * TM;
             if (it > 0 && !mbar_wait(&sh.lfree, (it - 1) & 1, abort_flag)) break;
-            const int rows = min(TM, L - r0);
-            const uint32_t bl = (uint32_t)(rows * p.ld), bv = (uint32_t)(L * TD);
-            mbar_expect_tx(&sh.load, bl + bv);
-            bulk_g2s(LG, p.logits + ((size_t)bh * L + r0) * p.ld, bl, &sh.load);
-            bulk_g2s(VS, p.v + (size_t)bh * L * TD, bv, &sh.load);
-            ++loads;
+            const uint32_t bl = (uint32_t)(min(TM, L - r0) * p.ld);
+            mbar_expect_tx(&sh.lload, bl);
+            bulk_g2s(LG, p.logits + ((size_t)bh * L + r0) * p.ld, bl, &sh.lload);
+            ++lloads;
+            const int64_t nxt = tile + gridDim.x;
+            if (nxt < ntiles) {
+                const int64_t bhn = nxt / tpb;
+                const int r0n = (int)(nxt % tpb) * TM;
+                prefetch_l2(p.logits + ((size_t)bhn * L + r0n) * p.ld, (uint32_t)(min(TM, L - r0n) * p.ld));
+                if (bhn != bh) prefetch_l2(p.v + (size_t)bhn * L * TD, bv);
+            }
+            if (it > 0 && !mbar_wait(&sh.vfree, (it - 1) & 1, abort_flag)) break;
+            mbar_expect_tx(&sh.vload, bv);
+            bulk_g2s(VS, p.v + (size_t)bh * L * TD, bv, &sh.vload);
+            ++vloads;
             bool ok = true;
             for (int kb = 0; kb < nkb; ++kb, ++g) {
                 const int slot = (int)(g % TSTAGES);
@@ -426,7 +475,10 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
         // drain: every MMA issued by this thread has completed, every load issued has landed
         mma_commit(&sh.fin);
         mbar_wait(&sh.fin, 0, abort_flag, false);
-        if (*abort_flag && loads > 0) mbar_wait(&sh.load, (loads - 1) & 1, abort_flag, false);
+        if (*abort_flag) {
+            if (lloads > 0) mbar_wait(&sh.lload, (lloads - 1) & 1, abort_flag, false);
+            if (vloads > 0) mbar_wait(&sh.vload, (vloads - 1) & 1, abort_flag, false);
+        }
     }
     tc_fence_before();
     __syncthreads();
@@ -441,6 +493,16 @@ size_t tc_smem_bytes(int L, int64_t ld)
            (size_t)kLutSize * TCOPIES * 4;
 }
 
+template <int NKB>
+cudaError_t tc_launch(const TcParams &p, size_t smem, int grid, cudaStream_t st)
+{
+    cudaError_t e = cudaFuncSetAttribute(lis_attn_tc_kernel<NKB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    lis_attn_tc_kernel<NKB><<<grid, TSOFT + 32, smem, st>>>(p);
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
@@ -453,13 +515,21 @@ bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
 {
     TcParams p{a.logits, a.ld_logit, a.s_logit, b.v, b.acc, b.BH, a.L};
-    size_t smem = tc_smem_bytes(a.L, a.ld_logit);
-    cudaError_t e = cudaFuncSetAttribute(lis_attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    int64_t ntiles = b.BH * ((a.L + TM - 1) / TM);
-    int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());
-    lis_attn_tc_kernel<<<grid, TSOFT + 32, smem, st>>>(p);
-    return cudaGetLastError();
+    const size_t smem = tc_smem_bytes(a.L, a.ld_logit);
+    const int64_t ntiles = b.BH * ((a.L + TM - 1) / TM);
+    const int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());
+    switch ((a.L + TKB - 1) / TKB) {
+    case 1: return tc_launch<1>(p, smem, grid, st);
+    case 2: return tc_launch<2>(p, smem, grid, st);
+    case 3: return tc_launch<3>(p, smem, grid, st);
+    case 4: return tc_launch<4>(p, smem, grid, st);
+    case 5: return tc_launch<5>(p, smem, grid, st);
+    case 6: return tc_launch<6>(p, smem, grid, st);
+    case 7: return tc_launch<7>(p, smem, grid, st);
+    case 8: return tc_launch<8>(p, smem, grid, st);
+    case 9: return tc_launch<9>(p, smem, grid, st);
+    default: return tc_launch<10>(p, smem, grid, st);
+    }
 }
 
 cudaError_t read_clear_device_status(int *status, cudaStream_t st)
