@@ -83,6 +83,28 @@ FQVIT_API int fqvit_calibrate_ptf(const float *x, int64_t rows, int32_t C, int64
                         double *sse_opt, void *workspace, size_t ws_bytes, void *stream);
 
 /*
+ * Same calibration as fqvit_calibrate_ptf, for callers that cannot allocate
+ * device memory: code that must not allocate once it runs (real-time or
+ * certified inference with a fixed memory budget) and code whose device memory
+ * is owned by another allocator that gives out no extra buffer.  There is no
+ * counterpart in the paper; it is an interface of this library.
+ *   - No workspace argument: the kernels use a fixed 160 KiB array of device
+ *     memory that the library reserves on every GPU that loads it, for as long
+ *     as it stays loaded.  The call allocates nothing.
+ *   - Limit: C * (K + 1) <= 16384 (e.g. C = 4096 at K = 3); larger problems
+ *     return FQVIT_ERR_UNSUPPORTED -- use fqvit_calibrate_ptf with a workspace.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress); make that first call before any stream capture.
+ *   - All calls share the array, which keeps the last call's contents (no
+ *     call needs it zeroed).  Calls whose kernels overlap on the GPU race on
+ *     it: do not run two of them concurrently.
+ * Arguments, outputs and results are those of fqvit_calibrate_ptf.
+ */
+FQVIT_API int fqvit_calibrate_ptf_noalloc(const float *x, int64_t rows, int32_t C, int64_t ld_x,
+                                          int32_t bits, int32_t K, float *s, int32_t *zp,
+                                          uint8_t *alpha, double *sse_opt, void *stream);
+
+/*
  * PTF quantizer (Eq. 7): xq[r][c] = clip(rint(x[r][c] / (2^alpha_c s)) + zp, 0, 255),
  * fp32 quotient, ties to even.  x [rows, C] fp32, alpha [C] (device),
  * xq [rows, C] uint8 with stride ld_q.

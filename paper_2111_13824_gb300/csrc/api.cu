@@ -57,6 +57,12 @@ int sm_count()
     return cached[dev];
 }
 
+int record_error(int code, const char *msg)
+{
+    if (code == FQVIT_OK) return ok();
+    return fail(code, "%s", msg);
+}
+
 }  // namespace fqvit
 
 extern "C" {

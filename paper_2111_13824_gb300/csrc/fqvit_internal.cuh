@@ -10,6 +10,9 @@ namespace fqvit {
 // Number of SMs of the current device (cached per device).
 int sm_count();
 
+// Sets the thread's fqvit_last_error message (empty for FQVIT_OK); returns code.
+int record_error(int code, const char *msg);
+
 // ---- PTF calibration / quantizer (ptf.cu) ---------------------------------
 size_t calibrate_workspace_bytes(int64_t rows, int C, int K);
 cudaError_t launch_calibrate(const float *x, int64_t rows, int C, int64_t ld_x, int K, float *s,

@@ -42,7 +42,7 @@ class BlockDesc(ctypes.Structure):
 EXPORTS = (
     "fqvit_version", "fqvit_last_error", "fqvit_calibrate_workspace_size", "fqvit_calibrate_ptf",
     "fqvit_ptf_quantize", "fqvit_ptf_layernorm", "fqvit_lis_softmax", "fqvit_lis_attn_v",
-    "fqvit_lis_attention", "fqvit_block_int", "fqvit_sync_status",
+    "fqvit_lis_attention", "fqvit_block_int", "fqvit_sync_status", "fqvit_calibrate_ptf_noalloc",
 )
 
 
@@ -73,6 +73,7 @@ def load(path: str | Path | None = None):
                                 ctypes.c_int),
         "fqvit_block_int": ([P, P], ctypes.c_int),
         "fqvit_sync_status": ([P], ctypes.c_int),
+        "fqvit_calibrate_ptf_noalloc": ([P, i64, i32, i64, i32, i32, P, P, P, P, P], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -141,6 +142,19 @@ def calibrate_ptf(x: torch.Tensor, K: int = 3, bits: int = 8, sse: torch.Tensor 
     _check(load().fqvit_calibrate_ptf(_p(x), rows, C, _ld(x), bits, K, _p(s), _p(zp), _p(alpha), _p(sse),
                                       _p(workspace), workspace.numel() * workspace.element_size(),
                                       _stream(stream)))
+    return s, zp, alpha
+
+
+def calibrate_ptf_noalloc(x: torch.Tensor, K: int = 3, bits: int = 8, sse: torch.Tensor | None = None,
+                          stream=None):
+    """fqvit_calibrate_ptf_noalloc: calibration with the library's fixed scratch (no workspace)."""
+    rows, C = x.shape
+    dev = x.device
+    s = torch.empty(1, dtype=torch.float32, device=dev)
+    zp = torch.empty(1, dtype=torch.int32, device=dev)
+    alpha = torch.empty(C, dtype=torch.uint8, device=dev)
+    _check(load().fqvit_calibrate_ptf_noalloc(_p(x), rows, C, _ld(x), bits, K, _p(s), _p(zp), _p(alpha), _p(sse),
+                                              _stream(stream)))
     return s, zp, alpha
 
 
