@@ -183,7 +183,9 @@ struct TcShared {
 
 constexpr int TPARTS = 4;                      // threads per query row
 constexpr int TSOFT = TM * TPARTS;             // softmax threads (16 warps)
-constexpr int TPRODUCER_WARP = TSOFT / 32;     // warp 16: loads + MMA issue
+constexpr int TPRODUCER_WARP = TSOFT / 32;     // warp 16: MMA issue
+constexpr int TLOAD_WARP = TPRODUCER_WARP + 1; // warp 17: bulk copies of logits and V
+constexpr int TTHREADS = (TLOAD_WARP + 1) * 32;
 constexpr int TMAXKB = TMAXLD / TKB + 1;       // key blocks of the longest row
 
 // fp16 exponent field (30 - code) of the operand 2^(15-code) for an i-exp
@@ -224,7 +226,7 @@ __device__ __forceinline__ uint32_t iexp_at(uint32_t lutq, uint32_t w)
 }
 
 template <int NKB>
-__global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
+__global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
 {
     extern __shared__ unsigned char dsm_raw[];
     __shared__ TcShared sh;
@@ -423,13 +425,11 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
                 }
             }
         }
-    } else if (warp == TPRODUCER_WARP && lane == 0) {
-        // ---------------- staged loads (logits as soon as the previous tile's are in registers,
-        // V once its previous copy is converted), L2 prefetch of the next tile, MMA issue
-        uint32_t g = 0;
+    } else if (warp == TLOAD_WARP && lane == 0) {
+        // ---------------- bulk copies: a tile's logits as soon as the previous tile's are in
+        // registers, its V once the previous V is converted; L2 prefetch of the tile after
         int it = 0;
         int lloads = 0, vloads = 0;
-        const int nkb = (L + TKB - 1) / TKB;
         const uint32_t bv = (uint32_t)(L * TD);
         for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
             const int64_t bh = tile / tpb;
@@ -450,6 +450,16 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
             mbar_expect_tx(&sh.vload, bv);
             bulk_g2s(VS, p.v + (size_t)bh * L * TD, bv, &sh.vload);
             ++vloads;
+        }
+        // drain: every copy issued has landed before the block exits
+        if (lloads > 0) mbar_wait(&sh.lload, (lloads - 1) & 1, abort_flag, false);
+        if (vloads > 0) mbar_wait(&sh.vload, (vloads - 1) & 1, abort_flag, false);
+    } else if (warp == TPRODUCER_WARP && lane == 0) {
+        // ---------------- MMA issue
+        uint32_t g = 0;
+        int it = 0;
+        const int nkb = (L + TKB - 1) / TKB;
+        for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
             bool ok = true;
             for (int kb = 0; kb < nkb; ++kb, ++g) {
                 const int slot = (int)(g % TSTAGES);
@@ -472,13 +482,9 @@ __global__ void __launch_bounds__(TSOFT + 32, 1) lis_attn_tc_kernel(TcParams p)
             if (!ok) break;
             mma_commit(&sh.accfull);
         }
-        // drain: every MMA issued by this thread has completed, every load issued has landed
+        // drain: every MMA issued by this thread has completed
         mma_commit(&sh.fin);
         mbar_wait(&sh.fin, 0, abort_flag, false);
-        if (*abort_flag) {
-            if (lloads > 0) mbar_wait(&sh.lload, (lloads - 1) & 1, abort_flag, false);
-            if (vloads > 0) mbar_wait(&sh.vload, (vloads - 1) & 1, abort_flag, false);
-        }
     }
     tc_fence_before();
     __syncthreads();
@@ -499,7 +505,7 @@ cudaError_t tc_launch(const TcParams &p, size_t smem, int grid, cudaStream_t st)
     cudaError_t e = cudaFuncSetAttribute(lis_attn_tc_kernel<NKB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
-    lis_attn_tc_kernel<NKB><<<grid, TSOFT + 32, smem, st>>>(p);
+    lis_attn_tc_kernel<NKB><<<grid, TTHREADS, smem, st>>>(p);
     return cudaGetLastError();
 }
 
