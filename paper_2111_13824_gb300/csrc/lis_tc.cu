@@ -11,16 +11,24 @@
 // instruction) with the accumulator in tensor memory.
 //
 // One CTA per SM walks (head, 128-row tile) work items.  Roles:
-//   warps 0-3 (thread = query row): the row maximum and i-exp row sum
-//     (phase A), then per block of 64 keys the 4-bit codes written as fp16
-//     operands 2^(15-code) into a 128B-swizzled K-major shared-memory tile,
-//     and the block's V rows converted to fp16 (128B-swizzled, MN-major);
-//     finally the epilogue reads the row's 64 accumulators from tensor memory.
-//   warp 4, lane 0: bulk asynchronous copies of the tile's logits and the
-//     head's V into shared memory, and the MMA issue.
-// Ring of 3 operand stages, mbarrier hand-offs.  Every wait is bounded: after
-// two seconds the kernel records a timeout status, drains what it issued and
-// returns (the host reads the status with fqvit_sync_status).
+//   warps 0-15 (four threads per query row; warp w serves rows 32 (w % 4) ..
+//     and the keys 16 (w / 4) .. +15 of every block of 64 keys): the tile's
+//     logits go from shared memory into registers, the row maximum and the
+//     i-exp row sum are combined over the four threads of a row through
+//     shared memory, the row's 256 possible operands are tabulated, and every
+//     4-bit code is written, as the fp16 operand 2^(15-code) looked up in that
+//     table, straight into tensor memory (the A operand: row = lane, K-major
+//     pairs per column).  The same threads convert a head's V rows to fp16
+//     (128B-swizzled, MN-major shared-memory tile, the B operand) and, one
+//     tile later, read the accumulators back from tensor memory.
+//   warp 16, lane 0: issues the tile's MMAs (four per key block) once every
+//     operand is written, and commits them to an mbarrier.
+//   warp 17, lane 0: bulk asynchronous copy of the next tile's logits into
+//     shared memory as soon as the current tile is in registers, plus L2
+//     prefetches of what follows.
+// Every wait is bounded: after two seconds the kernel records a timeout
+// status, drains what it issued and returns (the host reads the status with
+// fqvit_sync_status).
 #include "fqvit_internal.cuh"
 #include "lis_common.cuh"
 
@@ -35,12 +43,10 @@ namespace {
 using namespace lis;
 
 constexpr int TM = 128;        // query rows per tile (MMA M)
-constexpr int TKB = 64;        // keys per operand stage
-constexpr int TSTAGES = 3;
+constexpr int TKB = 64;        // keys per key block
 constexpr int TD = 64;         // head dimension (MMA N)
 constexpr int TMAXLD = 592;    // largest logit row stride handled here
 constexpr int TCOPIES = 32;    // replicas of the i-exp table (one per lane)
-constexpr int A_SLOT = TM * TKB * 2;
 constexpr int B_SLOT = TKB * TD * 2;
 constexpr unsigned long long kTimeoutNs = 2000000000ull;
 
@@ -89,24 +95,34 @@ __device__ __forceinline__ bool mbar_try(uint64_t *b, uint32_t parity)
     return ok != 0;
 }
 
-// Bounded wait with exponential back-off (sleeping warps leave the issue slots
-// to working ones); false on timeout or (honor_abort) when another role gave up.
+// try_wait that may suspend the thread until the phase completes, for at most ns nanoseconds
+__device__ __forceinline__ bool mbar_try_for(uint64_t *b, uint32_t parity, uint32_t ns)
+{
+    uint32_t ok;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; selp.u32 %0, 1, 0, p; }"
+        : "=r"(ok)
+        : "r"(sa(b)), "r"(parity), "r"(ns)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait: the thread sleeps in the barrier (woken when the phase completes) in slices of
+// at most 50 us; false on timeout or (honor_abort) when another role gave up.
 __device__ __noinline__ bool mbar_wait(uint64_t *b, uint32_t parity, volatile int *abort_flag,
                                        bool honor_abort = true)
 {
     if (mbar_try(b, parity)) return true;
     const uint64_t t0 = gtimer();
-    uint32_t ns = 32;
     for (;;) {
-        __nanosleep(ns);
-        if (mbar_try(b, parity)) return true;
-        if (ns < 1024) ns <<= 1;
+        if (mbar_try_for(b, parity, 50000)) return true;
         if (honor_abort && *abort_flag) return false;
         if (gtimer() - t0 > kTimeoutNs) {
             *abort_flag = 1;
             atomicExch(&g_device_status, 5);
             return false;
         }
+        __nanosleep(64);
     }
 }
 
@@ -141,14 +157,6 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint3
 // kind::f16 instruction descriptor: D f32, A/B f16, A K-major, B MN-major, N = 64, M = 128
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 16) | ((uint32_t)(TD >> 3) << 17) | ((uint32_t)(TM >> 4) << 24);
 
-__device__ __forceinline__ void mma_f16(uint32_t dt, uint64_t ad, uint64_t bd, uint32_t accumulate)
-{
-    asm volatile(
-        "{ .reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p; }" ::"r"(dt),
-        "l"(ad), "l"(bd), "r"(kIdesc), "r"(accumulate)
-        : "memory");
-}
-
 __device__ __forceinline__ void mma_commit(uint64_t *b)
 {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(sa(b))
@@ -157,14 +165,13 @@ __device__ __forceinline__ void mma_commit(uint64_t *b)
 
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16])
 {
+    __syncwarp();
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
           "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
         : "r"(taddr));
 }
-
-__device__ __forceinline__ uint32_t fp16_operand(uint32_t code) { return (30u - code) << 10; }  // 2^(15-code)
 
 // int8 x 2 (bytes b0, b1 of w ^ 0x80808080) -> half2 exact
 __device__ __forceinline__ uint32_t i8x2_to_h2(uint32_t xw, uint32_t sel)
@@ -175,18 +182,27 @@ __device__ __forceinline__ uint32_t i8x2_to_h2(uint32_t xw, uint32_t sel)
     return *reinterpret_cast<uint32_t *>(&h);
 }
 
-struct TcShared {
-    uint64_t lload, vload, full[TSTAGES], empty[TSTAGES], accfull, accempty, lfree, vfree, fin;
-    uint32_t tmem;
-    int abort_flag;
-};
-
 constexpr int TPARTS = 4;                      // threads per query row
 constexpr int TSOFT = TM * TPARTS;             // softmax threads (16 warps)
 constexpr int TPRODUCER_WARP = TSOFT / 32;     // warp 16: MMA issue
-constexpr int TLOAD_WARP = TPRODUCER_WARP + 1; // warp 17: bulk copies of logits and V
+constexpr int TLOAD_WARP = TPRODUCER_WARP + 1; // warp 17: bulk copies of the logits
 constexpr int TTHREADS = (TLOAD_WARP + 1) * 32;
-constexpr int TMAXKB = TMAXLD / TKB + 1;       // key blocks of the longest row
+constexpr int TA_COL = TD;                     // D: columns 0..63; A of key block kb: 64 + 32 kb ..
+
+// tensor-memory columns for NKB key blocks (a power of two >= 32)
+__host__ __device__ constexpr int tmem_cols(int nkb)
+{
+    return TA_COL + 32 * nkb <= 128 ? 128 : TA_COL + 32 * nkb <= 256 ? 256 : 512;
+}
+
+struct TcShared {
+    uint64_t lload, lfree, afull, mmadone, fin;
+    IexpC c;
+    uint32_t tmem;
+    int abort_flag;
+    int rising;  // some i-exp value exceeds the one before it (floored constants)
+    int stop;    // set (never cleared) by a softmax thread whose wait gave up
+};
 
 // fp16 exponent field (30 - code) of the operand 2^(15-code) for an i-exp
 // value e of a row with 2S = hi + lo (G = bits of hi); see the file comment
@@ -202,11 +218,43 @@ __device__ __forceinline__ uint32_t operand_exp(uint32_t e, int G, float hi, flo
     return (uint32_t)max(31 - k + (int)le, 15);
 }
 
+// Named barrier 1 over the TSOFT softmax threads.  Every softmax thread reaches every one of
+// these barriers (the waits before them are bounded), so they end.  bar.sync is warp-aligned:
+// lanes of a row-dependent branch meet first.
+__device__ __forceinline__ void soft_bar()
+{
+    __syncwarp();
+    asm volatile("bar.sync 1, %0;" ::"n"(TSOFT) : "memory");
+}
+
+// mbar_wait with one verdict for the whole warp (the callers go on to
+// warp-collective tcgen05 instructions)
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t *b, uint32_t parity, volatile int *abort_flag)
+{
+    return __all_sync(0xFFFFFFFFu, mbar_wait(b, parity, abort_flag));
+}
+
 __device__ __forceinline__ uint32_t lds32(uint32_t a)
 {
     uint32_t v;
-    asm("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(a));
+    asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
     return v;
+}
+
+// byte permute with the sign-replicate selector bit honoured
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel)
+{
+    uint32_t y;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(y) : "r"(a), "r"(b), "r"(sel));
+    return y;
+}
+
+// lane-wise maximum of two pairs of signed 16-bit integers
+__device__ __forceinline__ uint32_t vmax16x2(uint32_t a, uint32_t b)
+{
+    uint32_t d;
+    asm("max.s16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
 }
 
 // byte j of w, sign-extended
@@ -218,49 +266,88 @@ __device__ __forceinline__ int sbyte(uint32_t w)
     return (int)y;
 }
 
-// i-exp value of byte J of w: table entry m - q of this lane
+// i-exp value of byte J of w: table entry m - q of this lane's replica
 template <int J>
 __device__ __forceinline__ uint32_t iexp_at(uint32_t lutq, uint32_t w)
 {
-    return lds32(lutq - 128u * (uint32_t)sbyte<J>(w));
+    return lds32(lutq - (uint32_t)(TCOPIES * 4) * (uint32_t)sbyte<J>(w));
 }
 
+// warp-collective (.sync.aligned): the whole warp, converged, writes its 32 lanes
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8])
+{
+    __syncwarp();
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(r[0]),
+                 "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+                 : "memory");
+}
+
+__device__ __forceinline__ void mma_f16_ta(uint32_t dt, uint32_t at, uint64_t bd, uint32_t accumulate)
+{
+    asm volatile(
+        "{ .reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p; }" ::"r"(dt),
+        "r"(at), "l"(bd), "r"(kIdesc), "r"(accumulate)
+        : "memory");
+}
+
+// Per tile (128 query rows of one head):
+//   copy warp:  logits tile -> shared memory (bulk copy), L2 prefetch of the next tile (and of
+//               the next head's V)
+//   softmax:    thread (row r, part q) takes keys 64 kb + 16 q .. +15 of every key block into
+//               registers; the row maximum and the i-exp row sum are combined over the four parts
+//               through shared memory.  The row's operands then go into a table indexed by the
+//               raw logit byte: word j of row r (OT[j][r], so that the 32 rows of a warp sit in
+//               32 different banks) holds, in byte b, 4 (30 - code) for the logit byte 4 j + b.
+//               Codes only depend on the row maximum, the row sum and the logit, so one table
+//               serves the whole row; it is filled by the four parts together, evaluating the
+//               code at the two ends of each word first: where the i-exp values never rise
+//               with the distance to the maximum, codes are monotone in the logit and equal
+//               ends fill the word (the floored constants of a few scales break this; those
+//               evaluate every byte).  Every logit then costs one table load; two loads
+//               and one byte permute give the fp16 pair 2^(15-code) that goes to tensor memory
+//               (A, K-major rows = lanes).  V of a head -> fp16 in shared memory (B, MN-major)
+//               whenever the head changes.
+//   MMA thread: after all operands of the tile are written, 4 MMAs per key block, one commit
+//   epilogue:   one tile later, all 16 warps read the accumulators (16 columns each)
+// Each CTA takes a contiguous range of tiles, so that consecutive tiles share a head.
 template <int NKB>
 __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
 {
     extern __shared__ unsigned char dsm_raw[];
     __shared__ TcShared sh;
     unsigned char *base = dsm_raw + ((1024u - (sa(dsm_raw) & 1023u)) & 1023u);
-    unsigned char *As = base;
-    unsigned char *Bs = As + TSTAGES * A_SLOT;
-    int8_t *LG = (int8_t *)(Bs + TSTAGES * B_SLOT);
-    int8_t *VS = LG + (size_t)TM * p.ld;
-    uint32_t *LUT = (uint32_t *)(VS + (((size_t)p.L * TD + 15) & ~(size_t)15));
+    unsigned char *Bs = base;                                   // NKB x 8 KB
+    uint32_t *OT = (uint32_t *)(Bs + NKB * B_SLOT);             // 64 x TM operand-table words
+    uint32_t *LUT = OT + 64 * TM;                               // 256 x TCOPIES
+    int *red_max = (int *)(LUT + 256 * TCOPIES);
+    unsigned long long *red_sum = (unsigned long long *)(red_max + TPARTS * TM);
+    int8_t *LG = (int8_t *)(red_sum + TPARTS * TM);             // TM x ld
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile int *abort_flag = &sh.abort_flag;
+    volatile int *stop_flag = &sh.stop;
     if (tid == 0) {
         mbar_init(&sh.lload, 1);
-        mbar_init(&sh.vload, 1);
-        mbar_init(&sh.vfree, TSOFT);
-        for (int s = 0; s < TSTAGES; ++s) {
-            mbar_init(&sh.full[s], TSOFT);
-            mbar_init(&sh.empty[s], 1);
-        }
-        mbar_init(&sh.accfull, 1);
-        mbar_init(&sh.accempty, TM);
         mbar_init(&sh.lfree, TSOFT);
+        mbar_init(&sh.afull, TSOFT);
+        mbar_init(&sh.mmadone, 1);
         mbar_init(&sh.fin, 1);
         sh.abort_flag = 0;
+        sh.rising = 0;
+        sh.stop = 0;
+        sh.c = iexp_consts(p.s);
     }
     if (warp == TPRODUCER_WARP) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(&sh.tmem)),
-                     "r"(TD));
+                     "r"(tmem_cols(NKB)));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
+    __syncthreads();
     {
-        const IexpC c = iexp_consts(p.s);
-        for (int i = tid; i < kLutSize * TCOPIES; i += blockDim.x) LUT[i] = iexp_neg(i / TCOPIES, c);
+        const IexpC c = sh.c;
+        for (int i = tid; i < 256 * TCOPIES; i += blockDim.x) LUT[i] = iexp_neg(i / TCOPIES, c);
+        for (int d = tid; d < 255; d += blockDim.x)
+            if (iexp_neg(d, c) < iexp_neg(d + 1, c)) sh.rising = 1;
     }
     tc_fence_before();
     __syncthreads();
@@ -270,20 +357,51 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     const int L = p.L;
     const int tpb = (L + TM - 1) / TM;
     const int64_t ntiles = p.BH * tpb;
+    const int64_t t_begin = (int64_t)blockIdx.x * ntiles / gridDim.x;
+    const int64_t t_end = (int64_t)(blockIdx.x + 1) * ntiles / gridDim.x;
+    // (head, first row) of tile t_begin; every role steps it by one tile per iteration
+    const int64_t bh_begin = t_begin / tpb;
+    const int r0_begin = (int)(t_begin - bh_begin * tpb) * TM;
 
     if (tid < TSOFT) {
-        // ---------------- softmax: thread = (query row r, 16-key quarter q of every 64-key block)
-        const int r = tid >> 2, q = tid & 3;
-        const int kk = tid >> 3, ci = tid & 7;  // V conversion: key kk of a block, values 8ci..8ci+7
+        const int r = tid & (TM - 1), q = tid >> 7;   // warp (q, r / 32): lanes = rows = TMEM lanes
+        const int kk = tid >> 3, ci = tid & 7;        // V conversion: key kk of a block, values 8 ci .. +7
         const uint32_t lut_lane = sa(LUT) + 4u * (uint32_t)lane;
-        uint32_t g = 0;
+        const uint32_t ot_base = sa(OT);
+        const uint32_t r4 = 4u * (uint32_t)r;
+        const uint32_t tlane = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+        const bool small_e = LUT[0] < (1u << 28);    // e(0) is the largest i-exp value
+        const bool monotone = !sh.rising;            // codes never fall as d grows
         int it = 0;
-        for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
-            const int64_t bh = tile / tpb;
-            const int row = (int)(tile % tpb) * TM + r;
+        bool epi_bad = false;
+        int64_t prev_bh = -1, conv_bh = -1;
+        int prev_r0 = 0;
+        // accumulators of the previous tile: warp w reads rows 32 (w % 4) .., columns 16 (w / 4) ..
+        auto epilogue = [&](int tit, int64_t ebh, int er0) -> bool {
+            if (!mbar_wait_warp(&sh.mmadone, tit & 1, abort_flag)) return false;
+            tc_fence_after();
+            uint32_t v[16];
+            tmem_ld16(tlane + 16 * (warp >> 2), v);
+            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+            const int erow = er0 + (warp & 3) * 32 + lane;
+            if (erow < L) {
+                int4 *dst = reinterpret_cast<int4 *>(p.acc + ((size_t)ebh * L + erow) * TD + 16 * (warp >> 2));
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                    dst[c] = make_int4(__float2int_rn(__uint_as_float(v[4 * c + 0])),
+                                       __float2int_rn(__uint_as_float(v[4 * c + 1])),
+                                       __float2int_rn(__uint_as_float(v[4 * c + 2])),
+                                       __float2int_rn(__uint_as_float(v[4 * c + 3])));
+            }
+            return true;
+        };
+        bool failed = false;
+        int64_t bh = bh_begin;
+        int r0 = r0_begin;
+        for (int64_t tile = t_begin; tile < t_end; ++tile, ++it, r0 = r0 + TM < L ? r0 + TM : (++bh, 0)) {
+            const int row = r0 + r;
             const bool valid = row < L;
-            if (!mbar_wait(&sh.lload, it & 1, abort_flag)) break;
-            // the row's keys 64 kb + 16 q .. +15 of every block, from the staged tile
+            bool bad = !mbar_wait_warp(&sh.lload, it & 1, abort_flag);
             const int8_t *lr = LG + (size_t)r * p.ld + 16 * q;
             uint4 w[NKB];
 #pragma unroll
@@ -306,16 +424,26 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                     w[kb] = make_uint4(ww[0], ww[1], ww[2], ww[3]);
                 }
             }
-            fence_async_smem();
-            mbar_arrive(&sh.lfree);  // the staged logits are in registers now: the next tile may load
-            // phase A: row maximum and i-exp row sum
-            uint32_t mx = 0x80808080u;
+            if (!bad) {
+                fence_async_smem();
+                mbar_arrive(&sh.lfree);  // the staged logits are in registers: the next tile may load
+            }
+            // ---- row maximum over the four parts
+            // signed 16-bit lanes: the high byte of the larger lane is the larger byte, so lanes of w
+            // carry bytes 1 and 3 and lanes of w << 8 bytes 0 and 2
+            uint32_t mo = 0x80008000u, me = 0x80008000u;
 #pragma unroll
-            for (int kb = 0; kb < NKB; ++kb)
-                mx = __vmaxs4(mx, __vmaxs4(__vmaxs4(w[kb].x, w[kb].y), __vmaxs4(w[kb].z, w[kb].w)));
-            int m = max(max(sbyte<0>(mx), sbyte<1>(mx)), max(sbyte<2>(mx), sbyte<3>(mx)));
-            m = max(m, __shfl_xor_sync(0xffffffffu, m, 1));
-            m = max(m, __shfl_xor_sync(0xffffffffu, m, 2));
+            for (int kb = 0; kb < NKB; ++kb) {
+                mo = vmax16x2(vmax16x2(mo, w[kb].x), vmax16x2(w[kb].y, vmax16x2(w[kb].z, w[kb].w)));
+                me = vmax16x2(vmax16x2(me, w[kb].x << 8), vmax16x2(w[kb].y << 8, vmax16x2(w[kb].z << 8, w[kb].w << 8)));
+            }
+            int m = max(max(sbyte<1>(mo), sbyte<3>(mo)), max(sbyte<1>(me), sbyte<3>(me)));
+            red_max[q * TM + r] = m;
+            if (bad || epi_bad) *stop_flag = 1;
+            soft_bar();
+            if (*stop_flag) { failed = true; break; }  // every softmax thread leaves here together
+            m = max(max(red_max[r], red_max[TM + r]), max(red_max[2 * TM + r], red_max[3 * TM + r]));
+            // ---- i-exp row sum over the four parts
             const uint32_t lutq = lut_lane + (uint32_t)(m * TCOPIES * 4);
             unsigned long long S = 0;
             if (valid) {
@@ -324,11 +452,21 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                     const int k0 = kb * TKB + 16 * q;
                     const uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
                     if (k0 + 16 <= L) {
+                        if (small_e) {  // 16 values below 2^28: a 32-bit partial sum is exact
+                            uint32_t a = 0;
 #pragma unroll
-                        for (int b = 0; b < 4; ++b) {
-                            const uint32_t e0 = iexp_at<0>(lutq, ww[b]), e1 = iexp_at<1>(lutq, ww[b]);
-                            const uint32_t e2 = iexp_at<2>(lutq, ww[b]), e3 = iexp_at<3>(lutq, ww[b]);
-                            S += (unsigned long long)(e0 + e1) + (unsigned long long)(e2 + e3);  // each e < 2^31
+                            for (int b = 0; b < 4; ++b) {
+                                a += iexp_at<0>(lutq, ww[b]) + iexp_at<1>(lutq, ww[b]);
+                                a += iexp_at<2>(lutq, ww[b]) + iexp_at<3>(lutq, ww[b]);
+                            }
+                            S += a;
+                        } else {
+#pragma unroll
+                            for (int b = 0; b < 4; ++b) {
+                                const uint32_t e0 = iexp_at<0>(lutq, ww[b]), e1 = iexp_at<1>(lutq, ww[b]);
+                                const uint32_t e2 = iexp_at<2>(lutq, ww[b]), e3 = iexp_at<3>(lutq, ww[b]);
+                                S += (unsigned long long)(e0 + e1) + (unsigned long long)(e2 + e3);  // e < 2^31
+                            }
                         }
                     } else if (k0 < L) {
                         const int n = L - k0;
@@ -342,147 +480,133 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                     }
                 }
             }
-            S += __shfl_xor_sync(0xffffffffu, S, 1);
-            S += __shfl_xor_sync(0xffffffffu, S, 2);
-            const RowSum rs = make_rowsum(S);
-            // phase B: the row's operands and the block's V, per 64-key block
-            if (!mbar_wait(&sh.vload, it & 1, abort_flag)) break;
-            bool stop = false;
-#pragma unroll
-            for (int kb = 0; kb < NKB; ++kb) {
-                const int slot = (int)(g % TSTAGES);
-                if (g >= TSTAGES && !mbar_wait(&sh.empty[slot], ((g / TSTAGES) - 1) & 1, abort_flag)) {
-                    stop = true;
-                    break;
-                }
-                const int k0 = kb * TKB + 16 * q;
-                uint32_t o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                if (valid && k0 < L) {
-                    const uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
-                    uint32_t x[16];
-#pragma unroll
-                    for (int b = 0; b < 4; ++b) {
-                        x[4 * b + 0] = operand_exp(iexp_at<0>(lutq, ww[b]), rs.hibits, rs.hi, rs.lo);
-                        x[4 * b + 1] = operand_exp(iexp_at<1>(lutq, ww[b]), rs.hibits, rs.hi, rs.lo);
-                        x[4 * b + 2] = operand_exp(iexp_at<2>(lutq, ww[b]), rs.hibits, rs.hi, rs.lo);
-                        x[4 * b + 3] = operand_exp(iexp_at<3>(lutq, ww[b]), rs.hibits, rs.hi, rs.lo);
+            red_sum[q * TM + r] = S;
+            soft_bar();
+            S = red_sum[r] + red_sum[TM + r] + red_sum[2 * TM + r] + red_sum[3 * TM + r];
+            // ---- this row's operand table: words q, q + 4, .., q + 60
+            if (valid) {
+                const RowSum rs = make_rowsum(S);
+                auto E_at = [&](int x) -> uint32_t {
+                    return operand_exp(lds32(lut_lane + (uint32_t)((m - x) * (TCOPIES * 4))), rs.hibits, rs.hi, rs.lo);
+                };
+#pragma unroll 2
+                for (int i = 0; i < 16; ++i) {
+                    const int j = q + 4 * i;
+                    const int xlo = (int)(int8_t)(uint8_t)(4 * j);  // logits of word j: xlo .. xlo + 3
+                    if (xlo > m) continue;                          // no key of this row reads it
+                    const int hb = min(3, m - xlo);                 // bytes above hb exceed the maximum
+                    const uint32_t E0 = E_at(xlo), Eh = E_at(xlo + hb);
+                    uint32_t word;
+                    if (E0 == Eh && monotone) {
+                        word = (4u * E0) * 0x01010101u;
+                    } else {
+                        const uint32_t E1 = hb > 1 ? E_at(xlo + 1) : Eh;
+                        const uint32_t E2 = hb > 2 ? E_at(xlo + 2) : Eh;
+                        word = 4u * (E0 | (E1 << 8) | (E2 << 16) | (Eh << 24));
                     }
-                    if (k0 + 16 > L) {  // keys at or past L get a zero operand
-                        const int n = L - k0;
-#pragma unroll
-                        for (int j = 0; j < 16; ++j)
-                            if (j >= n) x[j] = 0;
-                    }
-#pragma unroll
-                    for (int b = 0; b < 8; ++b) o[b] = __byte_perm(x[2 * b], x[2 * b + 1], 0x5410) << 10;
+                    OT[j * TM + r] = word;
                 }
-                unsigned char *arow = As + slot * A_SLOT + (r >> 3) * 1024 + (r & 7) * 128;
-                *reinterpret_cast<uint4 *>(arow + (((2 * q) ^ (r & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
-                *reinterpret_cast<uint4 *>(arow + (((2 * q + 1) ^ (r & 7)) << 4)) = make_uint4(o[4], o[5], o[6], o[7]);
-                {
+            }
+            soft_bar();
+            // ---- the previous tile's accumulators (its MMAs also release A and B)
+            if (prev_bh >= 0 && !epilogue(it - 1, prev_bh, prev_r0)) {
+                epi_bad = true;  // the next tile's first barrier ends the loop for all
+                continue;
+            }
+            // ---- V of a new head -> fp16 B
+            if (bh != conv_bh) {
+#pragma unroll
+                for (int kb = 0; kb < NKB; ++kb) {
                     const int key = kb * TKB + kk;
                     uint4 v4 = make_uint4(0, 0, 0, 0);
                     if (key < L) {
-                        const uint2 vw = *reinterpret_cast<const uint2 *>(VS + (size_t)key * TD + 8 * ci);
+                        const uint2 vw = __ldg(reinterpret_cast<const uint2 *>(p.v + ((size_t)bh * L + key) * TD + 8 * ci));
                         const uint32_t x0 = vw.x ^ 0x80808080u, x1 = vw.y ^ 0x80808080u;
                         v4.x = i8x2_to_h2(x0, 0x5140);
                         v4.y = i8x2_to_h2(x0, 0x7362);
                         v4.z = i8x2_to_h2(x1, 0x5140);
                         v4.w = i8x2_to_h2(x1, 0x7362);
                     }
-                    *reinterpret_cast<uint4 *>(Bs + slot * B_SLOT + kk * 128 + ((ci ^ (kk & 7)) << 4)) = v4;
+                    *reinterpret_cast<uint4 *>(Bs + kb * B_SLOT + kk * 128 + ((ci ^ (kk & 7)) << 4)) = v4;
                 }
-                fence_async_smem();
-                mbar_arrive(&sh.full[slot]);
-                ++g;
+                conv_bh = bh;
             }
-            if (stop || *abort_flag) break;
+            // ---- operands of this row's keys -> tensor memory
+#pragma unroll
+            for (int kb = 0; kb < NKB; ++kb) {
+                const int k0 = kb * TKB + 16 * q;
+                uint32_t o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                if (valid && k0 < L) {
+                    const uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
+#pragma unroll
+                    for (int b = 0; b < 4; ++b) {
+                        const uint32_t v = ww[b];
+                        // word (byte >> 2) of this row, then byte (byte & 3) of it into the high byte
+                        // of each fp16 half; the low bytes copy the sign of a table byte (zero)
+                        const uint32_t t0 = lds32(ot_base + (((v << 7) & 0x7E00u) | r4));
+                        const uint32_t t1 = lds32(ot_base + (((v >> 1) & 0x7E00u) | r4));
+                        const uint32_t t2 = lds32(ot_base + (((v >> 9) & 0x7E00u) | r4));
+                        const uint32_t t3 = lds32(ot_base + (((v >> 17) & 0x7E00u) | r4));
+                        o[2 * b] = prmt(t0, t1, ((v << 4) & 0x3030u) | 0x4808u);
+                        o[2 * b + 1] = prmt(t2, t3, ((v >> 12) & 0x3030u) | 0x4808u);
+                    }
+                    if (k0 + 16 > L) {  // keys at or past L get a zero operand
+                        const int n = L - k0;
+#pragma unroll
+                        for (int c = 0; c < 8; ++c) {
+                            if (2 * c >= n)
+                                o[c] = 0;
+                            else if (2 * c + 1 == n)
+                                o[c] &= 0xFFFFu;
+                        }
+                    }
+                }
+                tmem_st8(tlane + TA_COL + 32 * kb + 8 * q, o);
+            }
+            __syncwarp();
+            asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+            tc_fence_before();
             fence_async_smem();
-            mbar_arrive(&sh.vfree);  // the staged V of this tile is no longer read
-            if (warp < 4) {
-                // epilogue by warps 0-3 (tensor-memory lanes 32w..32w+31 = rows); the
-                // other warps go on to the next tile meanwhile
-                if (!mbar_wait(&sh.accfull, it & 1, abort_flag)) break;
-                tc_fence_after();
-                uint32_t v[4][16];
-                const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-#pragma unroll
-                for (int j = 0; j < 4; ++j) tmem_ld16(trow + 16 * j, v[j]);
-                asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-                tc_fence_before();
-                mbar_arrive(&sh.accempty);
-                const int erow = (int)(tile % tpb) * TM + tid;
-                if (erow < L) {
-                    int4 *dst = reinterpret_cast<int4 *>(p.acc + ((size_t)bh * L + erow) * TD);
-#pragma unroll
-                    for (int j = 0; j < 4; ++j)
-#pragma unroll
-                        for (int c = 0; c < 4; ++c)
-                            dst[4 * j + c] = make_int4(__float2int_rn(__uint_as_float(v[j][4 * c + 0])),
-                                                       __float2int_rn(__uint_as_float(v[j][4 * c + 1])),
-                                                       __float2int_rn(__uint_as_float(v[j][4 * c + 2])),
-                                                       __float2int_rn(__uint_as_float(v[j][4 * c + 3])));
-                }
-            }
+            mbar_arrive(&sh.afull);
+            prev_bh = bh;
+            prev_r0 = r0;
         }
+        if (!failed && !*abort_flag && prev_bh >= 0) epilogue(it - 1, prev_bh, prev_r0);
     } else if (warp == TLOAD_WARP && lane == 0) {
-        // ---------------- bulk copies: a tile's logits as soon as the previous tile's are in
-        // registers, its V once the previous V is converted; L2 prefetch of the tile after
-        int it = 0;
-        int lloads = 0, vloads = 0;
-        const uint32_t bv = (uint32_t)(L * TD);
-        for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
-            const int64_t bh = tile / tpb;
-            const int r0 = (int)(tile % tpb) * TM;
+        // ---------------- logits tiles (each as soon as the previous one is in registers)
+        int it = 0, lloads = 0;
+        int64_t bh = bh_begin;
+        int r0 = r0_begin;
+        for (int64_t tile = t_begin; tile < t_end; ++tile, ++it, r0 = r0 + TM < L ? r0 + TM : (++bh, 0)) {
             if (it > 0 && !mbar_wait(&sh.lfree, (it - 1) & 1, abort_flag)) break;
             const uint32_t bl = (uint32_t)(min(TM, L - r0) * p.ld);
             mbar_expect_tx(&sh.lload, bl);
             bulk_g2s(LG, p.logits + ((size_t)bh * L + r0) * p.ld, bl, &sh.lload);
             ++lloads;
-            const int64_t nxt = tile + gridDim.x;
-            if (nxt < ntiles) {
-                const int64_t bhn = nxt / tpb;
-                const int r0n = (int)(nxt % tpb) * TM;
+            if (it == 0) prefetch_l2(p.v + (size_t)bh * L * TD, (uint32_t)(L * TD));
+            if (tile + 1 < t_end) {
+                const int64_t bhn = r0 + TM < L ? bh : bh + 1;
+                const int r0n = r0 + TM < L ? r0 + TM : 0;
                 prefetch_l2(p.logits + ((size_t)bhn * L + r0n) * p.ld, (uint32_t)(min(TM, L - r0n) * p.ld));
-                if (bhn != bh) prefetch_l2(p.v + (size_t)bhn * L * TD, bv);
+                if (bhn != bh) prefetch_l2(p.v + (size_t)bhn * L * TD, (uint32_t)(L * TD));
             }
-            if (it > 0 && !mbar_wait(&sh.vfree, (it - 1) & 1, abort_flag)) break;
-            mbar_expect_tx(&sh.vload, bv);
-            bulk_g2s(VS, p.v + (size_t)bh * L * TD, bv, &sh.vload);
-            ++vloads;
         }
-        // drain: every copy issued has landed before the block exits
         if (lloads > 0) mbar_wait(&sh.lload, (lloads - 1) & 1, abort_flag, false);
-        if (vloads > 0) mbar_wait(&sh.vload, (vloads - 1) & 1, abort_flag, false);
     } else if (warp == TPRODUCER_WARP && lane == 0) {
-        // ---------------- MMA issue
-        uint32_t g = 0;
+        // ---------------- MMA issue: the whole tile once its operands are in place
         int it = 0;
         const int nkb = (L + TKB - 1) / TKB;
-        for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
-            bool ok = true;
-            for (int kb = 0; kb < nkb; ++kb, ++g) {
-                const int slot = (int)(g % TSTAGES);
-                if (!mbar_wait(&sh.full[slot], (g / TSTAGES) & 1, abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                if (kb == 0 && it > 0 && !mbar_wait(&sh.accempty, (it - 1) & 1, abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t a0 = sa(As + slot * A_SLOT), b0 = sa(Bs + slot * B_SLOT);
+        for (int64_t tile = t_begin; tile < t_end; ++tile, ++it) {
+            if (!mbar_wait(&sh.afull, it & 1, abort_flag)) break;
+            tc_fence_after();
+            const uint32_t b0 = sa(Bs);
+            for (int kb = 0; kb < nkb; ++kb)
 #pragma unroll
                 for (int s = 0; s < TKB / 16; ++s)
-                    mma_f16(tmem, smem_desc(a0 + 32 * s, 16, 1024), smem_desc(b0 + 2048 * s, 1024, 1024),
-                            (kb | s) != 0);
-                mma_commit(&sh.empty[slot]);
-            }
-            if (!ok) break;
-            mma_commit(&sh.accfull);
+                    mma_f16_ta(tmem, tmem + TA_COL + 32 * kb + 8 * s,
+                               smem_desc(b0 + kb * B_SLOT + 2048 * s, 1024, 1024), (kb | s) != 0);
+            mma_commit(&sh.mmadone);
         }
-        // drain: every MMA issued by this thread has completed
         mma_commit(&sh.fin);
         mbar_wait(&sh.fin, 0, abort_flag, false);
     }
@@ -490,13 +614,14 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     __syncthreads();
     tc_fence_after();
     if (warp == TPRODUCER_WARP)
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TD));
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tmem_cols(NKB)));
 }
 
 size_t tc_smem_bytes(int L, int64_t ld)
 {
-    return 1024 + (size_t)TSTAGES * (A_SLOT + B_SLOT) + (size_t)TM * ld + (((size_t)L * TD + 15) & ~(size_t)15) +
-           (size_t)kLutSize * TCOPIES * 4;
+    const int nkb = (L + TKB - 1) / TKB;
+    return 1024 + (size_t)nkb * B_SLOT + (size_t)64 * TM * 4 + (size_t)256 * TCOPIES * 4 +
+           (size_t)TPARTS * TM * (4 + 8) + (size_t)TM * ld;
 }
 
 template <int NKB>

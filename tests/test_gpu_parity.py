@@ -391,3 +391,29 @@ def test_tensor_core_exact_at_the_accumulator_bound(L):
         assert not ov
         assert np.array_equal(np_(acc), ao), (L, s, vv)
         assert np.abs(ao).max() < 2 ** 24
+
+
+# scales whose floored i-exp constants (Algorithm 1) make e(d) rise once per
+# period of d: there the 4-bit code is not monotone in the logit
+_RISING_SCALES = (float(np.float32(0.008350185749701165)), float(np.float32(0.01732846078509329)))
+
+
+@pytest.mark.parametrize("s", _RISING_SCALES + (0.5, 0.3, 0.0625, 0.0078125))
+def test_tensor_core_operand_table_at_any_scale(s):
+    """Per-row operand tables against the oracle: large scales change the code
+    every few logit steps, and at the rising scales codes may fall back."""
+    if s in _RISING_SCALES:
+        e = [oracle.iexp(-d, s) for d in range(256)]
+        assert any(e[i] < e[i + 1] for i in range(255))
+    rng = np.random.default_rng(11)
+    L, BH, ld = 300, 4, 304
+    x = rng.integers(-128, 128, (BH * L, ld), dtype=np.int8)
+    x[::3] = rng.integers(60, 90, (x[::3].shape), dtype=np.int8)          # narrow rows
+    x[1::7] = rng.integers(-128, -100, (x[1::7].shape), dtype=np.int8)    # rows far below 0
+    v = rng.integers(-128, 128, (BH, L, 64), dtype=np.int8)
+    acc = fqvit.lis_attention(torch.from_numpy(x).to(DEV), s, torch.from_numpy(v).to(DEV), 0)
+    fqvit.sync_status()
+    co, _ = oracle.lis_softmax(x, L, s)
+    ao, ov = oracle.lis_attn_v(co, v, 0)
+    assert not ov
+    assert np.array_equal(np_(acc), ao)
