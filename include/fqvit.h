@@ -105,6 +105,45 @@ FQVIT_API int fqvit_calibrate_ptf_noalloc(const float *x, int64_t rows, int32_t 
                                           uint8_t *alpha, double *sse_opt, void *stream);
 
 /*
+ * Sharded calibration: the batch of fqvit_calibrate_ptf split by rows over
+ * `world` ranks (one GPU each), with the same s, zp and alpha on every rank.
+ * Eqs. 8-9 need the global range and Eq. 10 sums over all rows, so the batch
+ * is calibrated in three stages with two exchanges in between (done by the
+ * caller, e.g. torch.distributed):
+ *   1. fqvit_calibrate_minmax on each rank's rows -> its (min, max);
+ *      all-reduce MIN / MAX -> the global range (exact: any split gives the
+ *      unsplit range, hence the unsplit s and zp);
+ *   2. fqvit_calibrate_sse_partial on each rank's rows with the global range
+ *      -> its err_c(a) sums (ascending row order within the rank, fp64);
+ *      all-gather;
+ *   3. fqvit_calibrate_combine (host) -> the per-rank sums added in rank
+ *      order starting from 0.0, alpha_c = the smallest a with the least
+ *      total, and s, zp of the global range.
+ * Every rank combining the same gathered sums gets identical results; one
+ * rank reproduces fqvit_calibrate_ptf exactly.  Sums of several ranks differ
+ * from the unsplit sequential sum only by fp64 rounding.
+ */
+
+/* Stage 1.  mnmx (device, float[2]) <- exact (min, max) of x [rows, C].
+ * workspace: device, >= fqvit_calibrate_workspace_size(rows, C, 0) bytes,
+ * 8-byte aligned.  Shapes as fqvit_calibrate_ptf; x must be finite. */
+FQVIT_API int fqvit_calibrate_minmax(const float *x, int64_t rows, int32_t C, int64_t ld_x, float *mnmx,
+                                     void *workspace, size_t ws_bytes, void *stream);
+
+/* Stage 2.  sse (device, double[C][K+1]) <- err_c(a) of Eq. 10 over the
+ * rows of x for the global range mnmx (device, float[2], min <= max).
+ * workspace: device, >= 64 bytes, 8-byte aligned.  bits == 8, 0 <= K <= 7. */
+FQVIT_API int fqvit_calibrate_sse_partial(const float *x, int64_t rows, int32_t C, int64_t ld_x, int32_t bits,
+                                          int32_t K, const float *mnmx, double *sse, void *workspace,
+                                          size_t ws_bytes, void *stream);
+
+/* Stage 3, host only (no GPU call).  sse_parts: host double[world][C][K+1]
+ * in rank order; (mn, mx): the global range.  Outputs (host): s, zp,
+ * alpha[C]; sse_total[C][K+1] if not NULL.  INVALID_ARG if mn > mx. */
+FQVIT_API int fqvit_calibrate_combine(const double *sse_parts, int32_t world, int32_t C, int32_t K, float mn,
+                                      float mx, float *s, int32_t *zp, uint8_t *alpha, double *sse_total);
+
+/*
  * PTF quantizer (Eq. 7): xq[r][c] = clip(rint(x[r][c] / (2^alpha_c s)) + zp, 0, 255),
  * fp32 quotient, ties to even.  x [rows, C] fp32, alpha [C] (device),
  * xq [rows, C] uint8 with stride ld_q.

@@ -43,6 +43,12 @@ def _load():
     i64, i32, f32 = ctypes.c_int64, ctypes.c_int32, ctypes.c_float
     lib.or_calibrate_ptf.argtypes = [P, i64, i32, i64, i32, P, P, P, P]
     lib.or_calibrate_ptf.restype = ctypes.c_int
+    lib.or_calibrate_minmax.argtypes = [P, i64, i32, i64, P, P]
+    lib.or_calibrate_minmax.restype = ctypes.c_int
+    lib.or_calibrate_scale.argtypes = [f32, f32, i32, P, P, P]
+    lib.or_calibrate_scale.restype = None
+    lib.or_calibrate_sse.argtypes = [P, i64, i32, i64, i32, f32, f32, P]
+    lib.or_calibrate_sse.restype = ctypes.c_int
     lib.or_ptf_quantize.argtypes = [P, i64, i32, i64, f32, i32, P, P, i64]
     lib.or_ptf_quantize.restype = ctypes.c_int
     lib.or_ptf_layernorm.argtypes = [P, i64, i32, i64, i32, P, P, P, f32, i32, P, i64, P, P]
@@ -98,6 +104,66 @@ def calibrate_ptf(x: np.ndarray, K: int = 3):
     if rc:
         raise ValueError("or_calibrate_ptf rejected its arguments")
     return float(s[0]), int(zp[0]), alpha, sse
+
+
+def calibrate_minmax(x: np.ndarray):
+    """Exact fp32 (min, max) over every element of x."""
+    x = _c(x, np.float32)
+    rows, C = x.shape
+    mn = np.zeros(1, np.float32)
+    mx = np.zeros(1, np.float32)
+    if _load().or_calibrate_minmax(_ptr(x), rows, C, C, _ptr(mn), _ptr(mx)):
+        raise ValueError("or_calibrate_minmax rejected its arguments")
+    return float(mn[0]), float(mx[0])
+
+
+def calibrate_scale(mn: float, mx: float, K: int = 3):
+    """Eqs. 8-9 from a range: (s0 = 2^K s, s, zp)."""
+    s0 = np.zeros(1, np.float32)
+    s = np.zeros(1, np.float32)
+    zp = np.zeros(1, np.int32)
+    _load().or_calibrate_scale(mn, mx, K, _ptr(s0), _ptr(s), _ptr(zp))
+    return float(s0[0]), float(s[0]), int(zp[0])
+
+
+def calibrate_sse(x: np.ndarray, K: int, mn: float, mx: float) -> np.ndarray:
+    """Eq. 10 over the rows of x (ascending, fp64) for the range (mn, mx): [C, K+1]."""
+    x = _c(x, np.float32)
+    rows, C = x.shape
+    sse = np.zeros((C, K + 1), np.float64)
+    if _load().or_calibrate_sse(_ptr(x), rows, C, C, K, mn, mx, _ptr(sse)):
+        raise ValueError("or_calibrate_sse rejected its arguments")
+    return sse
+
+
+def calibrate_ptf_sharded(shards, K: int = 3):
+    """Eqs. 8-10 over a calibration batch split by rows into shards (rank order).
+
+    The range is the min / max over all shards (exact, so any split gives the
+    unsplit range and hence the same s and zp).  Each shard sums its own rows
+    in ascending order in fp64; the per-shard sums are then added in shard
+    order, starting from 0.0, and alpha_c is the smallest factor with the
+    least total.  One shard reproduces ``calibrate_ptf`` exactly.
+    Returns (s, zp, alpha[C] uint8, sse[C, K+1] float64).
+    """
+    shards = [s for s in shards if s.shape[0] > 0]
+    if not shards:
+        raise ValueError("no calibration rows")
+    ranges = [calibrate_minmax(x) for x in shards]
+    mn = min(r[0] for r in ranges)
+    mx = max(r[1] for r in ranges)
+    _, s, zp = calibrate_scale(mn, mx, K)
+    total = np.zeros((shards[0].shape[1], K + 1), np.float64)
+    for x in shards:
+        total = total + calibrate_sse(x, K, mn, mx)
+    alpha = np.zeros(total.shape[0], np.uint8)
+    for c in range(total.shape[0]):
+        best = 0
+        for a in range(1, K + 1):
+            if total[c, a] < total[c, best]:
+                best = a
+        alpha[c] = best
+    return s, zp, alpha, total
 
 
 def ptf_quantize(x: np.ndarray, s: float, zp: int, alpha: np.ndarray) -> np.ndarray:

@@ -92,11 +92,11 @@ OR_EXPORT void or_set_num_threads(int n)
  *  nearest even) and the square and the sum are fp64, summed in ascending
  *  row order.  alpha_c is the smallest alpha attaining the minimum.
  */
-OR_EXPORT int or_calibrate_ptf(const float *x, int64_t rows, int32_t C, int64_t ld,
-                               int32_t K, float *s_out, int32_t *zp_out,
-                               uint8_t *alpha, double *sse /* C*(K+1) or NULL */)
+/* exact fp32 minimum and maximum over all elements */
+OR_EXPORT int or_calibrate_minmax(const float *x, int64_t rows, int32_t C, int64_t ld, float *mn_out,
+                                  float *mx_out)
 {
-    if (!x || rows < 1 || C < 1 || ld < C || K < 0 || K > 7) return 1;
+    if (!x || rows < 1 || C < 1 || ld < C) return 1;
     float mn = x[0], mx = x[0];
     for (int64_t r = 0; r < rows; ++r)
         for (int32_t c = 0; c < C; ++c) {
@@ -104,20 +104,34 @@ OR_EXPORT int or_calibrate_ptf(const float *x, int64_t rows, int32_t C, int64_t 
             if (v < mn) mn = v;
             if (v > mx) mx = v;
         }
+    *mn_out = mn;
+    *mx_out = mx;
+    return 0;
+}
+
+/* Eqs. 8-9 from the range: s0 = (max - min) / 255 is 2^K s, zp from s0 */
+OR_EXPORT void or_calibrate_scale(float mn, float mx, int32_t K, float *s0_out, float *s_out,
+                                  int32_t *zp_out)
+{
     float range = mx - mn;
     if (range == 0.0f) range = 1.0f;
     float s0 = range / 255.0f;
-    float s = ldexpf(s0, -K);
     float t = -mn / s0;
-    float zr = clamp_f32(rintf(t), 0.0f, 255.0f);
-    int32_t zp = (int32_t)zr;
-    *s_out = s;
-    *zp_out = zp;
+    *s0_out = s0;
+    *s_out = ldexpf(s0, -K);
+    *zp_out = (int32_t)clamp_f32(rintf(t), 0.0f, 255.0f);
+}
 
+/* Eq. 10 for every channel and factor, rows summed in ascending order */
+OR_EXPORT int or_calibrate_sse(const float *x, int64_t rows, int32_t C, int64_t ld, int32_t K,
+                               float mn, float mx, double *sse /* C*(K+1) */)
+{
+    if (!x || !sse || rows < 1 || C < 1 || ld < C || K < 0 || K > 7) return 1;
+    float s0, s;
+    int32_t zp;
+    or_calibrate_scale(mn, mx, K, &s0, &s, &zp);
 #pragma omp parallel for schedule(static)
     for (int32_t c = 0; c < C; ++c) {
-        double best = 0.0;
-        int best_a = 0;
         for (int32_t a = 0; a <= K; ++a) {
             float sa = ldexpf(s0, a - K); /* 2^a * s, exact */
             double err = 0.0;
@@ -129,14 +143,32 @@ OR_EXPORT int or_calibrate_ptf(const float *x, int64_t rows, int32_t C, int64_t 
                 float d = v - dq;
                 err += (double)d * (double)d;
             }
-            if (sse) sse[(int64_t)c * (K + 1) + a] = err;
-            if (a == 0 || err < best) {
-                best = err;
-                best_a = a;
-            }
+            sse[(int64_t)c * (K + 1) + a] = err;
         }
+    }
+    return 0;
+}
+
+OR_EXPORT int or_calibrate_ptf(const float *x, int64_t rows, int32_t C, int64_t ld,
+                               int32_t K, float *s_out, int32_t *zp_out,
+                               uint8_t *alpha, double *sse /* C*(K+1) or NULL */)
+{
+    if (!x || !alpha || rows < 1 || C < 1 || ld < C || K < 0 || K > 7) return 1;
+    float mn, mx, s0;
+    or_calibrate_minmax(x, rows, C, ld, &mn, &mx);
+    or_calibrate_scale(mn, mx, K, &s0, s_out, zp_out);
+    double *err = (double *)malloc(sizeof(double) * (size_t)C * (size_t)(K + 1));
+    if (!err) return 1;
+    or_calibrate_sse(x, rows, C, ld, K, mn, mx, err);
+    for (int32_t c = 0; c < C; ++c) {
+        const double *e = err + (int64_t)c * (K + 1);
+        int best_a = 0;
+        for (int32_t a = 1; a <= K; ++a)
+            if (e[a] < e[best_a]) best_a = a;
         alpha[c] = (uint8_t)best_a;
     }
+    if (sse) memcpy(sse, err, sizeof(double) * (size_t)C * (size_t)(K + 1));
+    free(err);
     return 0;
 }
 

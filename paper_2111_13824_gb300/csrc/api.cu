@@ -108,6 +108,68 @@ int fqvit_calibrate_ptf(const float *x, int64_t rows, int32_t C, int64_t ld_x, i
                        "calibrate_ptf");
 }
 
+int fqvit_calibrate_minmax(const float *x, int64_t rows, int32_t C, int64_t ld_x, float *mnmx, void *workspace,
+                           size_t ws_bytes, void *stream)
+{
+    if (!x || !mnmx || !workspace) return fail(FQVIT_ERR_INVALID_ARG, "calibrate_minmax: NULL pointer");
+    if (rows < 1 || C < 1 || C > 8192 || ld_x < C)
+        return fail(FQVIT_ERR_INVALID_ARG, "calibrate_minmax: bad shape rows=%lld C=%d ld_x=%lld", (long long)rows,
+                    C, (long long)ld_x);
+    if (!aligned(x, 4) || !aligned(mnmx, 4) || !aligned(workspace, 8))
+        return fail(FQVIT_ERR_INVALID_ARG, "calibrate_minmax: misaligned pointer");
+    size_t need = fqvit::calibrate_workspace_bytes(rows, C, 0);
+    if (ws_bytes < need)
+        return fail(FQVIT_ERR_INVALID_ARG, "calibrate_minmax: workspace %zu bytes, need %zu", ws_bytes, need);
+    return cuda_status(fqvit::launch_calibrate_minmax(x, rows, C, ld_x, mnmx, workspace, as_stream(stream)),
+                       "calibrate_minmax");
+}
+
+int fqvit_calibrate_sse_partial(const float *x, int64_t rows, int32_t C, int64_t ld_x, int32_t bits, int32_t K,
+                                const float *mnmx, double *sse, void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!x || !mnmx || !sse || !workspace) return fail(FQVIT_ERR_INVALID_ARG, "calibrate_sse_partial: NULL pointer");
+    if (rows < 1 || C < 1 || C > 8192 || ld_x < C)
+        return fail(FQVIT_ERR_INVALID_ARG, "calibrate_sse_partial: bad shape rows=%lld C=%d ld_x=%lld",
+                    (long long)rows, C, (long long)ld_x);
+    if (bits != 8) return fail(FQVIT_ERR_UNSUPPORTED, "calibrate_sse_partial: bits=%d (only 8)", bits);
+    if (K < 0 || K > 7) return fail(FQVIT_ERR_UNSUPPORTED, "calibrate_sse_partial: K=%d (0..7)", K);
+    if (!aligned(x, 4) || !aligned(mnmx, 4) || !aligned(sse, 8) || !aligned(workspace, 8))
+        return fail(FQVIT_ERR_INVALID_ARG, "calibrate_sse_partial: misaligned pointer");
+    if (ws_bytes < 64) return fail(FQVIT_ERR_INVALID_ARG, "calibrate_sse_partial: workspace %zu bytes, need 64", ws_bytes);
+    return cuda_status(
+        fqvit::launch_calibrate_sse_partial(x, rows, C, ld_x, K, mnmx, sse, workspace, as_stream(stream)),
+        "calibrate_sse_partial");
+}
+
+int fqvit_calibrate_combine(const double *sse_parts, int32_t world, int32_t C, int32_t K, float mn, float mx,
+                            float *s, int32_t *zp, uint8_t *alpha, double *sse_total)
+{
+    if (!sse_parts || !s || !zp || !alpha) return fail(FQVIT_ERR_INVALID_ARG, "calibrate_combine: NULL pointer");
+    if (world < 1 || C < 1 || C > 8192) return fail(FQVIT_ERR_INVALID_ARG, "calibrate_combine: world=%d C=%d", world, C);
+    if (K < 0 || K > 7) return fail(FQVIT_ERR_UNSUPPORTED, "calibrate_combine: K=%d (0..7)", K);
+    if (!(mn <= mx) || !(mx - mn < 3.0e38f))
+        return fail(FQVIT_ERR_INVALID_ARG, "calibrate_combine: range [%g, %g] is empty or not finite", (double)mn,
+                    (double)mx);
+    const int64_t n = (int64_t)C * (K + 1);
+    for (int32_t c = 0; c < C; ++c) {
+        int best = 0;
+        double best_e = 0.0;
+        for (int32_t a = 0; a <= K; ++a) {
+            double t = 0.0;  // rank order, starting from zero: one rank gives its own sums back
+            for (int32_t r = 0; r < world; ++r) t += sse_parts[r * n + (int64_t)c * (K + 1) + a];
+            if (sse_total) sse_total[(int64_t)c * (K + 1) + a] = t;
+            if (a == 0 || t < best_e) {
+                best_e = t;
+                best = a;
+            }
+        }
+        alpha[c] = (uint8_t)best;
+    }
+    float s0;
+    fqvit::calib_scale(mn, mx, K, s0, *s, *zp);
+    return fail(FQVIT_OK, "");
+}
+
 int fqvit_ptf_quantize(const float *x, int64_t rows, int32_t C, int64_t ld_x, float s, int32_t zp,
                        const uint8_t *alpha, uint8_t *xq, int64_t ld_q, void *stream)
 {

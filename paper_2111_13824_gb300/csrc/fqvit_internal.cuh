@@ -15,6 +15,32 @@ int record_error(int code, const char *msg);
 
 // ---- PTF calibration / quantizer (ptf.cu) ---------------------------------
 size_t calibrate_workspace_bytes(int64_t rows, int C, int K);
+
+// Eqs. 8-9 from the calibration range, shared by the device path and the host
+// combine of sharded calibration: s0 = (mx - mn) / 255 (a zero range counts
+// as 1) is 2^K s, zp = clip(rint(-mn / s0), 0, 255).  Every operation is a
+// single IEEE round-to-nearest one, so host and device agree bit for bit.
+__host__ __device__ inline void calib_scale(float mn, float mx, int K, float &s0, float &s, int32_t &zp)
+{
+    float range = mx - mn;
+    if (range == 0.0f) range = 1.0f;
+    s0 = range / 255.0f;
+#ifdef __CUDA_ARCH__
+    s = s0 * __int_as_float((127 - K) << 23);  // s0 / 2^K, exact
+#else
+    s = ldexpf(s0, -K);
+#endif
+    const float t = -mn / s0;
+    zp = (int32_t)fminf(fmaxf(rintf(t), 0.0f), 255.0f);
+}
+
+// Per-rank stages of a calibration batch split by rows (sharded calibration):
+// the shard's exact (min, max) into mnmx[2], and the shard's Eq. 10 sums for
+// the global range mnmx[2] into sse[C][K+1].
+cudaError_t launch_calibrate_minmax(const float *x, int64_t rows, int C, int64_t ld_x, float *mnmx, void *ws,
+                                    cudaStream_t st);
+cudaError_t launch_calibrate_sse_partial(const float *x, int64_t rows, int C, int64_t ld_x, int K,
+                                         const float *mnmx, double *sse, void *ws, cudaStream_t st);
 cudaError_t launch_calibrate(const float *x, int64_t rows, int C, int64_t ld_x, int K, float *s,
                              int32_t *zp, uint8_t *alpha, double *sse, void *ws,
                              cudaStream_t st);

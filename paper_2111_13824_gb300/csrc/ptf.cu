@@ -1,7 +1,10 @@
 // ptf.cu -- Power-of-Two Factor calibration (Sec. 3.2, Eqs. 8-10) and the
 // PTF quantizer (Eq. 7) on sm_103a.
 //
-// Calibration runs in four launches on the caller's stream:
+// Calibration runs in four launches on the caller's stream (a calibration
+// batch split by rows over several ranks runs the first and third per rank,
+// with the range and the sums exchanged in between; see
+// fqvit_calibrate_minmax / _sse_partial / _combine):
 //   1. per-block min / max of the calibration batch (exact fp32 compares),
 //   2. one block folds the partials into s, zp (Eqs. 8-9),
 //   3. one thread per (channel, factor) sums the squared quantization error
@@ -76,17 +79,44 @@ __global__ void calib_finalize_kernel(const float2 *__restrict__ part, int npart
         mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
     }
     if (threadIdx.x == 0) {
-        float range = __fsub_rn(mx, mn);
-        if (range == 0.0f) range = 1.0f;
-        float s0 = __fdiv_rn(range, 255.0f);
-        float s = __fmul_rn(s0, pow2f(-K));
-        float t = __fdiv_rn(-mn, s0);
-        float z = fminf(fmaxf(rintf(t), 0.0f), 255.0f);
+        float s0, s;
+        int32_t zp;
+        calib_scale(mn, mx, K, s0, s, zp);
         *s_out = s;
-        *zp_out = (int32_t)z;
+        *zp_out = zp;
         *ws_s0 = s0;
-        *ws_zp = (int32_t)z;
+        *ws_zp = zp;
     }
+}
+
+// Folds the min / max partials of one shard into mnmx[2].
+__global__ void minmax_final_kernel(const float2 *__restrict__ part, int nparts, float *__restrict__ mnmx)
+{
+    float mn = FLT_MAX, mx = -FLT_MAX;
+    for (int i = threadIdx.x; i < nparts; i += 32) {
+        float2 p = part[i];
+        mn = fminf(mn, p.x);
+        mx = fmaxf(mx, p.y);
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+        mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    }
+    if (threadIdx.x == 0) {
+        mnmx[0] = mn;
+        mnmx[1] = mx;
+    }
+}
+
+// s0 and zp of a given (global) range, for the Eq. 10 sums of one shard.
+__global__ void calib_setscale_kernel(const float *__restrict__ mnmx, int K, float *__restrict__ ws_s0,
+                                      int32_t *__restrict__ ws_zp)
+{
+    float s0, s;
+    int32_t zp;
+    calib_scale(mnmx[0], mnmx[1], K, s0, s, zp);
+    *ws_s0 = s0;
+    *ws_zp = zp;
 }
 
 // Eq. 10, one thread per (channel c, factor a): sum over rows of
@@ -169,6 +199,15 @@ __global__ void quantize_kernel(const float *__restrict__ x, int64_t rows, int C
     }
 }
 
+// blocks of the min / max pass
+int minmax_blocks(int64_t rows)
+{
+    int nparts = (int)(rows < kMaxPartials ? rows : kMaxPartials);
+    int nsm = sm_count();
+    if (nparts > 4 * nsm) nparts = 4 * nsm;
+    return nparts < 1 ? 1 : nparts;
+}
+
 }  // namespace
 
 size_t calibrate_workspace_bytes(int64_t rows, int C, int K)
@@ -186,15 +225,34 @@ cudaError_t launch_calibrate(const float *x, int64_t rows, int C, int64_t ld_x, 
     float2 *part = reinterpret_cast<float2 *>(w + kWsHeader);
     double *sse_buf = sse ? sse : reinterpret_cast<double *>(w + kWsHeader + sizeof(float2) * kMaxPartials);
 
-    int nparts = (int)(rows < kMaxPartials ? rows : kMaxPartials);
-    int nsm = sm_count();
-    if (nparts > 4 * nsm) nparts = 4 * nsm;
-    if (nparts < 1) nparts = 1;
+    const int nparts = minmax_blocks(rows);
     minmax_partial_kernel<<<nparts, 256, 0, st>>>(x, rows, C, ld_x, part);
     calib_finalize_kernel<<<1, 32, 0, st>>>(part, nparts, K, s, zp, ws_s0, ws_zp);
     dim3 g((C + 31) / 32, K + 1);
     calib_sse_kernel<<<g, 32, 0, st>>>(x, rows, C, ld_x, K, ws_s0, ws_zp, sse_buf);
     calib_argmin_kernel<<<(C + 127) / 128, 128, 0, st>>>(sse_buf, C, K, alpha);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_calibrate_minmax(const float *x, int64_t rows, int C, int64_t ld_x, float *mnmx, void *ws,
+                                    cudaStream_t st)
+{
+    float2 *part = reinterpret_cast<float2 *>(static_cast<char *>(ws) + kWsHeader);
+    const int nparts = minmax_blocks(rows);
+    minmax_partial_kernel<<<nparts, 256, 0, st>>>(x, rows, C, ld_x, part);
+    minmax_final_kernel<<<1, 32, 0, st>>>(part, nparts, mnmx);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_calibrate_sse_partial(const float *x, int64_t rows, int C, int64_t ld_x, int K,
+                                         const float *mnmx, double *sse, void *ws, cudaStream_t st)
+{
+    char *w = static_cast<char *>(ws);
+    float *ws_s0 = reinterpret_cast<float *>(w);
+    int32_t *ws_zp = reinterpret_cast<int32_t *>(w + 4);
+    calib_setscale_kernel<<<1, 1, 0, st>>>(mnmx, K, ws_s0, ws_zp);
+    dim3 g((C + 31) / 32, K + 1);
+    calib_sse_kernel<<<g, 32, 0, st>>>(x, rows, C, ld_x, K, ws_s0, ws_zp, sse);
     return cudaGetLastError();
 }
 

@@ -43,6 +43,7 @@ EXPORTS = (
     "fqvit_version", "fqvit_last_error", "fqvit_calibrate_workspace_size", "fqvit_calibrate_ptf",
     "fqvit_ptf_quantize", "fqvit_ptf_layernorm", "fqvit_lis_softmax", "fqvit_lis_attn_v",
     "fqvit_lis_attention", "fqvit_block_int", "fqvit_sync_status", "fqvit_calibrate_ptf_noalloc",
+    "fqvit_calibrate_minmax", "fqvit_calibrate_sse_partial", "fqvit_calibrate_combine",
 )
 
 
@@ -74,6 +75,9 @@ def load(path: str | Path | None = None):
         "fqvit_block_int": ([P, P], ctypes.c_int),
         "fqvit_sync_status": ([P], ctypes.c_int),
         "fqvit_calibrate_ptf_noalloc": ([P, i64, i32, i64, i32, i32, P, P, P, P, P], ctypes.c_int),
+        "fqvit_calibrate_minmax": ([P, i64, i32, i64, P, P, sz, P], ctypes.c_int),
+        "fqvit_calibrate_sse_partial": ([P, i64, i32, i64, i32, i32, P, P, P, sz, P], ctypes.c_int),
+        "fqvit_calibrate_combine": ([P, i32, i32, i32, f32, f32, P, P, P, P], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -156,6 +160,57 @@ def calibrate_ptf_noalloc(x: torch.Tensor, K: int = 3, bits: int = 8, sse: torch
     _check(load().fqvit_calibrate_ptf_noalloc(_p(x), rows, C, _ld(x), bits, K, _p(s), _p(zp), _p(alpha), _p(sse),
                                               _stream(stream)))
     return s, zp, alpha
+
+
+def _workspace(rows: int, C: int, K: int, dev) -> torch.Tensor:
+    nbytes = calibrate_workspace_size(rows, C, K)
+    return torch.empty(max(nbytes, 64) // 8 + 1, dtype=torch.float64, device=dev)
+
+
+def calibrate_minmax(x: torch.Tensor, workspace: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Stage 1 of sharded calibration: device float32[2] = (min, max) of x."""
+    rows, C = x.shape
+    mnmx = torch.empty(2, dtype=torch.float32, device=x.device)
+    if workspace is None:
+        workspace = _workspace(rows, C, 0, x.device)
+    _check(load().fqvit_calibrate_minmax(_p(x), rows, C, _ld(x), _p(mnmx), _p(workspace),
+                                         workspace.numel() * workspace.element_size(), _stream(stream)))
+    return mnmx
+
+
+def calibrate_sse_partial(x: torch.Tensor, K: int, mnmx: torch.Tensor, bits: int = 8,
+                          sse: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
+                          stream=None) -> torch.Tensor:
+    """Stage 2: device float64[C, K+1] of Eq. 10 over the rows of x for the global range mnmx."""
+    rows, C = x.shape
+    if sse is None:
+        sse = torch.empty(C, K + 1, dtype=torch.float64, device=x.device)
+    if workspace is None:
+        workspace = _workspace(rows, C, 0, x.device)
+    _check(load().fqvit_calibrate_sse_partial(_p(x), rows, C, _ld(x), bits, K, _p(mnmx), _p(sse), _p(workspace),
+                                              workspace.numel() * workspace.element_size(), _stream(stream)))
+    return sse
+
+
+def calibrate_combine(sse_parts: torch.Tensor, mn: float, mx: float, K: int):
+    """Stage 3 (host, no GPU): sse_parts float64 [world, C, K+1] on the CPU, in rank order.
+
+    Returns (s float, zp int, alpha uint8[C] CPU tensor, sse_total float64 [C, K+1] CPU tensor).
+    """
+    if sse_parts.device.type != "cpu" or sse_parts.dtype != torch.float64 or sse_parts.dim() != 3:
+        raise ValueError("sse_parts must be a CPU float64 tensor [world, C, K+1]")
+    parts = sse_parts.contiguous()
+    world, C, k1 = parts.shape
+    if k1 != K + 1:
+        raise ValueError("sse_parts has the wrong factor count")
+    s = ctypes.c_float()
+    zp = ctypes.c_int32()
+    alpha = torch.empty(C, dtype=torch.uint8)
+    total = torch.empty(C, K + 1, dtype=torch.float64)
+    _check(load().fqvit_calibrate_combine(ctypes.c_void_p(parts.data_ptr()), world, C, K, float(mn), float(mx),
+                                          ctypes.byref(s), ctypes.byref(zp), ctypes.c_void_p(alpha.data_ptr()),
+                                          ctypes.c_void_p(total.data_ptr())))
+    return float(s.value), int(zp.value), alpha, total
 
 
 def ptf_quantize(x: torch.Tensor, s: float, zp: int, alpha: torch.Tensor, out: torch.Tensor | None = None,
