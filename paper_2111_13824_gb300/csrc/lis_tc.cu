@@ -32,6 +32,7 @@
 #include "fqvit_internal.cuh"
 #include "lis_common.cuh"
 
+#include <cuda.h>
 #include <cuda_fp16.h>
 
 namespace fqvit {
@@ -45,7 +46,6 @@ using namespace lis;
 constexpr int TM = 128;        // query rows per tile (MMA M)
 constexpr int TKB = 64;        // keys per key block
 constexpr int TD = 64;         // head dimension (MMA N)
-constexpr int TMAXLD = 592;    // largest logit row stride handled here
 constexpr int TCOPIES = 32;    // replicas of the i-exp table (one per lane)
 constexpr int B_SLOT = TKB * TD * 2;
 constexpr unsigned long long kTimeoutNs = 2000000000ull;
@@ -77,11 +77,6 @@ __device__ __forceinline__ void mbar_init(uint64_t *b, uint32_t n)
 __device__ __forceinline__ void mbar_arrive(uint64_t *b)
 {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(sa(b)) : "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint64_t *b, uint32_t bytes)
-{
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(sa(b)), "r"(bytes) : "memory");
 }
 
 __device__ __forceinline__ bool mbar_try(uint64_t *b, uint32_t parity)
@@ -131,14 +126,6 @@ __device__ __forceinline__ void prefetch_l2(const void *src, uint32_t bytes)
     asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
 }
 
-__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *b)
-{
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(sa(dst)),
-        "l"(src), "r"(bytes), "r"(sa(b))
-        : "memory");
-}
-
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
@@ -182,12 +169,19 @@ __device__ __forceinline__ uint32_t i8x2_to_h2(uint32_t xw, uint32_t sel)
     return *reinterpret_cast<uint32_t *>(&h);
 }
 
-constexpr int TPARTS = 4;                      // threads per query row
-constexpr int TSOFT = TM * TPARTS;             // softmax threads (16 warps)
-constexpr int TPRODUCER_WARP = TSOFT / 32;     // warp 16: MMA issue
-constexpr int TLOAD_WARP = TPRODUCER_WARP + 1; // warp 17: bulk copies of the logits
+constexpr int TPARTS = 4;                         // threads per query row
+constexpr int TSOFT = TM * TPARTS;                // softmax threads (16 warps)
+constexpr int TPRODUCER_WARP = TSOFT / 32;        // warp 16: MMA issue
+constexpr int TLOAD_WARP = TPRODUCER_WARP + 1;    // warp 17: bulk copies of the logits, L2 prefetch
 constexpr int TTHREADS = (TLOAD_WARP + 1) * 32;
-constexpr int TA_COL = TD;                     // D: columns 0..63; A of key block kb: 64 + 32 kb ..
+constexpr int TMAXKB = 10;                        // key blocks of the longest row (L <= 640)
+constexpr int TA_COL = TD;                        // D: columns 0..63; A of key block kb: 64 + 32 kb ..
+// The logits tile doubles as scratch between the row sums and the table: accumulator staging
+// (two 128-row x 128-byte halves in the 128-byte swizzle of the output tensor map) and the
+// row thresholds.
+constexpr int SCR_STAGE = 2 * TM * 128;           // 32 KB
+constexpr int SCR_THR = SCR_STAGE;                // int32 [16][TM]
+constexpr int SCR_BYTES = SCR_THR + 16 * TM * 4;  // 40 KB
 
 // tensor-memory columns for NKB key blocks (a power of two >= 32)
 __host__ __device__ constexpr int tmem_cols(int nkb)
@@ -290,38 +284,67 @@ __device__ __forceinline__ void mma_f16_ta(uint32_t dt, uint32_t at, uint64_t bd
         : "memory");
 }
 
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *b)
+{
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(sa(dst)),
+        "l"(src), "r"(bytes), "r"(sa(b))
+        : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *b, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(sa(b)), "r"(bytes) : "memory");
+}
+
+// tensor store of one 128-row x 32-column half tile of accumulators (rows past L are clipped
+// by the tensor map), in a bulk group
+__device__ __forceinline__ void tma_store_acc(const CUtensorMap *map, const void *ssrc, int col, int row, int head)
+{
+    asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(col), "r"(row), "r"(head), "r"(sa(ssrc))
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
 // Per tile (128 query rows of one head):
-//   copy warp:  logits tile -> shared memory (bulk copy), L2 prefetch of the next tile (and of
-//               the next head's V)
+//   copy warp:  logits tile -> shared memory (bulk copy) once the previous tile's table is built,
+//               L2 prefetch of the next tile (and of the next head's V)
 //   softmax:    thread (row r, part q) takes keys 64 kb + 16 q .. +15 of every key block into
 //               registers; the row maximum and the i-exp row sum are combined over the four parts
-//               through shared memory.  The row's operands then go into a table indexed by the
-//               raw logit byte: word j of row r (OT[j][r], so that the 32 rows of a warp sit in
-//               32 different banks) holds, in byte b, 4 (30 - code) for the logit byte 4 j + b.
-//               Codes only depend on the row maximum, the row sum and the logit, so one table
-//               serves the whole row; it is filled by the four parts together, evaluating the
-//               code at the two ends of each word first: where the i-exp values never rise
-//               with the distance to the maximum, codes are monotone in the logit and equal
-//               ends fill the word (the floored constants of a few scales break this; those
-//               evaluate every byte).  Every logit then costs one table load; two loads
-//               and one byte permute give the fp16 pair 2^(15-code) that goes to tensor memory
-//               (A, K-major rows = lanes).  V of a head -> fp16 in shared memory (B, MN-major)
-//               whenever the head changes.
+//               through shared memory.  Then the previous tile's accumulators come back from
+//               tensor memory into a staging tile (128-byte swizzle) and leave as two tensor
+//               stores.  The row's operands go into a table indexed by the raw logit byte: word j
+//               of row r (OT[j][r], so that the 32 rows of a warp sit in 32 different banks)
+//               holds, in byte b, 4 (30 - code) for the logit byte 4 j + b.  Codes only depend on
+//               the row maximum, the row sum and the logit, so one table serves the whole row.
+//               Where the i-exp values never rise with the distance d to the maximum,
+//               code(d) = #{k <= 15 : d >= delta_k} for the row's thresholds delta_k (the first d
+//               with e(d) D_k <= 2S): the four parts find them by binary search, histogram them
+//               into the table words and turn each word into its codes with a byte prefix sum
+//               (a multiply by 0x01010101); the floored constants of a few scales break the
+//               monotony, and those evaluate every entry.  Every logit then costs one table
+//               load; two loads and one byte permute give the fp16 pair 2^(15-code) that goes to
+//               tensor memory (A, K-major rows = lanes).  V of a head -> fp16 in shared memory
+//               (B, MN-major) whenever the head changes.
 //   MMA thread: after all operands of the tile are written, 4 MMAs per key block, one commit
-//   epilogue:   one tile later, all 16 warps read the accumulators (16 columns each)
 // Each CTA takes a contiguous range of tiles, so that consecutive tiles share a head.
 template <int NKB>
-__global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
+__global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, const __grid_constant__ CUtensorMap acc_map)
 {
     extern __shared__ unsigned char dsm_raw[];
     __shared__ TcShared sh;
+    __shared__ __align__(16) uint32_t OT[64 * TM];              // operand table: word j of row r at [j][r]
     unsigned char *base = dsm_raw + ((1024u - (sa(dsm_raw) & 1023u)) & 1023u);
     unsigned char *Bs = base;                                   // NKB x 8 KB
-    uint32_t *OT = (uint32_t *)(Bs + NKB * B_SLOT);             // 64 x TM operand-table words
-    uint32_t *LUT = OT + 64 * TM;                               // 256 x TCOPIES
-    int *red_max = (int *)(LUT + 256 * TCOPIES);
+    uint32_t *LUT = (uint32_t *)(Bs + NKB * B_SLOT);            // 256 x TCOPIES
+    int *red_max = (int *)(LUT + 256 * TCOPIES);                // TPARTS x TM
     unsigned long long *red_sum = (unsigned long long *)(red_max + TPARTS * TM);
-    int8_t *LG = (int8_t *)(red_sum + TPARTS * TM);             // TM x ld
+    unsigned char *LG = (unsigned char *)(red_sum + TPARTS * TM);  // TM x ld logits, then scratch
+    int *thr = (int *)(LG + SCR_THR);                           // 16 x TM: delta_k of each row
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile int *abort_flag = &sh.abort_flag;
@@ -358,58 +381,57 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     const int tpb = (L + TM - 1) / TM;
     const int64_t ntiles = p.BH * tpb;
     const int64_t t_begin = (int64_t)blockIdx.x * ntiles / gridDim.x;
-    const int64_t t_end = (int64_t)(blockIdx.x + 1) * ntiles / gridDim.x;
+    const int ncta_tiles = (int)((int64_t)(blockIdx.x + 1) * ntiles / gridDim.x - t_begin);
     // (head, first row) of tile t_begin; every role steps it by one tile per iteration
-    const int64_t bh_begin = t_begin / tpb;
-    const int r0_begin = (int)(t_begin - bh_begin * tpb) * TM;
+    const int bh_begin = (int)(t_begin / tpb);
+    const int r0_begin = (int)(t_begin - (int64_t)bh_begin * tpb) * TM;
 
     if (tid < TSOFT) {
         const int r = tid & (TM - 1), q = tid >> 7;   // warp (q, r / 32): lanes = rows = TMEM lanes
         const int kk = tid >> 3, ci = tid & 7;        // V conversion: key kk of a block, values 8 ci .. +7
         const uint32_t lut_lane = sa(LUT) + 4u * (uint32_t)lane;
-        const uint32_t ot_base = sa(OT);
         const uint32_t r4 = 4u * (uint32_t)r;
+        const unsigned char *otb = reinterpret_cast<const unsigned char *>(OT);
         const uint32_t tlane = tmem + ((uint32_t)((warp & 3) * 32) << 16);
         const bool small_e = LUT[0] < (1u << 28);    // e(0) is the largest i-exp value
         const bool monotone = !sh.rising;            // codes never fall as d grows
+        const int xs = (int)(int8_t)(uint8_t)(64 * q);  // part q's table words 16 q .. +15: logits xs .. xs + 63
         int it = 0;
-        bool epi_bad = false;
-        int64_t prev_bh = -1, conv_bh = -1;
+        bool epi_bad = false, failed = false;
+        int prev_bh = -1, conv_bh = -1;
         int prev_r0 = 0;
-        // accumulators of the previous tile: warp w reads rows 32 (w % 4) .., columns 16 (w / 4) ..
-        auto epilogue = [&](int tit, int64_t ebh, int er0) -> bool {
+        // accumulators of tile tit into the staging halves: warp w, rows 32 (w % 4) .., columns 16 (w / 4) ..
+        auto epilogue = [&](int tit) -> bool {
             if (!mbar_wait_warp(&sh.mmadone, tit & 1, abort_flag)) return false;
             tc_fence_after();
             uint32_t v[16];
             tmem_ld16(tlane + 16 * (warp >> 2), v);
             asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-            const int erow = er0 + (warp & 3) * 32 + lane;
-            if (erow < L) {
-                int4 *dst = reinterpret_cast<int4 *>(p.acc + ((size_t)ebh * L + erow) * TD + 16 * (warp >> 2));
+            unsigned char *half = LG + (q >> 1) * (TM * 128) + r * 128;
 #pragma unroll
-                for (int c = 0; c < 4; ++c)
-                    dst[c] = make_int4(__float2int_rn(__uint_as_float(v[4 * c + 0])),
-                                       __float2int_rn(__uint_as_float(v[4 * c + 1])),
-                                       __float2int_rn(__uint_as_float(v[4 * c + 2])),
-                                       __float2int_rn(__uint_as_float(v[4 * c + 3])));
-            }
+            for (int c = 0; c < 4; ++c)
+                *reinterpret_cast<int4 *>(half + (((4 * (q & 1) + c) ^ (r & 7)) << 4)) =
+                    make_int4(__float2int_rn(__uint_as_float(v[4 * c + 0])),
+                              __float2int_rn(__uint_as_float(v[4 * c + 1])),
+                              __float2int_rn(__uint_as_float(v[4 * c + 2])),
+                              __float2int_rn(__uint_as_float(v[4 * c + 3])));
+            fence_async_smem();  // read by the tensor stores after the next barrier
             return true;
         };
-        bool failed = false;
-        int64_t bh = bh_begin;
+        int bh = bh_begin;
         int r0 = r0_begin;
-        for (int64_t tile = t_begin; tile < t_end; ++tile, ++it, r0 = r0 + TM < L ? r0 + TM : (++bh, 0)) {
+        for (; it < ncta_tiles; ++it, r0 = r0 + TM < L ? r0 + TM : (++bh, 0)) {
             const int row = r0 + r;
             const bool valid = row < L;
-            bool bad = !mbar_wait_warp(&sh.lload, it & 1, abort_flag);
-            const int8_t *lr = LG + (size_t)r * p.ld + 16 * q;
+            const bool lbad = !mbar_wait_warp(&sh.lload, it & 1, abort_flag);
+            const unsigned char *lr = LG + (size_t)r * p.ld + 16 * q;
             uint4 w[NKB];
 #pragma unroll
             for (int kb = 0; kb < NKB; ++kb) {
                 const int k0 = kb * TKB + 16 * q;
                 w[kb] = (valid && k0 < L) ? *reinterpret_cast<const uint4 *>(lr + kb * TKB)
                                           : make_uint4(0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u);
-                if (k0 < L && k0 + 16 > L) {  // keys at or past L: -128 (no effect on the max)
+                if (valid && k0 < L && k0 + 16 > L) {  // keys at or past L: -128 (no effect on the max)
                     const int n = L - k0;
                     uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
 #pragma unroll
@@ -424,10 +446,6 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                     w[kb] = make_uint4(ww[0], ww[1], ww[2], ww[3]);
                 }
             }
-            if (!bad) {
-                fence_async_smem();
-                mbar_arrive(&sh.lfree);  // the staged logits are in registers: the next tile may load
-            }
             // ---- row maximum over the four parts
             // signed 16-bit lanes: the high byte of the larger lane is the larger byte, so lanes of w
             // carry bytes 1 and 3 and lanes of w << 8 bytes 0 and 2
@@ -439,7 +457,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
             }
             int m = max(max(sbyte<1>(mo), sbyte<3>(mo)), max(sbyte<1>(me), sbyte<3>(me)));
             red_max[q * TM + r] = m;
-            if (bad || epi_bad) *stop_flag = 1;
+            if (lbad || epi_bad) *stop_flag = 1;
             soft_bar();
             if (*stop_flag) { failed = true; break; }  // every softmax thread leaves here together
             m = max(max(red_max[r], red_max[TM + r]), max(red_max[2 * TM + r], red_max[3 * TM + r]));
@@ -481,38 +499,99 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                 }
             }
             red_sum[q * TM + r] = S;
+            // the table words of the previous tile are dead: clear this part's words for the histogram
+            if (valid && monotone) {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) OT[(16 * q + i) * TM + r] = 0u;
+            }
             soft_bar();
             S = red_sum[r] + red_sum[TM + r] + red_sum[2 * TM + r] + red_sum[3 * TM + r];
-            // ---- this row's operand table: words q, q + 4, .., q + 60
-            if (valid) {
-                const RowSum rs = make_rowsum(S);
-                auto E_at = [&](int x) -> uint32_t {
-                    return operand_exp(lds32(lut_lane + (uint32_t)((m - x) * (TCOPIES * 4))), rs.hibits, rs.hi, rs.lo);
+            const RowSum rs = make_rowsum(S);
+            // ---- the previous tile's accumulators (its MMAs also release A and B) -> staging
+            bool staged = false;
+            if (prev_bh >= 0) {
+                if (!epilogue(it - 1))
+                    epi_bad = true;
+                else
+                    staged = true;
+            }
+            // ---- this row's thresholds: part q finds delta_k for k = q + 1, q + 5, q + 9, q + 13,
+            //      the four binary searches interleaved
+            if (valid && monotone) {
+                float Dk[4];
+                int lo[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int k = q + 1 + 4 * i;
+                    Dk[i] = k == 1 ? 3.0f : (float)(3 * (1 << (min(k, 15) - 1)) - 1);
+                    lo[i] = 0;
+                }
+                // e(d) D_k <= 2S, exact: one rounding of an exact product minus hi, against lo
+                auto hit = [&](int d, float D) -> bool {
+                    const float ef = __uint2float_rn(lds32(lut_lane + (uint32_t)(d * (TCOPIES * 4))));
+                    return __fmaf_rn(ef, D, -rs.hi) <= rs.lo;
                 };
-#pragma unroll 2
-                for (int i = 0; i < 16; ++i) {
-                    const int j = q + 4 * i;
-                    const int xlo = (int)(int8_t)(uint8_t)(4 * j);  // logits of word j: xlo .. xlo + 3
-                    if (xlo > m) continue;                          // no key of this row reads it
-                    const int hb = min(3, m - xlo);                 // bytes above hb exceed the maximum
-                    const uint32_t E0 = E_at(xlo), Eh = E_at(xlo + hb);
-                    uint32_t word;
-                    if (E0 == Eh && monotone) {
-                        word = (4u * E0) * 0x01010101u;
-                    } else {
-                        const uint32_t E1 = hb > 1 ? E_at(xlo + 1) : Eh;
-                        const uint32_t E2 = hb > 2 ? E_at(xlo + 2) : Eh;
-                        word = 4u * (E0 | (E1 << 8) | (E2 << 16) | (Eh << 24));
-                    }
-                    OT[j * TM + r] = word;
+#pragma unroll
+                for (int step = 128; step >= 1; step >>= 1)
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        if (!hit(lo[i] + step - 1, Dk[i])) lo[i] += step;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int k = q + 1 + 4 * i;
+                    if (lo[i] == 255 && !hit(255, Dk[i])) lo[i] = 256;
+                    if (k <= 15) thr[(k - 1) * TM + r] = lo[i];
                 }
             }
             soft_bar();
-            // ---- the previous tile's accumulators (its MMAs also release A and B)
-            if (prev_bh >= 0 && !epilogue(it - 1, prev_bh, prev_r0)) {
-                epi_bad = true;  // the next tile's first barrier ends the loop for all
-                continue;
+            // ---- staged accumulators leave as two tensor stores
+            if (tid == 0 && staged) {
+                tma_store_acc(&acc_map, LG, 0, prev_r0, prev_bh);
+                tma_store_acc(&acc_map, LG + TM * 128, 32, prev_r0, prev_bh);
+                bulk_commit();
             }
+            // ---- this row's operand table
+            if (valid) {
+                if (monotone) {
+                    // E(x) = 30 - code(x) = 15 + #{k : m - delta_k < x}.  Histogram of the thresholds
+                    // m - delta_k over this part's logits (byte x - xs of the words), counting those
+                    // below xs, then per word the exclusive byte prefix sum.
+                    int n = 0;
+#pragma unroll
+                    for (int k = 0; k < 15; ++k) {
+                        const int t = m - thr[k * TM + r] - xs;
+                        n += t < 0 ? 1 : 0;
+                        if ((unsigned)t < 64u) OT[(16 * q + (t >> 2)) * TM + r] += 1u << (8 * (t & 3));
+                    }
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        uint32_t *wp = &OT[(16 * q + i) * TM + r];
+                        const uint32_t h = *wp;
+                        *wp = 0x3C3C3C3Cu + 4u * ((uint32_t)n * 0x01010101u + (h << 8) * 0x01010101u);
+                        n += (int)((h * 0x01010101u) >> 24);
+                    }
+                } else {
+                    auto E_at = [&](int x) -> uint32_t {
+                        return operand_exp(lds32(lut_lane + (uint32_t)((m - x) * (TCOPIES * 4))), rs.hibits, rs.hi, rs.lo);
+                    };
+#pragma unroll 2
+                    for (int i = 0; i < 16; ++i) {
+                        const int j = q + 4 * i;
+                        const int xlo = (int)(int8_t)(uint8_t)(4 * j);  // logits of word j: xlo .. xlo + 3
+                        if (xlo > m) continue;                          // no key of this row reads it
+                        const int hb = min(3, m - xlo);                 // bytes above hb exceed the maximum
+                        const uint32_t E0 = E_at(xlo);
+                        const uint32_t E1 = hb >= 1 ? E_at(xlo + 1) : E0;
+                        const uint32_t E2 = hb >= 2 ? E_at(xlo + 2) : E1;
+                        const uint32_t E3 = hb >= 3 ? E_at(xlo + 3) : E2;
+                        OT[j * TM + r] = 4u * (E0 | (E1 << 8) | (E2 << 16) | (E3 << 24));
+                    }
+                }
+            }
+            if (tid == 0) bulk_wait_read();  // the staging tile is read out before the next logits land
+            soft_bar();
+            mbar_arrive(&sh.lfree);  // the logits tile and its scratch are free: the next tile may load
+            if (epi_bad) continue;   // the next tile's first barrier ends the loop for all
             // ---- V of a new head -> fp16 B
             if (bh != conv_bh) {
 #pragma unroll
@@ -543,10 +622,10 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                         const uint32_t v = ww[b];
                         // word (byte >> 2) of this row, then byte (byte & 3) of it into the high byte
                         // of each fp16 half; the low bytes copy the sign of a table byte (zero)
-                        const uint32_t t0 = lds32(ot_base + (((v << 7) & 0x7E00u) | r4));
-                        const uint32_t t1 = lds32(ot_base + (((v >> 1) & 0x7E00u) | r4));
-                        const uint32_t t2 = lds32(ot_base + (((v >> 9) & 0x7E00u) | r4));
-                        const uint32_t t3 = lds32(ot_base + (((v >> 17) & 0x7E00u) | r4));
+                        const uint32_t t0 = *reinterpret_cast<const uint32_t *>(otb + (((v << 7) & 0x7E00u) | r4));
+                        const uint32_t t1 = *reinterpret_cast<const uint32_t *>(otb + (((v >> 1) & 0x7E00u) | r4));
+                        const uint32_t t2 = *reinterpret_cast<const uint32_t *>(otb + (((v >> 9) & 0x7E00u) | r4));
+                        const uint32_t t3 = *reinterpret_cast<const uint32_t *>(otb + (((v >> 17) & 0x7E00u) | r4));
                         o[2 * b] = prmt(t0, t1, ((v << 4) & 0x3030u) | 0x4808u);
                         o[2 * b + 1] = prmt(t2, t3, ((v >> 12) & 0x3030u) | 0x4808u);
                     }
@@ -571,21 +650,30 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
             prev_bh = bh;
             prev_r0 = r0;
         }
-        if (!failed && !*abort_flag && prev_bh >= 0) epilogue(it - 1, prev_bh, prev_r0);
+        // the last tile's accumulators (the copy warp loads nothing more: LG is free)
+        bool staged = false;
+        if (!failed && prev_bh >= 0) staged = epilogue(it - 1);
+        soft_bar();  // reached by every softmax thread
+        if (tid == 0 && staged) {
+            tma_store_acc(&acc_map, LG, 0, prev_r0, prev_bh);
+            tma_store_acc(&acc_map, LG + TM * 128, 32, prev_r0, prev_bh);
+            bulk_commit();
+        }
+        if (tid == 0) bulk_wait_all();  // every accumulator this CTA stored has landed
     } else if (warp == TLOAD_WARP && lane == 0) {
-        // ---------------- logits tiles (each as soon as the previous one is in registers)
-        int it = 0, lloads = 0;
-        int64_t bh = bh_begin;
+        // ---------------- logits tiles (each once the previous tile's table is built), L2 prefetch
+        int bh = bh_begin;
         int r0 = r0_begin;
-        for (int64_t tile = t_begin; tile < t_end; ++tile, ++it, r0 = r0 + TM < L ? r0 + TM : (++bh, 0)) {
+        int lloads = 0;
+        prefetch_l2(p.v + (size_t)bh * L * TD, (uint32_t)(L * TD));
+        for (int it = 0; it < ncta_tiles; ++it, r0 = r0 + TM < L ? r0 + TM : (++bh, 0)) {
             if (it > 0 && !mbar_wait(&sh.lfree, (it - 1) & 1, abort_flag)) break;
             const uint32_t bl = (uint32_t)(min(TM, L - r0) * p.ld);
             mbar_expect_tx(&sh.lload, bl);
             bulk_g2s(LG, p.logits + ((size_t)bh * L + r0) * p.ld, bl, &sh.lload);
             ++lloads;
-            if (it == 0) prefetch_l2(p.v + (size_t)bh * L * TD, (uint32_t)(L * TD));
-            if (tile + 1 < t_end) {
-                const int64_t bhn = r0 + TM < L ? bh : bh + 1;
+            if (it + 1 < ncta_tiles) {
+                const int bhn = r0 + TM < L ? bh : bh + 1;
                 const int r0n = r0 + TM < L ? r0 + TM : 0;
                 prefetch_l2(p.logits + ((size_t)bhn * L + r0n) * p.ld, (uint32_t)(min(TM, L - r0n) * p.ld));
                 if (bhn != bh) prefetch_l2(p.v + (size_t)bhn * L * TD, (uint32_t)(L * TD));
@@ -594,9 +682,8 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
         if (lloads > 0) mbar_wait(&sh.lload, (lloads - 1) & 1, abort_flag, false);
     } else if (warp == TPRODUCER_WARP && lane == 0) {
         // ---------------- MMA issue: the whole tile once its operands are in place
-        int it = 0;
         const int nkb = (L + TKB - 1) / TKB;
-        for (int64_t tile = t_begin; tile < t_end; ++tile, ++it) {
+        for (int it = 0; it < ncta_tiles; ++it) {
             if (!mbar_wait(&sh.afull, it & 1, abort_flag)) break;
             tc_fence_after();
             const uint32_t b0 = sa(Bs);
@@ -620,17 +707,46 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
 size_t tc_smem_bytes(int L, int64_t ld)
 {
     const int nkb = (L + TKB - 1) / TKB;
-    return 1024 + (size_t)nkb * B_SLOT + (size_t)64 * TM * 4 + (size_t)256 * TCOPIES * 4 +
-           (size_t)TPARTS * TM * (4 + 8) + (size_t)TM * ld;
+    const size_t lg = (size_t)TM * ld > (size_t)SCR_BYTES ? (size_t)TM * ld : (size_t)SCR_BYTES;
+    return 1024 + (size_t)nkb * B_SLOT + (size_t)256 * TCOPIES * 4 + (size_t)TPARTS * TM * (4 + 8) + lg;
+}
+
+// static shared memory of the kernel: the operand table and the control block
+constexpr size_t kTcStaticSmem = (size_t)64 * TM * 4 + 256;
+
+// The accumulators as a 3-d tensor [BH][L][64] of int32 for the tensor stores: boxes of
+// 32 columns x 128 rows x 1 head in the 128-byte swizzle; rows past L are clipped.
+cudaError_t make_acc_map(CUtensorMap *map, int32_t *acc, int64_t BH, int L)
+{
+    using EncodeFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+    static EncodeFn encode = nullptr;
+    if (!encode) {
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+        if (e != cudaSuccess) return e;
+        if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+        encode = reinterpret_cast<EncodeFn>(fn);
+    }
+    const cuuint64_t dims[3] = {(cuuint64_t)TD, (cuuint64_t)L, (cuuint64_t)BH};
+    const cuuint64_t strides[2] = {(cuuint64_t)TD * 4, (cuuint64_t)L * TD * 4};
+    const cuuint32_t box[3] = {32, TM, 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_INT32, 3, acc, dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
 template <int NKB>
-cudaError_t tc_launch(const TcParams &p, size_t smem, int grid, cudaStream_t st)
+cudaError_t tc_launch(const TcParams &p, const CUtensorMap &map, size_t smem, int grid, cudaStream_t st)
 {
     cudaError_t e = cudaFuncSetAttribute(lis_attn_tc_kernel<NKB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
-    lis_attn_tc_kernel<NKB><<<grid, TTHREADS, smem, st>>>(p);
+    lis_attn_tc_kernel<NKB><<<grid, TTHREADS, smem, st>>>(p, map);
     return cudaGetLastError();
 }
 
@@ -638,28 +754,32 @@ cudaError_t tc_launch(const TcParams &p, size_t smem, int grid, cudaStream_t st)
 
 bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
 {
-    return b.d == TD && a.bias == nullptr && a.codes == nullptr && b.zp_v == 0 && a.ld_logit <= TMAXLD &&
+    return b.d == TD && a.bias == nullptr && a.codes == nullptr && b.zp_v == 0 && a.L <= TMAXKB * TKB &&
            a.ld_logit % 16 == 0 && b.ld_v == TD && b.ld_acc == TD && ((uintptr_t)a.logits % 16) == 0 &&
-           ((uintptr_t)b.v % 16) == 0 && ((uintptr_t)b.acc % 16) == 0 && tc_smem_bytes(a.L, a.ld_logit) <= 232448;
+           ((uintptr_t)b.v % 16) == 0 && ((uintptr_t)b.acc % 16) == 0 &&
+           tc_smem_bytes(a.L, a.ld_logit) + kTcStaticSmem <= 232448;
 }
 
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
 {
     TcParams p{a.logits, a.ld_logit, a.s_logit, b.v, b.acc, b.BH, a.L};
+    CUtensorMap map;
+    cudaError_t e = make_acc_map(&map, b.acc, b.BH, a.L);
+    if (e != cudaSuccess) return e;
     const size_t smem = tc_smem_bytes(a.L, a.ld_logit);
     const int64_t ntiles = b.BH * ((a.L + TM - 1) / TM);
     const int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());
     switch ((a.L + TKB - 1) / TKB) {
-    case 1: return tc_launch<1>(p, smem, grid, st);
-    case 2: return tc_launch<2>(p, smem, grid, st);
-    case 3: return tc_launch<3>(p, smem, grid, st);
-    case 4: return tc_launch<4>(p, smem, grid, st);
-    case 5: return tc_launch<5>(p, smem, grid, st);
-    case 6: return tc_launch<6>(p, smem, grid, st);
-    case 7: return tc_launch<7>(p, smem, grid, st);
-    case 8: return tc_launch<8>(p, smem, grid, st);
-    case 9: return tc_launch<9>(p, smem, grid, st);
-    default: return tc_launch<10>(p, smem, grid, st);
+    case 1: return tc_launch<1>(p, map, smem, grid, st);
+    case 2: return tc_launch<2>(p, map, smem, grid, st);
+    case 3: return tc_launch<3>(p, map, smem, grid, st);
+    case 4: return tc_launch<4>(p, map, smem, grid, st);
+    case 5: return tc_launch<5>(p, map, smem, grid, st);
+    case 6: return tc_launch<6>(p, map, smem, grid, st);
+    case 7: return tc_launch<7>(p, map, smem, grid, st);
+    case 8: return tc_launch<8>(p, map, smem, grid, st);
+    case 9: return tc_launch<9>(p, map, smem, grid, st);
+    default: return tc_launch<10>(p, map, smem, grid, st);
     }
 }
 
