@@ -260,11 +260,11 @@ __device__ __forceinline__ int sbyte(uint32_t w)
     return (int)y;
 }
 
-// i-exp value of byte J of w: table entry m - q of this lane's replica
+// i-exp value of byte J of w: table entry m - q of this lane's replica (lutq points at entry m)
 template <int J>
-__device__ __forceinline__ uint32_t iexp_at(uint32_t lutq, uint32_t w)
+__device__ __forceinline__ uint32_t iexp_at(const uint32_t *lutq, uint32_t w)
 {
-    return lds32(lutq - (uint32_t)(TCOPIES * 4) * (uint32_t)sbyte<J>(w));
+    return lutq[-TCOPIES * sbyte<J>(w)];
 }
 
 // warp-collective (.sync.aligned): the whole warp, converged, writes its 32 lanes
@@ -462,7 +462,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, co
             if (*stop_flag) { failed = true; break; }  // every softmax thread leaves here together
             m = max(max(red_max[r], red_max[TM + r]), max(red_max[2 * TM + r], red_max[3 * TM + r]));
             // ---- i-exp row sum over the four parts
-            const uint32_t lutq = lut_lane + (uint32_t)(m * TCOPIES * 4);
+            const uint32_t *lutq = LUT + lane + m * TCOPIES;
             unsigned long long S = 0;
             if (valid) {
 #pragma unroll
