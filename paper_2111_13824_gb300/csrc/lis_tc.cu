@@ -32,6 +32,7 @@
 #include "fqvit_internal.cuh"
 #include "lis_common.cuh"
 
+#include <cmath>
 #include <cuda.h>
 #include <cuda_fp16.h>
 
@@ -332,7 +333,9 @@ __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wa
 //               (B, MN-major) whenever the head changes.
 //   MMA thread: after all operands of the tile are written, 4 MMAs per key block, one commit
 // Each CTA takes a contiguous range of tiles, so that consecutive tiles share a head.
-template <int NKB>
+// SMALL_E: every i-exp value is below 2^28 (decided on the host from the scale), so 16 of them
+// sum exactly in 32 bits
+template <int NKB, bool SMALL_E>
 __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, const __grid_constant__ CUtensorMap acc_map)
 {
     extern __shared__ unsigned char dsm_raw[];
@@ -393,9 +396,14 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, co
         const uint32_t r4 = 4u * (uint32_t)r;
         const unsigned char *otb = reinterpret_cast<const unsigned char *>(OT);
         const uint32_t tlane = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-        const bool small_e = LUT[0] < (1u << 28);    // e(0) is the largest i-exp value
         const bool monotone = !sh.rising;            // codes never fall as d grows
         const int xs = (int)(int8_t)(uint8_t)(64 * q);  // part q's table words 16 q .. +15: logits xs .. xs + 63
+        int npad = 0;  // keys at or past L inside this part's last partial block (summed as -128, then removed)
+#pragma unroll
+        for (int kb = 0; kb < NKB; ++kb) {
+            const int k0 = kb * TKB + 16 * q;
+            if (k0 < L && k0 + 16 > L) npad = k0 + 16 - L;
+        }
         int it = 0;
         bool epi_bad = false, failed = false;
         int prev_bh = -1, conv_bh = -1;
@@ -467,10 +475,9 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, co
             if (valid) {
 #pragma unroll
                 for (int kb = 0; kb < NKB; ++kb) {
-                    const int k0 = kb * TKB + 16 * q;
-                    const uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
-                    if (k0 + 16 <= L) {
-                        if (small_e) {  // 16 values below 2^28: a 32-bit partial sum is exact
+                    if (kb * TKB + 16 * q < L) {
+                        const uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
+                        if (SMALL_E) {  // 16 values below 2^28: a 32-bit partial sum is exact
                             uint32_t a = 0;
 #pragma unroll
                             for (int b = 0; b < 4; ++b) {
@@ -486,17 +493,9 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, co
                                 S += (unsigned long long)(e0 + e1) + (unsigned long long)(e2 + e3);  // e < 2^31
                             }
                         }
-                    } else if (k0 < L) {
-                        const int n = L - k0;
-#pragma unroll
-                        for (int b = 0; b < 4; ++b) {
-                            if (4 * b + 0 < n) S += iexp_at<0>(lutq, ww[b]);
-                            if (4 * b + 1 < n) S += iexp_at<1>(lutq, ww[b]);
-                            if (4 * b + 2 < n) S += iexp_at<2>(lutq, ww[b]);
-                            if (4 * b + 3 < n) S += iexp_at<3>(lutq, ww[b]);
-                        }
                     }
                 }
+                S -= (unsigned long long)npad * lutq[128 * TCOPIES];  // the padding bytes, -128 each
             }
             red_sum[q * TM + r] = S;
             // the table words of the previous tile are dead: clear this part's words for the histogram
@@ -740,14 +739,31 @@ cudaError_t make_acc_map(CUtensorMap *map, int32_t *acc, int64_t BH, int L)
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-template <int NKB>
+template <int NKB, bool SMALL_E>
 cudaError_t tc_launch(const TcParams &p, const CUtensorMap &map, size_t smem, int grid, cudaStream_t st)
 {
-    cudaError_t e = cudaFuncSetAttribute(lis_attn_tc_kernel<NKB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(lis_attn_tc_kernel<NKB, SMALL_E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
-    lis_attn_tc_kernel<NKB><<<grid, TTHREADS, smem, st>>>(p, map);
+    lis_attn_tc_kernel<NKB, SMALL_E><<<grid, TTHREADS, smem, st>>>(p, map);
     return cudaGetLastError();
+}
+
+template <int NKB>
+cudaError_t tc_launch_e(bool small_e, const TcParams &p, const CUtensorMap &map, size_t smem, int grid, cudaStream_t st)
+{
+    return small_e ? tc_launch<NKB, true>(p, map, smem, grid, st) : tc_launch<NKB, false>(p, map, smem, grid, st);
+}
+
+// Whether every i-exp value of the scale is below 2^28: the largest is e(0) = (q_b^2 + q_c) 2^15,
+// with the constants of Algorithm 1 computed exactly as the kernels do (fp64, one rounding per
+// operation), so host and device agree.
+bool small_iexp(float s)
+{
+    const double sd = (double)s;
+    const double qb = floor(1.353 / sd);
+    const double qc = floor(0.344 / (0.3585 * (sd * sd)));
+    return (qb * qb + qc) * 32768.0 < 268435456.0;
 }
 
 }  // namespace
@@ -769,17 +785,18 @@ cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaSt
     const size_t smem = tc_smem_bytes(a.L, a.ld_logit);
     const int64_t ntiles = b.BH * ((a.L + TM - 1) / TM);
     const int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());
+    const bool se = small_iexp(a.s_logit);
     switch ((a.L + TKB - 1) / TKB) {
-    case 1: return tc_launch<1>(p, map, smem, grid, st);
-    case 2: return tc_launch<2>(p, map, smem, grid, st);
-    case 3: return tc_launch<3>(p, map, smem, grid, st);
-    case 4: return tc_launch<4>(p, map, smem, grid, st);
-    case 5: return tc_launch<5>(p, map, smem, grid, st);
-    case 6: return tc_launch<6>(p, map, smem, grid, st);
-    case 7: return tc_launch<7>(p, map, smem, grid, st);
-    case 8: return tc_launch<8>(p, map, smem, grid, st);
-    case 9: return tc_launch<9>(p, map, smem, grid, st);
-    default: return tc_launch<10>(p, map, smem, grid, st);
+    case 1: return tc_launch_e<1>(se, p, map, smem, grid, st);
+    case 2: return tc_launch_e<2>(se, p, map, smem, grid, st);
+    case 3: return tc_launch_e<3>(se, p, map, smem, grid, st);
+    case 4: return tc_launch_e<4>(se, p, map, smem, grid, st);
+    case 5: return tc_launch_e<5>(se, p, map, smem, grid, st);
+    case 6: return tc_launch_e<6>(se, p, map, smem, grid, st);
+    case 7: return tc_launch_e<7>(se, p, map, smem, grid, st);
+    case 8: return tc_launch_e<8>(se, p, map, smem, grid, st);
+    case 9: return tc_launch_e<9>(se, p, map, smem, grid, st);
+    default: return tc_launch_e<10>(se, p, map, smem, grid, st);
     }
 }
 
