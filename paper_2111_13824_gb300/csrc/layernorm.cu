@@ -204,35 +204,53 @@ __global__ void __launch_bounds__(kWarps * 32)
             if (a.m1) a.m1[row] = M1;
             if (a.m2) a.m2[row] = M2;
         }
-        const bool fast = ln_row_fast(sh, r, t);
+        const bool fast = ln_row_fast(sh, r, t);  // warp-uniform: one evaluation per row, chosen outside the loops
         uint4 *dst = reinterpret_cast<uint4 *>(a.yq + row * a.ld_out);
         // pass 2: requantization
+        if (fast) {
 #pragma unroll
-        for (int i = 0; i < CPL; ++i) {
-            int ch = lane + 32 * i;
-            if (ch < nch) {
-                uint4 al4 = *reinterpret_cast<const uint4 *>(al_s + ch * 16);
-                uint32_t w[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
-                uint32_t aw[4] = {al4.x, al4.y, al4.z, al4.w};
-                uint32_t o[4] = {0, 0, 0, 0};
-                const float4 *g4 = reinterpret_cast<const float4 *>(gs_s + ch * 16);
-                const float4 *b4 = reinterpret_cast<const float4 *>(bs_s + ch * 16);
+            for (int i = 0; i < CPL; ++i) {
+                int ch = lane + 32 * i;
+                if (ch < nch) {
+                    uint4 al4 = *reinterpret_cast<const uint4 *>(al_s + ch * 16);
+                    uint32_t w[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+                    uint32_t aw[4] = {al4.x, al4.y, al4.z, al4.w};
+                    uint32_t o[4] = {0, 0, 0, 0};
+                    const float4 *g4 = reinterpret_cast<const float4 *>(gs_s + ch * 16);
+                    const float4 *b4 = reinterpret_cast<const float4 *>(bs_s + ch * 16);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    float4 g = g4[q], b = b4[q];
-                    float gg[4] = {g.x, g.y, g.z, g.w};
-                    float bb[4] = {b.x, b.y, b.z, b.w};
+                    for (int q = 0; q < 4; ++q) {
+                        float4 g = g4[q], b = b4[q];
+                        float gg[4] = {g.x, g.y, g.z, g.w};
+                        float bb[4] = {b.x, b.y, b.z, b.w};
 #pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        int x = (w[q] >> (8 * k)) & 0xFF;
-                        int al = (aw[q] >> (8 * k)) & 0xFF;
-                        int xh = (x - a.zp_in) << al;
-                        uint32_t y = fast ? ln_fast(gg[k], bb[k], r, t, xh, zh)
-                                          : (uint32_t)ln_exact(gg[k], bb[k], r, t, xh, a.zp_out);
-                        o[q] |= y << (8 * k);
+                        for (int k = 0; k < 4; ++k) {
+                            int x = (w[q] >> (8 * k)) & 0xFF;
+                            int al = (aw[q] >> (8 * k)) & 0xFF;
+                            int xh = (x - a.zp_in) << al;
+                            o[q] |= ln_fast(gg[k], bb[k], r, t, xh, zh) << (8 * k);
+                        }
                     }
+                    __stcs(dst + ch, make_uint4(o[0], o[1], o[2], o[3]));
                 }
-                __stcs(dst + ch, make_uint4(o[0], o[1], o[2], o[3]));
+            }
+        } else {
+#pragma unroll
+            for (int i = 0; i < CPL; ++i) {
+                int ch = lane + 32 * i;
+                if (ch < nch) {
+                    uint32_t o0 = 0, o1 = 0, o2 = 0, o3 = 0;
+#pragma unroll 1
+                    for (int k = 0; k < 16; ++k) {
+                        const int c = ch * 16 + k;
+                        const uint32_t wk = k < 8 ? (k < 4 ? v[i].x : v[i].y) : (k < 12 ? v[i].z : v[i].w);
+                        int x = (wk >> (8 * (k & 3))) & 0xFF;
+                        int xh = (x - a.zp_in) << al_s[c];
+                        const uint32_t y = (uint32_t)ln_exact(gs_s[c], bs_s[c], r, t, xh, a.zp_out) << (8 * (k & 3));
+                        if (k < 4) o0 |= y; else if (k < 8) o1 |= y; else if (k < 12) o2 |= y; else o3 |= y;
+                    }
+                    __stcs(dst + ch, make_uint4(o0, o1, o2, o3));
+                }
             }
         }
     }
