@@ -154,14 +154,27 @@ __global__ void __launch_bounds__(kWarps * 32)
     const float zh = (float)a.zp_out + 0.5f;
     const float Cf = (float)a.C;
 
-    for (int64_t row = (int64_t)blockIdx.x * kWarps + warp; row < a.rows;
-         row += (int64_t)gridDim.x * kWarps) {
-        const uint4 *src = reinterpret_cast<const uint4 *>(a.xq + row * a.ld_in);
+    const int64_t rstep = (int64_t)gridDim.x * kWarps;
+    int64_t row = (int64_t)blockIdx.x * kWarps + warp;
+    // the row's 16-byte chunks, loaded one row ahead so that the HBM latency overlaps the work
+    uint4 nv[CPL];
+#pragma unroll
+    for (int i = 0; i < CPL; ++i) {
+        int ch = lane + 32 * i;
+        nv[i] = (row < a.rows && ch < nch) ? __ldcs(reinterpret_cast<const uint4 *>(a.xq + row * a.ld_in) + ch)
+                                           : make_uint4(0, 0, 0, 0);
+    }
+    for (; row < a.rows; row += rstep) {
         uint4 v[CPL];
 #pragma unroll
-        for (int i = 0; i < CPL; ++i) {
-            int ch = lane + 32 * i;
-            v[i] = ch < nch ? __ldcs(src + ch) : make_uint4(0, 0, 0, 0);
+        for (int i = 0; i < CPL; ++i) v[i] = nv[i];
+        if (row + rstep < a.rows) {
+            const uint4 *nsrc = reinterpret_cast<const uint4 *>(a.xq + (row + rstep) * a.ld_in);
+#pragma unroll
+            for (int i = 0; i < CPL; ++i) {
+                int ch = lane + 32 * i;
+                if (ch < nch) nv[i] = __ldcs(nsrc + ch);
+            }
         }
         // pass 1: integer statistics
         int m1 = 0;
@@ -305,10 +318,19 @@ cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st)
 {
     size_t smem = (size_t)a.C * (2 * sizeof(float) + 1);
     smem = (smem + 15) & ~(size_t)15;
-    int nsm = sm_count();
-    int64_t want = (a.rows + kWarps - 1) / kWarps;
-    int64_t cap = (int64_t)nsm * 8;
-    int blocks = (int)(want < cap ? want : cap);
+    const int nsm = sm_count();
+    const int64_t want = (a.rows + kWarps - 1) / kWarps;
+    // Every block first derives the per-channel constants (three correctly rounded divisions per
+    // channel), so the grid is the number of blocks that are resident at once: each block then
+    // walks many rows.
+    auto blocks_for = [&](const void *fn) -> int {
+        int per_sm = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kWarps * 32, smem) != cudaSuccess ||
+            per_sm < 1)
+            per_sm = 1;
+        const int64_t cap = (int64_t)nsm * per_sm;
+        return (int)(want < cap ? want : cap);
+    };
     bool vec = (a.C % 16 == 0) && (a.ld_in % 16 == 0) && (a.ld_out % 16 == 0) &&
                ((uintptr_t)a.xq % 16 == 0) && ((uintptr_t)a.yq % 16 == 0) && a.C <= 4096;
     if (vec) {
@@ -318,7 +340,7 @@ cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st)
     case N:                                                                                \
         cudaFuncSetAttribute(ln_vec_kernel<N>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
                              (int)smem);                                                   \
-        ln_vec_kernel<N><<<blocks, kWarps * 32, smem, st>>>(a);                            \
+        ln_vec_kernel<N><<<blocks_for((const void *)ln_vec_kernel<N>), kWarps * 32, smem, st>>>(a); \
         return cudaGetLastError();
             FQ_LN_CASE(1)
             FQ_LN_CASE(2)
@@ -334,7 +356,7 @@ cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st)
         }
     }
     cudaFuncSetAttribute(ln_generic_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    ln_generic_kernel<<<blocks, kWarps * 32, smem, st>>>(a);
+    ln_generic_kernel<<<blocks_for((const void *)ln_generic_kernel), kWarps * 32, smem, st>>>(a);
     return cudaGetLastError();
 }
 
