@@ -19,13 +19,13 @@
 //     4-bit code is written, as the fp16 operand 2^(15-code) looked up in that
 //     table, straight into tensor memory (the A operand: row = lane, K-major
 //     pairs per column).  The same threads convert a head's V rows to fp16
-//     (128B-swizzled, MN-major shared-memory tile, the B operand) and, one
-//     tile later, read the accumulators back from tensor memory.
-//   warp 16, lane 0: issues the tile's MMAs (four per key block) once every
-//     operand is written, and commits them to an mbarrier.
-//   warp 17, lane 0: bulk asynchronous copy of the next tile's logits into
-//     shared memory as soon as the current tile is in registers, plus L2
-//     prefetches of what follows.
+//     (128B-swizzled, MN-major shared-memory tile, the B operand).
+//   warps 16-19 (one per tensor-memory lane quarter): read each tile's
+//     accumulators out of tensor memory as soon as its MMAs complete and store
+//     the int32 rows (32-byte stores) while the softmax warps work on the next
+//     tile; warp 16, lane 0 also issues the tile's MMAs (four per key block)
+//     once every operand is written, warp 17, lane 0 the bulk copy of the next
+//     tile's logits into shared memory, plus L2 prefetches.
 // Every wait is bounded: after two seconds the kernel records a timeout
 // status, drains what it issued and returns (the host reads the status with
 // fqvit_sync_status).
@@ -33,7 +33,6 @@
 #include "lis_common.cuh"
 
 #include <cmath>
-#include <cuda.h>
 #include <cuda_fp16.h>
 
 namespace fqvit {
@@ -151,15 +150,6 @@ __device__ __forceinline__ void mma_commit(uint64_t *b)
                  : "memory");
 }
 
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16])
-{
-    __syncwarp();
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr));
-}
 
 // int8 x 2 (bytes b0, b1 of w ^ 0x80808080) -> half2 exact
 __device__ __forceinline__ uint32_t i8x2_to_h2(uint32_t xw, uint32_t sel)
@@ -172,17 +162,14 @@ __device__ __forceinline__ uint32_t i8x2_to_h2(uint32_t xw, uint32_t sel)
 
 constexpr int TPARTS = 4;                         // threads per query row
 constexpr int TSOFT = TM * TPARTS;                // softmax threads (16 warps)
-constexpr int TPRODUCER_WARP = TSOFT / 32;        // warp 16: MMA issue
-constexpr int TLOAD_WARP = TPRODUCER_WARP + 1;    // warp 17: bulk copies of the logits, L2 prefetch
-constexpr int TTHREADS = (TLOAD_WARP + 1) * 32;
+constexpr int TEPI_WARP = TSOFT / 32;             // warps 16..19: accumulator read-out, one per lane quarter
+constexpr int TMMA_WARP = TEPI_WARP;              //   warp 16 lane 0 also issues the MMAs
+constexpr int TCOPY_WARP = TEPI_WARP + 1;         //   warp 17 lane 0 also copies the logits tiles
+constexpr int TTHREADS = TSOFT + 128;
 constexpr int TMAXKB = 10;                        // key blocks of the longest row (L <= 640)
 constexpr int TA_COL = TD;                        // D: columns 0..63; A of key block kb: 64 + 32 kb ..
-// The logits tile doubles as scratch between the row sums and the table: accumulator staging
-// (two 128-row x 128-byte halves in the 128-byte swizzle of the output tensor map) and the
-// row thresholds.
-constexpr int SCR_STAGE = 2 * TM * 128;           // 32 KB
-constexpr int SCR_THR = SCR_STAGE;                // int32 [16][TM]
-constexpr int SCR_BYTES = SCR_THR + 16 * TM * 4;  // 40 KB
+constexpr int SCR_THR = 0;                        // the logits tile doubles as threshold scratch: int32 [16][TM]
+constexpr int SCR_BYTES = 16 * TM * 4;
 
 // tensor-memory columns for NKB key blocks (a power of two >= 32)
 __host__ __device__ constexpr int tmem_cols(int nkb)
@@ -197,6 +184,7 @@ struct TcShared {
     int abort_flag;
     int rising;  // some i-exp value exceeds the one before it (floored constants)
     int stop;    // set (never cleared) by a softmax thread whose wait gave up
+    int ew_stop; // the same for the read-out warps
 };
 
 // fp16 exponent field (30 - code) of the operand 2^(15-code) for an i-exp
@@ -298,45 +286,61 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t *b, uint32_t bytes)
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(sa(b)), "r"(bytes) : "memory");
 }
 
-// tensor store of one 128-row x 32-column half tile of accumulators (rows past L are clipped
-// by the tensor map), in a bulk group
-__device__ __forceinline__ void tma_store_acc(const CUtensorMap *map, const void *ssrc, int col, int row, int head)
+// 32 bytes of int32 to global memory (32-byte aligned)
+__device__ __forceinline__ void stg256(int32_t *p, const int (&v)[8])
 {
-    asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
-                     reinterpret_cast<uint64_t>(map)),
-                 "r"(col), "r"(row), "r"(head), "r"(sa(ssrc))
+    asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(v[0]), "r"(v[1]), "r"(v[2]),
+                 "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
                  : "memory");
 }
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32])
+{
+    __syncwarp();
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+}
+
+// Named barrier 2 over the 128 read-out threads
+__device__ __forceinline__ void epi_bar()
+{
+    __syncwarp();
+    asm volatile("bar.sync 2, 128;" ::: "memory");
+}
 
 // Per tile (128 query rows of one head):
-//   copy warp:  logits tile -> shared memory (bulk copy) once the previous tile's table is built,
-//               L2 prefetch of the next tile (and of the next head's V)
+//   copy (warp 17, lane 0): logits tile -> shared memory (bulk copy) once the previous tile's
+//               table is built, L2 prefetch of the tile after it (and of the next head's V)
 //   softmax:    thread (row r, part q) takes keys 64 kb + 16 q .. +15 of every key block into
 //               registers; the row maximum and the i-exp row sum are combined over the four parts
-//               through shared memory.  Then the previous tile's accumulators come back from
-//               tensor memory into a staging tile (128-byte swizzle) and leave as two tensor
-//               stores.  The row's operands go into a table indexed by the raw logit byte: word j
-//               of row r (OT[j][r], so that the 32 rows of a warp sit in 32 different banks)
-//               holds, in byte b, 4 (30 - code) for the logit byte 4 j + b.  Codes only depend on
-//               the row maximum, the row sum and the logit, so one table serves the whole row.
-//               Where the i-exp values never rise with the distance d to the maximum,
-//               code(d) = #{k <= 15 : d >= delta_k} for the row's thresholds delta_k (the first d
-//               with e(d) D_k <= 2S): the four parts find them by binary search, histogram them
-//               into the table words and turn each word into its codes with a byte prefix sum
-//               (a multiply by 0x01010101); the floored constants of a few scales break the
-//               monotony, and those evaluate every entry.  Every logit then costs one table
-//               load; two loads and one byte permute give the fp16 pair 2^(15-code) that goes to
-//               tensor memory (A, K-major rows = lanes).  V of a head -> fp16 in shared memory
-//               (B, MN-major) whenever the head changes.
-//   MMA thread: after all operands of the tile are written, 4 MMAs per key block, one commit
+//               through shared memory.  The row's operands go into a table indexed by the raw
+//               logit byte: word j of row r (OT[j][r], so that the 32 rows of a warp sit in 32
+//               different banks) holds, in byte b, 4 (30 - code) for the logit byte 4 j + b.
+//               Codes only depend on the row maximum, the row sum and the logit, so one table
+//               serves the whole row.  Where the i-exp values never rise with the distance d to
+//               the maximum, code(d) = #{k <= 15 : d >= delta_k} for the row's thresholds delta_k
+//               (the first d with e(d) D_k <= 2S): the four parts find them by binary search,
+//               histogram them into the table words and turn each word into its codes with a
+//               byte prefix sum (a multiply by 0x01010101); the floored constants of a few scales
+//               break the monotony, and those evaluate every entry.  Every logit then costs one
+//               table load; two loads and one byte permute give the fp16 pair 2^(15-code) that
+//               goes to tensor memory (A, K-major rows = lanes) once the previous tile's MMAs are
+//               done.  V of a head -> fp16 in shared memory (B, MN-major) whenever the head
+//               changes.
+//   MMA (warp 16, lane 0): after all operands of the tile are written, 4 MMAs per key block,
+//               one commit
+//   read-out (warps 16-19): the tile's accumulators, while the softmax warps work on the next
 // Each CTA takes a contiguous range of tiles, so that consecutive tiles share a head.
 // SMALL_E: every i-exp value is below 2^28 (decided on the host from the scale), so 16 of them
 // sum exactly in 32 bits
 template <int NKB, bool SMALL_E>
-__global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, const __grid_constant__ CUtensorMap acc_map)
+__global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
 {
     extern __shared__ unsigned char dsm_raw[];
     __shared__ TcShared sh;
@@ -361,9 +365,10 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, co
         sh.abort_flag = 0;
         sh.rising = 0;
         sh.stop = 0;
+        sh.ew_stop = 0;
         sh.c = iexp_consts(p.s);
     }
-    if (warp == TPRODUCER_WARP) {
+    if (warp == TMMA_WARP) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(&sh.tmem)),
                      "r"(tmem_cols(NKB)));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
@@ -405,27 +410,8 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, co
             if (k0 < L && k0 + 16 > L) npad = k0 + 16 - L;
         }
         int it = 0;
-        bool epi_bad = false, failed = false;
-        int prev_bh = -1, conv_bh = -1;
-        int prev_r0 = 0;
-        // accumulators of tile tit into the staging halves: warp w, rows 32 (w % 4) .., columns 16 (w / 4) ..
-        auto epilogue = [&](int tit) -> bool {
-            if (!mbar_wait_warp(&sh.mmadone, tit & 1, abort_flag)) return false;
-            tc_fence_after();
-            uint32_t v[16];
-            tmem_ld16(tlane + 16 * (warp >> 2), v);
-            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-            unsigned char *half = LG + (q >> 1) * (TM * 128) + r * 128;
-#pragma unroll
-            for (int c = 0; c < 4; ++c)
-                *reinterpret_cast<int4 *>(half + (((4 * (q & 1) + c) ^ (r & 7)) << 4)) =
-                    make_int4(__float2int_rn(__uint_as_float(v[4 * c + 0])),
-                              __float2int_rn(__uint_as_float(v[4 * c + 1])),
-                              __float2int_rn(__uint_as_float(v[4 * c + 2])),
-                              __float2int_rn(__uint_as_float(v[4 * c + 3])));
-            fence_async_smem();  // read by the tensor stores after the next barrier
-            return true;
-        };
+        bool wait_bad = false;
+        int conv_bh = -1;
         int bh = bh_begin;
         int r0 = r0_begin;
         for (; it < ncta_tiles; ++it, r0 = r0 + TM < L ? r0 + TM : (++bh, 0)) {
@@ -465,9 +451,9 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, co
             }
             int m = max(max(sbyte<1>(mo), sbyte<3>(mo)), max(sbyte<1>(me), sbyte<3>(me)));
             red_max[q * TM + r] = m;
-            if (lbad || epi_bad) *stop_flag = 1;
+            if (lbad || wait_bad) *stop_flag = 1;
             soft_bar();
-            if (*stop_flag) { failed = true; break; }  // every softmax thread leaves here together
+            if (*stop_flag) break;  // every softmax thread leaves here together
             m = max(max(red_max[r], red_max[TM + r]), max(red_max[2 * TM + r], red_max[3 * TM + r]));
             // ---- i-exp row sum over the four parts
             const uint32_t *lutq = LUT + lane + m * TCOPIES;
@@ -506,14 +492,6 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, co
             soft_bar();
             S = red_sum[r] + red_sum[TM + r] + red_sum[2 * TM + r] + red_sum[3 * TM + r];
             const RowSum rs = make_rowsum(S);
-            // ---- the previous tile's accumulators (its MMAs also release A and B) -> staging
-            bool staged = false;
-            if (prev_bh >= 0) {
-                if (!epilogue(it - 1))
-                    epi_bad = true;
-                else
-                    staged = true;
-            }
             // ---- this row's thresholds: part q finds delta_k for k = q + 1, q + 5, q + 9, q + 13,
             //      the four binary searches interleaved
             if (valid && monotone) {
@@ -543,12 +521,6 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, co
                 }
             }
             soft_bar();
-            // ---- staged accumulators leave as two tensor stores
-            if (tid == 0 && staged) {
-                tma_store_acc(&acc_map, LG, 0, prev_r0, prev_bh);
-                tma_store_acc(&acc_map, LG + TM * 128, 32, prev_r0, prev_bh);
-                bulk_commit();
-            }
             // ---- this row's operand table
             if (valid) {
                 if (monotone) {
@@ -587,10 +559,13 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, co
                     }
                 }
             }
-            if (tid == 0) bulk_wait_read();  // the staging tile is read out before the next logits land
             soft_bar();
             mbar_arrive(&sh.lfree);  // the logits tile and its scratch are free: the next tile may load
-            if (epi_bad) continue;   // the next tile's first barrier ends the loop for all
+            // the previous tile's MMAs have read A and B: they may be rewritten
+            if (it > 0 && !mbar_wait_warp(&sh.mmadone, (it - 1) & 1, abort_flag)) {
+                wait_bad = true;  // the next tile's first barrier ends the loop for all
+                continue;
+            }
             // ---- V of a new head -> fp16 B
             if (bh != conv_bh) {
 #pragma unroll
@@ -646,60 +621,88 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p, co
             tc_fence_before();
             fence_async_smem();
             mbar_arrive(&sh.afull);
-            prev_bh = bh;
-            prev_r0 = r0;
         }
-        // the last tile's accumulators (the copy warp loads nothing more: LG is free)
-        bool staged = false;
-        if (!failed && prev_bh >= 0) staged = epilogue(it - 1);
-        soft_bar();  // reached by every softmax thread
-        if (tid == 0 && staged) {
-            tma_store_acc(&acc_map, LG, 0, prev_r0, prev_bh);
-            tma_store_acc(&acc_map, LG + TM * 128, 32, prev_r0, prev_bh);
-            bulk_commit();
-        }
-        if (tid == 0) bulk_wait_all();  // every accumulator this CTA stored has landed
-    } else if (warp == TLOAD_WARP && lane == 0) {
-        // ---------------- logits tiles (each once the previous tile's table is built), L2 prefetch
+    } else {
+        // ---------------- read-out warps (lane quarter eq), with the MMA issue and the logits copies
+        const int eq = warp & 3;
+        const uint32_t etl = tmem + ((uint32_t)(eq * 32) << 16);
+        volatile int *ew_stop = &sh.ew_stop;
+        const int nkb = (L + TKB - 1) / TKB;
         int bh = bh_begin;
         int r0 = r0_begin;
-        int lloads = 0;
-        prefetch_l2(p.v + (size_t)bh * L * TD, (uint32_t)(L * TD));
-        for (int it = 0; it < ncta_tiles; ++it, r0 = r0 + TM < L ? r0 + TM : (++bh, 0)) {
-            if (it > 0 && !mbar_wait(&sh.lfree, (it - 1) & 1, abort_flag)) break;
+        if (warp == TCOPY_WARP && lane == 0) {
+            prefetch_l2(p.v + (size_t)bh * L * TD, (uint32_t)(L * TD));
             const uint32_t bl = (uint32_t)(min(TM, L - r0) * p.ld);
             mbar_expect_tx(&sh.lload, bl);
             bulk_g2s(LG, p.logits + ((size_t)bh * L + r0) * p.ld, bl, &sh.lload);
-            ++lloads;
-            if (it + 1 < ncta_tiles) {
+        }
+        for (int it = 0; it < ncta_tiles; ++it, r0 = r0 + TM < L ? r0 + TM : (++bh, 0)) {
+            if (warp == TCOPY_WARP && lane == 0 && it + 1 < ncta_tiles) {
+                // the next tile's logits as soon as this tile's table is built
                 const int bhn = r0 + TM < L ? bh : bh + 1;
                 const int r0n = r0 + TM < L ? r0 + TM : 0;
-                prefetch_l2(p.logits + ((size_t)bhn * L + r0n) * p.ld, (uint32_t)(min(TM, L - r0n) * p.ld));
-                if (bhn != bh) prefetch_l2(p.v + (size_t)bhn * L * TD, (uint32_t)(L * TD));
+                if (mbar_wait(&sh.lfree, it & 1, abort_flag)) {
+                    const uint32_t bl = (uint32_t)(min(TM, L - r0n) * p.ld);
+                    mbar_expect_tx(&sh.lload, bl);
+                    bulk_g2s(LG, p.logits + ((size_t)bhn * L + r0n) * p.ld, bl, &sh.lload);
+                    if (bhn != bh) prefetch_l2(p.v + (size_t)bhn * L * TD, (uint32_t)(L * TD));
+                    if (it + 2 < ncta_tiles) {
+                        const int r0m = r0n + TM < L ? r0n + TM : 0;
+                        const int bhm = r0n + TM < L ? bhn : bhn + 1;
+                        prefetch_l2(p.logits + ((size_t)bhm * L + r0m) * p.ld, (uint32_t)(min(TM, L - r0m) * p.ld));
+                    }
+                }
             }
-        }
-        if (lloads > 0) mbar_wait(&sh.lload, (lloads - 1) & 1, abort_flag, false);
-    } else if (warp == TPRODUCER_WARP && lane == 0) {
-        // ---------------- MMA issue: the whole tile once its operands are in place
-        const int nkb = (L + TKB - 1) / TKB;
-        for (int it = 0; it < ncta_tiles; ++it) {
-            if (!mbar_wait(&sh.afull, it & 1, abort_flag)) break;
-            tc_fence_after();
-            const uint32_t b0 = sa(Bs);
-            for (int kb = 0; kb < nkb; ++kb)
+            if (warp == TMMA_WARP && lane == 0) {
+                // this tile's MMAs once its operands are in place
+                if (mbar_wait(&sh.afull, it & 1, abort_flag)) {
+                    tc_fence_after();
+                    const uint32_t b0 = sa(Bs);
+                    for (int kb = 0; kb < nkb; ++kb)
 #pragma unroll
-                for (int s = 0; s < TKB / 16; ++s)
-                    mma_f16_ta(tmem, tmem + TA_COL + 32 * kb + 8 * s,
-                               smem_desc(b0 + kb * B_SLOT + 2048 * s, 1024, 1024), (kb | s) != 0);
-            mma_commit(&sh.mmadone);
+                        for (int s = 0; s < TKB / 16; ++s)
+                            mma_f16_ta(tmem, tmem + TA_COL + 32 * kb + 8 * s,
+                                       smem_desc(b0 + kb * B_SLOT + 2048 * s, 1024, 1024), (kb | s) != 0);
+                    mma_commit(&sh.mmadone);
+                }
+            }
+            // this tile's accumulators: row 32 eq + lane of the tile, 64 columns in two halves
+            const bool ok = mbar_wait_warp(&sh.mmadone, it & 1, abort_flag);
+            if (ok) {
+                tc_fence_after();
+                const int row = r0 + 32 * eq + lane;
+                int32_t *dst = p.acc + ((size_t)bh * L + row) * TD;
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    uint32_t va[32];
+                    tmem_ld32(etl + 32 * h, va);
+                    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+                    if (row < L) {
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            int v8[8];
+#pragma unroll
+                            for (int j = 0; j < 8; ++j) v8[j] = __float2int_rn(__uint_as_float(va[8 * c + j]));
+                            stg256(dst + 32 * h + 8 * c, v8);
+                        }
+                    }
+                }
+            }
+            tc_fence_before();
+            if (!ok) *ew_stop = 1;
+            epi_bar();  // all four quarters have read D: the next tile's MMAs may overwrite it
+            if (*ew_stop) break;
         }
-        mma_commit(&sh.fin);
-        mbar_wait(&sh.fin, 0, abort_flag, false);
+        if (warp == TCOPY_WARP && lane == 0) mbar_wait(&sh.lload, (ncta_tiles - 1) & 1, abort_flag, false);
+        if (warp == TMMA_WARP && lane == 0) {  // every MMA issued has completed before tensor memory is freed
+            mma_commit(&sh.fin);
+            mbar_wait(&sh.fin, 0, abort_flag, false);
+        }
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == TPRODUCER_WARP)
+    if (warp == TMMA_WARP)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tmem_cols(NKB)));
 }
 
@@ -713,46 +716,20 @@ size_t tc_smem_bytes(int L, int64_t ld)
 // static shared memory of the kernel: the operand table and the control block
 constexpr size_t kTcStaticSmem = (size_t)64 * TM * 4 + 256;
 
-// The accumulators as a 3-d tensor [BH][L][64] of int32 for the tensor stores: boxes of
-// 32 columns x 128 rows x 1 head in the 128-byte swizzle; rows past L are clipped.
-cudaError_t make_acc_map(CUtensorMap *map, int32_t *acc, int64_t BH, int L)
-{
-    using EncodeFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
-                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-    static EncodeFn encode = nullptr;
-    if (!encode) {
-        void *fn = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
-        if (e != cudaSuccess) return e;
-        if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
-        encode = reinterpret_cast<EncodeFn>(fn);
-    }
-    const cuuint64_t dims[3] = {(cuuint64_t)TD, (cuuint64_t)L, (cuuint64_t)BH};
-    const cuuint64_t strides[2] = {(cuuint64_t)TD * 4, (cuuint64_t)L * TD * 4};
-    const cuuint32_t box[3] = {32, TM, 1};
-    const cuuint32_t estr[3] = {1, 1, 1};
-    CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_INT32, 3, acc, dims, strides, box, estr,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
-                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
-}
-
 template <int NKB, bool SMALL_E>
-cudaError_t tc_launch(const TcParams &p, const CUtensorMap &map, size_t smem, int grid, cudaStream_t st)
+cudaError_t tc_launch(const TcParams &p, size_t smem, int grid, cudaStream_t st)
 {
     cudaError_t e = cudaFuncSetAttribute(lis_attn_tc_kernel<NKB, SMALL_E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
-    lis_attn_tc_kernel<NKB, SMALL_E><<<grid, TTHREADS, smem, st>>>(p, map);
+    lis_attn_tc_kernel<NKB, SMALL_E><<<grid, TTHREADS, smem, st>>>(p);
     return cudaGetLastError();
 }
 
 template <int NKB>
-cudaError_t tc_launch_e(bool small_e, const TcParams &p, const CUtensorMap &map, size_t smem, int grid, cudaStream_t st)
+cudaError_t tc_launch_e(bool small_e, const TcParams &p, size_t smem, int grid, cudaStream_t st)
 {
-    return small_e ? tc_launch<NKB, true>(p, map, smem, grid, st) : tc_launch<NKB, false>(p, map, smem, grid, st);
+    return small_e ? tc_launch<NKB, true>(p, smem, grid, st) : tc_launch<NKB, false>(p, smem, grid, st);
 }
 
 // Whether every i-exp value of the scale is below 2^28: the largest is e(0) = (q_b^2 + q_c) 2^15,
@@ -772,31 +749,28 @@ bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
 {
     return b.d == TD && a.bias == nullptr && a.codes == nullptr && b.zp_v == 0 && a.L <= TMAXKB * TKB &&
            a.ld_logit % 16 == 0 && b.ld_v == TD && b.ld_acc == TD && ((uintptr_t)a.logits % 16) == 0 &&
-           ((uintptr_t)b.v % 16) == 0 && ((uintptr_t)b.acc % 16) == 0 &&
+           ((uintptr_t)b.v % 16) == 0 && ((uintptr_t)b.acc % 32) == 0 &&
            tc_smem_bytes(a.L, a.ld_logit) + kTcStaticSmem <= 232448;
 }
 
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
 {
     TcParams p{a.logits, a.ld_logit, a.s_logit, b.v, b.acc, b.BH, a.L};
-    CUtensorMap map;
-    cudaError_t e = make_acc_map(&map, b.acc, b.BH, a.L);
-    if (e != cudaSuccess) return e;
     const size_t smem = tc_smem_bytes(a.L, a.ld_logit);
     const int64_t ntiles = b.BH * ((a.L + TM - 1) / TM);
     const int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());
     const bool se = small_iexp(a.s_logit);
     switch ((a.L + TKB - 1) / TKB) {
-    case 1: return tc_launch_e<1>(se, p, map, smem, grid, st);
-    case 2: return tc_launch_e<2>(se, p, map, smem, grid, st);
-    case 3: return tc_launch_e<3>(se, p, map, smem, grid, st);
-    case 4: return tc_launch_e<4>(se, p, map, smem, grid, st);
-    case 5: return tc_launch_e<5>(se, p, map, smem, grid, st);
-    case 6: return tc_launch_e<6>(se, p, map, smem, grid, st);
-    case 7: return tc_launch_e<7>(se, p, map, smem, grid, st);
-    case 8: return tc_launch_e<8>(se, p, map, smem, grid, st);
-    case 9: return tc_launch_e<9>(se, p, map, smem, grid, st);
-    default: return tc_launch_e<10>(se, p, map, smem, grid, st);
+    case 1: return tc_launch_e<1>(se, p, smem, grid, st);
+    case 2: return tc_launch_e<2>(se, p, smem, grid, st);
+    case 3: return tc_launch_e<3>(se, p, smem, grid, st);
+    case 4: return tc_launch_e<4>(se, p, smem, grid, st);
+    case 5: return tc_launch_e<5>(se, p, smem, grid, st);
+    case 6: return tc_launch_e<6>(se, p, smem, grid, st);
+    case 7: return tc_launch_e<7>(se, p, smem, grid, st);
+    case 8: return tc_launch_e<8>(se, p, smem, grid, st);
+    case 9: return tc_launch_e<9>(se, p, smem, grid, st);
+    default: return tc_launch_e<10>(se, p, smem, grid, st);
     }
 }
 
