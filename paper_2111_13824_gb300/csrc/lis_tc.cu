@@ -210,6 +210,34 @@ __device__ __forceinline__ void soft_bar()
     asm volatile("bar.sync 1, %0;" ::"n"(TSOFT) : "memory");
 }
 
+// 2S = hi + lo with hi = fp32(2S) rounded to nearest even and lo exact (|lo| < 2^19), from
+// integer operations only (the same values as the fp32 conversions of make_rowsum)
+__device__ __forceinline__ RowSum split_2s(unsigned long long S)
+{
+    const unsigned long long s2 = 2ull * S;
+    RowSum rs;
+    if (s2 < (1ull << 24)) {
+        rs.hi = __uint2float_rn((uint32_t)s2);
+        rs.lo = 0.0f;
+    } else {
+        const int p = 63 - __clzll((long long)s2);  // 24 .. 42
+        const int sh = p - 23;
+        unsigned long long mant = s2 >> sh;         // 2^23 .. 2^24 - 1
+        const unsigned long long rem = s2 & ((1ull << sh) - 1), half = 1ull << (sh - 1);
+        if (rem > half || (rem == half && (mant & 1ull))) ++mant;
+        int e = p;
+        if (mant == (1ull << 24)) {
+            mant >>= 1;
+            ++e;
+        }
+        rs.hi = __int_as_float(((127 + e) << 23) | (int)(mant & 0x7FFFFFull));
+        const int lo = (int)((long long)s2 - (long long)(mant << (e - 23)));  // |lo| <= half < 2^19
+        rs.lo = __fsub_rn(__int_as_float(lo + 0x4B400000), 12582912.0f);    // exact below 2^22
+    }
+    rs.hibits = __float_as_int(rs.hi);
+    return rs;
+}
+
 // mbar_wait with one verdict for the whole warp (the callers go on to
 // warp-collective tcgen05 instructions)
 __device__ __forceinline__ bool mbar_wait_warp(uint64_t *b, uint32_t parity, volatile int *abort_flag)
@@ -345,6 +373,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     extern __shared__ unsigned char dsm_raw[];
     __shared__ TcShared sh;
     __shared__ __align__(16) uint32_t OT[64 * TM];              // operand table: word j of row r at [j][r]
+    __shared__ float LUTF[256];                                 // fp32 of the i-exp values (exact: <= 16 bits)
     unsigned char *base = dsm_raw + ((1024u - (sa(dsm_raw) & 1023u)) & 1023u);
     unsigned char *Bs = base;                                   // NKB x 8 KB
     uint32_t *LUT = (uint32_t *)(Bs + NKB * B_SLOT);            // 256 x TCOPIES
@@ -377,6 +406,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     {
         const IexpC c = sh.c;
         for (int i = tid; i < 256 * TCOPIES; i += blockDim.x) LUT[i] = iexp_neg(i / TCOPIES, c);
+        for (int d = tid; d < 256; d += blockDim.x) LUTF[d] = __uint2float_rn(iexp_neg(d, c));
         for (int d = tid; d < 255; d += blockDim.x)
             if (iexp_neg(d, c) < iexp_neg(d + 1, c)) sh.rising = 1;
     }
@@ -491,7 +521,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
             }
             soft_bar();
             S = red_sum[r] + red_sum[TM + r] + red_sum[2 * TM + r] + red_sum[3 * TM + r];
-            const RowSum rs = make_rowsum(S);
+            const RowSum rs = split_2s(S);
             // ---- this row's thresholds: part q finds delta_k for k = q + 1, q + 5, q + 9, q + 13,
             //      the four binary searches interleaved
             if (valid && monotone) {
@@ -504,10 +534,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                     lo[i] = 0;
                 }
                 // e(d) D_k <= 2S, exact: one rounding of an exact product minus hi, against lo
-                auto hit = [&](int d, float D) -> bool {
-                    const float ef = __uint2float_rn(lds32(lut_lane + (uint32_t)(d * (TCOPIES * 4))));
-                    return __fmaf_rn(ef, D, -rs.hi) <= rs.lo;
-                };
+                auto hit = [&](int d, float D) -> bool { return __fmaf_rn(LUTF[d], D, -rs.hi) <= rs.lo; };
 #pragma unroll
                 for (int step = 128; step >= 1; step >>= 1)
 #pragma unroll
@@ -713,8 +740,8 @@ size_t tc_smem_bytes(int L, int64_t ld)
     return 1024 + (size_t)nkb * B_SLOT + (size_t)256 * TCOPIES * 4 + (size_t)TPARTS * TM * (4 + 8) + lg;
 }
 
-// static shared memory of the kernel: the operand table and the control block
-constexpr size_t kTcStaticSmem = (size_t)64 * TM * 4 + 256;
+// static shared memory of the kernel: the operand table, the fp32 i-exp table, the control block
+constexpr size_t kTcStaticSmem = (size_t)64 * TM * 4 + 1024 + 256;
 
 template <int NKB, bool SMALL_E>
 cudaError_t tc_launch(const TcParams &p, size_t smem, int grid, cudaStream_t st)
