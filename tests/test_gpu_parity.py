@@ -417,3 +417,24 @@ def test_tensor_core_operand_table_at_any_scale(s):
     ao, ov = oracle.lis_attn_v(co, v, 0)
     assert not ov
     assert np.array_equal(np_(acc), ao)
+
+
+@pytest.mark.parametrize("L", [63, 64, 65, 577])
+def test_tensor_core_ignores_row_padding(L):
+    """Bytes of a logit row past L (up to the row stride) are not keys: filling them with
+    random values must not change anything."""
+    rng = np.random.default_rng(L)
+    BH = 3
+    ld = (L + 15) // 16 * 16 + 32
+    x = np.zeros((BH * L, ld), np.int8)
+    x[:, :L] = rng.integers(-128, 128, (BH * L, L), dtype=np.int8)
+    v = rng.integers(-128, 128, (BH, L, 64), dtype=np.int8)
+    xg = x.copy()
+    xg[:, L:] = rng.integers(-128, 128, (BH * L, ld - L), dtype=np.int8)
+    for s in (0.05, 0.3):
+        a0 = fqvit.lis_attention(torch.from_numpy(x).to(DEV), s, torch.from_numpy(v).to(DEV), 0)
+        a1 = fqvit.lis_attention(torch.from_numpy(xg).to(DEV), s, torch.from_numpy(v).to(DEV), 0)
+        fqvit.sync_status()
+        co, _ = oracle.lis_softmax(x, L, s)
+        ao, _ = oracle.lis_attn_v(co, v, 0)
+        assert np.array_equal(np_(a0), ao) and np.array_equal(np_(a1), ao)
