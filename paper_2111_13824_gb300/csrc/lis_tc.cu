@@ -1,14 +1,16 @@
 // lis_tc.cu -- fused Log-Int-Softmax + BitShift attention times values on
 // the 5th-generation tensor cores (tcgen05) of sm_103a.
 //
-// Eq. 15 is a matrix product: acc = P (V - zp_V) with P[i][j] = 2^(15 - code_ij).
-// Every P entry and every int8 value of V is exact in fp16, and for codes made
-// by Log-Int-Softmax sum_j 2^-code_j <= 3 + L 2^-15 (2^-code < 1.5 / q_rev and
-// q_rev >= S/e - 1/2), so with |V| <= 128 every partial sum of a row is an
-// integer below 2^24: fp16 operands with fp32 accumulation give the integer
-// result exactly.  The kernel therefore evaluates the shift-accumulate as
+// Eq. 15 is a matrix product: acc = P (V - zp_V) with P[i][j] = 2^(15 - code_ij),
+// computed as P V - zp_V (P 1).  Every P entry and every int8 value of V is exact
+// in fp16, and for codes made by Log-Int-Softmax sum_j 2^-code_j <= 3 + L 2^-15
+// (2^-code < 1.5 / q_rev and q_rev >= S/e - 1/2), so with |V| <= 128 every
+// partial sum of P V is an integer below 2^24, and the row sums P 1 (a second,
+// N = 16 product against a block of ones, only when zp_V != 0) stay below 2^17:
+// fp16 operands with fp32 accumulation give the integers exactly, and
+// zp_V (P 1) is subtracted in int32.  The kernel evaluates the products as
 // tcgen05.mma.kind::f16 (M = 128 query rows, N = 64 = d, K = 16 keys per
-// instruction) with the accumulator in tensor memory.
+// instruction) with the accumulators in tensor memory.
 //
 // One CTA per SM walks (head, 128-row tile) work items.  Roles:
 //   warps 0-15 (four threads per query row; warp w serves rows 32 (w % 4) ..
@@ -58,6 +60,7 @@ struct TcParams {
     int32_t *acc;
     int64_t BH;
     int L;
+    int zp;  // zero point of V (acc = sum_j 2^(15-code) (V - zp))
 };
 
 __device__ __forceinline__ uint32_t sa(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -143,6 +146,8 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint3
 
 // kind::f16 instruction descriptor: D f32, A/B f16, A K-major, B MN-major, N = 64, M = 128
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 16) | ((uint32_t)(TD >> 3) << 17) | ((uint32_t)(TM >> 4) << 24);
+// the row sums of P: N = 16, B K-major (a block of ones, so its layout does not matter)
+constexpr uint32_t kIdescOnes = (1u << 4) | ((uint32_t)(16 >> 3) << 17) | ((uint32_t)(TM >> 4) << 24);
 
 __device__ __forceinline__ void mma_commit(uint64_t *b)
 {
@@ -168,13 +173,15 @@ constexpr int TCOPY_WARP = TEPI_WARP + 1;         //   warp 17 lane 0 also copie
 constexpr int TTHREADS = TSOFT + 128;
 constexpr int TMAXKB = 10;                        // key blocks of the longest row (L <= 640)
 constexpr int TA_COL = TD;                        // D: columns 0..63; A of key block kb: 64 + 32 kb ..
+// row sums of P (only when zp_V != 0): 16 columns after A
+__host__ __device__ constexpr int tr_col(int nkb) { return TA_COL + 32 * nkb; }
 constexpr int SCR_THR = 0;                        // the logits tile doubles as threshold scratch: int32 [16][TM]
 constexpr int SCR_BYTES = 16 * TM * 4;
 
 // tensor-memory columns for NKB key blocks (a power of two >= 32)
 __host__ __device__ constexpr int tmem_cols(int nkb)
 {
-    return TA_COL + 32 * nkb <= 128 ? 128 : TA_COL + 32 * nkb <= 256 ? 256 : 512;
+    return tr_col(nkb) + 16 <= 128 ? 128 : tr_col(nkb) + 16 <= 256 ? 256 : 512;
 }
 
 struct TcShared {
@@ -293,12 +300,29 @@ __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8])
                  : "memory");
 }
 
-__device__ __forceinline__ void mma_f16_ta(uint32_t dt, uint32_t at, uint64_t bd, uint32_t accumulate)
+__device__ __forceinline__ void mma_f16_ta(uint32_t dt, uint32_t at, uint64_t bd, uint32_t accumulate,
+                                           uint32_t idesc = kIdesc)
 {
     asm volatile(
         "{ .reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p; }" ::"r"(dt),
-        "r"(at), "l"(bd), "r"(kIdesc), "r"(accumulate)
+        "r"(at), "l"(bd), "r"(idesc), "r"(accumulate)
         : "memory");
+}
+
+// shared-memory matrix descriptor without swizzle
+__device__ __forceinline__ uint64_t smem_desc_plain(uint32_t addr, uint32_t lbo, uint32_t sbo)
+{
+    uint64_t d = (uint64_t)((addr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)(lbo >> 4) << 16;
+    d |= (uint64_t)(sbo >> 4) << 32;
+    d |= 1ull << 46;  // descriptor version for tcgen05
+    return d;
+}
+
+__device__ __forceinline__ void tmem_ld1(uint32_t taddr, uint32_t &r)
+{
+    __syncwarp();
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(r) : "r"(taddr));
 }
 
 __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *b)
@@ -374,6 +398,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     __shared__ TcShared sh;
     __shared__ __align__(16) uint32_t OT[64 * TM];              // operand table: word j of row r at [j][r]
     __shared__ float LUTF[256];                                 // fp32 of the i-exp values (exact: <= 16 bits)
+    __shared__ __align__(128) uint32_t ONES[128];               // 16 x 16 fp16 ones: B of the row sums of P
     unsigned char *base = dsm_raw + ((1024u - (sa(dsm_raw) & 1023u)) & 1023u);
     unsigned char *Bs = base;                                   // NKB x 8 KB
     uint32_t *LUT = (uint32_t *)(Bs + NKB * B_SLOT);            // 256 x TCOPIES
@@ -407,9 +432,11 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
         const IexpC c = sh.c;
         for (int i = tid; i < 256 * TCOPIES; i += blockDim.x) LUT[i] = iexp_neg(i / TCOPIES, c);
         for (int d = tid; d < 256; d += blockDim.x) LUTF[d] = __uint2float_rn(iexp_neg(d, c));
+        for (int i = tid; i < 128; i += blockDim.x) ONES[i] = 0x3C003C00u;
         for (int d = tid; d < 255; d += blockDim.x)
             if (iexp_neg(d, c) < iexp_neg(d + 1, c)) sh.rising = 1;
     }
+    fence_async_smem();  // ONES is read by the MMAs
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -685,11 +712,23 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                 if (mbar_wait(&sh.afull, it & 1, abort_flag)) {
                     tc_fence_after();
                     const uint32_t b0 = sa(Bs);
-                    for (int kb = 0; kb < nkb; ++kb)
+                    const uint64_t ones = smem_desc_plain(sa(ONES), 128, 256);
+                    if (p.zp == 0) {
+                        for (int kb = 0; kb < nkb; ++kb)
 #pragma unroll
-                        for (int s = 0; s < TKB / 16; ++s)
-                            mma_f16_ta(tmem, tmem + TA_COL + 32 * kb + 8 * s,
-                                       smem_desc(b0 + kb * B_SLOT + 2048 * s, 1024, 1024), (kb | s) != 0);
+                            for (int s = 0; s < TKB / 16; ++s)
+                                mma_f16_ta(tmem, tmem + TA_COL + 32 * kb + 8 * s,
+                                           smem_desc(b0 + kb * B_SLOT + 2048 * s, 1024, 1024), (kb | s) != 0);
+                    } else {
+                        for (int kb = 0; kb < nkb; ++kb)
+#pragma unroll
+                            for (int s = 0; s < TKB / 16; ++s) {
+                                mma_f16_ta(tmem, tmem + TA_COL + 32 * kb + 8 * s,
+                                           smem_desc(b0 + kb * B_SLOT + 2048 * s, 1024, 1024), (kb | s) != 0);
+                                mma_f16_ta(tmem + tr_col(NKB), tmem + TA_COL + 32 * kb + 8 * s, ones,
+                                           (kb | s) != 0, kIdescOnes);
+                            }
+                    }
                     mma_commit(&sh.mmadone);
                 }
             }
@@ -699,6 +738,14 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                 tc_fence_after();
                 const int row = r0 + 32 * eq + lane;
                 int32_t *dst = p.acc + ((size_t)bh * L + row) * TD;
+                // zp (sum_j 2^(15-code_j)), an exact integer below 2^24 times |zp| <= 255
+                int zsum = 0;
+                if (p.zp != 0) {
+                    uint32_t rs;
+                    tmem_ld1(etl + tr_col(NKB), rs);
+                    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+                    zsum = p.zp * __float2int_rn(__uint_as_float(rs));
+                }
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
                     uint32_t va[32];
@@ -709,7 +756,8 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                         for (int c = 0; c < 4; ++c) {
                             int v8[8];
 #pragma unroll
-                            for (int j = 0; j < 8; ++j) v8[j] = __float2int_rn(__uint_as_float(va[8 * c + j]));
+                            for (int j = 0; j < 8; ++j)
+                                v8[j] = __float2int_rn(__uint_as_float(va[8 * c + j])) - zsum;
                             stg256(dst + 32 * h + 8 * c, v8);
                         }
                     }
@@ -741,7 +789,7 @@ size_t tc_smem_bytes(int L, int64_t ld)
 }
 
 // static shared memory of the kernel: the operand table, the fp32 i-exp table, the control block
-constexpr size_t kTcStaticSmem = (size_t)64 * TM * 4 + 1024 + 256;
+constexpr size_t kTcStaticSmem = (size_t)64 * TM * 4 + 1024 + 512 + 256;
 
 template <int NKB, bool SMALL_E>
 cudaError_t tc_launch(const TcParams &p, size_t smem, int grid, cudaStream_t st)
@@ -774,7 +822,7 @@ bool small_iexp(float s)
 
 bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
 {
-    return b.d == TD && a.bias == nullptr && a.codes == nullptr && b.zp_v == 0 && a.L <= TMAXKB * TKB &&
+    return b.d == TD && a.bias == nullptr && a.codes == nullptr && a.L <= TMAXKB * TKB &&
            a.ld_logit % 16 == 0 && b.ld_v == TD && b.ld_acc == TD && ((uintptr_t)a.logits % 16) == 0 &&
            ((uintptr_t)b.v % 16) == 0 && ((uintptr_t)b.acc % 32) == 0 &&
            tc_smem_bytes(a.L, a.ld_logit) + kTcStaticSmem <= 232448;
@@ -782,7 +830,7 @@ bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
 
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
 {
-    TcParams p{a.logits, a.ld_logit, a.s_logit, b.v, b.acc, b.BH, a.L};
+    TcParams p{a.logits, a.ld_logit, a.s_logit, b.v, b.acc, b.BH, a.L, b.zp_v};
     const size_t smem = tc_smem_bytes(a.L, a.ld_logit);
     const int64_t ntiles = b.BH * ((a.L + TM - 1) / TM);
     const int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());

@@ -438,3 +438,27 @@ def test_tensor_core_ignores_row_padding(L):
         co, _ = oracle.lis_softmax(x, L, s)
         ao, _ = oracle.lis_attn_v(co, v, 0)
         assert np.array_equal(np_(a0), ao) and np.array_equal(np_(a1), ao)
+
+
+@pytest.mark.parametrize("zp", [-255, -7, 3, 128, 255])
+def test_fused_attention_with_v_zero_point(zp, monkeypatch):
+    """acc = sum_j 2^(15-code) (V - zp_V) with an asymmetric V (Eq. 15): the tensor-core
+    path (P V - zp P 1) and the CUDA-core path against the oracle."""
+    rng = np.random.default_rng(1000 + zp)
+    for L in (49, 197, 577):
+        BH = 2
+        ld = (L + 15) // 16 * 16
+        x = np.zeros((BH * L, ld), np.int8)
+        x[:, :L] = rng.integers(-128, 128, (BH * L, L), dtype=np.int8)
+        v = rng.integers(-128, 128, (BH, L, 64), dtype=np.int8)
+        co, _ = oracle.lis_softmax(x, L, 0.06)
+        ao, ov = oracle.lis_attn_v(co, v, zp)
+        assert not ov
+        acc = fqvit.lis_attention(torch.from_numpy(x).to(DEV), 0.06, torch.from_numpy(v).to(DEV), zp)
+        fqvit.sync_status()
+        assert np.array_equal(np_(acc), ao), (L, zp)
+        monkeypatch.setenv("FQVIT_ATTN_PATH", "cuda_core")
+        acc2 = fqvit.lis_attention(torch.from_numpy(x).to(DEV), 0.06, torch.from_numpy(v).to(DEV), zp)
+        fqvit.sync_status()
+        monkeypatch.delenv("FQVIT_ATTN_PATH")
+        assert np.array_equal(np_(acc2), ao), (L, zp)
