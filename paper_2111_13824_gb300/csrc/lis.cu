@@ -94,11 +94,11 @@ __device__ void softmax_row(const int8_t *__restrict__ src, int L, const uint32_
 }
 
 template <int NW, bool BIAS>
-__global__ void __launch_bounds__(256) lis_softmax_kernel(LisArgs a)
+__global__ void __launch_bounds__(256) lis_softmax_kernel(LisArgs a, IexpC ic)
 {
     __shared__ uint32_t lut[kLutSize];
     extern __shared__ int8_t btab_all[];  // [heads][(2w-1)^2] when BIAS
-    build_lut(lut, a.s_logit);
+    build_lut(lut, ic);
     const int nb = (2 * a.window - 1) * (2 * a.window - 1);
     if (BIAS)
         for (int i = threadIdx.x; i < a.heads * nb; i += blockDim.x) btab_all[i] = a.bias[i];
@@ -182,7 +182,7 @@ __global__ void __launch_bounds__(256) lis_attn_v_kernel(AttnVArgs a)
 
 // Fused: codes of 32 rows into shared memory, then the accumulate.
 template <int NW, bool BIAS, int CPT>
-__global__ void __launch_bounds__(256) lis_attention_kernel(LisArgs la, AttnVArgs a)
+__global__ void __launch_bounds__(256) lis_attention_kernel(LisArgs la, AttnVArgs a, IexpC ic)
 {
     extern __shared__ __align__(16) unsigned char sm[];
     __shared__ uint32_t lut[kLutSize];
@@ -194,7 +194,7 @@ __global__ void __launch_bounds__(256) lis_attention_kernel(LisArgs la, AttnVArg
     int8_t *btab_all = reinterpret_cast<int8_t *>(sm + off);
     const int nb = (2 * la.window - 1) * (2 * la.window - 1);
 
-    build_lut(lut, la.s_logit);
+    build_lut(lut, ic);
     if (BIAS)
         for (int i = threadIdx.x; i < la.heads * nb; i += blockDim.x) btab_all[i] = la.bias[i];
     const int64_t bh = blockIdx.y;
@@ -245,7 +245,7 @@ cudaError_t softmax_launch(const LisArgs &a, cudaStream_t st)
     if (smem > 48 * 1024)
         cudaFuncSetAttribute(lis_softmax_kernel<NW, BIAS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
-    lis_softmax_kernel<NW, BIAS><<<blocks, 256, smem, st>>>(a);
+    lis_softmax_kernel<NW, BIAS><<<blocks, 256, smem, st>>>(a, iexp_consts_host(a.s_logit));
     return cudaGetLastError();
 }
 
@@ -275,11 +275,11 @@ cudaError_t fused_launch(const LisArgs &la, const AttnVArgs &a, cudaStream_t st)
     if (a.d == 64) {
         cudaFuncSetAttribute(lis_attention_kernel<NW, BIAS, 8>,
                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        lis_attention_kernel<NW, BIAS, 8><<<g, 256, smem, st>>>(la, a);
+        lis_attention_kernel<NW, BIAS, 8><<<g, 256, smem, st>>>(la, a, iexp_consts_host(la.s_logit));
     } else {
         cudaFuncSetAttribute(lis_attention_kernel<NW, BIAS, 4>,
                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        lis_attention_kernel<NW, BIAS, 4><<<g, 256, smem, st>>>(la, a);
+        lis_attention_kernel<NW, BIAS, 4><<<g, 256, smem, st>>>(la, a, iexp_consts_host(la.s_logit));
     }
     return cudaGetLastError();
 }

@@ -5,6 +5,8 @@
 
 #include <stdint.h>
 
+#include <cmath>
+
 namespace fqvit {
 namespace lis {
 
@@ -13,18 +15,6 @@ constexpr int kLutSize = 288;  // q~ in [-287, 0]
 struct IexpC {
     int q_ln2, q_b, q_c;
 };
-
-// Algorithm 1 constants, fp64 as in the oracle's definition.
-__device__ __forceinline__ IexpC iexp_consts(float s)
-{
-    const double ln2 = 0.693147180559945309417232121458176568;
-    double sd = (double)s;
-    IexpC c;
-    c.q_ln2 = (int)floor(__ddiv_rn(-ln2, sd));
-    c.q_b = (int)floor(__ddiv_rn(1.353, sd));
-    c.q_c = (int)floor(__ddiv_rn(0.344, __dmul_rn(0.3585, __dmul_rn(sd, sd))));
-    return c;
-}
 
 // e(-t) for t in [0, 287], n = 15
 __device__ __forceinline__ uint32_t iexp_neg(int t, IexpC c)
@@ -39,9 +29,21 @@ __device__ __forceinline__ uint32_t iexp_neg(int t, IexpC c)
     return qL << (15 - z);
 }
 
-__device__ __forceinline__ void build_lut(uint32_t *lut, float s)
+// Algorithm 1 constants of a scale, fp64 with one IEEE rounding per operation as in the
+// oracle's definition; computed on the host once per launch (fp64 is slow on the device).
+__host__ inline IexpC iexp_consts_host(float s)
 {
-    IexpC c = iexp_consts(s);
+    const double ln2 = 0.693147180559945309417232121458176568;
+    const double sd = (double)s;
+    IexpC c;
+    c.q_ln2 = (int)floor(-ln2 / sd);
+    c.q_b = (int)floor(1.353 / sd);
+    c.q_c = (int)floor(0.344 / (0.3585 * (sd * sd)));
+    return c;
+}
+
+__device__ __forceinline__ void build_lut(uint32_t *lut, IexpC c)
+{
     for (int t = threadIdx.x; t < kLutSize; t += blockDim.x) lut[t] = iexp_neg(t, c);
 }
 

@@ -61,6 +61,7 @@ struct TcParams {
     int64_t BH;
     int L;
     int zp;  // zero point of V (acc = sum_j 2^(15-code) (V - zp))
+    IexpC ic;  // Algorithm 1 constants of the scale
 };
 
 __device__ __forceinline__ uint32_t sa(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -420,7 +421,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
         sh.rising = 0;
         sh.stop = 0;
         sh.ew_stop = 0;
-        sh.c = iexp_consts(p.s);
+        sh.c = p.ic;
     }
     if (warp == TMMA_WARP) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(&sh.tmem)),
@@ -807,16 +808,8 @@ cudaError_t tc_launch_e(bool small_e, const TcParams &p, size_t smem, int grid, 
     return small_e ? tc_launch<NKB, true>(p, smem, grid, st) : tc_launch<NKB, false>(p, smem, grid, st);
 }
 
-// Whether every i-exp value of the scale is below 2^28: the largest is e(0) = (q_b^2 + q_c) 2^15,
-// with the constants of Algorithm 1 computed exactly as the kernels do (fp64, one rounding per
-// operation), so host and device agree.
-bool small_iexp(float s)
-{
-    const double sd = (double)s;
-    const double qb = floor(1.353 / sd);
-    const double qc = floor(0.344 / (0.3585 * (sd * sd)));
-    return (qb * qb + qc) * 32768.0 < 268435456.0;
-}
+// Whether every i-exp value of the scale is below 2^28: the largest is e(0) = (q_b^2 + q_c) 2^15.
+bool small_iexp(const IexpC &c) { return ((double)c.q_b * c.q_b + c.q_c) * 32768.0 < 268435456.0; }
 
 }  // namespace
 
@@ -830,11 +823,11 @@ bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
 
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
 {
-    TcParams p{a.logits, a.ld_logit, a.s_logit, b.v, b.acc, b.BH, a.L, b.zp_v};
+    TcParams p{a.logits, a.ld_logit, a.s_logit, b.v, b.acc, b.BH, a.L, b.zp_v, iexp_consts_host(a.s_logit)};
     const size_t smem = tc_smem_bytes(a.L, a.ld_logit);
     const int64_t ntiles = b.BH * ((a.L + TM - 1) / TM);
     const int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());
-    const bool se = small_iexp(a.s_logit);
+    const bool se = small_iexp(p.ic);
     switch ((a.L + TKB - 1) / TKB) {
     case 1: return tc_launch_e<1>(se, p, smem, grid, st);
     case 2: return tc_launch_e<2>(se, p, smem, grid, st);
