@@ -105,11 +105,19 @@ cudaError_t launch_lis_attention(const LisArgs &a, const AttnVArgs &b, cudaStrea
 bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b);
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st);
 
+// tensor-core fused path for rows of at most 64 keys, two heads per MMA tile, with
+// the optional relative-position bias (lis_win.cu)
+bool lis_attention_win_eligible(const LisArgs &a, const AttnVArgs &b);
+cudaError_t launch_lis_attention_win(const LisArgs &a, const AttnVArgs &b, cudaStream_t st);
+cudaError_t read_clear_win_status(int *status);
+
 // Synchronizes st, returns the device status word (0 ok, 5 a bounded wait
 // timed out) and clears it.
 cudaError_t read_clear_device_status(int *status, cudaStream_t st);
 
-// Attention implementation choice: 0 automatic, 1 CUDA cores only (FQVIT_ATTN_PATH=cuda_core).
+// Attention implementation choice: 0 automatic, 1 CUDA cores only (FQVIT_ATTN_PATH=cuda_core),
+// 2 no short-row kernel (FQVIT_ATTN_PATH=no_window: rows of at most 64 keys take the
+// one-head-per-tile tensor-core kernel when it applies).
 int attention_path_override();
 
 }  // namespace fqvit

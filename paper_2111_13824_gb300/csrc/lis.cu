@@ -324,12 +324,16 @@ cudaError_t launch_lis_attn_v(const AttnVArgs &a, cudaStream_t st)
 int attention_path_override()
 {
     const char *e = getenv("FQVIT_ATTN_PATH");
-    return (e && strcmp(e, "cuda_core") == 0) ? 1 : 0;
+    if (e && strcmp(e, "cuda_core") == 0) return 1;
+    if (e && strcmp(e, "no_window") == 0) return 2;
+    return 0;
 }
 
 cudaError_t launch_lis_attention(const LisArgs &la, const AttnVArgs &a, cudaStream_t st)
 {
-    if (attention_path_override() == 0 && lis_attention_tc_eligible(la, a)) return launch_lis_attention_tc(la, a, st);
+    const int path = attention_path_override();
+    if (path == 0 && lis_attention_win_eligible(la, a)) return launch_lis_attention_win(la, a, st);
+    if (path != 1 && lis_attention_tc_eligible(la, a)) return launch_lis_attention_tc(la, a, st);
     return la.bias ? fused_dispatch<true>(la, a, st) : fused_dispatch<false>(la, a, st);
 }
 

@@ -10,7 +10,7 @@
 namespace fqvit {
 namespace lis {
 
-constexpr int kLutSize = 288;  // q~ in [-287, 0]
+constexpr int kLutSize = 511;  // q~ in [-510, 0]: int8 logits plus an int8 bias, minus the maximum
 
 struct IexpC {
     int q_ln2, q_b, q_c;

@@ -1,0 +1,505 @@
+// lis_win.cu -- fused Log-Int-Softmax + BitShift attention times values on the
+// tcgen05 tensor cores for short rows: L <= 64 keys, as in windowed attention
+// (7 x 7 windows: L = 49), with an optional relative-position bias.
+//
+// The product is the one of lis_tc.cu: acc = P (V - zp_V) with
+// P[i][j] = 2^(15 - code_ij) exact in fp16 and fp32 accumulation exact for
+// codes made by Log-Int-Softmax (Eq. 15, Algorithm 2).  A tile of the MMA
+// (M = 128 rows) holds two heads: head slot h in {0, 1} owns tensor-memory
+// lanes 64 h .. 64 h + 63 (query row i at lane 64 h + i) and keys
+// 64 h .. 64 h + 63 of the K = 128 reduction.  A is block diagonal: a row's
+// operands sit in its own slot's 32 tensor-memory columns (two keys per
+// column) and the other slot's columns hold zeros, written once.  B holds the
+// two heads' V rows as fp16 (rows = keys, 128-byte swizzled, MN-major), so
+// one tile is 8 MMAs of K = 16.  With d = 32, B's columns 32 .. 63 are free:
+// column 32 holds 1 for every key, which makes column 32 of D the row sum of
+// P, and acc = P V - zp_V (P 1) needs no second product.
+//
+// A CTA runs up to four independent groups of 128 threads; thread r of a
+// group serves query row r & 63 of head slot r >> 6, owns tensor-memory lane r
+// of the group's 128 columns (D: 0..63, A: 64..127) and converts V's key row
+// r & 63 of its slot.  Per tile a thread takes its row into registers, adds
+// the bias, finds the maximum and the i-exp row sum, waits for the group's
+// previous MMAs, stores their accumulators, writes its operands and its V row,
+// and after a group barrier one thread issues the tile's MMAs.
+//
+// i-exp table: e(d) for the distance d = max - q~ in [0, ne), replicated for
+// each of the 32 lanes (one 256-byte line per d: 32 copies of e, then 32 of
+// fp32 e), so lookups are free of bank conflicts and a byte permute forms the
+// address.  Distances past 15 |q_ln2| all give e(15 |q_ln2|) (the clamp of
+// Algorithm 1), so d is clamped to ne - 1.
+//
+// Every wait is bounded (two seconds), after which the group stops, records a
+// timeout status and the kernel drains what it issued.
+#include "fqvit_internal.cuh"
+#include "lis_common.cuh"
+#include "tc_common.cuh"
+
+#include <cstdlib>
+#include <cstring>
+
+namespace fqvit {
+
+namespace {
+
+using namespace lis;
+using namespace tc;
+
+constexpr int WMAXG = 4;                 // groups per CTA
+constexpr int WB_BYTES = 128 * 128;      // B of a group: 128 keys x 64 fp16, 128B-swizzled (16 KB)
+constexpr int WBIAS_ROW = 64;            // bytes per bias row (keys 0..63, 16-byte chunks swizzled)
+
+struct WinParams {
+    const int8_t *logits;
+    int64_t ld;
+    const int8_t *v;
+    int64_t ld_v;
+    int32_t *acc;
+    int64_t ld_acc;
+    const int8_t *bias;  // [heads][(2w-1)^2] or nullptr
+    int heads;
+    int window;
+    int64_t BH;
+    int L;
+    int zp;
+    IexpC ic;
+    int ne;  // table entries: distances 0 .. ne - 1
+    int ng;  // groups per CTA
+};
+
+struct WinShared {
+    uint64_t mmadone[WMAXG];
+    uint64_t fin[WMAXG];
+    uint32_t tmem;
+    int abort_flag;
+    int stop[WMAXG][2];  // set (never cleared) when a wait of iteration parity [.][it & 1] gave up
+};
+
+__device__ __forceinline__ void group_bar(int g)
+{
+    __syncwarp();
+    asm volatile("bar.sync %0, 128;" ::"r"(1 + g) : "memory");
+}
+
+__device__ __forceinline__ uint32_t win_tmem_cols(int ng) { return ng == 1 ? 128u : ng == 2 ? 256u : 512u; }
+
+// the i-exp table line of the distance in the low (SEL = 0x5104) or high (0x5324) half of a
+// pair word, for this lane: 256 d + 4 lane
+template <uint32_t SEL>
+__device__ __forceinline__ uint32_t lut_off(uint32_t dpair, uint32_t lane4)
+{
+    return prmt(dpair, lane4, SEL);
+}
+
+template <int D, bool BIAS, bool SMALL_E>
+__global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams p)
+{
+    extern __shared__ unsigned char dsm_raw[];
+    __shared__ WinShared sh;
+    __shared__ uint32_t e_tmp[512];
+    unsigned char *base = dsm_raw + ((1024u - (sa(dsm_raw) & 1023u)) & 1023u);
+    unsigned char *Bs_all = base;                                             // ng x 16 KB
+    const unsigned char *LUTB = Bs_all + p.ng * WB_BYTES;                     // ne x 256 B
+    unsigned char *BR = Bs_all + p.ng * WB_BYTES + (size_t)p.ne * 256;        // heads x L x 64 B
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int g = tid >> 7, r = tid & 127;
+    const int h = r >> 6, i = r & 63;
+    const int L = p.L;
+    volatile int *abort_flag = &sh.abort_flag;
+
+    if (tid == 0) {
+        for (int k = 0; k < p.ng; ++k) {
+            mbar_init(&sh.mmadone[k], 1);
+            mbar_init(&sh.fin[k], 1);
+            sh.stop[k][0] = sh.stop[k][1] = 0;
+        }
+        sh.abort_flag = 0;
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(&sh.tmem)),
+                     "r"(win_tmem_cols(p.ng)));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    for (int d = tid; d < p.ne; d += blockDim.x) e_tmp[d] = iexp_neg(d, p.ic);
+    // B: zeros, and (d = 32) fp16 1 in column 32 of every key row below L
+    for (int x = tid; x < p.ng * WB_BYTES / 16; x += blockDim.x) {
+        const int kk = (x >> 3) & 127, pos = x & 7, ci = pos ^ (kk & 7);
+        uint4 z = make_uint4(0, 0, 0, 0);
+        if (D == 32 && ci == 4 && (kk & 63) < L) z.x = 0x3C00u;
+        *reinterpret_cast<uint4 *>(Bs_all + 16 * x) = z;
+    }
+    // bias rows: byte j of row (head, query) = bias + 128 for keys j < L, 0 past L; the 16-byte
+    // chunk c of a row sits at position c ^ ((query >> 1) & 3)
+    if (BIAS) {
+        const int nb = 2 * p.window - 1;
+        for (int x = tid; x < p.heads * L * 16; x += blockDim.x) {
+            const int row = x >> 4, wj = x & 15;
+            const int hh = row / L, qi = row - hh * L;
+            uint32_t word = 0;
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+                const int j = 4 * wj + b;
+                if (j < L) word |= (uint32_t)((int)p.bias[hh * nb * nb + relpos_idx(qi, j, p.window)] + 128) << (8 * b);
+            }
+            const int pc = (wj >> 2) ^ ((qi >> 1) & 3);
+            *reinterpret_cast<uint32_t *>(BR + (size_t)row * WBIAS_ROW + 16 * pc + 4 * (wj & 3)) = word;
+        }
+    }
+    __syncthreads();
+    for (int x = tid; x < p.ne * 64; x += blockDim.x) {
+        const uint32_t e = e_tmp[x >> 6];
+        reinterpret_cast<uint32_t *>(const_cast<unsigned char *>(LUTB))[x] =
+            (x & 32) ? __float_as_uint(__uint2float_rn(e)) : e;
+    }
+    fence_async_smem();  // B is read by the MMAs
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+
+    const uint32_t tmem = sh.tmem;
+    const uint32_t tD = tmem + 128u * (uint32_t)g + ((uint32_t)((warp & 3) * 32) << 16);  // this warp's lanes
+    const uint32_t tA = tD + 64u;
+    unsigned char *Bg = Bs_all + g * WB_BYTES;
+    const uint32_t lane4 = (uint32_t)lane << 2;
+    const int nq = (L + 15) >> 4;  // 16-byte chunks of a row that hold keys
+    const int nw = (L + 3) >> 2;   // words that hold keys
+    uint32_t cm[4];                // byte masks of the last chunk's words: keys below L
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int j0 = 16 * (nq - 1) + 4 * k, n = L - j0;
+        cm[k] = n >= 4 ? 0xFFFFFFFFu : n <= 0 ? 0u : (0xFFFFFFFFu >> (32 - 8 * n));
+    }
+    // A starts as zeros: the other slot's columns and the own slot's keys past the last
+    // 16-key chunk are never written again
+    {
+        const uint32_t z[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+#pragma unroll
+        for (int c = 0; c < 8; ++c) tmem_st8(tA + 8u * c, z);
+        tmem_wait_st();
+    }
+    tc_fence_before();
+    group_bar(g);
+
+    const int64_t ntiles = (p.BH + 1) >> 1;
+    const int64_t gstride = (int64_t)gridDim.x * p.ng;
+    const uint32_t cap2 = (uint32_t)(p.ne - 1) * 0x10001u;
+
+    auto load_row = [&](int64_t t, uint4 (&w)[4], uint4 (&vv)[D / 16]) {
+        const int64_t bh = 2 * t + h;
+        const bool ok = t < ntiles && bh < p.BH && i < L;
+        const int8_t *lr = p.logits + ((size_t)bh * L + i) * p.ld;
+        const int8_t *vr = p.v + ((size_t)bh * L + i) * p.ld_v;
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+            w[c] = (ok && c < nq) ? __ldg(reinterpret_cast<const uint4 *>(lr) + c) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+        for (int c = 0; c < D / 16; ++c) vv[c] = ok ? __ldg(reinterpret_cast<const uint4 *>(vr) + c) : make_uint4(0, 0, 0, 0);
+    };
+
+    // accumulators of tile t (rows of this thread): D columns 0 .. D-1 (and 32 = P 1 when D = 32)
+    auto store_acc = [&](int64_t t) {
+        const int64_t bh = 2 * t + h;
+        const bool ok = bh < p.BH && i < L;
+        int zsum = 0;
+        if (D == 32 && p.zp != 0) {
+            uint32_t x;
+            tmem_ld1(tD + 32u, x);
+            tmem_wait_ld();
+            zsum = p.zp * __float2int_rn(__uint_as_float(x));
+        }
+        int32_t *dst = p.acc + ((size_t)bh * L + i) * p.ld_acc;
+#pragma unroll
+        for (int hf = 0; hf < D / 16; ++hf) {
+            uint32_t va[16];
+            tmem_ld16(tD + 16u * hf, va);
+            tmem_wait_ld();
+            if (ok) {
+#pragma unroll
+                for (int c = 0; c < 2; ++c) {
+                    int v8[8];
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) v8[j] = __float2int_rn(__uint_as_float(va[8 * c + j])) - zsum;
+                    stg256(dst + 16 * hf + 8 * c, v8);
+                }
+            }
+        }
+    };
+
+    uint4 nw4[4], nv[D / 16];
+    int64_t t = (int64_t)blockIdx.x * p.ng + g;
+    load_row(t, nw4, nv);
+    int it = 0;
+    int64_t prev = -1;
+    bool stopped = false;
+    for (; t < ntiles; t += gstride, ++it) {
+        uint4 w[4], vv[D / 16];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) w[c] = nw4[c];
+#pragma unroll
+        for (int c = 0; c < D / 16; ++c) vv[c] = nv[c];
+        load_row(t + gstride, nw4, nv);  // the next tile's row, in flight during this one
+
+        const int64_t bh = 2 * t + h;
+        const bool valid = bh < p.BH && i < L;
+        // ---- q + 128 per byte, keys past L zeroed
+        uint32_t u[16];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const uint32_t ww[4] = {w[c].x, w[c].y, w[c].z, w[c].w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                uint32_t x = ww[k] ^ 0x80808080u;
+                if (c == nq - 1) x &= cm[k];
+                if (c >= nq) x = 0u;
+                u[4 * c + k] = x;
+            }
+        }
+        // ---- pairs of 16-bit lanes v = q + bias + 256 (0 for keys past L):
+        //      vp[2j] holds keys (4j, 4j+2), vp[2j+1] keys (4j+1, 4j+3)
+        uint32_t vp[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) vp[k] = 0u;
+        if (BIAS) {
+            const int hh = (int)(bh % p.heads);
+            const int qi = i < L ? i : L - 1;
+            const unsigned char *br = BR + ((size_t)hh * L + qi) * WBIAS_ROW;
+            const int sw = (qi >> 1) & 3;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const uint4 b4 = *reinterpret_cast<const uint4 *>(br + 16 * (c ^ sw));
+                const uint32_t bb[4] = {b4.x, b4.y, b4.z, b4.w};
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int j = 4 * c + k;
+                    if (j < nw) {
+                        vp[2 * j] = prmt(u[j], 0u, 0x4240u) + prmt(bb[k], 0u, 0x4240u);
+                        vp[2 * j + 1] = prmt(u[j], 0u, 0x4341u) + prmt(bb[k], 0u, 0x4341u);
+                    }
+                }
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                if (j < nw) {
+                    vp[2 * j] = prmt(u[j], 0u, 0x4240u);
+                    vp[2 * j + 1] = prmt(u[j], 0u, 0x4341u);
+                }
+            }
+        }
+        // ---- row maximum, then distances d = max - v clamped to the table
+        uint32_t mx = vmax16x2u(vp[0], vp[1]);
+#pragma unroll
+        for (int k = 2; k < 32; k += 2) mx = vmax16x2u(mx, vmax16x2u(vp[k], vp[k + 1]));
+        const uint32_t m = max(mx & 0xFFFFu, mx >> 16);
+        const uint32_t m2 = m * 0x10001u;
+#pragma unroll
+        for (int k = 0; k < 32; ++k) vp[k] = vmin16x2u(m2 - vp[k], cap2);
+        // ---- i-exp row sum over the words that hold keys (padding keys of the last word have
+        //      d = max; they are taken out below)
+        unsigned long long S = 0;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            if (c < nq) {
+                uint32_t a = 0;
+                unsigned long long a64 = 0;
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    if (4 * c + (k >> 1) < nw) {
+                        const uint32_t dp = vp[8 * c + k];
+                        const uint32_t e0 = *reinterpret_cast<const uint32_t *>(LUTB + lut_off<0x5104u>(dp, lane4));
+                        const uint32_t e1 = *reinterpret_cast<const uint32_t *>(LUTB + lut_off<0x5324u>(dp, lane4));
+                        if (SMALL_E)
+                            a += e0 + e1;
+                        else
+                            a64 += (unsigned long long)e0 + e1;
+                    }
+                }
+                S += SMALL_E ? (unsigned long long)a : a64;
+            }
+        }
+        {
+            const uint32_t dm = m < (uint32_t)(p.ne - 1) ? m : (uint32_t)(p.ne - 1);
+            const uint32_t epad = *reinterpret_cast<const uint32_t *>(LUTB + ((dm << 8) | lane4));
+            S -= (unsigned long long)(4 * nw - L) * epad;
+        }
+        const RowSum rs = split_2s(S);
+
+        // ---- the previous tile's MMAs are done: its accumulators out, A and B free
+        bool ok = true;
+        if (it > 0) {
+            ok = mbar_wait_warp(&sh.mmadone[g], (it - 1) & 1, abort_flag);
+            if (ok) {
+                tc_fence_after();
+                store_acc(prev);
+            }
+        }
+        if (ok) {
+            // ---- operands 2^(15 - code) of this row's keys -> tensor memory (own slot)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                if (c >= nq) continue;  // keys past the row: zero operands since the start
+                uint32_t o[8];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int j = 4 * c + k;
+                    if (j >= nw) {
+                        o[2 * k] = o[2 * k + 1] = 0u;
+                        continue;
+                    }
+                    const uint32_t de = vp[2 * j], dod = vp[2 * j + 1];
+                    const float f0 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5104u>(de, lane4));
+                    const float f2 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5324u>(de, lane4));
+                    const float f1 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5104u>(dod, lane4));
+                    const float f3 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5324u>(dod, lane4));
+                    const uint32_t E0 = operand_exp_f(f0, rs.hibits, rs.hi, rs.lo);
+                    const uint32_t E1 = operand_exp_f(f1, rs.hibits, rs.hi, rs.lo);
+                    const uint32_t E2 = operand_exp_f(f2, rs.hibits, rs.hi, rs.lo);
+                    const uint32_t E3 = operand_exp_f(f3, rs.hibits, rs.hi, rs.lo);
+                    o[2 * k] = (E0 << 10) | (E1 << 26);
+                    o[2 * k + 1] = (E2 << 10) | (E3 << 26);
+                }
+                tmem_st8(tA + 32u * (uint32_t)h + 8u * c, o);
+            }
+            // ---- V key row i of this slot -> fp16 B (row 64 h + i, chunk ci at ci ^ (row & 7))
+            if (valid) {
+                const int kk = 64 * h + i;
+                unsigned char *brow = Bg + kk * 128;
+#pragma unroll
+                for (int c = 0; c < D / 16; ++c) {
+                    const uint32_t x0 = vv[c].x ^ 0x80808080u, x1 = vv[c].y ^ 0x80808080u;
+                    const uint32_t x2 = vv[c].z ^ 0x80808080u, x3 = vv[c].w ^ 0x80808080u;
+                    uint4 lo, hi;
+                    lo.x = i8x2_to_h2(x0, 0x5140);
+                    lo.y = i8x2_to_h2(x0, 0x7362);
+                    lo.z = i8x2_to_h2(x1, 0x5140);
+                    lo.w = i8x2_to_h2(x1, 0x7362);
+                    hi.x = i8x2_to_h2(x2, 0x5140);
+                    hi.y = i8x2_to_h2(x2, 0x7362);
+                    hi.z = i8x2_to_h2(x3, 0x5140);
+                    hi.w = i8x2_to_h2(x3, 0x7362);
+                    *reinterpret_cast<uint4 *>(brow + (((2 * c) ^ (kk & 7)) << 4)) = lo;
+                    *reinterpret_cast<uint4 *>(brow + (((2 * c + 1) ^ (kk & 7)) << 4)) = hi;
+                }
+            }
+            tmem_wait_st();
+        }
+        fence_async_smem();
+        tc_fence_before();
+        if (!ok) sh.stop[g][it & 1] = 1;
+        group_bar(g);
+        if (*(volatile int *)&sh.stop[g][it & 1]) {
+            stopped = true;
+            break;
+        }
+        if (r == 0) {
+            tc_fence_after();
+            const uint32_t dcol = tmem + 128u * (uint32_t)g, acol = dcol + 64u;
+            const uint32_t b0 = sa(Bg);
+#pragma unroll
+            for (int kb = 0; kb < 2; ++kb)
+#pragma unroll
+                for (int s = 0; s < 4; ++s)
+                    mma_f16_ta(dcol, acol + 32u * kb + 8u * s, smem_desc(b0 + kb * 8192 + 2048 * s, 1024, 1024),
+                               (kb | s) != 0);
+            mma_commit(&sh.mmadone[g]);
+        }
+        prev = t;
+    }
+    if (!stopped && it > 0) {
+        if (mbar_wait_warp(&sh.mmadone[g], (it - 1) & 1, abort_flag)) {
+            tc_fence_after();
+            store_acc(prev);
+        }
+    }
+    if (r == 0) {  // every MMA this group issued has completed before tensor memory is freed
+        mma_commit(&sh.fin[g]);
+        mbar_wait(&sh.fin[g], 0, abort_flag, false);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(win_tmem_cols(p.ng)));
+}
+
+constexpr size_t kWinStaticSmem = 512 * 4 + sizeof(WinShared) + 256;
+constexpr size_t kSmemLimit = 232448;
+
+size_t win_smem_bytes(int ng, int ne, int heads, int L, bool bias)
+{
+    return 1024 + (size_t)ng * WB_BYTES + (size_t)ne * 256 + (bias ? (size_t)heads * L * WBIAS_ROW : 0);
+}
+
+// table entries: distances up to 255 (510 with a bias), and none past the clamp 15 |q_ln2|
+int win_table_entries(const IexpC &c, bool bias)
+{
+    const int dmax = bias ? 510 : 255;
+    const int clamp = 15 * -c.q_ln2;
+    return (clamp < dmax ? clamp : dmax) + 1;
+}
+
+int win_groups(int ne, int heads, int L, bool bias)
+{
+    for (int ng = WMAXG; ng >= 1; --ng)
+        if (win_smem_bytes(ng, ne, heads, L, bias) + kWinStaticSmem <= kSmemLimit) return ng;
+    return 0;
+}
+
+bool small_iexp_w(const IexpC &c) { return ((double)c.q_b * c.q_b + c.q_c) * 32768.0 < 268435456.0; }
+
+template <int D, bool BIAS, bool SMALL_E>
+cudaError_t win_launch(const WinParams &p, size_t smem, int grid, cudaStream_t st)
+{
+    cudaError_t e = cudaFuncSetAttribute(lis_attn_win_kernel<D, BIAS, SMALL_E>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    lis_attn_win_kernel<D, BIAS, SMALL_E><<<grid, 128 * p.ng, smem, st>>>(p);
+    return cudaGetLastError();
+}
+
+template <int D>
+cudaError_t win_launch_d(bool bias, bool small_e, const WinParams &p, size_t smem, int grid, cudaStream_t st)
+{
+    if (bias) return small_e ? win_launch<D, true, true>(p, smem, grid, st) : win_launch<D, true, false>(p, smem, grid, st);
+    return small_e ? win_launch<D, false, true>(p, smem, grid, st) : win_launch<D, false, false>(p, smem, grid, st);
+}
+
+}  // namespace
+
+bool lis_attention_win_eligible(const LisArgs &a, const AttnVArgs &b)
+{
+    if (a.L > 64 || a.codes != nullptr || a.rowsum != nullptr) return false;
+    if (!(b.d == 32 || (b.d == 64 && b.zp_v == 0))) return false;
+    if (a.ld_logit % 16 != 0 || ((uintptr_t)a.logits % 16) != 0) return false;
+    if (b.ld_v % 16 != 0 || ((uintptr_t)b.v % 16) != 0) return false;
+    if (b.ld_acc % 8 != 0 || ((uintptr_t)b.acc % 32) != 0) return false;
+    const bool bias = a.bias != nullptr;
+    const IexpC c = iexp_consts_host(a.s_logit);
+    return win_groups(win_table_entries(c, bias), a.heads, a.L, bias) > 0;
+}
+
+cudaError_t launch_lis_attention_win(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
+{
+    const bool bias = a.bias != nullptr;
+    WinParams p{a.logits, a.ld_logit, b.v, b.ld_v, b.acc, b.ld_acc, a.bias, a.heads, a.window, b.BH, a.L, b.zp_v,
+                iexp_consts_host(a.s_logit), 0, 0};
+    p.ne = win_table_entries(p.ic, bias);
+    p.ng = win_groups(p.ne, a.heads, a.L, bias);
+    const size_t smem = win_smem_bytes(p.ng, p.ne, a.heads, a.L, bias);
+    const int64_t ntiles = (b.BH + 1) / 2;
+    const int64_t want = (ntiles + p.ng - 1) / p.ng;
+    const int grid = (int)(want < sm_count() ? want : sm_count());
+    const bool se = small_iexp_w(p.ic);
+    return b.d == 32 ? win_launch_d<32>(bias, se, p, smem, grid, st) : win_launch_d<64>(bias, se, p, smem, grid, st);
+}
+
+cudaError_t read_clear_win_status(int *status)
+{
+    int zero = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(status, g_status, sizeof(int));
+    if (e != cudaSuccess) return e;
+    return cudaMemcpyToSymbol(g_status, &zero, sizeof(int));
+}
+
+}  // namespace fqvit
