@@ -91,16 +91,32 @@ __device__ __forceinline__ uint32_t lut_off(uint32_t dpair, uint32_t lane4)
     return prmt(dpair, lane4, SEL);
 }
 
-template <int D, bool BIAS, bool SMALL_E>
+// fp16 exponent field (30 - code) of the operand 2^(15-code), as operand_exp_f with D_k read
+// from a table (dk[k] = D_k for k = 1 .. 63; k <= 43 since 2S < 2^43 and e >= 1)
+__device__ __forceinline__ uint32_t operand_exp_tab(float ef, int G, float hi, float lo, const float *dk)
+{
+    const int k = (G - __float_as_int(ef)) >> 23;
+    const float t = __fmaf_rn(ef, dk[k], -hi);
+    uint32_t le;  // 0xFFFFFFFF when e D_k <= 2S
+    asm("set.le.u32.f32 %0, %1, %2;" : "=r"(le) : "f"(t), "f"(lo));
+    return (uint32_t)max(31 - k + (int)le, 15);
+}
+
+// NQ: 16-key chunks of a row (L in 16 (NQ - 1) + 1 .. 16 NQ)
+template <int D, bool BIAS, bool SMALL_E, int NQ>
 __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams p)
 {
-    extern __shared__ unsigned char dsm_raw[];
+    extern __shared__ __align__(16) unsigned char dsm_raw[];
     __shared__ WinShared sh;
     __shared__ uint32_t e_tmp[512];
-    unsigned char *base = dsm_raw + ((1024u - (sa(dsm_raw) & 1023u)) & 1023u);
-    unsigned char *Bs_all = base;                                             // ng x 16 KB
-    const unsigned char *LUTB = Bs_all + p.ng * WB_BYTES;                     // ne x 256 B
-    unsigned char *BR = Bs_all + p.ng * WB_BYTES + (size_t)p.ne * 256;        // heads x L x 64 B
+    __shared__ float dk[64];
+    __shared__ int koff[64], qbase[64];  // relative-position offsets (bias only)
+    // the table first, at the fixed start of dynamic shared memory (lookups add no base), then
+    // B (1024-byte aligned for the 128-byte swizzle) and the bias rows
+    const unsigned char *LUTB = dsm_raw;                                      // ne x 256 B
+    const uint32_t bs_off = (uint32_t)p.ne * 256u;
+    unsigned char *Bs_all = dsm_raw + bs_off + ((1024u - ((sa(dsm_raw) + bs_off) & 1023u)) & 1023u);  // ng x 16 KB
+    unsigned char *BR = Bs_all + p.ng * WB_BYTES;                             // heads x L x 64 B
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = tid >> 7, r = tid & 127;
@@ -121,36 +137,54 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
                      "r"(win_tmem_cols(p.ng)));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
+    // set-up, phase 1: i-exp values, the D_k table, the raw bias table (into the B area, free
+    // until phase 3) and the index offsets of the relative positions
     for (int d = tid; d < p.ne; d += blockDim.x) e_tmp[d] = iexp_neg(d, p.ic);
-    // B: zeros, and (d = 32) fp16 1 in column 32 of every key row below L
+    for (int k = tid; k < 64; k += blockDim.x)  // D_1 = 3, D_k = 3 2^(k-1) - 1 (exact up to k = 24)
+        dk[k] = k <= 1 ? 3.0f : __fsub_rn(__int_as_float(((k + 127) << 23) | 0x400000), 1.0f);
+    const int nb = 2 * p.window - 1;
+    if (BIAS) {
+        for (int x = tid; x < p.heads * nb * nb; x += blockDim.x) Bs_all[x] = (unsigned char)p.bias[x];
+        // entry of (query i, key j) = qbase[i] - koff[j]: (y_i - y_j + w - 1) nb + (x_i - x_j + w - 1)
+        for (int j = tid; j < L; j += blockDim.x) {
+            const int y = j / p.window, x = j - y * p.window;
+            koff[j] = y * nb + x;
+            qbase[j] = (y + p.window - 1) * nb + x + p.window - 1;
+        }
+    }
+    __syncthreads();
+    // phase 2: bias rows (byte j of row (head, query) = bias + 128 for keys j < L, 0 past L; the
+    // 16-byte chunk c of a row sits at position c ^ ((query >> 1) & 3)) and the replicated table
+    if (BIAS) {
+        // thread: word wj (keys 4 wj .. +3) of rows tid / 16, + blockDim / 16, ...
+        const int wj = tid & 15, rstep = blockDim.x >> 4;
+        int kof[4];
+#pragma unroll
+        for (int b = 0; b < 4; ++b) kof[b] = 4 * wj + b < L ? koff[4 * wj + b] : -1;
+        int row = tid >> 4, hh = row / L, qi = row - hh * L;
+        for (; row < p.heads * L; row += rstep) {
+            const unsigned char *tab = Bs_all + hh * nb * nb + qbase[qi];
+            uint32_t word = 0;
+#pragma unroll
+            for (int b = 0; b < 4; ++b)
+                if (kof[b] >= 0) word |= (uint32_t)(((int)(int8_t)tab[-kof[b]] + 128) & 0xFF) << (8 * b);
+            const int pc = (wj >> 2) ^ ((qi >> 1) & 3);
+            *reinterpret_cast<uint32_t *>(BR + (size_t)row * WBIAS_ROW + 16 * pc + 4 * (wj & 3)) = word;
+            for (qi += rstep; qi >= L; qi -= L) ++hh;
+        }
+    }
+    for (int x = tid; x < p.ne * 16; x += blockDim.x) {  // 16 bytes: 4 copies of e (parts 0-7) or fp32 e
+        const uint32_t e = e_tmp[x >> 4];
+        const uint32_t w = (x & 8) ? __float_as_uint(__uint2float_rn(e)) : e;
+        reinterpret_cast<uint4 *>(const_cast<unsigned char *>(LUTB))[x] = make_uint4(w, w, w, w);
+    }
+    __syncthreads();
+    // phase 3: B of every group: zeros, and (d = 32) fp16 1 in column 32 of every key row below L
     for (int x = tid; x < p.ng * WB_BYTES / 16; x += blockDim.x) {
         const int kk = (x >> 3) & 127, pos = x & 7, ci = pos ^ (kk & 7);
         uint4 z = make_uint4(0, 0, 0, 0);
         if (D == 32 && ci == 4 && (kk & 63) < L) z.x = 0x3C00u;
         *reinterpret_cast<uint4 *>(Bs_all + 16 * x) = z;
-    }
-    // bias rows: byte j of row (head, query) = bias + 128 for keys j < L, 0 past L; the 16-byte
-    // chunk c of a row sits at position c ^ ((query >> 1) & 3)
-    if (BIAS) {
-        const int nb = 2 * p.window - 1;
-        for (int x = tid; x < p.heads * L * 16; x += blockDim.x) {
-            const int row = x >> 4, wj = x & 15;
-            const int hh = row / L, qi = row - hh * L;
-            uint32_t word = 0;
-#pragma unroll
-            for (int b = 0; b < 4; ++b) {
-                const int j = 4 * wj + b;
-                if (j < L) word |= (uint32_t)((int)p.bias[hh * nb * nb + relpos_idx(qi, j, p.window)] + 128) << (8 * b);
-            }
-            const int pc = (wj >> 2) ^ ((qi >> 1) & 3);
-            *reinterpret_cast<uint32_t *>(BR + (size_t)row * WBIAS_ROW + 16 * pc + 4 * (wj & 3)) = word;
-        }
-    }
-    __syncthreads();
-    for (int x = tid; x < p.ne * 64; x += blockDim.x) {
-        const uint32_t e = e_tmp[x >> 6];
-        reinterpret_cast<uint32_t *>(const_cast<unsigned char *>(LUTB))[x] =
-            (x & 32) ? __float_as_uint(__uint2float_rn(e)) : e;
     }
     fence_async_smem();  // B is read by the MMAs
     tc_fence_before();
@@ -162,12 +196,11 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
     const uint32_t tA = tD + 64u;
     unsigned char *Bg = Bs_all + g * WB_BYTES;
     const uint32_t lane4 = (uint32_t)lane << 2;
-    const int nq = (L + 15) >> 4;  // 16-byte chunks of a row that hold keys
-    const int nw = (L + 3) >> 2;   // words that hold keys
+    const int nw = (L + 3) >> 2;   // words that hold keys (all but the last chunk's are full)
     uint32_t cm[4];                // byte masks of the last chunk's words: keys below L
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-        const int j0 = 16 * (nq - 1) + 4 * k, n = L - j0;
+        const int j0 = 16 * (NQ - 1) + 4 * k, n = L - j0;
         cm[k] = n >= 4 ? 0xFFFFFFFFu : n <= 0 ? 0u : (0xFFFFFFFFu >> (32 - 8 * n));
     }
     // A starts as zeros: the other slot's columns and the own slot's keys past the last
@@ -181,26 +214,26 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
     tc_fence_before();
     group_bar(g);
 
-    const int64_t ntiles = (p.BH + 1) >> 1;
-    const int64_t gstride = (int64_t)gridDim.x * p.ng;
+    const int ntiles = (int)((p.BH + 1) >> 1);  // BH <= 65535
+    const int BH = (int)p.BH;
+    const int gstride = (int)gridDim.x * p.ng;
     const uint32_t cap2 = (uint32_t)(p.ne - 1) * 0x10001u;
+    const int qi = i < L ? i : L - 1;  // bias row of this thread (rows past L read the last one)
+    const int sw = (qi >> 1) & 3;
+    const int hstep = (int)((2 * (int64_t)gstride) % p.heads);  // head of the bias table: +2 gstride per tile
 
-    auto load_row = [&](int64_t t, uint4 (&w)[4], uint4 (&vv)[D / 16]) {
-        const int64_t bh = 2 * t + h;
-        const bool ok = t < ntiles && bh < p.BH && i < L;
+    auto load_row = [&](int t, uint4 (&w)[NQ]) {
+        const int bh = 2 * t + h;
+        const bool ok = t < ntiles && bh < BH && i < L;
         const int8_t *lr = p.logits + ((size_t)bh * L + i) * p.ld;
-        const int8_t *vr = p.v + ((size_t)bh * L + i) * p.ld_v;
 #pragma unroll
-        for (int c = 0; c < 4; ++c)
-            w[c] = (ok && c < nq) ? __ldg(reinterpret_cast<const uint4 *>(lr) + c) : make_uint4(0, 0, 0, 0);
-#pragma unroll
-        for (int c = 0; c < D / 16; ++c) vv[c] = ok ? __ldg(reinterpret_cast<const uint4 *>(vr) + c) : make_uint4(0, 0, 0, 0);
+        for (int c = 0; c < NQ; ++c) w[c] = ok ? __ldg(reinterpret_cast<const uint4 *>(lr) + c) : make_uint4(0, 0, 0, 0);
     };
 
     // accumulators of tile t (rows of this thread): D columns 0 .. D-1 (and 32 = P 1 when D = 32)
-    auto store_acc = [&](int64_t t) {
-        const int64_t bh = 2 * t + h;
-        const bool ok = bh < p.BH && i < L;
+    auto store_acc = [&](int t) {
+        const int bh = 2 * t + h;
+        const bool ok = bh < BH && i < L;
         int zsum = 0;
         if (D == 32 && p.zp != 0) {
             uint32_t x;
@@ -226,97 +259,80 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
         }
     };
 
-    uint4 nw4[4], nv[D / 16];
-    int64_t t = (int64_t)blockIdx.x * p.ng + g;
-    load_row(t, nw4, nv);
+    uint4 nw4[NQ];
+    int t = (int)blockIdx.x * p.ng + g;
+    int hh = BIAS ? (int)((2 * (int64_t)t + h) % p.heads) : 0;
+    load_row(t, nw4);
     int it = 0;
-    int64_t prev = -1;
+    int prev = -1;
     bool stopped = false;
-    for (; t < ntiles; t += gstride, ++it) {
-        uint4 w[4], vv[D / 16];
+    for (; t < ntiles; t += gstride, ++it, hh = (hh + hstep >= p.heads ? hh + hstep - p.heads : hh + hstep)) {
+        uint4 w[NQ];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) w[c] = nw4[c];
-#pragma unroll
-        for (int c = 0; c < D / 16; ++c) vv[c] = nv[c];
-        load_row(t + gstride, nw4, nv);  // the next tile's row, in flight during this one
+        for (int c = 0; c < NQ; ++c) w[c] = nw4[c];
+        load_row(t + gstride, nw4);  // the next tile's logits, in flight during this one
 
-        const int64_t bh = 2 * t + h;
-        const bool valid = bh < p.BH && i < L;
-        // ---- q + 128 per byte, keys past L zeroed
-        uint32_t u[16];
+        const int bh = 2 * t + h;
+        const bool valid = bh < BH && i < L;
+        // ---- q + 128 per byte, keys past L zeroed (only the last chunk has any)
+        uint32_t u[4 * NQ];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < NQ; ++c) {
             const uint32_t ww[4] = {w[c].x, w[c].y, w[c].z, w[c].w};
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                uint32_t x = ww[k] ^ 0x80808080u;
-                if (c == nq - 1) x &= cm[k];
-                if (c >= nq) x = 0u;
-                u[4 * c + k] = x;
-            }
+            for (int k = 0; k < 4; ++k) u[4 * c + k] = (ww[k] ^ 0x80808080u) & (c == NQ - 1 ? cm[k] : 0xFFFFFFFFu);
         }
         // ---- pairs of 16-bit lanes v = q + bias + 256 (0 for keys past L):
         //      vp[2j] holds keys (4j, 4j+2), vp[2j+1] keys (4j+1, 4j+3)
-        uint32_t vp[32];
-#pragma unroll
-        for (int k = 0; k < 32; ++k) vp[k] = 0u;
+        uint32_t vp[8 * NQ];
         if (BIAS) {
-            const int hh = (int)(bh % p.heads);
-            const int qi = i < L ? i : L - 1;
             const unsigned char *br = BR + ((size_t)hh * L + qi) * WBIAS_ROW;
-            const int sw = (qi >> 1) & 3;
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
+            for (int c = 0; c < NQ; ++c) {
                 const uint4 b4 = *reinterpret_cast<const uint4 *>(br + 16 * (c ^ sw));
                 const uint32_t bb[4] = {b4.x, b4.y, b4.z, b4.w};
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
                     const int j = 4 * c + k;
-                    if (j < nw) {
-                        vp[2 * j] = prmt(u[j], 0u, 0x4240u) + prmt(bb[k], 0u, 0x4240u);
-                        vp[2 * j + 1] = prmt(u[j], 0u, 0x4341u) + prmt(bb[k], 0u, 0x4341u);
-                    }
+                    vp[2 * j] = prmt(u[j], 0u, 0x4240u) + prmt(bb[k], 0u, 0x4240u);
+                    vp[2 * j + 1] = prmt(u[j], 0u, 0x4341u) + prmt(bb[k], 0u, 0x4341u);
                 }
             }
         } else {
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-                if (j < nw) {
-                    vp[2 * j] = prmt(u[j], 0u, 0x4240u);
-                    vp[2 * j + 1] = prmt(u[j], 0u, 0x4341u);
-                }
+            for (int j = 0; j < 4 * NQ; ++j) {
+                vp[2 * j] = prmt(u[j], 0u, 0x4240u);
+                vp[2 * j + 1] = prmt(u[j], 0u, 0x4341u);
             }
         }
-        // ---- row maximum, then distances d = max - v clamped to the table
+        // ---- row maximum (keys past L are 0), then distances d = max - v clamped to the table
         uint32_t mx = vmax16x2u(vp[0], vp[1]);
 #pragma unroll
-        for (int k = 2; k < 32; k += 2) mx = vmax16x2u(mx, vmax16x2u(vp[k], vp[k + 1]));
+        for (int k = 2; k < 8 * NQ; k += 2) mx = vmax16x2u(mx, vmax16x2u(vp[k], vp[k + 1]));
         const uint32_t m = max(mx & 0xFFFFu, mx >> 16);
         const uint32_t m2 = m * 0x10001u;
 #pragma unroll
-        for (int k = 0; k < 32; ++k) vp[k] = vmin16x2u(m2 - vp[k], cap2);
+        for (int k = 0; k < 8 * NQ; ++k) vp[k] = vmin16x2u(m2 - vp[k], cap2);
         // ---- i-exp row sum over the words that hold keys (padding keys of the last word have
         //      d = max; they are taken out below)
         unsigned long long S = 0;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            if (c < nq) {
-                uint32_t a = 0;
-                unsigned long long a64 = 0;
+        for (int c = 0; c < NQ; ++c) {
+            uint32_t a = 0;
+            unsigned long long a64 = 0;
 #pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    if (4 * c + (k >> 1) < nw) {
-                        const uint32_t dp = vp[8 * c + k];
-                        const uint32_t e0 = *reinterpret_cast<const uint32_t *>(LUTB + lut_off<0x5104u>(dp, lane4));
-                        const uint32_t e1 = *reinterpret_cast<const uint32_t *>(LUTB + lut_off<0x5324u>(dp, lane4));
-                        if (SMALL_E)
-                            a += e0 + e1;
-                        else
-                            a64 += (unsigned long long)e0 + e1;
-                    }
+            for (int k = 0; k < 8; ++k) {
+                if (c < NQ - 1 || 4 * c + (k >> 1) < nw) {
+                    const uint32_t dp = vp[8 * c + k];
+                    const uint32_t e0 = *reinterpret_cast<const uint32_t *>(LUTB + lut_off<0x5104u>(dp, lane4));
+                    const uint32_t e1 = *reinterpret_cast<const uint32_t *>(LUTB + lut_off<0x5324u>(dp, lane4));
+                    if (SMALL_E)
+                        a += e0 + e1;
+                    else
+                        a64 += (unsigned long long)e0 + e1;
                 }
-                S += SMALL_E ? (unsigned long long)a : a64;
             }
+            S += SMALL_E ? (unsigned long long)a : a64;
         }
         {
             const uint32_t dm = m < (uint32_t)(p.ne - 1) ? m : (uint32_t)(p.ne - 1);
@@ -324,6 +340,13 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
             S -= (unsigned long long)(4 * nw - L) * epad;
         }
         const RowSum rs = split_2s(S);
+        // V key row i of this slot (used after the operands: its latency hides behind them)
+        uint4 vv[D / 16];
+        {
+            const int8_t *vr = p.v + ((size_t)bh * L + i) * p.ld_v;
+#pragma unroll
+            for (int c = 0; c < D / 16; ++c) vv[c] = valid ? __ldg(reinterpret_cast<const uint4 *>(vr) + c) : make_uint4(0, 0, 0, 0);
+        }
 
         // ---- the previous tile's MMAs are done: its accumulators out, A and B free
         bool ok = true;
@@ -335,15 +358,15 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
             }
         }
         if (ok) {
-            // ---- operands 2^(15 - code) of this row's keys -> tensor memory (own slot)
+            // ---- operands 2^(15 - code) of this row's keys -> tensor memory (own slot); chunks
+            //      past NQ keep the zeros written at the start
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                if (c >= nq) continue;  // keys past the row: zero operands since the start
+            for (int c = 0; c < NQ; ++c) {
                 uint32_t o[8];
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
                     const int j = 4 * c + k;
-                    if (j >= nw) {
+                    if (c == NQ - 1 && j >= nw) {
                         o[2 * k] = o[2 * k + 1] = 0u;
                         continue;
                     }
@@ -352,10 +375,10 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
                     const float f2 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5324u>(de, lane4));
                     const float f1 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5104u>(dod, lane4));
                     const float f3 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5324u>(dod, lane4));
-                    const uint32_t E0 = operand_exp_f(f0, rs.hibits, rs.hi, rs.lo);
-                    const uint32_t E1 = operand_exp_f(f1, rs.hibits, rs.hi, rs.lo);
-                    const uint32_t E2 = operand_exp_f(f2, rs.hibits, rs.hi, rs.lo);
-                    const uint32_t E3 = operand_exp_f(f3, rs.hibits, rs.hi, rs.lo);
+                    const uint32_t E0 = operand_exp_tab(f0, rs.hibits, rs.hi, rs.lo, dk);
+                    const uint32_t E1 = operand_exp_tab(f1, rs.hibits, rs.hi, rs.lo, dk);
+                    const uint32_t E2 = operand_exp_tab(f2, rs.hibits, rs.hi, rs.lo, dk);
+                    const uint32_t E3 = operand_exp_tab(f3, rs.hibits, rs.hi, rs.lo, dk);
                     o[2 * k] = (E0 << 10) | (E1 << 26);
                     o[2 * k + 1] = (E2 << 10) | (E3 << 26);
                 }
@@ -423,7 +446,7 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(win_tmem_cols(p.ng)));
 }
 
-constexpr size_t kWinStaticSmem = 512 * 4 + sizeof(WinShared) + 256;
+constexpr size_t kWinStaticSmem = 512 * 4 + 64 * 4 * 3 + sizeof(WinShared) + 256;
 constexpr size_t kSmemLimit = 232448;
 
 size_t win_smem_bytes(int ng, int ne, int heads, int L, bool bias)
@@ -439,23 +462,38 @@ int win_table_entries(const IexpC &c, bool bias)
     return (clamp < dmax ? clamp : dmax) + 1;
 }
 
-int win_groups(int ne, int heads, int L, bool bias)
+// groups per CTA that fit shared memory; the raw bias table (heads x (2w-1)^2 bytes) is
+// staged in the groups' B area during the set-up
+int win_groups(int ne, int heads, int L, int window, bool bias)
 {
+    const size_t tab = bias ? (size_t)heads * (2 * window - 1) * (2 * window - 1) : 0;
     for (int ng = WMAXG; ng >= 1; --ng)
-        if (win_smem_bytes(ng, ne, heads, L, bias) + kWinStaticSmem <= kSmemLimit) return ng;
+        if (win_smem_bytes(ng, ne, heads, L, bias) + kWinStaticSmem <= kSmemLimit && tab <= (size_t)ng * WB_BYTES)
+            return ng;
     return 0;
 }
 
 bool small_iexp_w(const IexpC &c) { return ((double)c.q_b * c.q_b + c.q_c) * 32768.0 < 268435456.0; }
 
+template <int D, bool BIAS, bool SMALL_E, int NQ>
+cudaError_t win_launch_q(const WinParams &p, size_t smem, int grid, cudaStream_t st)
+{
+    cudaError_t e = cudaFuncSetAttribute(lis_attn_win_kernel<D, BIAS, SMALL_E, NQ>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    lis_attn_win_kernel<D, BIAS, SMALL_E, NQ><<<grid, 128 * p.ng, smem, st>>>(p);
+    return cudaGetLastError();
+}
+
 template <int D, bool BIAS, bool SMALL_E>
 cudaError_t win_launch(const WinParams &p, size_t smem, int grid, cudaStream_t st)
 {
-    cudaError_t e = cudaFuncSetAttribute(lis_attn_win_kernel<D, BIAS, SMALL_E>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    lis_attn_win_kernel<D, BIAS, SMALL_E><<<grid, 128 * p.ng, smem, st>>>(p);
-    return cudaGetLastError();
+    switch ((p.L + 15) >> 4) {
+    case 1: return win_launch_q<D, BIAS, SMALL_E, 1>(p, smem, grid, st);
+    case 2: return win_launch_q<D, BIAS, SMALL_E, 2>(p, smem, grid, st);
+    case 3: return win_launch_q<D, BIAS, SMALL_E, 3>(p, smem, grid, st);
+    default: return win_launch_q<D, BIAS, SMALL_E, 4>(p, smem, grid, st);
+    }
 }
 
 template <int D>
@@ -476,7 +514,7 @@ bool lis_attention_win_eligible(const LisArgs &a, const AttnVArgs &b)
     if (b.ld_acc % 8 != 0 || ((uintptr_t)b.acc % 32) != 0) return false;
     const bool bias = a.bias != nullptr;
     const IexpC c = iexp_consts_host(a.s_logit);
-    return win_groups(win_table_entries(c, bias), a.heads, a.L, bias) > 0;
+    return win_groups(win_table_entries(c, bias), a.heads, a.L, a.window, bias) > 0;
 }
 
 cudaError_t launch_lis_attention_win(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
@@ -485,7 +523,7 @@ cudaError_t launch_lis_attention_win(const LisArgs &a, const AttnVArgs &b, cudaS
     WinParams p{a.logits, a.ld_logit, b.v, b.ld_v, b.acc, b.ld_acc, a.bias, a.heads, a.window, b.BH, a.L, b.zp_v,
                 iexp_consts_host(a.s_logit), 0, 0};
     p.ne = win_table_entries(p.ic, bias);
-    p.ng = win_groups(p.ne, a.heads, a.L, bias);
+    p.ng = win_groups(p.ne, a.heads, a.L, a.window, bias);
     const size_t smem = win_smem_bytes(p.ng, p.ne, a.heads, a.L, bias);
     const int64_t ntiles = (b.BH + 1) / 2;
     const int64_t want = (ntiles + p.ng - 1) / p.ng;
