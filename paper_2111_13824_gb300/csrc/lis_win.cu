@@ -21,7 +21,9 @@
 // r & 63 of its slot.  Per tile a thread takes its row into registers, adds
 // the bias, finds the maximum and the i-exp row sum, waits for the group's
 // previous MMAs, stores their accumulators, writes its operands and its V row,
-// and after a group barrier one thread issues the tile's MMAs.
+// and arrives on the group's mbarrier; the thread whose arrival count makes a
+// multiple of 128 issues the tile's MMAs once all arrivals are in, so no
+// thread waits for the group's slowest at a barrier.
 //
 // i-exp table: e(d) for the distance d = max - q~ in [0, ne), replicated for
 // each of the 32 lanes (one 256-byte line per d: 32 copies of e, then 32 of
@@ -68,18 +70,13 @@ struct WinParams {
 };
 
 struct WinShared {
-    uint64_t mmadone[WMAXG];
-    uint64_t fin[WMAXG];
+    uint64_t afull[WMAXG];    // a group's 128 threads wrote A and B and read D
+    uint64_t mmadone[WMAXG];  // the group's MMAs completed
+    uint32_t arrivals[WMAXG]; // arrivals so far: the one that makes a multiple of 128 issues the MMAs
+    int issued[WMAXG];        // tiles whose MMAs were issued
     uint32_t tmem;
     int abort_flag;
-    int stop[WMAXG][2];  // set (never cleared) when a wait of iteration parity [.][it & 1] gave up
 };
-
-__device__ __forceinline__ void group_bar(int g)
-{
-    __syncwarp();
-    asm volatile("bar.sync %0, 128;" ::"r"(1 + g) : "memory");
-}
 
 __device__ __forceinline__ uint32_t win_tmem_cols(int ng) { return ng == 1 ? 128u : ng == 2 ? 256u : 512u; }
 
@@ -126,9 +123,10 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
 
     if (tid == 0) {
         for (int k = 0; k < p.ng; ++k) {
+            mbar_init(&sh.afull[k], 128);
             mbar_init(&sh.mmadone[k], 1);
-            mbar_init(&sh.fin[k], 1);
-            sh.stop[k][0] = sh.stop[k][1] = 0;
+            sh.arrivals[k] = 0;
+            sh.issued[k] = 0;
         }
         sh.abort_flag = 0;
     }
@@ -161,8 +159,10 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
         int kof[4];
 #pragma unroll
         for (int b = 0; b < 4; ++b) kof[b] = 4 * wj + b < L ? koff[4 * wj + b] : -1;
-        int row = tid >> 4, hh = row / L, qi = row - hh * L;
-        for (; row < p.heads * L; row += rstep) {
+        const int nrows = p.heads * L;
+#pragma unroll 4
+        for (int row = tid >> 4; row < nrows; row += rstep) {
+            const int hh = row / L, qi = row - hh * L;
             const unsigned char *tab = Bs_all + hh * nb * nb + qbase[qi];
             uint32_t word = 0;
 #pragma unroll
@@ -170,7 +170,6 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
                 if (kof[b] >= 0) word |= (uint32_t)(((int)(int8_t)tab[-kof[b]] + 128) & 0xFF) << (8 * b);
             const int pc = (wj >> 2) ^ ((qi >> 1) & 3);
             *reinterpret_cast<uint32_t *>(BR + (size_t)row * WBIAS_ROW + 16 * pc + 4 * (wj & 3)) = word;
-            for (qi += rstep; qi >= L; qi -= L) ++hh;
         }
     }
     for (int x = tid; x < p.ne * 16; x += blockDim.x) {  // 16 bytes: 4 copies of e (parts 0-7) or fp32 e
@@ -192,6 +191,11 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
     tc_fence_after();
 
     const uint32_t tmem = sh.tmem;
+    const int ntiles = (int)((p.BH + 1) >> 1);  // BH <= 65535
+    const int BH = (int)p.BH;
+    const int gstride = (int)gridDim.x * p.ng;
+
+    {
     const uint32_t tD = tmem + 128u * (uint32_t)g + ((uint32_t)((warp & 3) * 32) << 16);  // this warp's lanes
     const uint32_t tA = tD + 64u;
     unsigned char *Bg = Bs_all + g * WB_BYTES;
@@ -204,19 +208,14 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
         cm[k] = n >= 4 ? 0xFFFFFFFFu : n <= 0 ? 0u : (0xFFFFFFFFu >> (32 - 8 * n));
     }
     // A starts as zeros: the other slot's columns and the own slot's keys past the last
-    // 16-key chunk are never written again
+    // 16-key chunk are never written again (the first arrival on afull comes after this)
     {
         const uint32_t z[8] = {0, 0, 0, 0, 0, 0, 0, 0};
 #pragma unroll
         for (int c = 0; c < 8; ++c) tmem_st8(tA + 8u * c, z);
         tmem_wait_st();
     }
-    tc_fence_before();
-    group_bar(g);
 
-    const int ntiles = (int)((p.BH + 1) >> 1);  // BH <= 65535
-    const int BH = (int)p.BH;
-    const int gstride = (int)gridDim.x * p.ng;
     const uint32_t cap2 = (uint32_t)(p.ne - 1) * 0x10001u;
     const int qi = i < L ? i : L - 1;  // bias row of this thread (rows past L read the last one)
     const int sw = (qi >> 1) & 3;
@@ -243,18 +242,15 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
         }
         int32_t *dst = p.acc + ((size_t)bh * L + i) * p.ld_acc;
 #pragma unroll
-        for (int hf = 0; hf < D / 16; ++hf) {
-            uint32_t va[16];
-            tmem_ld16(tD + 16u * hf, va);
+        for (int c = 0; c < D / 8; ++c) {
+            uint32_t va[8];
+            tmem_ld8(tD + 8u * c, va);
             tmem_wait_ld();
             if (ok) {
+                int v8[8];
 #pragma unroll
-                for (int c = 0; c < 2; ++c) {
-                    int v8[8];
-#pragma unroll
-                    for (int j = 0; j < 8; ++j) v8[j] = __float2int_rn(__uint_as_float(va[8 * c + j])) - zsum;
-                    stg256(dst + 16 * hf + 8 * c, v8);
-                }
+                for (int j = 0; j < 8; ++j) v8[j] = __float2int_rn(__uint_as_float(va[j])) - zsum;
+                stg256(dst + 8 * c, v8);
             }
         }
     };
@@ -349,83 +345,80 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
         }
 
         // ---- the previous tile's MMAs are done: its accumulators out, A and B free
-        bool ok = true;
         if (it > 0) {
-            ok = mbar_wait_warp(&sh.mmadone[g], (it - 1) & 1, abort_flag);
-            if (ok) {
-                tc_fence_after();
-                store_acc(prev);
+            if (!mbar_wait_warp(&sh.mmadone[g], (it - 1) & 1, abort_flag)) {
+                stopped = true;  // the abort flag is set: the other warps' waits end too
+                break;
+            }
+            tc_fence_after();
+            store_acc(prev);
+        }
+        // ---- operands 2^(15 - code) of this row's keys -> tensor memory (own slot), 16 keys at a
+        //      time; chunks past NQ keep the zeros of the start
+#pragma unroll
+        for (int c = 0; c < NQ; ++c) {
+            uint32_t o[8];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int j = 4 * c + k;
+                if (c == NQ - 1 && j >= nw) {
+                    o[2 * k] = o[2 * k + 1] = 0u;
+                    continue;
+                }
+                const uint32_t de = vp[2 * j], dod = vp[2 * j + 1];
+                const float f0 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5104u>(de, lane4));
+                const float f2 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5324u>(de, lane4));
+                const float f1 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5104u>(dod, lane4));
+                const float f3 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5324u>(dod, lane4));
+                const uint32_t E0 = operand_exp_tab(f0, rs.hibits, rs.hi, rs.lo, dk);
+                const uint32_t E1 = operand_exp_tab(f1, rs.hibits, rs.hi, rs.lo, dk);
+                const uint32_t E2 = operand_exp_tab(f2, rs.hibits, rs.hi, rs.lo, dk);
+                const uint32_t E3 = operand_exp_tab(f3, rs.hibits, rs.hi, rs.lo, dk);
+                o[2 * k] = (E0 << 10) | (E1 << 26);
+                o[2 * k + 1] = (E2 << 10) | (E3 << 26);
+            }
+            tmem_st8(tA + 32u * (uint32_t)h + 8u * c, o);
+        }
+        // ---- V key row i of this slot -> fp16 B (row 64 h + i, chunk ci at ci ^ (row & 7))
+        if (valid) {
+            const int kk = 64 * h + i;
+            unsigned char *brow = Bg + kk * 128;
+#pragma unroll
+            for (int c = 0; c < D / 16; ++c) {
+                const uint32_t x0 = vv[c].x ^ 0x80808080u, x1 = vv[c].y ^ 0x80808080u;
+                const uint32_t x2 = vv[c].z ^ 0x80808080u, x3 = vv[c].w ^ 0x80808080u;
+                uint4 lo, hi;
+                lo.x = i8x2_to_h2(x0, 0x5140);
+                lo.y = i8x2_to_h2(x0, 0x7362);
+                lo.z = i8x2_to_h2(x1, 0x5140);
+                lo.w = i8x2_to_h2(x1, 0x7362);
+                hi.x = i8x2_to_h2(x2, 0x5140);
+                hi.y = i8x2_to_h2(x2, 0x7362);
+                hi.z = i8x2_to_h2(x3, 0x5140);
+                hi.w = i8x2_to_h2(x3, 0x7362);
+                *reinterpret_cast<uint4 *>(brow + (((2 * c) ^ (kk & 7)) << 4)) = lo;
+                *reinterpret_cast<uint4 *>(brow + (((2 * c + 1) ^ (kk & 7)) << 4)) = hi;
             }
         }
-        if (ok) {
-            // ---- operands 2^(15 - code) of this row's keys -> tensor memory (own slot); chunks
-            //      past NQ keep the zeros written at the start
-#pragma unroll
-            for (int c = 0; c < NQ; ++c) {
-                uint32_t o[8];
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    const int j = 4 * c + k;
-                    if (c == NQ - 1 && j >= nw) {
-                        o[2 * k] = o[2 * k + 1] = 0u;
-                        continue;
-                    }
-                    const uint32_t de = vp[2 * j], dod = vp[2 * j + 1];
-                    const float f0 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5104u>(de, lane4));
-                    const float f2 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5324u>(de, lane4));
-                    const float f1 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5104u>(dod, lane4));
-                    const float f3 = *reinterpret_cast<const float *>(LUTB + 128 + lut_off<0x5324u>(dod, lane4));
-                    const uint32_t E0 = operand_exp_tab(f0, rs.hibits, rs.hi, rs.lo, dk);
-                    const uint32_t E1 = operand_exp_tab(f1, rs.hibits, rs.hi, rs.lo, dk);
-                    const uint32_t E2 = operand_exp_tab(f2, rs.hibits, rs.hi, rs.lo, dk);
-                    const uint32_t E3 = operand_exp_tab(f3, rs.hibits, rs.hi, rs.lo, dk);
-                    o[2 * k] = (E0 << 10) | (E1 << 26);
-                    o[2 * k + 1] = (E2 << 10) | (E3 << 26);
-                }
-                tmem_st8(tA + 32u * (uint32_t)h + 8u * c, o);
-            }
-            // ---- V key row i of this slot -> fp16 B (row 64 h + i, chunk ci at ci ^ (row & 7))
-            if (valid) {
-                const int kk = 64 * h + i;
-                unsigned char *brow = Bg + kk * 128;
-#pragma unroll
-                for (int c = 0; c < D / 16; ++c) {
-                    const uint32_t x0 = vv[c].x ^ 0x80808080u, x1 = vv[c].y ^ 0x80808080u;
-                    const uint32_t x2 = vv[c].z ^ 0x80808080u, x3 = vv[c].w ^ 0x80808080u;
-                    uint4 lo, hi;
-                    lo.x = i8x2_to_h2(x0, 0x5140);
-                    lo.y = i8x2_to_h2(x0, 0x7362);
-                    lo.z = i8x2_to_h2(x1, 0x5140);
-                    lo.w = i8x2_to_h2(x1, 0x7362);
-                    hi.x = i8x2_to_h2(x2, 0x5140);
-                    hi.y = i8x2_to_h2(x2, 0x7362);
-                    hi.z = i8x2_to_h2(x3, 0x5140);
-                    hi.w = i8x2_to_h2(x3, 0x7362);
-                    *reinterpret_cast<uint4 *>(brow + (((2 * c) ^ (kk & 7)) << 4)) = lo;
-                    *reinterpret_cast<uint4 *>(brow + (((2 * c + 1) ^ (kk & 7)) << 4)) = hi;
-                }
-            }
-            tmem_wait_st();
-        }
+        tmem_wait_st();
         fence_async_smem();
         tc_fence_before();
-        if (!ok) sh.stop[g][it & 1] = 1;
-        group_bar(g);
-        if (*(volatile int *)&sh.stop[g][it & 1]) {
-            stopped = true;
-            break;
-        }
-        if (r == 0) {
-            tc_fence_after();
-            const uint32_t dcol = tmem + 128u * (uint32_t)g, acol = dcol + 64u;
-            const uint32_t b0 = sa(Bg);
+        mbar_arrive(&sh.afull[g]);  // A, B written and D read: the tile's MMAs may go
+        if (atomicAdd(&sh.arrivals[g], 1u) % 128u == 127u) {
+            // the last thread to count issues the tile's MMAs once every arrival is in
+            if (mbar_wait(&sh.afull[g], (uint32_t)(it & 1), abort_flag)) {
+                tc_fence_after();
+                const uint32_t dcol = tmem + 128u * (uint32_t)g, acol = dcol + 64u;
+                const uint32_t b0 = sa(Bg);
 #pragma unroll
-            for (int kb = 0; kb < 2; ++kb)
+                for (int kb = 0; kb < 2; ++kb)
 #pragma unroll
-                for (int s = 0; s < 4; ++s)
-                    mma_f16_ta(dcol, acol + 32u * kb + 8u * s, smem_desc(b0 + kb * 8192 + 2048 * s, 1024, 1024),
-                               (kb | s) != 0);
-            mma_commit(&sh.mmadone[g]);
+                    for (int s2 = 0; s2 < 4; ++s2)
+                        mma_f16_ta(dcol, acol + 32u * kb + 8u * s2, smem_desc(b0 + kb * 8192 + 2048 * s2, 1024, 1024),
+                                   (kb | s2) != 0);
+                mma_commit(&sh.mmadone[g]);
+                sh.issued[g] = it + 1;
+            }
         }
         prev = t;
     }
@@ -435,10 +428,10 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
             store_acc(prev);
         }
     }
-    if (r == 0) {  // every MMA this group issued has completed before tensor memory is freed
-        mma_commit(&sh.fin[g]);
-        mbar_wait(&sh.fin[g], 0, abort_flag, false);
     }
+    // every MMA issued has completed before tensor memory is freed (after a timeout too)
+    __syncthreads();
+    if (tid < p.ng && sh.issued[tid] > 0) mbar_wait(&sh.mmadone[tid], (uint32_t)((sh.issued[tid] - 1) & 1), abort_flag, false);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
