@@ -7,7 +7,12 @@ resident in HBM (7.4 GB for ViT-L/384, far above the 129 MB L2, so no flush
 is needed between steps).  Calibration and quantization of the LayerNorm
 input are offline (setup), as in post-training quantization.
 
-Prints ONE JSON line (rank 0).  See the design doc for the byte model.
+Algorithmic bytes per layer: LayerNorm 2 bytes per element (int8 in and out)
+plus 9 bytes of per-channel parameters; attention 1 byte per logit, 1 per V
+element and 4 per int32 accumulator (the 4-bit codes stay on chip).  The K
+timed steps run as one CUDA graph (--no-graph: eager launches).
+
+Prints ONE JSON line (rank 0).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config vit_l384]
                   [--impl reference] [--no-e2e] [--no-cpu]
@@ -226,11 +231,51 @@ def bench_gpu(args):
             run_layer(fqvit, ly)
     torch.cuda.synchronize()
 
-    attn_events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                   for _ in range(args.steps * len(layers))]
-    ln_events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                 for _ in range(args.steps * len(layers))]
+    # The K timed steps go into one CUDA graph (launches and their timing events), so that
+    # the host's per-call enqueue cost stays out of the timed region; eager launches when the
+    # graph cannot be built (a PyTorch without external events, or a capture error).
+    use_graph = not args.no_graph
+    ev_kw = dict(enable_timing=True)
+    if use_graph:
+        try:
+            torch.cuda.Event(enable_timing=True, external=True)
+            ev_kw["external"] = True
+        except TypeError:
+            use_graph = False
+    attn_events = [(torch.cuda.Event(**ev_kw), torch.cuda.Event(**ev_kw)) for _ in range(args.steps * len(layers))]
+    ln_events = [(torch.cuda.Event(**ev_kw), torch.cuda.Event(**ev_kw)) for _ in range(args.steps * len(layers))]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def enqueue_steps():
+        k = 0
+        for _ in range(args.steps):
+            for ly in layers:
+                ln_events[k][0].record()
+                fqvit.ptf_layernorm(ly["xq"], ly["zp"], ly["alpha"], ly["gamma"], ly["beta"], ly["s_out"],
+                                    ly["zp_out"], out=ly["yq"])
+                ln_events[k][1].record()
+                attn_events[k][0].record()
+                fqvit.lis_attention(ly["logits"], ly["s_logit"], ly["v"], 0, acc=ly["acc"], bias=ly["bias"],
+                                    heads=ly["heads"], window=ly["window"])
+                attn_events[k][1].record()
+                k += 1
+
+    graph = None
+    if use_graph:
+        try:
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph):
+                enqueue_steps()
+            graph.replay()  # upload and one untimed pass
+            torch.cuda.synchronize()
+        except Exception as exc:  # noqa: BLE001 - any capture failure falls back to eager launches
+            print(f"bench: CUDA graph unavailable ({type(exc).__name__}: {exc}); eager launches", file=sys.stderr)
+            graph = None
+            torch.cuda.synchronize()
+            attn_events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                           for _ in range(args.steps * len(layers))]
+            ln_events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                         for _ in range(args.steps * len(layers))]
     clocks = ClockSampler(local)
     if ws > 1:
         torch.distributed.barrier()
@@ -238,18 +283,10 @@ def bench_gpu(args):
     clocks.start()
     time.sleep(0.3)  # let the sampler start before the timed region
     start.record()
-    k = 0
-    for _ in range(args.steps):
-        for ly in layers:
-            ln_events[k][0].record()
-            fqvit.ptf_layernorm(ly["xq"], ly["zp"], ly["alpha"], ly["gamma"], ly["beta"], ly["s_out"],
-                                ly["zp_out"], out=ly["yq"])
-            ln_events[k][1].record()
-            attn_events[k][0].record()
-            fqvit.lis_attention(ly["logits"], ly["s_logit"], ly["v"], 0, acc=ly["acc"], bias=ly["bias"],
-                                heads=ly["heads"], window=ly["window"])
-            attn_events[k][1].record()
-            k += 1
+    if graph is not None:
+        graph.replay()
+    else:
+        enqueue_steps()
     end.record()
     torch.cuda.synchronize()
     clk = clocks.stop()
@@ -307,14 +344,15 @@ def bench_gpu(args):
             "l2": f"inputs {step_bytes / 1e9:.2f} GB per step, larger than the 129 MB L2 (no flush)",
             "logit_sigma": args.sigma,
             "parallelism": f"replicas x{ws} (independent batches, no collective)",
+            "launch": "cuda_graph" if graph is not None else "eager",
         },
         "hbm_gbs": round(stack_gbs, 1),
         "hbm_frac": round(stack_gbs / peak, 4),
         "kernels": {
             "attention": {"gbs": round(attn_gbs, 1), "ms_per_launch": round(sum(attn_ms) / len(attn_ms), 5),
-                          "bytes_per_launch": ab[0]},
+                          "bytes_per_launch": round(sum(ab) / len(ab))},
             "layernorm": {"gbs": round(ln_gbs, 1), "ms_per_launch": round(sum(ln_ms) / len(ln_ms), 5),
-                          "bytes_per_launch": lb[0]},
+                          "bytes_per_launch": round(sum(lb) / len(lb))},
         },
         "roofline": {"kernel": dominant, "bound": "hbm", "achieved": round(dom_gbs, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(dom_gbs / peak, 4), "traffic": traffic,
@@ -477,6 +515,7 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--traffic", default=None, help="JSON {kernel: dram bytes per launch} from an ncu capture")
     ap.add_argument("--layers", type=int, default=0, help="time only the first N layers (profiling cases)")
+    ap.add_argument("--no-graph", action="store_true", help="launch the timed steps eagerly instead of as one CUDA graph")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

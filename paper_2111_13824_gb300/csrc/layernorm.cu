@@ -85,12 +85,6 @@ __device__ __forceinline__ uint32_t ln_fast(float gs, float bs, float r, float t
     return (uint32_t)__float_as_int(__fadd_rd(y, 12582912.0f)) & 0xFFu;
 }
 
-__device__ __forceinline__ float warp_sum_f(float v)
-{
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    return v;
-}
-
 // per-launch channel constants, computed by every block into shared memory
 __device__ void ln_prologue(const LnArgs &a, float *gs_s, float *bs_s, uint8_t *al_s, LnShared &sh)
 {
@@ -136,8 +130,10 @@ __device__ __forceinline__ bool ln_row_fast(const LnShared &sh, float r, float t
     return (sh.kappa + fabsf(t)) * 1.001f < 16384.0f * r;
 }
 
-// Vector path: C % 16 == 0, rows 16-byte aligned.  CPL = chunks per lane.
-template <int CPL>
+// Vector path: C % 16 == 0, rows 16-byte aligned.  A segment of S lanes (a power of two) serves
+// one row, so a warp carries 32 / S rows (short rows do not leave lanes idle); CPL = 16-byte
+// chunks per lane, chunk sl + S i of the row for segment lane sl.
+template <int S, int CPL>
 __global__ void __launch_bounds__(kWarps * 32)
     ln_vec_kernel(LnArgs a)
 {
@@ -148,23 +144,28 @@ __global__ void __launch_bounds__(kWarps * 32)
     __shared__ LnShared sh;
     ln_prologue(a, gs_s, bs_s, al_s, sh);
 
+    constexpr int RPW = 32 / S;  // rows per warp
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
+    const int sl = lane & (S - 1), seg = lane / S;
     const int nch = a.C >> 4;
     const float zh = (float)a.zp_out + 0.5f;
     const float Cf = (float)a.C;
 
-    const int64_t rstep = (int64_t)gridDim.x * kWarps;
-    int64_t row = (int64_t)blockIdx.x * kWarps + warp;
+    // every lane of a warp runs every iteration (the segment reductions are warp shuffles);
+    // rows past the end only skip their loads and stores
+    const int64_t rstep = (int64_t)gridDim.x * kWarps * RPW;
+    int64_t row = ((int64_t)blockIdx.x * kWarps + warp) * RPW + seg;
     // the row's 16-byte chunks, loaded one row ahead so that the HBM latency overlaps the work
     uint4 nv[CPL];
 #pragma unroll
     for (int i = 0; i < CPL; ++i) {
-        int ch = lane + 32 * i;
+        int ch = sl + S * i;
         nv[i] = (row < a.rows && ch < nch) ? __ldcs(reinterpret_cast<const uint4 *>(a.xq + row * a.ld_in) + ch)
                                            : make_uint4(0, 0, 0, 0);
     }
-    for (; row < a.rows; row += rstep) {
+    for (; row - seg < a.rows; row += rstep) {  // warp-uniform: the warp's first row is in range
+        const bool rv = row < a.rows;
         uint4 v[CPL];
 #pragma unroll
         for (int i = 0; i < CPL; ++i) v[i] = nv[i];
@@ -172,7 +173,7 @@ __global__ void __launch_bounds__(kWarps * 32)
             const uint4 *nsrc = reinterpret_cast<const uint4 *>(a.xq + (row + rstep) * a.ld_in);
 #pragma unroll
             for (int i = 0; i < CPL; ++i) {
-                int ch = lane + 32 * i;
+                int ch = sl + S * i;
                 if (ch < nch) nv[i] = __ldcs(nsrc + ch);
             }
         }
@@ -181,8 +182,8 @@ __global__ void __launch_bounds__(kWarps * 32)
         unsigned long long m2 = 0;
 #pragma unroll
         for (int i = 0; i < CPL; ++i) {
-            int ch = lane + 32 * i;
-            if (ch < nch) {
+            int ch = sl + S * i;
+            if (rv && ch < nch) {
                 uint4 al4 = *reinterpret_cast<const uint4 *>(al_s + ch * 16);
                 uint32_t w[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
                 uint32_t aw[4] = {al4.x, al4.y, al4.z, al4.w};
@@ -201,10 +202,12 @@ __global__ void __launch_bounds__(kWarps * 32)
                 m2 += p2;
             }
         }
-        for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+        for (int o = S / 2; o > 0; o >>= 1) {
             m1 += __shfl_xor_sync(0xffffffffu, m1, o);
             m2 += __shfl_xor_sync(0xffffffffu, m2, o);
         }
+        if (!rv) continue;
         long long M1 = m1, M2 = (long long)m2;
         long long D = (long long)a.C * M2 - M1 * M1;
         float r = 0.0f, t = 0.0f;
@@ -213,17 +216,17 @@ __global__ void __launch_bounds__(kWarps * 32)
             r = __fdiv_rn(Cf, sd);
             t = __fdiv_rn(__ll2float_rn(M1), sd);
         }
-        if (lane == 0) {
+        if (sl == 0) {
             if (a.m1) a.m1[row] = M1;
             if (a.m2) a.m2[row] = M2;
         }
-        const bool fast = ln_row_fast(sh, r, t);  // warp-uniform: one evaluation per row, chosen outside the loops
+        const bool fast = ln_row_fast(sh, r, t);  // one evaluation per row, chosen outside the loops
         uint4 *dst = reinterpret_cast<uint4 *>(a.yq + row * a.ld_out);
         // pass 2: requantization
         if (fast) {
 #pragma unroll
             for (int i = 0; i < CPL; ++i) {
-                int ch = lane + 32 * i;
+                int ch = sl + S * i;
                 if (ch < nch) {
                     uint4 al4 = *reinterpret_cast<const uint4 *>(al_s + ch * 16);
                     uint32_t w[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
@@ -250,7 +253,7 @@ __global__ void __launch_bounds__(kWarps * 32)
         } else {
 #pragma unroll
             for (int i = 0; i < CPL; ++i) {
-                int ch = lane + 32 * i;
+                int ch = sl + S * i;
                 if (ch < nch) {
                     uint32_t o0 = 0, o1 = 0, o2 = 0, o3 = 0;
 #pragma unroll 1
@@ -319,7 +322,7 @@ cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st)
     size_t smem = (size_t)a.C * (2 * sizeof(float) + 1);
     smem = (smem + 15) & ~(size_t)15;
     const int nsm = sm_count();
-    const int64_t want = (a.rows + kWarps - 1) / kWarps;
+    int64_t want = (a.rows + kWarps - 1) / kWarps;
     // Every block first derives the per-channel constants (three correctly rounded divisions per
     // channel), so the grid is the number of blocks that are resident at once: each block then
     // walks many rows.
@@ -334,26 +337,40 @@ cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st)
     bool vec = (a.C % 16 == 0) && (a.ld_in % 16 == 0) && (a.ld_out % 16 == 0) &&
                ((uintptr_t)a.xq % 16 == 0) && ((uintptr_t)a.yq % 16 == 0) && a.C <= 4096;
     if (vec) {
-        int cpl = (a.C / 16 + 31) / 32;
-        switch (cpl) {
-#define FQ_LN_CASE(N)                                                                      \
-    case N:                                                                                \
-        cudaFuncSetAttribute(ln_vec_kernel<N>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
-                             (int)smem);                                                   \
-        ln_vec_kernel<N><<<blocks_for((const void *)ln_vec_kernel<N>), kWarps * 32, smem, st>>>(a); \
-        return cudaGetLastError();
-            FQ_LN_CASE(1)
-            FQ_LN_CASE(2)
-            FQ_LN_CASE(3)
-            FQ_LN_CASE(4)
-            FQ_LN_CASE(5)
-            FQ_LN_CASE(6)
-            FQ_LN_CASE(7)
-            FQ_LN_CASE(8)
-#undef FQ_LN_CASE
-        default:
-            break;
+        // segment width: the smallest power of two lanes holding the row's 16-byte chunks, at most 32
+        const int nch = a.C / 16;
+        int S = 1;
+        while (S < nch && S < 32) S <<= 1;
+        const int cpl = (nch + S - 1) / S;
+        const int rpw = 32 / S;
+        want = (a.rows + (int64_t)kWarps * rpw - 1) / ((int64_t)kWarps * rpw);
+#define FQ_LN_LAUNCH(SS, N)                                                                      \
+    {                                                                                           \
+        cudaFuncSetAttribute(ln_vec_kernel<SS, N>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
+        ln_vec_kernel<SS, N><<<blocks_for((const void *)ln_vec_kernel<SS, N>), kWarps * 32, smem, st>>>(a); \
+        return cudaGetLastError();                                                              \
+    }
+        if (S < 32) {
+            switch (S) {
+            case 1: FQ_LN_LAUNCH(1, 1)
+            case 2: FQ_LN_LAUNCH(2, 1)
+            case 4: FQ_LN_LAUNCH(4, 1)
+            case 8: FQ_LN_LAUNCH(8, 1)
+            default: FQ_LN_LAUNCH(16, 1)
+            }
         }
+        switch (cpl) {
+        case 1: FQ_LN_LAUNCH(32, 1)
+        case 2: FQ_LN_LAUNCH(32, 2)
+        case 3: FQ_LN_LAUNCH(32, 3)
+        case 4: FQ_LN_LAUNCH(32, 4)
+        case 5: FQ_LN_LAUNCH(32, 5)
+        case 6: FQ_LN_LAUNCH(32, 6)
+        case 7: FQ_LN_LAUNCH(32, 7)
+        case 8: FQ_LN_LAUNCH(32, 8)
+        default: break;
+        }
+#undef FQ_LN_LAUNCH
     }
     cudaFuncSetAttribute(ln_generic_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     ln_generic_kernel<<<blocks_for((const void *)ln_generic_kernel), kWarps * 32, smem, st>>>(a);

@@ -123,6 +123,14 @@ def test_layernorm_matches_oracle(rows, C):
     _assert_ln(_ln_case(rows + C, rows, C))
 
 
+@pytest.mark.parametrize("rows,C", [(1001, 32), (777, 48), (513, 64), (2049, 80), (333, 128), (99, 256),
+                                    (50001, 96), (40003, 192), (7, 16), (3, 48)])
+def test_layernorm_rows_per_warp(rows, C):
+    """Short rows share a warp (a segment of lanes per row): every segment width, row counts
+    that leave the last warp partly empty, and enough rows for many passes per warp."""
+    _assert_ln(_ln_case(rows * 7 + C, rows, C))
+
+
 def test_layernorm_strided_rows():
     _assert_ln(_ln_case(5, 200, 192), ld_in=208, ld_out=224)
     _assert_ln(_ln_case(6, 200, 192), ld_in=193, ld_out=195)
