@@ -85,8 +85,14 @@ __device__ __forceinline__ uint32_t ln_fast(float gs, float bs, float r, float t
     return (uint32_t)__float_as_int(__fadd_rd(y, 12582912.0f)) & 0xFFu;
 }
 
-// per-launch channel constants, computed by every block into shared memory
-__device__ void ln_prologue(const LnArgs &a, float *gs_s, float *bs_s, uint8_t *al_s, LnShared &sh)
+// Shared-memory position of channel c's constants: the four 16-byte units of each 16-channel chunk
+// ch are permuted (unit q at q ^ ((ch >> 1) & 3)), so that eight lanes reading unit q of eight
+// consecutive chunks touch eight different bank groups.  A permutation of 0 .. C-1 for C % 16 == 0;
+// the vector path uses it, the generic path (any C) the identity.
+__device__ __forceinline__ int ln_sidx(int c) { return (c & ~15) + ((((c >> 2) & 3) ^ ((c >> 5) & 3)) << 2) + (c & 3); }
+
+// per-launch channel constants, computed by every block into shared memory (swizzled: ln_sidx)
+__device__ void ln_prologue(const LnArgs &a, float *gs_s, float *bs_s, uint8_t *al_s, LnShared &sh, bool swz)
 {
     if (threadIdx.x == 0) {
         sh.gsmax = 0.0f;
@@ -100,8 +106,9 @@ __device__ void ln_prologue(const LnArgs &a, float *gs_s, float *bs_s, uint8_t *
     for (int c = threadIdx.x; c < a.C; c += blockDim.x) {
         float gs = __fdiv_rn(a.gamma[c], a.s_out);
         float bs = __fdiv_rn(a.beta[c], a.s_out);
-        gs_s[c] = gs;
-        bs_s[c] = bs;
+        const int sc = swz ? ln_sidx(c) : c;
+        gs_s[sc] = gs;
+        bs_s[sc] = bs;
         int al = a.alpha[c];
         al_s[c] = (uint8_t)al;
         amax = max(amax, al);
@@ -142,7 +149,7 @@ __global__ void __launch_bounds__(kWarps * 32)
     float *bs_s = gs_s + a.C;
     uint8_t *al_s = reinterpret_cast<uint8_t *>(bs_s + a.C);
     __shared__ LnShared sh;
-    ln_prologue(a, gs_s, bs_s, al_s, sh);
+    ln_prologue(a, gs_s, bs_s, al_s, sh, true);
 
     constexpr int RPW = 32 / S;  // rows per warp
     const int lane = threadIdx.x & 31;
@@ -234,9 +241,10 @@ __global__ void __launch_bounds__(kWarps * 32)
                     uint32_t o[4] = {0, 0, 0, 0};
                     const float4 *g4 = reinterpret_cast<const float4 *>(gs_s + ch * 16);
                     const float4 *b4 = reinterpret_cast<const float4 *>(bs_s + ch * 16);
+                    const int qs = (ch >> 1) & 3;
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
-                        float4 g = g4[q], b = b4[q];
+                        float4 g = g4[q ^ qs], b = b4[q ^ qs];
                         float gg[4] = {g.x, g.y, g.z, g.w};
                         float bb[4] = {b.x, b.y, b.z, b.w};
 #pragma unroll
@@ -262,7 +270,8 @@ __global__ void __launch_bounds__(kWarps * 32)
                         const uint32_t wk = k < 8 ? (k < 4 ? v[i].x : v[i].y) : (k < 12 ? v[i].z : v[i].w);
                         int x = (wk >> (8 * (k & 3))) & 0xFF;
                         int xh = (x - a.zp_in) << al_s[c];
-                        const uint32_t y = (uint32_t)ln_exact(gs_s[c], bs_s[c], r, t, xh, a.zp_out) << (8 * (k & 3));
+                        const int sc = ln_sidx(c);
+                        const uint32_t y = (uint32_t)ln_exact(gs_s[sc], bs_s[sc], r, t, xh, a.zp_out) << (8 * (k & 3));
                         if (k < 4) o0 |= y; else if (k < 8) o1 |= y; else if (k < 12) o2 |= y; else o3 |= y;
                     }
                     __stcs(dst + ch, make_uint4(o0, o1, o2, o3));
@@ -280,7 +289,7 @@ __global__ void __launch_bounds__(kWarps * 32) ln_generic_kernel(LnArgs a)
     float *bs_s = gs_s + a.C;
     uint8_t *al_s = reinterpret_cast<uint8_t *>(bs_s + a.C);
     __shared__ LnShared sh;
-    ln_prologue(a, gs_s, bs_s, al_s, sh);
+    ln_prologue(a, gs_s, bs_s, al_s, sh, false);
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     for (int64_t row = (int64_t)blockIdx.x * kWarps + warp; row < a.rows;
