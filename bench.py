@@ -66,16 +66,16 @@ def attn_bytes(BH, L, d):
     return BH * (L * L + L * d + 4 * L * d)
 
 
-def recorded_traffic(kernel):
-    """DRAM bytes per launch from the committed ncu record, if the kernel's sources
-    are unchanged since that capture (else None)."""
+def recorded_traffic(config, kernel):
+    """DRAM bytes per launch (mean over the step's layers) from the committed ncu record of this
+    config, if the kernel's sources are unchanged since that capture (else None)."""
     import hashlib
 
     path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
-        rec = json.load(f).get(kernel)
+        rec = json.load(f).get(config, {}).get(kernel)
     if not rec:
         return None
     h = hashlib.sha256()
@@ -311,7 +311,7 @@ def bench_gpu(args):
     stack_gbs = step_bytes / (ms_per_step / 1e3) / 1e9
     dominant = "attention" if sum(attn_ms) >= sum(ln_ms) else "layernorm"
     dom_gbs = attn_gbs if dominant == "attention" else ln_gbs
-    traffic = recorded_traffic(dominant)
+    traffic = recorded_traffic(args.config, dominant)
     if args.traffic:
         traffic = json.loads(args.traffic).get(dominant)
 
