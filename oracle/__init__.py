@@ -62,6 +62,8 @@ def _load():
     lib.or_lis_softmax.argtypes = [P, i64, i32, i64, f32, i32, P, i32, i32, P, i64, P]
     lib.or_lis_softmax.restype = ctypes.c_int
     lib.or_lis_attn_v.argtypes = [P, i64, P, i64, i32, i64, i32, i32, P, i64]
+    lib.or_attn_requant.restype = ctypes.c_int
+    lib.or_attn_requant.argtypes = [P, i64, i32, i64, f32, f32, i32, P, i64]
     lib.or_lis_attn_v.restype = ctypes.c_int
     lib.or_num_threads.argtypes = []
     lib.or_num_threads.restype = ctypes.c_int
@@ -242,3 +244,16 @@ def lis_attn_v(codes: np.ndarray, v: np.ndarray, zp_v: int = 0):
     if rc not in (0, 3):
         raise ValueError("or_lis_attn_v rejected its arguments")
     return acc, rc == 3
+
+
+def attn_requant(acc: np.ndarray, s_v: float, s_out: float, zp_out: int) -> np.ndarray:
+    """8-bit requantization of the attention output (Eq. 3 with the dyadic multiplier of the
+    LayerNorm output stage): int32 [..., d] -> uint8 [..., d]."""
+    acc = _c(acc, np.int32)
+    d = acc.shape[-1]
+    rows = acc.size // d
+    y = np.zeros(acc.shape, np.uint8)
+    rc = _load().or_attn_requant(_ptr(acc), rows, d, d, float(s_v), float(s_out), int(zp_out), _ptr(y), d)
+    if rc != 0:
+        raise ValueError("or_attn_requant rejected its arguments")
+    return y

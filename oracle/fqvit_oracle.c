@@ -407,6 +407,51 @@ OR_EXPORT int or_lis_softmax(const int8_t *logits, int64_t n_rows, int32_t L, in
 }
 
 /* ------------------------------------------------------------------ */
+/* 8-bit requantization of the attention output                        */
+/* ------------------------------------------------------------------ */
+
+/*
+ * The attention output acc (real value acc * s_v / 2^15, Eq. 15) quantized to
+ * the next layer's 8-bit activation (Eq. 3: scale s_out, zero point zp_out),
+ * with the dyadic multiplier of the supplement's LayerNorm output stage (the
+ * requantization with A = M, B = 0):
+ *   M  = (s_v / s_out) / 2^15        (one fp32 division, then an exact scaling)
+ *   N1 = 7 - floor(log2 M)  (at most 31),   N2 = floor(M 2^N1)
+ *   y  = clip(floor((N2 acc + 2^(N1-1)) / 2^N1) + zp_out, 0, 255)   for N1 > 0
+ *   y  = clip(N2 acc 2^min(-N1, 10) + zp_out, 0, 255)                for N1 <= 0
+ * The readings are those of or_ptf_layernorm: the division by 2^N1 rounds half
+ * up (floor of the value plus one half), the result is clipped to 8 bits.
+ * acc [rows][ld_acc] (d values per row), y [rows][ld_y].
+ */
+OR_EXPORT int or_attn_requant(const int32_t *acc, int64_t rows, int32_t d, int64_t ld_acc, float s_v, float s_out,
+                              int32_t zp_out, uint8_t *y, int64_t ld_y)
+{
+    if (!acc || !y || rows < 1 || d < 1 || !(s_v > 0.0f) || !(s_out > 0.0f)) return 1;
+    const float M = ldexpf(s_v / s_out, -15);
+    if (!(M > 0.0f)) return 1;
+    int N1 = 7 - ilogbf(M);
+    if (N1 > 31) N1 = 31;
+    const int64_t N2 = (int64_t)floorf(ldexpf(M, N1));
+    for (int64_t r = 0; r < rows; ++r) {
+        for (int32_t t = 0; t < d; ++t) {
+            const int64_t num = N2 * (int64_t)acc[r * ld_acc + t];
+            int64_t R;
+            if (N1 > 0)
+                R = floor_div_pow2(num + ((int64_t)1 << (N1 - 1)), N1);
+            else if (N1 == 0)
+                R = num;
+            else {
+                int sh = -N1;
+                if (sh > 10) sh = 10;
+                R = num * ((int64_t)1 << sh);
+            }
+            y[r * ld_y + t] = (uint8_t)clamp_i64(R + zp_out, 0, 255);
+        }
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
 /* Eq. 15 and the supplement's Attn.V: BitShift attention times values */
 /* ------------------------------------------------------------------ */
 
