@@ -246,6 +246,27 @@ FQVIT_API int fqvit_lis_attention(const int8_t *logits, int64_t ld_logit, float 
                         int32_t *acc, int64_t ld_acc, uint8_t *codes_opt, int64_t ld_codes,
                         void *stream);
 
+/*
+ * The fused attention with its output requantized to 8 bits for the next
+ * layer (the activation quantizer of Eq. 3, scale s_out, zero point zp_out),
+ * evaluated with the dyadic multiplier of the supplement's LayerNorm output
+ * stage: the real output acc * s_v / 2^15 (Eq. 15) becomes
+ *   M  = (s_v / s_out) / 2^15   (one fp32 division, then an exact scaling),
+ *   N1 = 7 - floor(log2 M) (at most 31),  N2 = floor(M 2^N1)  (8 bits),
+ *   out = clip(floor((N2 acc + 2^(N1-1)) / 2^N1) + zp_out, 0, 255)  (N1 > 0),
+ *   out = clip(N2 acc 2^min(-N1, 10) + zp_out, 0, 255)             (N1 <= 0).
+ * The int32 accumulators are not written.  out: uint8 [BH][L][ld_out]
+ * (device, caller-owned), ld_out >= d.  Other arguments as in
+ * fqvit_lis_attention.  Errors: INVALID_ARG for a NULL out, ld_out < d,
+ * s_v or s_out not positive and finite, zp_out outside 0..255; UNSUPPORTED
+ * when M leaves the fp32 range; otherwise as fqvit_lis_attention.
+ */
+FQVIT_API int fqvit_lis_attention_q(const int8_t *logits, int64_t ld_logit, float s_logit,
+                          int32_t n_shift, const fqvit_relpos_bias *bias_opt, const int8_t *v,
+                          int64_t ld_v, int32_t zp_v, int64_t BH, int32_t L, int32_t d,
+                          float s_v, float s_out, int32_t zp_out, uint8_t *out, int64_t ld_out,
+                          void *stream);
+
 /* ------------------------------------------------------------------ */
 /* One layer: norm1 LayerNorm and the attention core (Fig. 4 dataflow) */
 /* ------------------------------------------------------------------ */

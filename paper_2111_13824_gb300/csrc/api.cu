@@ -241,16 +241,17 @@ int fqvit_lis_softmax(const int8_t *logits, int64_t n_rows, int32_t L, int64_t l
     return cuda_status(fqvit::launch_lis_softmax(a, as_stream(stream)), "lis_softmax");
 }
 
+// acc == nullptr with need_acc false: the output is checked by the caller (8-bit path)
 static int check_attnv(const int8_t *v, int64_t ld_v, int32_t zp_v, int64_t BH, int32_t L, int32_t d,
-                       const int32_t *acc, int64_t ld_acc, const char *who)
+                       const int32_t *acc, int64_t ld_acc, const char *who, bool need_acc = true)
 {
-    if (!v || !acc) return fail(FQVIT_ERR_INVALID_ARG, "%s: NULL pointer", who);
+    if (!v || (need_acc && !acc)) return fail(FQVIT_ERR_INVALID_ARG, "%s: NULL pointer", who);
     if (BH < 1 || L < 1 || BH > 65535) return fail(FQVIT_ERR_INVALID_ARG, "%s: bad shape BH=%lld L=%d", who, (long long)BH, L);
     if (L > 1024) return fail(FQVIT_ERR_UNSUPPORTED, "%s: L=%d (at most 1024)", who, L);
     if (d != 32 && d != 64) return fail(FQVIT_ERR_UNSUPPORTED, "%s: d=%d (32 or 64)", who, d);
-    if (ld_v < d || ld_acc < d) return fail(FQVIT_ERR_INVALID_ARG, "%s: stride below d", who);
+    if (ld_v < d || (need_acc && ld_acc < d)) return fail(FQVIT_ERR_INVALID_ARG, "%s: stride below d", who);
     if (zp_v < -255 || zp_v > 255) return fail(FQVIT_ERR_UNSUPPORTED, "%s: |zp_v| > 255", who);
-    if (!aligned(acc, 4)) return fail(FQVIT_ERR_INVALID_ARG, "%s: misaligned acc", who);
+    if (need_acc && !aligned(acc, 4)) return fail(FQVIT_ERR_INVALID_ARG, "%s: misaligned acc", who);
     return FQVIT_OK;
 }
 
@@ -280,6 +281,38 @@ int fqvit_lis_attention(const int8_t *logits, int64_t ld_logit, float s_logit, i
                       bias_opt ? bias_opt->window : 0, codes_opt, ld_codes, nullptr};
     fqvit::AttnVArgs a{nullptr, 0, v, ld_v, zp_v, BH, L, d, acc, ld_acc, nullptr};
     return cuda_status(fqvit::launch_lis_attention(la, a, as_stream(stream)), "lis_attention");
+}
+
+int fqvit_lis_attention_q(const int8_t *logits, int64_t ld_logit, float s_logit, int32_t n_shift,
+                          const fqvit_relpos_bias *bias_opt, const int8_t *v, int64_t ld_v, int32_t zp_v,
+                          int64_t BH, int32_t L, int32_t d, float s_v, float s_out, int32_t zp_out, uint8_t *out,
+                          int64_t ld_out, void *stream)
+{
+    if (!out) return fail(FQVIT_ERR_INVALID_ARG, "lis_attention_q: NULL output");
+    if (ld_out < d) return fail(FQVIT_ERR_INVALID_ARG, "lis_attention_q: ld_out < d");
+    if (!(s_v > 0.0f) || !(s_v < 3.0e38f) || !(s_out > 0.0f) || !(s_out < 3.0e38f))
+        return fail(FQVIT_ERR_INVALID_ARG, "lis_attention_q: s_v and s_out must be positive and finite");
+    if (zp_out < 0 || zp_out > 255) return fail(FQVIT_ERR_INVALID_ARG, "lis_attention_q: zp_out outside 0..255");
+    // the multiplier M = (s_v / s_out) / 2^15 as N2 / 2^N1 with 8 significant bits
+    const float M = ldexpf(s_v / s_out, -15);
+    if (!(M > 0.0f) || !(M < 1.0e30f)) return fail(FQVIT_ERR_UNSUPPORTED, "lis_attention_q: s_v / s_out out of range");
+    int n1 = 7 - ilogbf(M);
+    if (n1 > 31) n1 = 31;
+    const int n2 = (int)floorf(ldexpf(M, n1));
+    int rc = check_attnv(v, ld_v, zp_v, BH, L, d, nullptr, 0, "lis_attention_q", false);
+    if (rc) return rc;
+    rc = check_lis(logits, BH * L, L, ld_logit, s_logit, n_shift, bias_opt, "lis_attention_q");
+    if (rc) return rc;
+    fqvit::LisArgs la{logits, BH * L, L, ld_logit, s_logit,
+                      bias_opt ? bias_opt->table : nullptr, bias_opt ? bias_opt->heads : 1,
+                      bias_opt ? bias_opt->window : 0, nullptr, 0, nullptr};
+    fqvit::AttnVArgs a{nullptr, 0, v, ld_v, zp_v, BH, L, d, nullptr, 0, nullptr};
+    a.out8 = out;
+    a.ld_out8 = ld_out;
+    a.rq_n1 = n1 < -10 ? -10 : n1;
+    a.rq_n2 = n2;
+    a.rq_zp = zp_out;
+    return cuda_status(fqvit::launch_lis_attention(la, a, as_stream(stream)), "lis_attention_q");
 }
 
 int fqvit_block_int(const fqvit_block_desc *b, void *stream)

@@ -95,6 +95,13 @@ struct AttnVArgs {
     int32_t *acc;
     int64_t ld_acc;
     int32_t *range_flag;
+    // 8-bit output instead of acc (fused attention only): y = clip(((n2 acc + 2^(n1-1)) >> n1)
+    // + zp, 0, 255) for n1 > 0, clip(n2 acc 2^-n1 + zp, 0, 255) for -10 <= n1 <= 0
+    uint8_t *out8 = nullptr;
+    int64_t ld_out8 = 0;
+    int rq_n1 = 0;
+    int rq_n2 = 0;
+    int rq_zp = 0;
 };
 cudaError_t launch_lis_attn_v(const AttnVArgs &a, cudaStream_t st);
 

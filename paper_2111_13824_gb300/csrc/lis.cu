@@ -229,6 +229,12 @@ __global__ void __launch_bounds__(256) lis_attention_kernel(LisArgs la, AttnVArg
     int acc[CPT];
     long long wsum;
     attnv_row<CPT>(cs + r * ldc, vs, a.L, a.d, g * CPT, a.zp_v, acc, wsum);
+    if (a.out8) {  // 8-bit output for the next layer instead of the accumulators
+        uint8_t *d8 = a.out8 + (bh * a.L + row) * a.ld_out8 + g * CPT;
+#pragma unroll
+        for (int k = 0; k < CPT; ++k) d8[k] = (uint8_t)requant8(acc[k], a.rq_n1, a.rq_n2, a.rq_zp);
+        return;
+    }
     int32_t *dst = a.acc + (bh * a.L + row) * a.ld_acc + g * CPT;
 #pragma unroll
     for (int k = 0; k < CPT; ++k) dst[k] = acc[k];

@@ -72,6 +72,16 @@ __device__ __forceinline__ uint32_t lis_code(uint32_t e, const RowSum &rs)
     return (uint32_t)(k - 1 + (t <= rs.lo ? 1 : 0));
 }
 
+// 8-bit requantization of an attention accumulator by the dyadic multiplier n2 / 2^n1 (n1 in
+// [-10, 31]; the division rounds half up), plus the zero point, clipped to 0 .. 255
+__device__ __forceinline__ uint32_t requant8(int acc, int n1, int n2, int zp)
+{
+    const long long num = (long long)n2 * acc;
+    long long R = n1 > 0 ? (num + (1LL << (n1 - 1))) >> n1 : num * (1LL << -n1);
+    R += zp;
+    return (uint32_t)(R < 0 ? 0 : (R > 255 ? 255 : R));
+}
+
 __device__ __forceinline__ int relpos_idx(int i, int j, int w)
 {
     int yi = i / w, xi = i - yi * w, yj = j / w, xj = j - yj * w;

@@ -61,6 +61,9 @@ struct TcParams {
     int L;
     int zp;  // zero point of V (acc = sum_j 2^(15-code) (V - zp))
     IexpC ic;  // Algorithm 1 constants of the scale
+    uint8_t *out8;  // when not null: 8-bit outputs (requant8 with n1, n2, zp8) instead of acc
+    int64_t ld_out8;
+    int n1, n2, zp8;
 };
 
 constexpr int TPARTS = 4;                         // threads per query row
@@ -485,7 +488,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
             if (ok) {
                 tc_fence_after();
                 const int row = r0 + 32 * eq + lane;
-                int32_t *dst = p.acc + ((size_t)bh * L + row) * TD;
+                int32_t *dst = p.out8 ? nullptr : p.acc + ((size_t)bh * L + row) * TD;
                 // zp (sum_j 2^(15-code_j)), an exact integer below 2^24 times |zp| <= 255
                 int zsum = 0;
                 if (p.zp != 0) {
@@ -499,7 +502,20 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                     uint32_t va[32];
                     tmem_ld32(etl + 32 * h, va);
                     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-                    if (row < L) {
+                    if (row < L && p.out8) {  // 8-bit outputs: 32 bytes of this half of the row
+                        uint32_t wq[8];
+#pragma unroll
+                        for (int c = 0; c < 8; ++c) {
+                            wq[c] = 0;
+#pragma unroll
+                            for (int k = 0; k < 4; ++k)
+                                wq[c] |= requant8(__float2int_rn(__uint_as_float(va[4 * c + k])) - zsum, p.n1, p.n2,
+                                                  p.zp8) << (8 * k);
+                        }
+                        uint4 *d8 = reinterpret_cast<uint4 *>(p.out8 + ((size_t)bh * L + row) * p.ld_out8 + 32 * h);
+                        d8[0] = make_uint4(wq[0], wq[1], wq[2], wq[3]);
+                        d8[1] = make_uint4(wq[4], wq[5], wq[6], wq[7]);
+                    } else if (row < L) {
 #pragma unroll
                         for (int c = 0; c < 4; ++c) {
                             int v8[8];
@@ -562,15 +578,17 @@ bool small_iexp(const IexpC &c) { return ((double)c.q_b * c.q_b + c.q_c) * 32768
 
 bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
 {
+    const bool out_ok = b.out8 ? (b.ld_out8 % 16 == 0 && ((uintptr_t)b.out8 % 16) == 0)
+                               : (b.ld_acc == TD && ((uintptr_t)b.acc % 32) == 0);
     return b.d == TD && a.bias == nullptr && a.codes == nullptr && a.L <= TMAXKB * TKB &&
-           a.ld_logit % 16 == 0 && b.ld_v == TD && b.ld_acc == TD && ((uintptr_t)a.logits % 16) == 0 &&
-           ((uintptr_t)b.v % 16) == 0 && ((uintptr_t)b.acc % 32) == 0 &&
-           tc_smem_bytes(a.L, a.ld_logit) + kTcStaticSmem <= 232448;
+           a.ld_logit % 16 == 0 && b.ld_v == TD && out_ok && ((uintptr_t)a.logits % 16) == 0 &&
+           ((uintptr_t)b.v % 16) == 0 && tc_smem_bytes(a.L, a.ld_logit) + kTcStaticSmem <= 232448;
 }
 
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
 {
-    TcParams p{a.logits, a.ld_logit, a.s_logit, b.v, b.acc, b.BH, a.L, b.zp_v, iexp_consts_host(a.s_logit)};
+    TcParams p{a.logits, a.ld_logit, a.s_logit, b.v, b.acc, b.BH, a.L, b.zp_v, iexp_consts_host(a.s_logit),
+               b.out8, b.ld_out8, b.rq_n1, b.rq_n2, b.rq_zp};
     const size_t smem = tc_smem_bytes(a.L, a.ld_logit);
     const int64_t ntiles = b.BH * ((a.L + TM - 1) / TM);
     const int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());

@@ -67,6 +67,9 @@ struct WinParams {
     IexpC ic;
     int ne;  // table entries: distances 0 .. ne - 1
     int ng;  // groups per CTA
+    uint8_t *out8;  // when not null: 8-bit outputs (requant8 with n1, n2, zp8) instead of acc
+    int64_t ld_out8;
+    int n1, n2, zp8;
 };
 
 struct WinShared {
@@ -240,17 +243,24 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
             tmem_wait_ld();
             zsum = p.zp * __float2int_rn(__uint_as_float(x));
         }
-        int32_t *dst = p.acc + ((size_t)bh * L + i) * p.ld_acc;
 #pragma unroll
         for (int c = 0; c < D / 8; ++c) {
             uint32_t va[8];
             tmem_ld8(tD + 8u * c, va);
             tmem_wait_ld();
-            if (ok) {
+            if (ok && p.out8) {  // 8 bytes of 8-bit outputs
+                uint32_t lo = 0, hi = 0;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    lo |= requant8(__float2int_rn(__uint_as_float(va[j])) - zsum, p.n1, p.n2, p.zp8) << (8 * j);
+                    hi |= requant8(__float2int_rn(__uint_as_float(va[4 + j])) - zsum, p.n1, p.n2, p.zp8) << (8 * j);
+                }
+                *reinterpret_cast<uint2 *>(p.out8 + ((size_t)bh * L + i) * p.ld_out8 + 8 * c) = make_uint2(lo, hi);
+            } else if (ok) {
                 int v8[8];
 #pragma unroll
                 for (int j = 0; j < 8; ++j) v8[j] = __float2int_rn(__uint_as_float(va[j])) - zsum;
-                stg256(dst + 8 * c, v8);
+                stg256(p.acc + ((size_t)bh * L + i) * p.ld_acc + 8 * c, v8);
             }
         }
     };
@@ -504,7 +514,9 @@ bool lis_attention_win_eligible(const LisArgs &a, const AttnVArgs &b)
     if (!(b.d == 32 || (b.d == 64 && b.zp_v == 0))) return false;
     if (a.ld_logit % 16 != 0 || ((uintptr_t)a.logits % 16) != 0) return false;
     if (b.ld_v % 16 != 0 || ((uintptr_t)b.v % 16) != 0) return false;
-    if (b.ld_acc % 8 != 0 || ((uintptr_t)b.acc % 32) != 0) return false;
+    if (b.out8 ? (b.ld_out8 % 8 != 0 || ((uintptr_t)b.out8 % 8) != 0)
+               : (b.ld_acc % 8 != 0 || ((uintptr_t)b.acc % 32) != 0))
+        return false;
     const bool bias = a.bias != nullptr;
     const IexpC c = iexp_consts_host(a.s_logit);
     return win_groups(win_table_entries(c, bias), a.heads, a.L, a.window, bias) > 0;
@@ -514,7 +526,7 @@ cudaError_t launch_lis_attention_win(const LisArgs &a, const AttnVArgs &b, cudaS
 {
     const bool bias = a.bias != nullptr;
     WinParams p{a.logits, a.ld_logit, b.v, b.ld_v, b.acc, b.ld_acc, a.bias, a.heads, a.window, b.BH, a.L, b.zp_v,
-                iexp_consts_host(a.s_logit), 0, 0};
+                iexp_consts_host(a.s_logit), 0, 0, b.out8, b.ld_out8, b.rq_n1, b.rq_n2, b.rq_zp};
     p.ne = win_table_entries(p.ic, bias);
     p.ng = win_groups(p.ne, a.heads, a.L, a.window, bias);
     const size_t smem = win_smem_bytes(p.ng, p.ne, a.heads, a.L, bias);

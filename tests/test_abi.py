@@ -76,3 +76,18 @@ def test_relpos_bias_checks(lib):
     assert lib.fqvit_lis_softmax(fake, 3 * 49, 49, 64, 0.05, 15, ctypes.byref(bad), fake, 25, None, None) == 1
     b2 = fqvit.RelposBias(fake, 4, 7)
     assert lib.fqvit_lis_softmax(fake, 3 * 49, 49, 64, 0.05, 15, ctypes.byref(b2), fake, 25, None, None) == 1
+
+
+def test_requantized_attention_checks(lib):
+    """fqvit_lis_attention_q rejects bad output arguments before any launch."""
+    fake = ctypes.c_void_p(4096)
+    args = lambda s_v, s_out, zp, out, ld: lib.fqvit_lis_attention_q(  # noqa: E731
+        fake, 208, 0.05, 15, None, fake, 64, 0, 2, 197, 64, s_v, s_out, zp, out, ld, None)
+    assert args(0.05, 0.02, 0, None, 64) == 1
+    assert "NULL" in _err(lib)
+    assert args(0.05, 0.02, 0, fake, 32) == 1          # ld_out < d
+    assert args(0.0, 0.02, 0, fake, 64) == 1           # s_v not positive
+    assert args(0.05, float("inf"), 0, fake, 64) == 1  # s_out not finite
+    assert args(0.05, 0.02, 256, fake, 64) == 1        # zp_out outside 0..255
+    assert "zp_out" in _err(lib)
+    assert args(1e30, 1e-30, 0, fake, 64) == 2         # M leaves the fp32 range
