@@ -61,9 +61,13 @@ def ln_bytes(rows, C):
     return 2 * rows * C + 9 * C
 
 
-def attn_bytes(BH, L, d):
-    """Algorithmic bytes of one fused attention launch: 1 B / logit + 1 B / V element + 4 B / acc element."""
-    return BH * (L * L + L * d + 4 * L * d)
+OUT8_SV = 1.0 / 127.0  # V's scale for the 8-bit output option (any value: the work is the same)
+
+
+def attn_bytes(BH, L, d, out_bytes=4):
+    """Algorithmic bytes of one fused attention launch: 1 B / logit + 1 B / V element + 4 B / acc element
+    (1 B / output element with the 8-bit requantized output)."""
+    return BH * (L * L + L * d + out_bytes * L * d)
 
 
 def recorded_traffic(config, kernel):
@@ -103,6 +107,7 @@ def make_layers(cfg, device, sigma=1.0, limit=0):
             yq=torch.empty_like(xq), logits=a["logits"], s_logit=a["s_logit"], v=a["v"], bias=a["bias"],
             heads=a["heads"], window=a["window"],
             acc=torch.empty(a["BH"], a["L"], a["d"], dtype=torch.int32, device=device),
+            out8=torch.empty(a["BH"], a["L"], a["d"], dtype=torch.uint8, device=device),
             rows=st.rows, C=st.C, BH=st.BH, L=st.L, d=st.d))
         del d, a
     torch.cuda.synchronize()
@@ -255,8 +260,12 @@ def bench_gpu(args):
                                     ly["zp_out"], out=ly["yq"])
                 ln_events[k][1].record()
                 attn_events[k][0].record()
-                fqvit.lis_attention(ly["logits"], ly["s_logit"], ly["v"], 0, acc=ly["acc"], bias=ly["bias"],
-                                    heads=ly["heads"], window=ly["window"])
+                if args.out8:  # the output requantized to 8 bits (output scale = V's: M = 2^-15)
+                    fqvit.lis_attention_q(ly["logits"], ly["s_logit"], ly["v"], 0, OUT8_SV, OUT8_SV, 128,
+                                          out=ly["out8"], bias=ly["bias"], heads=ly["heads"], window=ly["window"])
+                else:
+                    fqvit.lis_attention(ly["logits"], ly["s_logit"], ly["v"], 0, acc=ly["acc"], bias=ly["bias"],
+                                        heads=ly["heads"], window=ly["window"])
                 attn_events[k][1].record()
                 k += 1
 
@@ -303,7 +312,7 @@ def bench_gpu(args):
     ln_ms = [a.elapsed_time(b) for a, b in ln_events]
     peak, peak_kind = peaks()
     # per-launch algorithmic bytes (averaged over the stack's layer shapes)
-    ab = [attn_bytes(ly["BH"], ly["L"], ly["d"]) for ly in layers]
+    ab = [attn_bytes(ly["BH"], ly["L"], ly["d"], 1 if args.out8 else 4) for ly in layers]
     lb = [ln_bytes(ly["rows"], ly["C"]) for ly in layers]
     attn_gbs = sum(ab) * args.steps / (sum(attn_ms) / 1e3) / 1e9
     ln_gbs = sum(lb) * args.steps / (sum(ln_ms) / 1e3) / 1e9
@@ -311,7 +320,7 @@ def bench_gpu(args):
     stack_gbs = step_bytes / (ms_per_step / 1e3) / 1e9
     dominant = "attention" if sum(attn_ms) >= sum(ln_ms) else "layernorm"
     dom_gbs = attn_gbs if dominant == "attention" else ln_gbs
-    traffic = recorded_traffic(args.config, dominant)
+    traffic = None if args.out8 else recorded_traffic(args.config, dominant)  # the record is of the int32 output
     if args.traffic:
         traffic = json.loads(args.traffic).get(dominant)
 
@@ -345,6 +354,7 @@ def bench_gpu(args):
             "logit_sigma": args.sigma,
             "parallelism": f"replicas x{ws} (independent batches, no collective)",
             "launch": "cuda_graph" if graph is not None else "eager",
+            "attention_output": "uint8 (requantized)" if args.out8 else "int32 accumulators",
         },
         "hbm_gbs": round(stack_gbs, 1),
         "hbm_frac": round(stack_gbs / peak, 4),
@@ -516,6 +526,8 @@ def main():
     ap.add_argument("--traffic", default=None, help="JSON {kernel: dram bytes per launch} from an ncu capture")
     ap.add_argument("--layers", type=int, default=0, help="time only the first N layers (profiling cases)")
     ap.add_argument("--no-graph", action="store_true", help="launch the timed steps eagerly instead of as one CUDA graph")
+    ap.add_argument("--out8", action="store_true",
+                    help="the attention output requantized to 8 bits (fqvit_lis_attention_q) instead of int32")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
