@@ -60,6 +60,8 @@ def _load():
     lib.or_ilog2.argtypes = [ctypes.c_uint64]
     lib.or_ilog2.restype = i32
     lib.or_lis_softmax.argtypes = [P, i64, i32, i64, f32, i32, P, i32, i32, P, i64, P]
+    lib.or_lis_softmax_masked.restype = ctypes.c_int
+    lib.or_lis_softmax_masked.argtypes = [P, i64, i32, i64, f32, i32, P, i32, i32, P, i32, i32, P, i64, P]
     lib.or_lis_softmax.restype = ctypes.c_int
     lib.or_lis_attn_v.argtypes = [P, i64, P, i64, i32, i64, i32, i32, P, i64]
     lib.or_attn_requant.restype = ctypes.c_int
@@ -215,8 +217,10 @@ def ilog2(x: int) -> int:
 
 
 def lis_softmax(logits: np.ndarray, L: int, s: float, n: int = 15, bias=None, heads: int = 1,
-                window: int = 7):
-    """Algorithm 2 over rows of int8 logits [n_rows, >=L].
+                window: int = 7, region=None, mask_value: int = 0):
+    """Algorithm 2 over rows of int8 logits [n_rows, >=L], with the optional relative-position
+    bias [heads, (2w-1)^2] and the optional shifted-window mask (region ids [n_windows, L]:
+    mask_value added where the query's and the key's regions differ).
 
     Returns (codes uint8 [n_rows, L], rowsum uint64 [n_rows])."""
     logits = _c(logits, np.int8)
@@ -224,8 +228,11 @@ def lis_softmax(logits: np.ndarray, L: int, s: float, n: int = 15, bias=None, he
     codes = np.zeros((n_rows, L), np.uint8)
     rowsum = np.zeros(n_rows, np.uint64)
     b = None if bias is None else _c(bias, np.int8)
-    rc = _load().or_lis_softmax(_ptr(logits), n_rows, L, ld, np.float32(s), n, _ptr(b),
-                                heads, window, _ptr(codes), L, _ptr(rowsum))
+    reg = None if region is None else _c(region, np.uint8)
+    nw = 1 if reg is None else reg.shape[0]
+    rc = _load().or_lis_softmax_masked(_ptr(logits), n_rows, L, ld, np.float32(s), n, _ptr(b),
+                                       heads, window, _ptr(reg), nw, int(mask_value), _ptr(codes), L,
+                                       _ptr(rowsum))
     if rc:
         raise ValueError("or_lis_softmax rejected its arguments")
     return codes, rowsum

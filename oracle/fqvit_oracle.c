@@ -360,14 +360,21 @@ static int32_t relpos_index(int32_t i, int32_t j, int32_t w)
  * to the int8 logit in integer arithmetic before the max.  Row r belongs
  * to head (r / L) % heads and query index r % L; the table is
  * [heads][(2w-1)^2] indexed by (dy + w-1)(2w-1) + (dx + w-1).
+ * Optional shifted-window mask (Swin, not in the paper): region ids
+ * [n_windows][L]; row r belongs to window (r / (L heads)) % n_windows, and
+ * key j of query i gets mask_value (logit units) added when their region ids
+ * in that window differ.  The i-exp clamp (Algorithm 1) bounds what a large
+ * negative mask does.
  * codes: one byte per code, row stride ld_codes.  rowsum: S per row.
  */
-OR_EXPORT int or_lis_softmax(const int8_t *logits, int64_t n_rows, int32_t L, int64_t ld,
-                             float s, int32_t n, const int8_t *bias, int32_t heads,
-                             int32_t window, uint8_t *codes, int64_t ld_codes,
-                             uint64_t *rowsum)
+OR_EXPORT int or_lis_softmax_masked(const int8_t *logits, int64_t n_rows, int32_t L, int64_t ld,
+                                    float s, int32_t n, const int8_t *bias, int32_t heads,
+                                    int32_t window, const uint8_t *region, int32_t n_windows,
+                                    int32_t mask_value, uint8_t *codes, int64_t ld_codes,
+                                    uint64_t *rowsum)
 {
-    if (!logits || !codes || n_rows < 1 || L < 1) return 1;
+    if (!logits || !codes || n_rows < 1 || L < 1 || heads < 1) return 1;
+    if (region && n_windows < 1) return 1;
     int64_t q_ln2, q_b, q_c;
     or_iexp_consts(s, &q_ln2, &q_b, &q_c);
     int32_t nb = (2 * window - 1) * (2 * window - 1);
@@ -380,10 +387,12 @@ OR_EXPORT int or_lis_softmax(const int8_t *logits, int64_t n_rows, int32_t L, in
             const int8_t *row = logits + r * ld;
             int32_t i = (int32_t)(r % L);
             int32_t h = bias ? (int32_t)((r / L) % heads) : 0;
-            int32_t m = -100000;
+            const uint8_t *reg = region ? region + ((r / ((int64_t)L * heads)) % n_windows) * L : NULL;
+            int32_t m = -2147483647;
             for (int32_t j = 0; j < L; ++j) {
                 int32_t q = row[j];
                 if (bias) q += bias[(int64_t)h * nb + relpos_index(i, j, window)];
+                if (reg && reg[i] != reg[j]) q += mask_value;
                 qv[j] = q;
                 if (q > m) m = q;
             }
@@ -404,6 +413,15 @@ OR_EXPORT int or_lis_softmax(const int8_t *logits, int64_t n_rows, int32_t L, in
         free(ev);
     }
     return 0;
+}
+
+OR_EXPORT int or_lis_softmax(const int8_t *logits, int64_t n_rows, int32_t L, int64_t ld,
+                             float s, int32_t n, const int8_t *bias, int32_t heads,
+                             int32_t window, uint8_t *codes, int64_t ld_codes,
+                             uint64_t *rowsum)
+{
+    return or_lis_softmax_masked(logits, n_rows, L, ld, s, n, bias, heads, window, NULL, 1, 0, codes, ld_codes,
+                                 rowsum);
 }
 
 /* ------------------------------------------------------------------ */
