@@ -192,6 +192,17 @@ typedef struct fqvit_relpos_bias {
     int32_t window;
 } fqvit_relpos_bias;
 
+/* Shifted-window attention mask (Swin, not in the paper): region ids
+ * [n_windows][L] uint8 (device); rows are ordered [batch][window][head]
+ * [query], so row r belongs to window (r / (L heads)) % n_windows.  Key j of
+ * query i gets mask_value (logit units, -32768 .. 0) added to its logit when
+ * region[w][i] != region[w][j]; the bias, if any, is added too. */
+typedef struct fqvit_window_mask {
+    const uint8_t *region;
+    int32_t n_windows;
+    int32_t mask_value;
+} fqvit_window_mask;
+
 /*
  * Log-Int-Softmax of n_rows rows of int8 logits (stride ld_logit bytes,
  * L keys per row; rows ordered [batch][head][query]):
@@ -266,6 +277,24 @@ FQVIT_API int fqvit_lis_attention_q(const int8_t *logits, int64_t ld_logit, floa
                           int64_t ld_v, int32_t zp_v, int64_t BH, int32_t L, int32_t d,
                           float s_v, float s_out, int32_t zp_out, uint8_t *out, int64_t ld_out,
                           void *stream);
+
+/*
+ * fqvit_lis_softmax and fqvit_lis_attention with a shifted-window mask
+ * (mask may be NULL: then they are those functions).  The mask requires
+ * n_rows (BH * L) to be a multiple of heads * L * n_windows, heads from
+ * bias_opt (1 without a bias).  Errors as those functions, plus INVALID_ARG
+ * for a NULL region, n_windows < 1, a row count that is not such a multiple,
+ * and UNSUPPORTED for mask_value outside -32768 .. 0.
+ */
+FQVIT_API int fqvit_lis_softmax_masked(const int8_t *logits, int64_t n_rows, int32_t L, int64_t ld_logit,
+                      float s_logit, int32_t n_shift, const fqvit_relpos_bias *bias_opt,
+                      const fqvit_window_mask *mask, uint8_t *codes, int64_t ld_codes,
+                      uint64_t *rowsum_opt, void *stream);
+FQVIT_API int fqvit_lis_attention_masked(const int8_t *logits, int64_t ld_logit, float s_logit,
+                        int32_t n_shift, const fqvit_relpos_bias *bias_opt,
+                        const fqvit_window_mask *mask, const int8_t *v, int64_t ld_v, int32_t zp_v,
+                        int64_t BH, int32_t L, int32_t d, int32_t *acc, int64_t ld_acc,
+                        uint8_t *codes_opt, int64_t ld_codes, void *stream);
 
 /* ------------------------------------------------------------------ */
 /* One layer: norm1 LayerNorm and the attention core (Fig. 4 dataflow) */

@@ -315,6 +315,68 @@ int fqvit_lis_attention_q(const int8_t *logits, int64_t ld_logit, float s_logit,
     return cuda_status(fqvit::launch_lis_attention(la, a, as_stream(stream)), "lis_attention_q");
 }
 
+static int check_mask(const fqvit_window_mask *mask, const fqvit_relpos_bias *bias, int64_t n_rows, int32_t L,
+                      const char *who)
+{
+    if (!mask) return FQVIT_OK;
+    if (!mask->region || mask->n_windows < 1) return fail(FQVIT_ERR_INVALID_ARG, "%s: bad window mask", who);
+    if (mask->mask_value < -32768 || mask->mask_value > 0)
+        return fail(FQVIT_ERR_UNSUPPORTED, "%s: mask_value outside -32768..0", who);
+    const int64_t heads = bias ? bias->heads : 1;
+    if (n_rows % (heads * L * (int64_t)mask->n_windows) != 0)
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: rows not a multiple of heads*L*n_windows", who);
+    return FQVIT_OK;
+}
+
+int fqvit_lis_softmax_masked(const int8_t *logits, int64_t n_rows, int32_t L, int64_t ld_logit, float s_logit,
+                             int32_t n_shift, const fqvit_relpos_bias *bias_opt, const fqvit_window_mask *mask,
+                             uint8_t *codes, int64_t ld_codes, uint64_t *rowsum_opt, void *stream)
+{
+    int rc = check_lis(logits, n_rows, L, ld_logit, s_logit, n_shift, bias_opt, "lis_softmax_masked");
+    if (rc) return rc;
+    rc = check_mask(mask, bias_opt, n_rows, L, "lis_softmax_masked");
+    if (rc) return rc;
+    if (!codes) return fail(FQVIT_ERR_INVALID_ARG, "lis_softmax_masked: NULL codes");
+    if (ld_codes < (L + 1) / 2) return fail(FQVIT_ERR_INVALID_ARG, "lis_softmax_masked: ld_codes < ceil(L/2)");
+    if (rowsum_opt && !aligned(rowsum_opt, 8))
+        return fail(FQVIT_ERR_INVALID_ARG, "lis_softmax_masked: misaligned rowsum");
+    fqvit::LisArgs a{logits, n_rows, L, ld_logit, s_logit,
+                     bias_opt ? bias_opt->table : nullptr, bias_opt ? bias_opt->heads : 1,
+                     bias_opt ? bias_opt->window : 0, codes, ld_codes,
+                     reinterpret_cast<uint64_t *>(rowsum_opt)};
+    if (mask) {
+        a.region = mask->region;
+        a.n_windows = mask->n_windows;
+        a.mask_value = mask->mask_value;
+    }
+    return cuda_status(fqvit::launch_lis_softmax(a, as_stream(stream)), "lis_softmax_masked");
+}
+
+int fqvit_lis_attention_masked(const int8_t *logits, int64_t ld_logit, float s_logit, int32_t n_shift,
+                               const fqvit_relpos_bias *bias_opt, const fqvit_window_mask *mask, const int8_t *v,
+                               int64_t ld_v, int32_t zp_v, int64_t BH, int32_t L, int32_t d, int32_t *acc,
+                               int64_t ld_acc, uint8_t *codes_opt, int64_t ld_codes, void *stream)
+{
+    int rc = check_attnv(v, ld_v, zp_v, BH, L, d, acc, ld_acc, "lis_attention_masked");
+    if (rc) return rc;
+    rc = check_lis(logits, BH * L, L, ld_logit, s_logit, n_shift, bias_opt, "lis_attention_masked");
+    if (rc) return rc;
+    rc = check_mask(mask, bias_opt, BH * L, L, "lis_attention_masked");
+    if (rc) return rc;
+    if (codes_opt && ld_codes < (L + 1) / 2)
+        return fail(FQVIT_ERR_INVALID_ARG, "lis_attention_masked: ld_codes < ceil(L/2)");
+    fqvit::LisArgs la{logits, BH * L, L, ld_logit, s_logit,
+                      bias_opt ? bias_opt->table : nullptr, bias_opt ? bias_opt->heads : 1,
+                      bias_opt ? bias_opt->window : 0, codes_opt, ld_codes, nullptr};
+    if (mask) {
+        la.region = mask->region;
+        la.n_windows = mask->n_windows;
+        la.mask_value = mask->mask_value;
+    }
+    fqvit::AttnVArgs a{nullptr, 0, v, ld_v, zp_v, BH, L, d, acc, ld_acc, nullptr};
+    return cuda_status(fqvit::launch_lis_attention(la, a, as_stream(stream)), "lis_attention_masked");
+}
+
 int fqvit_block_int(const fqvit_block_desc *b, void *stream)
 {
     if (!b) return fail(FQVIT_ERR_INVALID_ARG, "block_int: NULL descriptor");

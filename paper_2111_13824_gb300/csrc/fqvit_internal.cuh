@@ -80,6 +80,11 @@ struct LisArgs {
     uint8_t *codes;  // packed nibbles or nullptr
     int64_t ld_codes;
     uint64_t *rowsum;  // or nullptr
+    // shifted-window mask: region ids [n_windows][L] or nullptr; mask_value (-32768 .. 0) is added
+    // where a query's and a key's regions differ; window of row r: (r / (L heads)) % n_windows
+    const uint8_t *region = nullptr;
+    int n_windows = 1;
+    int mask_value = 0;
 };
 cudaError_t launch_lis_softmax(const LisArgs &a, cudaStream_t st);
 

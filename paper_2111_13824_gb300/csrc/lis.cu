@@ -31,10 +31,12 @@ using namespace lis;
 
 // Codes of one row by one warp.  Lane owns keys 4*(lane + 32 i) .. +3.
 // dst: packed nibbles (global or shared), written for bytes < ceil(L/2).
+// reg: the window's region ids [L] when a shifted-window mask is given (else nullptr): key j of
+// query qi gets mask_value where reg[j] != reg[qi]
 template <int NW, bool BIAS>
 __device__ void softmax_row(const int8_t *__restrict__ src, int L, const uint32_t *lut,
                             const int8_t *btab /* shared [(2w-1)^2] of this head */, int qi,
-                            int w, uint8_t *dst, uint64_t *rowsum_dst)
+                            int w, uint8_t *dst, uint64_t *rowsum_dst, const uint8_t *reg, int mask_value)
 {
     const int lane = threadIdx.x & 31;
     const int nwords = (L + 3) >> 2;
@@ -50,6 +52,7 @@ __device__ void softmax_row(const int8_t *__restrict__ src, int L, const uint32_
             int key = 4 * widx + b;
             int q = (int)(int8_t)(word >> (8 * b));
             if (BIAS && key < L) q += btab[relpos_idx(qi, key, w)];
+            if (reg && key < L && reg[key] != reg[qi]) q += mask_value;
             val[i][b] = q;
             if (key < L) m = max(m, q);
         }
@@ -62,7 +65,7 @@ __device__ void softmax_row(const int8_t *__restrict__ src, int L, const uint32_
 #pragma unroll
         for (int b = 0; b < 4; ++b) {
             int key = 4 * (lane + 32 * i) + b;
-            uint32_t ev = key < L ? lut[m - val[i][b]] : 0u;
+            uint32_t ev = key < L ? lut[min(m - val[i][b], kLutSize - 1)] : 0u;
             e[i][b] = ev;
             S += ev;
         }
@@ -107,14 +110,12 @@ __global__ void __launch_bounds__(256) lis_softmax_kernel(LisArgs a, IexpC ic)
     const int nwarps = blockDim.x >> 5;
     for (int64_t row = (int64_t)blockIdx.x * nwarps + warp; row < a.n_rows;
          row += (int64_t)gridDim.x * nwarps) {
-        int qi = 0;
+        const int qi = (int)(row % a.L);
         const int8_t *bt = nullptr;
-        if (BIAS) {
-            qi = (int)(row % a.L);
-            bt = btab_all + (int)((row / a.L) % a.heads) * nb;
-        }
+        if (BIAS) bt = btab_all + (int)((row / a.L) % a.heads) * nb;
+        const uint8_t *reg = a.region ? a.region + (row / ((int64_t)a.L * a.heads)) % a.n_windows * a.L : nullptr;
         softmax_row<NW, BIAS>(a.logits + row * a.ld_logit, a.L, lut, bt, qi, a.window,
-                              a.codes + row * a.ld_codes, a.rowsum ? a.rowsum + row : nullptr);
+                              a.codes + row * a.ld_codes, a.rowsum ? a.rowsum + row : nullptr, reg, a.mask_value);
     }
 }
 
@@ -211,8 +212,9 @@ __global__ void __launch_bounds__(256) lis_attention_kernel(LisArgs la, AttnVArg
         if (row < a.L) {
             int64_t grow = bh * a.L + row;
             const int8_t *bt = BIAS ? btab_all + (int)(bh % la.heads) * nb : nullptr;
+            const uint8_t *reg = la.region ? la.region + (bh / la.heads) % la.n_windows * a.L : nullptr;
             softmax_row<NW, BIAS>(la.logits + grow * la.ld_logit, a.L, lut, bt, row, la.window,
-                                  cs + r * ldc, la.rowsum ? la.rowsum + grow : nullptr);
+                                  cs + r * ldc, la.rowsum ? la.rowsum + grow : nullptr, reg, la.mask_value);
         }
     }
     __syncthreads();

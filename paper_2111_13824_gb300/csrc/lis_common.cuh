@@ -10,7 +10,10 @@
 namespace fqvit {
 namespace lis {
 
-constexpr int kLutSize = 511;  // q~ in [-510, 0]: int8 logits plus an int8 bias, minus the maximum
+// q~ in [-1335, 0]: int8 logits plus an int8 bias minus the maximum reach -510; with a window mask
+// further, but e(q~) is constant below the clamp 15 q_ln2 >= -1335 (scales >= 2^-7), so indices past
+// kLutSize - 1 read the last entry
+constexpr int kLutSize = 1336;
 
 struct IexpC {
     int q_ln2, q_b, q_c;

@@ -580,7 +580,7 @@ bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
 {
     const bool out_ok = b.out8 ? (b.ld_out8 % 16 == 0 && ((uintptr_t)b.out8 % 16) == 0)
                                : (b.ld_acc == TD && ((uintptr_t)b.acc % 32) == 0);
-    return b.d == TD && a.bias == nullptr && a.codes == nullptr && a.L <= TMAXKB * TKB &&
+    return b.d == TD && a.bias == nullptr && a.region == nullptr && a.codes == nullptr && a.L <= TMAXKB * TKB &&
            a.ld_logit % 16 == 0 && b.ld_v == TD && out_ok && ((uintptr_t)a.logits % 16) == 0 &&
            ((uintptr_t)b.v % 16) == 0 && tc_smem_bytes(a.L, a.ld_logit) + kTcStaticSmem <= 232448;
 }

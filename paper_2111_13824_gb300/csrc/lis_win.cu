@@ -70,6 +70,9 @@ struct WinParams {
     uint8_t *out8;  // when not null: 8-bit outputs (requant8 with n1, n2, zp8) instead of acc
     int64_t ld_out8;
     int n1, n2, zp8;
+    const uint8_t *region;  // shifted-window mask: region ids [n_windows][L] (MASK variants)
+    int n_windows;
+    int mask_c;  // |mask value| clamped to 1024 (exact: see the kernel)
 };
 
 struct WinShared {
@@ -102,8 +105,13 @@ __device__ __forceinline__ uint32_t operand_exp_tab(float ef, int G, float hi, f
     return (uint32_t)max(31 - k + (int)le, 15);
 }
 
-// NQ: 16-key chunks of a row (L in 16 (NQ - 1) + 1 .. 16 NQ)
-template <int D, bool BIAS, bool SMALL_E, int NQ>
+// NQ: 16-key chunks of a row (L in 16 (NQ - 1) + 1 .. 16 NQ).  MASK (with BIAS): the shifted-window
+// mask.  Logits then sit in the 16-bit lanes as v = q + bias + 1280 - (masked ? m_c : 0) with m_c the
+// mask magnitude clamped to 1024: a key masked by more still lands below every unmasked key (the
+// query's own key is never masked, v >= 1024) at a distance above 510 >= the table's last entry,
+// which is the clamp 15 |q_ln2| of Algorithm 1 (the launch requires 15 |q_ln2| <= 510), so its
+// i-exp value and the row maximum are those of the true mask.
+template <int D, bool BIAS, bool SMALL_E, int NQ, bool MASK>
 __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams p)
 {
     extern __shared__ __align__(16) unsigned char dsm_raw[];
@@ -117,6 +125,7 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
     const uint32_t bs_off = (uint32_t)p.ne * 256u;
     unsigned char *Bs_all = dsm_raw + bs_off + ((1024u - ((sa(dsm_raw) + bs_off) & 1023u)) & 1023u);  // ng x 16 KB
     unsigned char *BR = Bs_all + p.ng * WB_BYTES;                             // heads x L x 64 B
+    unsigned char *RG = BR + (BIAS ? (size_t)p.heads * p.L * WBIAS_ROW : 0);  // n_windows x 64 B region ids
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = tid >> 7, r = tid & 127;
@@ -181,6 +190,11 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
         reinterpret_cast<uint4 *>(const_cast<unsigned char *>(LUTB))[x] = make_uint4(w, w, w, w);
     }
     __syncthreads();
+    if (MASK)  // region ids, one 64-byte row per window (bytes past L: 0, never read as masked)
+        for (int x = tid; x < p.n_windows * 64; x += blockDim.x) {
+            const int wdx = x >> 6, j = x & 63;
+            RG[x] = j < L ? p.region[(size_t)wdx * L + j] : 0;
+        }
     // phase 3: B of every group: zeros, and (d = 32) fp16 1 in column 32 of every key row below L
     for (int x = tid; x < p.ng * WB_BYTES / 16; x += blockDim.x) {
         const int kk = (x >> 3) & 127, pos = x & 7, ci = pos ^ (kk & 7);
@@ -291,7 +305,29 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
         // ---- pairs of 16-bit lanes v = q + bias + 256 (0 for keys past L):
         //      vp[2j] holds keys (4j, 4j+2), vp[2j+1] keys (4j+1, 4j+3)
         uint32_t vp[8 * NQ];
-        if (BIAS) {
+        if (MASK) {
+            const unsigned char *br = BR + ((size_t)hh * L + qi) * WBIAS_ROW;
+            const unsigned char *rg = RG + (size_t)((bh / p.heads) % p.n_windows) * 64;
+            const uint32_t rib = (uint32_t)rg[qi] * 0x01010101u;
+#pragma unroll
+            for (int c = 0; c < NQ; ++c) {
+                const uint4 b4 = *reinterpret_cast<const uint4 *>(br + 16 * (c ^ sw));
+                const uint4 r4 = *reinterpret_cast<const uint4 *>(rg + 16 * c);
+                const uint32_t bb[4] = {b4.x, b4.y, b4.z, b4.w};
+                const uint32_t rr[4] = {r4.x, r4.y, r4.z, r4.w};
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int j = 4 * c + k;
+                    // byte nonzero: the key's region differs from the query's (keys past L: never)
+                    const uint32_t x = (rr[k] ^ rib) & (c == NQ - 1 ? cm[k] : 0xFFFFFFFFu);
+                    const uint32_t me = ((prmt(x, 0u, 0x4240u) + 0x7FFF7FFFu) >> 15) & 0x00010001u;
+                    const uint32_t mo = ((prmt(x, 0u, 0x4341u) + 0x7FFF7FFFu) >> 15) & 0x00010001u;
+                    vp[2 * j] = prmt(u[j], 0u, 0x4240u) + prmt(bb[k], 0u, 0x4240u) + 0x04000400u - me * (uint32_t)p.mask_c;
+                    vp[2 * j + 1] =
+                        prmt(u[j], 0u, 0x4341u) + prmt(bb[k], 0u, 0x4341u) + 0x04000400u - mo * (uint32_t)p.mask_c;
+                }
+            }
+        } else if (BIAS) {
             const unsigned char *br = BR + ((size_t)hh * L + qi) * WBIAS_ROW;
 #pragma unroll
             for (int c = 0; c < NQ; ++c) {
@@ -341,7 +377,8 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
             S += SMALL_E ? (unsigned long long)a : a64;
         }
         {
-            const uint32_t dm = m < (uint32_t)(p.ne - 1) ? m : (uint32_t)(p.ne - 1);
+            const uint32_t mp = MASK ? m - 1024u : m;  // padding keys sit at v = 1024 (MASK) or 0
+            const uint32_t dm = mp < (uint32_t)(p.ne - 1) ? mp : (uint32_t)(p.ne - 1);
             const uint32_t epad = *reinterpret_cast<const uint32_t *>(LUTB + ((dm << 8) | lane4));
             S -= (unsigned long long)(4 * nw - L) * epad;
         }
@@ -452,9 +489,10 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
 constexpr size_t kWinStaticSmem = 512 * 4 + 64 * 4 * 3 + sizeof(WinShared) + 256;
 constexpr size_t kSmemLimit = 232448;
 
-size_t win_smem_bytes(int ng, int ne, int heads, int L, bool bias)
+size_t win_smem_bytes(int ng, int ne, int heads, int L, bool bias, int mask_windows)
 {
-    return 1024 + (size_t)ng * WB_BYTES + (size_t)ne * 256 + (bias ? (size_t)heads * L * WBIAS_ROW : 0);
+    return 1024 + (size_t)ng * WB_BYTES + (size_t)ne * 256 + (bias ? (size_t)heads * L * WBIAS_ROW : 0) +
+           (size_t)mask_windows * 64;
 }
 
 // table entries: distances up to 255 (510 with a bias), and none past the clamp 15 |q_ln2|
@@ -467,43 +505,52 @@ int win_table_entries(const IexpC &c, bool bias)
 
 // groups per CTA that fit shared memory; the raw bias table (heads x (2w-1)^2 bytes) is
 // staged in the groups' B area during the set-up
-int win_groups(int ne, int heads, int L, int window, bool bias)
+int win_groups(int ne, int heads, int L, int window, bool bias, int mask_windows)
 {
     const size_t tab = bias ? (size_t)heads * (2 * window - 1) * (2 * window - 1) : 0;
     for (int ng = WMAXG; ng >= 1; --ng)
-        if (win_smem_bytes(ng, ne, heads, L, bias) + kWinStaticSmem <= kSmemLimit && tab <= (size_t)ng * WB_BYTES)
+        if (win_smem_bytes(ng, ne, heads, L, bias, mask_windows) + kWinStaticSmem <= kSmemLimit &&
+            tab <= (size_t)ng * WB_BYTES)
             return ng;
     return 0;
 }
 
 bool small_iexp_w(const IexpC &c) { return ((double)c.q_b * c.q_b + c.q_c) * 32768.0 < 268435456.0; }
 
-template <int D, bool BIAS, bool SMALL_E, int NQ>
+template <int D, bool BIAS, bool SMALL_E, int NQ, bool MASK>
 cudaError_t win_launch_q(const WinParams &p, size_t smem, int grid, cudaStream_t st)
 {
-    cudaError_t e = cudaFuncSetAttribute(lis_attn_win_kernel<D, BIAS, SMALL_E, NQ>,
+    cudaError_t e = cudaFuncSetAttribute(lis_attn_win_kernel<D, BIAS, SMALL_E, NQ, MASK>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    lis_attn_win_kernel<D, BIAS, SMALL_E, NQ><<<grid, 128 * p.ng, smem, st>>>(p);
+    lis_attn_win_kernel<D, BIAS, SMALL_E, NQ, MASK><<<grid, 128 * p.ng, smem, st>>>(p);
     return cudaGetLastError();
 }
 
-template <int D, bool BIAS, bool SMALL_E>
+template <int D, bool BIAS, bool SMALL_E, bool MASK>
 cudaError_t win_launch(const WinParams &p, size_t smem, int grid, cudaStream_t st)
 {
     switch ((p.L + 15) >> 4) {
-    case 1: return win_launch_q<D, BIAS, SMALL_E, 1>(p, smem, grid, st);
-    case 2: return win_launch_q<D, BIAS, SMALL_E, 2>(p, smem, grid, st);
-    case 3: return win_launch_q<D, BIAS, SMALL_E, 3>(p, smem, grid, st);
-    default: return win_launch_q<D, BIAS, SMALL_E, 4>(p, smem, grid, st);
+    case 1: return win_launch_q<D, BIAS, SMALL_E, 1, MASK>(p, smem, grid, st);
+    case 2: return win_launch_q<D, BIAS, SMALL_E, 2, MASK>(p, smem, grid, st);
+    case 3: return win_launch_q<D, BIAS, SMALL_E, 3, MASK>(p, smem, grid, st);
+    default: return win_launch_q<D, BIAS, SMALL_E, 4, MASK>(p, smem, grid, st);
     }
 }
 
+// (bias, mask): (no, no), (yes, no), (yes, yes); a mask needs the bias (the eligibility checks)
 template <int D>
-cudaError_t win_launch_d(bool bias, bool small_e, const WinParams &p, size_t smem, int grid, cudaStream_t st)
+cudaError_t win_launch_d(bool bias, bool mask, bool small_e, const WinParams &p, size_t smem, int grid,
+                         cudaStream_t st)
 {
-    if (bias) return small_e ? win_launch<D, true, true>(p, smem, grid, st) : win_launch<D, true, false>(p, smem, grid, st);
-    return small_e ? win_launch<D, false, true>(p, smem, grid, st) : win_launch<D, false, false>(p, smem, grid, st);
+    if (mask)
+        return small_e ? win_launch<D, true, true, true>(p, smem, grid, st)
+                       : win_launch<D, true, false, true>(p, smem, grid, st);
+    if (bias)
+        return small_e ? win_launch<D, true, true, false>(p, smem, grid, st)
+                       : win_launch<D, true, false, false>(p, smem, grid, st);
+    return small_e ? win_launch<D, false, true, false>(p, smem, grid, st)
+                   : win_launch<D, false, false, false>(p, smem, grid, st);
 }
 
 }  // namespace
@@ -519,22 +566,29 @@ bool lis_attention_win_eligible(const LisArgs &a, const AttnVArgs &b)
         return false;
     const bool bias = a.bias != nullptr;
     const IexpC c = iexp_consts_host(a.s_logit);
-    return win_groups(win_table_entries(c, bias), a.heads, a.L, a.window, bias) > 0;
+    const int mwin = a.region ? a.n_windows : 0;
+    // a mask needs the bias (the masked kernel variants) and the i-exp clamp inside the table
+    if (a.region && (!bias || 15 * -c.q_ln2 > 510)) return false;
+    return win_groups(win_table_entries(c, bias), a.heads, a.L, a.window, bias, mwin) > 0;
 }
 
 cudaError_t launch_lis_attention_win(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
 {
     const bool bias = a.bias != nullptr;
     WinParams p{a.logits, a.ld_logit, b.v, b.ld_v, b.acc, b.ld_acc, a.bias, a.heads, a.window, b.BH, a.L, b.zp_v,
-                iexp_consts_host(a.s_logit), 0, 0, b.out8, b.ld_out8, b.rq_n1, b.rq_n2, b.rq_zp};
+                iexp_consts_host(a.s_logit), 0, 0, b.out8, b.ld_out8, b.rq_n1, b.rq_n2, b.rq_zp,
+                a.region, a.n_windows, a.mask_value < -1024 ? 1024 : -a.mask_value};
+    const int mwin = a.region ? a.n_windows : 0;
     p.ne = win_table_entries(p.ic, bias);
-    p.ng = win_groups(p.ne, a.heads, a.L, a.window, bias);
-    const size_t smem = win_smem_bytes(p.ng, p.ne, a.heads, a.L, bias);
+    p.ng = win_groups(p.ne, a.heads, a.L, a.window, bias, mwin);
+    const size_t smem = win_smem_bytes(p.ng, p.ne, a.heads, a.L, bias, mwin);
     const int64_t ntiles = (b.BH + 1) / 2;
     const int64_t want = (ntiles + p.ng - 1) / p.ng;
     const int grid = (int)(want < sm_count() ? want : sm_count());
     const bool se = small_iexp_w(p.ic);
-    return b.d == 32 ? win_launch_d<32>(bias, se, p, smem, grid, st) : win_launch_d<64>(bias, se, p, smem, grid, st);
+    const bool mask = a.region != nullptr;
+    return b.d == 32 ? win_launch_d<32>(bias, mask, se, p, smem, grid, st)
+                     : win_launch_d<64>(bias, mask, se, p, smem, grid, st);
 }
 
 cudaError_t read_clear_win_status(int *status)

@@ -28,6 +28,10 @@ class RelposBias(ctypes.Structure):
     _fields_ = [("table", ctypes.c_void_p), ("heads", ctypes.c_int32), ("window", ctypes.c_int32)]
 
 
+class WindowMask(ctypes.Structure):
+    _fields_ = [("region", ctypes.c_void_p), ("n_windows", ctypes.c_int32), ("mask_value", ctypes.c_int32)]
+
+
 class BlockDesc(ctypes.Structure):
     _fields_ = [
         ("xq", ctypes.c_void_p), ("rows", ctypes.c_int64), ("C", ctypes.c_int32), ("zp_in", ctypes.c_int32),
@@ -45,6 +49,7 @@ EXPORTS = (
     "fqvit_lis_attention", "fqvit_lis_attention_q", "fqvit_block_int", "fqvit_sync_status",
     "fqvit_calibrate_ptf_noalloc",
     "fqvit_calibrate_minmax", "fqvit_calibrate_sse_partial", "fqvit_calibrate_combine",
+    "fqvit_lis_softmax_masked", "fqvit_lis_attention_masked",
 )
 
 
@@ -75,6 +80,9 @@ def load(path: str | Path | None = None):
                                   ctypes.c_int),
         "fqvit_lis_attention": ([P, i64, f32, i32, P, P, i64, i32, i64, i32, i32, P, i64, P, i64, P],
                                 ctypes.c_int),
+        "fqvit_lis_softmax_masked": ([P, i64, i32, i64, f32, i32, P, P, P, i64, P, P], ctypes.c_int),
+        "fqvit_lis_attention_masked": ([P, i64, f32, i32, P, P, P, i64, i32, i64, i32, i32, P, i64, P, i64, P],
+                                       ctypes.c_int),
         "fqvit_block_int": ([P, P], ctypes.c_int),
         "fqvit_sync_status": ([P], ctypes.c_int),
         "fqvit_calibrate_ptf_noalloc": ([P, i64, i32, i64, i32, i32, P, P, P, P, P], ctypes.c_int),
@@ -289,6 +297,51 @@ def lis_attention_q(logits: torch.Tensor, s_logit: float, v: torch.Tensor, zp_v:
                                         BH, L, d, float(s_v), float(s_out), int(zp_out), _p(out), out.stride(1),
                                         _stream(stream)))
     return out
+
+
+def _mask(region, mask_value):
+    if region is None:
+        return None
+    if not isinstance(region, torch.Tensor) or not region.is_cuda or region.dtype != torch.uint8:
+        raise ValueError("region: a uint8 device tensor [n_windows, L]")
+    if not region.is_contiguous():
+        raise ValueError("region must be contiguous")
+    return WindowMask(ctypes.c_void_p(region.data_ptr()), region.shape[0], int(mask_value))
+
+
+def lis_softmax_masked(logits: torch.Tensor, L: int, s_logit: float, region: torch.Tensor | None,
+                       mask_value: int, codes: torch.Tensor | None = None, rowsum: torch.Tensor | None = None,
+                       bias: torch.Tensor | None = None, heads: int = 1, window: int = 0, n_shift: int = 15,
+                       stream=None) -> torch.Tensor:
+    """LIS codes with a shifted-window mask (fqvit_lis_softmax_masked); region uint8 [n_windows, L]."""
+    n_rows = logits.shape[0]
+    if codes is None:
+        codes = torch.empty(n_rows, (L + 1) // 2, dtype=torch.uint8, device=logits.device)
+    b = _bias(bias, heads, window)
+    m = _mask(region, mask_value)
+    _check(load().fqvit_lis_softmax_masked(_p(logits), n_rows, L, _ld(logits), float(s_logit), n_shift,
+                                           ctypes.byref(b) if b is not None else None,
+                                           ctypes.byref(m) if m is not None else None, _p(codes), _ld(codes),
+                                           _p(rowsum), _stream(stream)))
+    return codes
+
+
+def lis_attention_masked(logits: torch.Tensor, s_logit: float, v: torch.Tensor, region: torch.Tensor | None,
+                         mask_value: int, zp_v: int = 0, acc: torch.Tensor | None = None,
+                         codes: torch.Tensor | None = None, bias: torch.Tensor | None = None, heads: int = 1,
+                         window: int = 0, n_shift: int = 15, stream=None) -> torch.Tensor:
+    """Fused attention with a shifted-window mask (fqvit_lis_attention_masked): int32 [BH, L, d]."""
+    BH, L, d = v.shape
+    if acc is None:
+        acc = torch.empty(BH, L, d, dtype=torch.int32, device=v.device)
+    b = _bias(bias, heads, window)
+    m = _mask(region, mask_value)
+    _check(load().fqvit_lis_attention_masked(_p(logits), _ld(logits), float(s_logit), n_shift,
+                                             ctypes.byref(b) if b is not None else None,
+                                             ctypes.byref(m) if m is not None else None, _p(v), v.stride(1),
+                                             int(zp_v), BH, L, d, _p(acc), acc.stride(1), _p(codes),
+                                             _ld(codes) if codes is not None else 0, _stream(stream)))
+    return acc
 
 
 def block_int(xq, zp_in, alpha, gamma, beta, s_out, zp_out, yq, logits, ld_logit, s_logit, v, zp_v, acc,

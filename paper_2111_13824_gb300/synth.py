@@ -26,6 +26,12 @@ S * 1000 + l, draws in this fixed order):
   keys (Sec. 3.3: 98.8 % of ViT-L attention values are below 1/16).
 * V: int8 uniform in [-128, 127], zero point 0.
 * Swin relative-position bias: int8 ``[H, (2w-1)^2]`` uniform in [-16, 16].
+* Swin shifted-window mask (odd blocks of a stage whose side exceeds the
+  window): region ids ``[n_windows, w*w]`` of the cyclically shifted map
+  (three bands per axis: below side - w, below side - shift, the rest;
+  id = 3 band_y + band_x), windows in raster order, tokens in raster order
+  inside a window; the mask value is -100 in real units, rounded to logit
+  units (``swin_mask_value``).
 
 Rows of logits are padded to a multiple of 16 bytes (``ld_logit``).
 """
@@ -182,3 +188,27 @@ def attn_inputs(cfg: Config, layer: int, device="cpu", sigma: float = 1.0, bh: i
     logits[:, :L] = qq.reshape(BH * L, L).to(torch.int8)
     return dict(logits=logits, ld_logit=ld, s_logit=s_logit, v=v.contiguous(), bias=bias,
                 heads=st.H, window=st.window, BH=BH, L=L, d=d)
+
+
+def shifted_window_regions(side: int, window: int, shift: int | None = None) -> torch.Tensor:
+    """Region ids uint8 [n_windows, window^2] of a side x side map shifted by ``shift``
+    (default window // 2); every token of a window carries its band pair 3 band_y + band_x."""
+    shift = window // 2 if shift is None else shift
+
+    def band(t):
+        return 0 if t < side - window else (1 if t < side - shift else 2)
+
+    nw = side // window
+    out = torch.empty(nw * nw, window * window, dtype=torch.uint8)
+    for wy in range(nw):
+        for wx in range(nw):
+            for ty in range(window):
+                for tx in range(window):
+                    y, x = wy * window + ty, wx * window + tx
+                    out[wy * nw + wx, ty * window + tx] = 3 * band(y) + band(x)
+    return out
+
+
+def swin_mask_value(s_logit: float, real: float = -100.0) -> int:
+    """The Swin mask (-100 in real units) in logit units, kept inside -32768 .. 0."""
+    return max(-32768, min(0, int(round(real / s_logit))))

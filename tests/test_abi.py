@@ -91,3 +91,23 @@ def test_requantized_attention_checks(lib):
     assert args(0.05, 0.02, 256, fake, 64) == 1        # zp_out outside 0..255
     assert "zp_out" in _err(lib)
     assert args(1e30, 1e-30, 0, fake, 64) == 2         # M leaves the fp32 range
+
+
+def test_window_mask_checks(lib):
+    """The masked entry points reject a bad mask before any launch; heads come from the bias."""
+    fake = ctypes.c_void_p(4096)
+    b = fqvit.RelposBias(fake, 3, 7)
+    soft = lambda m, rows=2 * 3 * 49: lib.fqvit_lis_softmax_masked(  # noqa: E731
+        fake, rows, 49, 64, 0.05, 15, ctypes.byref(b), m, fake, 25, None, None)
+    assert soft(ctypes.byref(fqvit.WindowMask(None, 2, -100))) == 1        # NULL region
+    assert "mask" in _err(lib)
+    assert soft(ctypes.byref(fqvit.WindowMask(fake, 0, -100))) == 1        # no windows
+    assert soft(ctypes.byref(fqvit.WindowMask(fake, 2, 1))) == 2           # positive mask value
+    assert soft(ctypes.byref(fqvit.WindowMask(fake, 2, -32769))) == 2      # below -32768
+    assert soft(ctypes.byref(fqvit.WindowMask(fake, 4, -100))) == 1        # rows not a multiple of 3*49*4
+    assert "n_windows" in _err(lib)
+    att = lambda m: lib.fqvit_lis_attention_masked(  # noqa: E731
+        fake, 64, 0.05, 15, ctypes.byref(b), m, fake, 32, 0, 2 * 3, 49, 32, fake, 32, None, 0, None)
+    assert att(ctypes.byref(fqvit.WindowMask(None, 2, -100))) == 1
+    assert att(ctypes.byref(fqvit.WindowMask(fake, 4, -100))) == 1
+    assert att(ctypes.byref(fqvit.WindowMask(fake, 2, -32769))) == 2
