@@ -106,6 +106,7 @@ def make_layers(cfg, device, sigma=1.0, limit=0):
             xq=xq, zp=zp_i, alpha=alpha, gamma=d["gamma"], beta=d["beta"], s_out=d["s_out"], zp_out=d["zp_out"],
             yq=torch.empty_like(xq), logits=a["logits"], s_logit=a["s_logit"], v=a["v"], bias=a["bias"],
             heads=a["heads"], window=a["window"],
+            region=synth.layer_window_mask(cfg, l, device=device), mask_value=synth.swin_mask_value(a["s_logit"]),
             acc=torch.empty(a["BH"], a["L"], a["d"], dtype=torch.int32, device=device),
             out8=torch.empty(a["BH"], a["L"], a["d"], dtype=torch.uint8, device=device),
             rows=st.rows, C=st.C, BH=st.BH, L=st.L, d=st.d))
@@ -114,14 +115,28 @@ def make_layers(cfg, device, sigma=1.0, limit=0):
     return layers
 
 
+def attention(fq, ly, out8=False):
+    """The layer's fused attention; Swin's shifted blocks take their window mask."""
+    kw = dict(bias=ly["bias"], heads=ly["heads"], window=ly["window"])
+    if ly["region"] is not None:
+        if out8:  # the output requantized to 8 bits (output scale = V's: M = 2^-15)
+            fq.lis_attention_masked_q(ly["logits"], ly["s_logit"], ly["v"], ly["region"], ly["mask_value"], 0,
+                                      OUT8_SV, OUT8_SV, 128, out=ly["out8"], **kw)
+        else:
+            fq.lis_attention_masked(ly["logits"], ly["s_logit"], ly["v"], ly["region"], ly["mask_value"], 0,
+                                    acc=ly["acc"], **kw)
+    elif out8:
+        fq.lis_attention_q(ly["logits"], ly["s_logit"], ly["v"], 0, OUT8_SV, OUT8_SV, 128, out=ly["out8"], **kw)
+    else:
+        fq.lis_attention(ly["logits"], ly["s_logit"], ly["v"], 0, acc=ly["acc"], **kw)
+
+
 def run_layer(fq, ly, ev=None):
     fq.ptf_layernorm(ly["xq"], ly["zp"], ly["alpha"], ly["gamma"], ly["beta"], ly["s_out"], ly["zp_out"],
                      out=ly["yq"])
     if ev is not None:
         ev[0].record()
-    bias = ly["bias"]
-    fq.lis_attention(ly["logits"], ly["s_logit"], ly["v"], 0, acc=ly["acc"], bias=bias, heads=ly["heads"],
-                     window=ly["window"])
+    attention(fq, ly)
     if ev is not None:
         ev[1].record()
 
@@ -260,12 +275,7 @@ def bench_gpu(args):
                                     ly["zp_out"], out=ly["yq"])
                 ln_events[k][1].record()
                 attn_events[k][0].record()
-                if args.out8:  # the output requantized to 8 bits (output scale = V's: M = 2^-15)
-                    fqvit.lis_attention_q(ly["logits"], ly["s_logit"], ly["v"], 0, OUT8_SV, OUT8_SV, 128,
-                                          out=ly["out8"], bias=ly["bias"], heads=ly["heads"], window=ly["window"])
-                else:
-                    fqvit.lis_attention(ly["logits"], ly["s_logit"], ly["v"], 0, acc=ly["acc"], bias=ly["bias"],
-                                        heads=ly["heads"], window=ly["window"])
+                attention(fqvit, ly, args.out8)
                 attn_events[k][1].record()
                 k += 1
 
@@ -355,6 +365,7 @@ def bench_gpu(args):
             "parallelism": f"replicas x{ws} (independent batches, no collective)",
             "launch": "cuda_graph" if graph is not None else "eager",
             "attention_output": "uint8 (requantized)" if args.out8 else "int32 accumulators",
+            "shifted_window_layers": sum(ly["region"] is not None for ly in layers),
         },
         "hbm_gbs": round(stack_gbs, 1),
         "hbm_frac": round(stack_gbs / peak, 4),

@@ -295,6 +295,13 @@ FQVIT_API int fqvit_lis_attention_masked(const int8_t *logits, int64_t ld_logit,
                         const fqvit_window_mask *mask, const int8_t *v, int64_t ld_v, int32_t zp_v,
                         int64_t BH, int32_t L, int32_t d, int32_t *acc, int64_t ld_acc,
                         uint8_t *codes_opt, int64_t ld_codes, void *stream);
+/* fqvit_lis_attention_q with a shifted-window mask (mask may be NULL); the
+ * mask's requirements and errors as fqvit_lis_attention_masked. */
+FQVIT_API int fqvit_lis_attention_masked_q(const int8_t *logits, int64_t ld_logit, float s_logit,
+                          int32_t n_shift, const fqvit_relpos_bias *bias_opt,
+                          const fqvit_window_mask *mask, const int8_t *v, int64_t ld_v, int32_t zp_v,
+                          int64_t BH, int32_t L, int32_t d, float s_v, float s_out, int32_t zp_out,
+                          uint8_t *out, int64_t ld_out, void *stream);
 
 /* ------------------------------------------------------------------ */
 /* One layer: norm1 LayerNorm and the attention core (Fig. 4 dataflow) */

@@ -283,38 +283,6 @@ int fqvit_lis_attention(const int8_t *logits, int64_t ld_logit, float s_logit, i
     return cuda_status(fqvit::launch_lis_attention(la, a, as_stream(stream)), "lis_attention");
 }
 
-int fqvit_lis_attention_q(const int8_t *logits, int64_t ld_logit, float s_logit, int32_t n_shift,
-                          const fqvit_relpos_bias *bias_opt, const int8_t *v, int64_t ld_v, int32_t zp_v,
-                          int64_t BH, int32_t L, int32_t d, float s_v, float s_out, int32_t zp_out, uint8_t *out,
-                          int64_t ld_out, void *stream)
-{
-    if (!out) return fail(FQVIT_ERR_INVALID_ARG, "lis_attention_q: NULL output");
-    if (ld_out < d) return fail(FQVIT_ERR_INVALID_ARG, "lis_attention_q: ld_out < d");
-    if (!(s_v > 0.0f) || !(s_v < 3.0e38f) || !(s_out > 0.0f) || !(s_out < 3.0e38f))
-        return fail(FQVIT_ERR_INVALID_ARG, "lis_attention_q: s_v and s_out must be positive and finite");
-    if (zp_out < 0 || zp_out > 255) return fail(FQVIT_ERR_INVALID_ARG, "lis_attention_q: zp_out outside 0..255");
-    // the multiplier M = (s_v / s_out) / 2^15 as N2 / 2^N1 with 8 significant bits
-    const float M = ldexpf(s_v / s_out, -15);
-    if (!(M > 0.0f) || !(M < 1.0e30f)) return fail(FQVIT_ERR_UNSUPPORTED, "lis_attention_q: s_v / s_out out of range");
-    int n1 = 7 - ilogbf(M);
-    if (n1 > 31) n1 = 31;
-    const int n2 = (int)floorf(ldexpf(M, n1));
-    int rc = check_attnv(v, ld_v, zp_v, BH, L, d, nullptr, 0, "lis_attention_q", false);
-    if (rc) return rc;
-    rc = check_lis(logits, BH * L, L, ld_logit, s_logit, n_shift, bias_opt, "lis_attention_q");
-    if (rc) return rc;
-    fqvit::LisArgs la{logits, BH * L, L, ld_logit, s_logit,
-                      bias_opt ? bias_opt->table : nullptr, bias_opt ? bias_opt->heads : 1,
-                      bias_opt ? bias_opt->window : 0, nullptr, 0, nullptr};
-    fqvit::AttnVArgs a{nullptr, 0, v, ld_v, zp_v, BH, L, d, nullptr, 0, nullptr};
-    a.out8 = out;
-    a.ld_out8 = ld_out;
-    a.rq_n1 = n1 < -10 ? -10 : n1;
-    a.rq_n2 = n2;
-    a.rq_zp = zp_out;
-    return cuda_status(fqvit::launch_lis_attention(la, a, as_stream(stream)), "lis_attention_q");
-}
-
 static int check_mask(const fqvit_window_mask *mask, const fqvit_relpos_bias *bias, int64_t n_rows, int32_t L,
                       const char *who)
 {
@@ -326,6 +294,64 @@ static int check_mask(const fqvit_window_mask *mask, const fqvit_relpos_bias *bi
     if (n_rows % (heads * L * (int64_t)mask->n_windows) != 0)
         return fail(FQVIT_ERR_INVALID_ARG, "%s: rows not a multiple of heads*L*n_windows", who);
     return FQVIT_OK;
+}
+
+// The attention with its output requantized to 8 bits, with or without a window mask.
+static int attention_q(const int8_t *logits, int64_t ld_logit, float s_logit, int32_t n_shift,
+                       const fqvit_relpos_bias *bias_opt, const fqvit_window_mask *mask, const int8_t *v,
+                       int64_t ld_v, int32_t zp_v, int64_t BH, int32_t L, int32_t d, float s_v, float s_out,
+                       int32_t zp_out, uint8_t *out, int64_t ld_out, void *stream, const char *who)
+{
+    if (!out) return fail(FQVIT_ERR_INVALID_ARG, "%s: NULL output", who);
+    if (ld_out < d) return fail(FQVIT_ERR_INVALID_ARG, "%s: ld_out < d", who);
+    if (!(s_v > 0.0f) || !(s_v < 3.0e38f) || !(s_out > 0.0f) || !(s_out < 3.0e38f))
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: s_v and s_out must be positive and finite", who);
+    if (zp_out < 0 || zp_out > 255) return fail(FQVIT_ERR_INVALID_ARG, "%s: zp_out outside 0..255", who);
+    // the multiplier M = (s_v / s_out) / 2^15 as N2 / 2^N1 with 8 significant bits
+    const float M = ldexpf(s_v / s_out, -15);
+    if (!(M > 0.0f) || !(M < 1.0e30f)) return fail(FQVIT_ERR_UNSUPPORTED, "%s: s_v / s_out out of range", who);
+    int n1 = 7 - ilogbf(M);
+    if (n1 > 31) n1 = 31;
+    const int n2 = (int)floorf(ldexpf(M, n1));
+    int rc = check_attnv(v, ld_v, zp_v, BH, L, d, nullptr, 0, who, false);
+    if (rc) return rc;
+    rc = check_lis(logits, BH * L, L, ld_logit, s_logit, n_shift, bias_opt, who);
+    if (rc) return rc;
+    rc = check_mask(mask, bias_opt, BH * L, L, who);
+    if (rc) return rc;
+    fqvit::LisArgs la{logits, BH * L, L, ld_logit, s_logit,
+                      bias_opt ? bias_opt->table : nullptr, bias_opt ? bias_opt->heads : 1,
+                      bias_opt ? bias_opt->window : 0, nullptr, 0, nullptr};
+    if (mask) {
+        la.region = mask->region;
+        la.n_windows = mask->n_windows;
+        la.mask_value = mask->mask_value;
+    }
+    fqvit::AttnVArgs a{nullptr, 0, v, ld_v, zp_v, BH, L, d, nullptr, 0, nullptr};
+    a.out8 = out;
+    a.ld_out8 = ld_out;
+    a.rq_n1 = n1 < -10 ? -10 : n1;
+    a.rq_n2 = n2;
+    a.rq_zp = zp_out;
+    return cuda_status(fqvit::launch_lis_attention(la, a, as_stream(stream)), who);
+}
+
+int fqvit_lis_attention_q(const int8_t *logits, int64_t ld_logit, float s_logit, int32_t n_shift,
+                          const fqvit_relpos_bias *bias_opt, const int8_t *v, int64_t ld_v, int32_t zp_v,
+                          int64_t BH, int32_t L, int32_t d, float s_v, float s_out, int32_t zp_out, uint8_t *out,
+                          int64_t ld_out, void *stream)
+{
+    return attention_q(logits, ld_logit, s_logit, n_shift, bias_opt, nullptr, v, ld_v, zp_v, BH, L, d, s_v, s_out,
+                       zp_out, out, ld_out, stream, "lis_attention_q");
+}
+
+int fqvit_lis_attention_masked_q(const int8_t *logits, int64_t ld_logit, float s_logit, int32_t n_shift,
+                                 const fqvit_relpos_bias *bias_opt, const fqvit_window_mask *mask, const int8_t *v,
+                                 int64_t ld_v, int32_t zp_v, int64_t BH, int32_t L, int32_t d, float s_v,
+                                 float s_out, int32_t zp_out, uint8_t *out, int64_t ld_out, void *stream)
+{
+    return attention_q(logits, ld_logit, s_logit, n_shift, bias_opt, mask, v, ld_v, zp_v, BH, L, d, s_v, s_out,
+                       zp_out, out, ld_out, stream, "lis_attention_masked_q");
 }
 
 int fqvit_lis_softmax_masked(const int8_t *logits, int64_t n_rows, int32_t L, int64_t ld_logit, float s_logit,

@@ -49,7 +49,7 @@ EXPORTS = (
     "fqvit_lis_attention", "fqvit_lis_attention_q", "fqvit_block_int", "fqvit_sync_status",
     "fqvit_calibrate_ptf_noalloc",
     "fqvit_calibrate_minmax", "fqvit_calibrate_sse_partial", "fqvit_calibrate_combine",
-    "fqvit_lis_softmax_masked", "fqvit_lis_attention_masked",
+    "fqvit_lis_softmax_masked", "fqvit_lis_attention_masked", "fqvit_lis_attention_masked_q",
 )
 
 
@@ -83,6 +83,8 @@ def load(path: str | Path | None = None):
         "fqvit_lis_softmax_masked": ([P, i64, i32, i64, f32, i32, P, P, P, i64, P, P], ctypes.c_int),
         "fqvit_lis_attention_masked": ([P, i64, f32, i32, P, P, P, i64, i32, i64, i32, i32, P, i64, P, i64, P],
                                        ctypes.c_int),
+        "fqvit_lis_attention_masked_q": ([P, i64, f32, i32, P, P, P, i64, i32, i64, i32, i32, f32, f32, i32, P,
+                                          i64, P], ctypes.c_int),
         "fqvit_block_int": ([P, P], ctypes.c_int),
         "fqvit_sync_status": ([P], ctypes.c_int),
         "fqvit_calibrate_ptf_noalloc": ([P, i64, i32, i64, i32, i32, P, P, P, P, P], ctypes.c_int),
@@ -342,6 +344,24 @@ def lis_attention_masked(logits: torch.Tensor, s_logit: float, v: torch.Tensor, 
                                              int(zp_v), BH, L, d, _p(acc), acc.stride(1), _p(codes),
                                              _ld(codes) if codes is not None else 0, _stream(stream)))
     return acc
+
+
+def lis_attention_masked_q(logits: torch.Tensor, s_logit: float, v: torch.Tensor, region: torch.Tensor | None,
+                           mask_value: int, zp_v: int, s_v: float, s_out: float, zp_out: int,
+                           out: torch.Tensor | None = None, bias: torch.Tensor | None = None, heads: int = 1,
+                           window: int = 0, n_shift: int = 15, stream=None) -> torch.Tensor:
+    """Masked fused attention, output requantized to 8 bits (fqvit_lis_attention_masked_q): uint8 [BH, L, d]."""
+    BH, L, d = v.shape
+    if out is None:
+        out = torch.empty(BH, L, d, dtype=torch.uint8, device=v.device)
+    b = _bias(bias, heads, window)
+    m = _mask(region, mask_value)
+    _check(load().fqvit_lis_attention_masked_q(_p(logits), _ld(logits), float(s_logit), n_shift,
+                                               ctypes.byref(b) if b is not None else None,
+                                               ctypes.byref(m) if m is not None else None, _p(v), v.stride(1),
+                                               int(zp_v), BH, L, d, float(s_v), float(s_out), int(zp_out), _p(out),
+                                               out.stride(1), _stream(stream)))
+    return out
 
 
 def block_int(xq, zp_in, alpha, gamma, beta, s_out, zp_out, yq, logits, ld_logit, s_logit, v, zp_v, acc,

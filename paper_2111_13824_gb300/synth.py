@@ -55,6 +55,7 @@ class Stage:
     layers: int        # how many layers of this shape
     calib_rows: int    # calibration rows (32 images)
     window: int = 0    # Swin window side (0 = no relative-position bias)
+    side: int = 0      # Swin feature-map side (tokens per image = side^2)
 
 
 @dataclass(frozen=True)
@@ -84,7 +85,7 @@ def _swin():
         tokens = side * side
         nwin = (side // w) ** 2
         stages.append(Stage(rows=B * tokens, C=C, BH=B * nwin * H, H=H, L=w * w, d=32,
-                            layers=depth, calib_rows=32 * tokens, window=w))
+                            layers=depth, calib_rows=32 * tokens, window=w, side=side))
     return Config(name="swin_s", seed=4, stages=tuple(stages), first_tokens=B * 56 * 56,
                   note="Swin-S, 7x7 windows, relative-position bias")
 
@@ -188,6 +189,22 @@ def attn_inputs(cfg: Config, layer: int, device="cpu", sigma: float = 1.0, bh: i
     logits[:, :L] = qq.reshape(BH * L, L).to(torch.int8)
     return dict(logits=logits, ld_logit=ld, s_logit=s_logit, v=v.contiguous(), bias=bias,
                 heads=st.H, window=st.window, BH=BH, L=L, d=d)
+
+
+def layer_window_mask(cfg: Config, layer: int, device="cpu"):
+    """(region ids uint8 [n_windows, L], n_windows) of a shifted-window layer, else None: in a
+    Swin stage the odd blocks shift their windows by window // 2, unless one window covers the map."""
+    st = layer_stage(cfg, layer)
+    if not st.window or st.side <= st.window:
+        return None
+    block = layer
+    for prev in cfg.stages:
+        if prev is st:
+            break
+        block -= prev.layers
+    if block % 2 == 0:
+        return None
+    return shifted_window_regions(st.side, st.window).to(device)
 
 
 def shifted_window_regions(side: int, window: int, shift: int | None = None) -> torch.Tensor:

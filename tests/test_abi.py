@@ -111,3 +111,8 @@ def test_window_mask_checks(lib):
     assert att(ctypes.byref(fqvit.WindowMask(None, 2, -100))) == 1
     assert att(ctypes.byref(fqvit.WindowMask(fake, 4, -100))) == 1
     assert att(ctypes.byref(fqvit.WindowMask(fake, 2, -32769))) == 2
+    attq = lambda m, zp=0: lib.fqvit_lis_attention_masked_q(  # noqa: E731
+        fake, 64, 0.05, 15, ctypes.byref(b), m, fake, 32, 0, 2 * 3, 49, 32, 0.05, 0.02, zp, fake, 32, None)
+    assert attq(ctypes.byref(fqvit.WindowMask(fake, 4, -100))) == 1
+    assert attq(ctypes.byref(fqvit.WindowMask(fake, 2, -100)), zp=300) == 1
+    assert "zp_out" in _err(lib)

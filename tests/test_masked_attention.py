@@ -172,3 +172,25 @@ def test_null_mask_is_the_plain_call():
     got = fqvit.lis_attention_masked(x, a["s_logit"], v, None, 0, bias=b, heads=3, window=7)
     fqvit.sync_status()
     assert torch.equal(got, want)
+
+
+def test_masked_requantized_output(path):
+    """fqvit_lis_attention_masked_q: the masked accumulators of the oracle, then its 8-bit
+    requantization."""
+    rng = np.random.default_rng(11)
+    heads, L, d = 3, 49, 32
+    region = synth.shifted_window_regions(14, 7).numpy()
+    nw = region.shape[0]
+    bias = rng.integers(-16, 17, size=(heads, 169), dtype=np.int8)
+    BH = 2 * nw * heads
+    x = _logits(rng, BH * L, L, 64)
+    v = rng.integers(-128, 128, size=(BH, L, d), dtype=np.int8)
+    for s, mv, (s_v, s_out, zp_out) in ((0.0347, -2882, (0.05, 0.02, 128)), (0.17, -588, (3 * 2 ** -10, 2 ** -3, 7)),
+                                        (0.0078125, -12800, (0.9, 0.0007, 60))):
+        _, _, ao = _oracle(x, L, s, v, 0, region, mv, bias=bias, heads=heads)
+        want = oracle.attn_requant(ao, s_v, s_out, zp_out)
+        out = fqvit.lis_attention_masked_q(torch.from_numpy(x).to(DEV), s, torch.from_numpy(v).to(DEV),
+                                           torch.from_numpy(region).to(DEV), mv, 0, s_v, s_out, zp_out,
+                                           bias=torch.from_numpy(bias).to(DEV), heads=heads, window=7)
+        fqvit.sync_status()
+        assert np.array_equal(out.cpu().numpy(), want), (s, mv)
