@@ -4,7 +4,9 @@ One step = the whole hot path over one batch: for each of the config's
 layers, the PTF integer LayerNorm (norm1) and the fused Log-Int-Softmax
 attention (codes -> BitShift attn.V), on per-layer synthetic inputs already
 resident in HBM (7.4 GB for ViT-L/384, far above the 129 MB L2, so no flush
-is needed between steps).  Calibration and quantization of the LayerNorm
+is needed between steps).  Swin-S adds its shifted-window mask on the odd
+blocks of stages 1-3 and the LayerNorm of each patch merging (4C channels)
+before stages 2-4.  Calibration and quantization of the LayerNorm
 input are offline (setup), as in post-training quantization.
 
 Algorithmic bytes per layer: LayerNorm 2 bytes per element (int8 in and out)
@@ -109,10 +111,31 @@ def make_layers(cfg, device, sigma=1.0, limit=0):
             region=synth.layer_window_mask(cfg, l, device=device), mask_value=synth.swin_mask_value(a["s_logit"]),
             acc=torch.empty(a["BH"], a["L"], a["d"], dtype=torch.int32, device=device),
             out8=torch.empty(a["BH"], a["L"], a["d"], dtype=torch.uint8, device=device),
-            rows=st.rows, C=st.C, BH=st.BH, L=st.L, d=st.d))
+            rows=st.rows, C=st.C, BH=st.BH, L=st.L, d=st.d, merge=None))
         del d, a
+    # Swin: the patch merging after stage i runs its LayerNorm (4C channels) before stage i+1
+    first = 0
+    for i, st in enumerate(cfg.stages):
+        if i > 0 and (i - 1) in synth.merge_stages(cfg) and first < len(layers):
+            layers[first]["merge"] = make_merge(cfg, i - 1, device)
+        first += st.layers
     torch.cuda.synchronize()
     return layers
+
+
+def make_merge(cfg, stage, device):
+    from paper_2111_13824_gb300 import fqvit
+
+    d = synth.merge_ln_inputs(cfg, stage, device=device)
+    s, zp, alpha = fqvit.calibrate_ptf(d["x_calib"], K=cfg.K)
+    zp_i, s_f = int(zp.item()), float(s.item())
+    xq = fqvit.ptf_quantize(d["x"], s_f, zp_i, alpha)
+    return dict(xq=xq, zp=zp_i, alpha=alpha, gamma=d["gamma"], beta=d["beta"], s_out=d["s_out"], zp_out=d["zp_out"],
+                yq=torch.empty_like(xq), rows=d["rows"], C=d["C"])
+
+
+def layernorm(fq, m):
+    fq.ptf_layernorm(m["xq"], m["zp"], m["alpha"], m["gamma"], m["beta"], m["s_out"], m["zp_out"], out=m["yq"])
 
 
 def attention(fq, ly, out8=False):
@@ -132,8 +155,9 @@ def attention(fq, ly, out8=False):
 
 
 def run_layer(fq, ly, ev=None):
-    fq.ptf_layernorm(ly["xq"], ly["zp"], ly["alpha"], ly["gamma"], ly["beta"], ly["s_out"], ly["zp_out"],
-                     out=ly["yq"])
+    if ly["merge"] is not None:
+        layernorm(fq, ly["merge"])
+    layernorm(fq, ly)
     if ev is not None:
         ev[0].record()
     attention(fq, ly)
@@ -189,8 +213,9 @@ class OracleSample:
     """A bounded sample of one layer for the CPU oracle, scaled to the whole step.
 
     Sample: the LayerNorm of `ln_rows` rows and the Log-Int-Softmax + BitShift
-    attn.V of `heads` attention heads of layer 0; the estimate scales each part to
-    the full layer and multiplies by the number of layers."""
+    attn.V of `heads` attention heads of layer 0; the estimate scales the first by
+    the LayerNorm elements of the whole step (every layer, and Swin's patch
+    mergings) and the second by the step's attention logits."""
 
     def __init__(self, cfg, heads=1, ln_rows=512, layer=0):
         import oracle
@@ -217,12 +242,24 @@ class OracleSample:
                               window=a["window"] or 7)
         o.lis_attn_v(co, self.v, 0)
         t2 = time.perf_counter()
-        layer = (t1 - t0) * self.st.rows / self.ln_rows + (t2 - t1) * self.st.BH / self.heads
-        return layer * self.cfg.layers, t2 - t0
+        ln_elems, logits = step_elements(self.cfg)
+        step = ((t1 - t0) * ln_elems / (self.ln_rows * self.st.C)
+                + (t2 - t1) * logits / (self.heads * self.st.L * self.st.L))
+        return step, t2 - t0
 
     def describe(self):
         return (f"layer 0: LayerNorm of {self.ln_rows} of {self.st.rows} rows and LIS + BitShift attn.V of "
-                f"{self.heads} of {self.st.BH} heads, scaled to the layer and x{self.cfg.layers} layers")
+                f"{self.heads} of {self.st.BH} heads, scaled to the step's LayerNorm elements and attention "
+                f"logits ({self.cfg.layers} layers" + (", patch mergings)" if synth.merge_stages(self.cfg) else ")"))
+
+
+def step_elements(cfg):
+    """(LayerNorm elements, attention logits) of one step over the whole config."""
+    ln = sum(st.layers * st.rows * st.C for st in cfg.stages)
+    for i in synth.merge_stages(cfg):
+        st = cfg.stages[i]
+        ln += (st.rows // 4) * 4 * st.C
+    return ln, sum(st.layers * st.BH * st.L * st.L for st in cfg.stages)
 
 
 # ------------------------------------------------------------------ main arms
@@ -266,10 +303,18 @@ def bench_gpu(args):
     ln_events = [(torch.cuda.Event(**ev_kw), torch.cuda.Event(**ev_kw)) for _ in range(args.steps * len(layers))]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
 
+    merges = [ly["merge"] for ly in layers if ly["merge"] is not None]
+    merge_events = [(torch.cuda.Event(**ev_kw), torch.cuda.Event(**ev_kw)) for _ in range(args.steps * len(merges))]
+
     def enqueue_steps():
-        k = 0
+        k = km = 0
         for _ in range(args.steps):
             for ly in layers:
+                if ly["merge"] is not None:
+                    merge_events[km][0].record()
+                    layernorm(fqvit, ly["merge"])
+                    merge_events[km][1].record()
+                    km += 1
                 ln_events[k][0].record()
                 fqvit.ptf_layernorm(ly["xq"], ly["zp"], ly["alpha"], ly["gamma"], ly["beta"], ly["s_out"],
                                     ly["zp_out"], out=ly["yq"])
@@ -295,6 +340,8 @@ def bench_gpu(args):
                            for _ in range(args.steps * len(layers))]
             ln_events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                          for _ in range(args.steps * len(layers))]
+            merge_events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                            for _ in range(args.steps * len(merges))]
     clocks = ClockSampler(local)
     if ws > 1:
         torch.distributed.barrier()
@@ -326,7 +373,9 @@ def bench_gpu(args):
     lb = [ln_bytes(ly["rows"], ly["C"]) for ly in layers]
     attn_gbs = sum(ab) * args.steps / (sum(attn_ms) / 1e3) / 1e9
     ln_gbs = sum(lb) * args.steps / (sum(ln_ms) / 1e3) / 1e9
-    step_bytes = sum(ab) + sum(lb)
+    mb = [ln_bytes(m["rows"], m["C"]) for m in merges]
+    merge_ms = [a.elapsed_time(b) for a, b in merge_events]
+    step_bytes = sum(ab) + sum(lb) + sum(mb)
     stack_gbs = step_bytes / (ms_per_step / 1e3) / 1e9
     dominant = "attention" if sum(attn_ms) >= sum(ln_ms) else "layernorm"
     dom_gbs = attn_gbs if dominant == "attention" else ln_gbs
@@ -366,6 +415,7 @@ def bench_gpu(args):
             "launch": "cuda_graph" if graph is not None else "eager",
             "attention_output": "uint8 (requantized)" if args.out8 else "int32 accumulators",
             "shifted_window_layers": sum(ly["region"] is not None for ly in layers),
+            "patch_merges": len(merges),
         },
         "hbm_gbs": round(stack_gbs, 1),
         "hbm_frac": round(stack_gbs / peak, 4),
@@ -374,13 +424,17 @@ def bench_gpu(args):
                           "bytes_per_launch": round(sum(ab) / len(ab))},
             "layernorm": {"gbs": round(ln_gbs, 1), "ms_per_launch": round(sum(ln_ms) / len(ln_ms), 5),
                           "bytes_per_launch": round(sum(lb) / len(lb))},
+            **({"patch_merge_layernorm": {
+                "gbs": round(sum(mb) * args.steps / (sum(merge_ms) / 1e3) / 1e9, 1),
+                "ms_per_launch": round(sum(merge_ms) / len(merge_ms), 5),
+                "bytes_per_launch": round(sum(mb) / len(mb))}} if merges else {}),
         },
         "roofline": {"kernel": dominant, "bound": "hbm", "achieved": round(dom_gbs, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(dom_gbs / peak, 4), "traffic": traffic,
                      "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
                      else "fallback"},
         "clocks": clk,
-        "gpu_launches": 2 * len(layers) * args.steps,
+        "gpu_launches": (2 * len(layers) + len(merges)) * args.steps,
     }
     if e2e is not None:
         line["e2e"] = e2e
@@ -400,9 +454,12 @@ def bench_e2e(fqvit, layers, tokens_per_step, args, dev, ws):
         h = {k: ly[k].cpu().pin_memory() for k in ("xq", "logits", "v")}
         h["yq"] = torch.empty_like(ly["yq"], device="cpu").pin_memory()
         h["acc"] = torch.empty_like(ly["acc"], device="cpu").pin_memory()
+        if ly["merge"] is not None:  # the patch merging's LayerNorm input and output
+            h["mxq"] = ly["merge"]["xq"].cpu().pin_memory()
+            h["myq"] = torch.empty_like(ly["merge"]["yq"], device="cpu").pin_memory()
         host.append(h)
-    h2d = sum(h[k].numel() * h[k].element_size() for h in host for k in ("xq", "logits", "v"))
-    d2h = sum(h[k].numel() * h[k].element_size() for h in host for k in ("yq", "acc"))
+    h2d = sum(h[k].numel() * h[k].element_size() for h in host for k in ("xq", "logits", "v", "mxq") if k in h)
+    d2h = sum(h[k].numel() * h[k].element_size() for h in host for k in ("yq", "acc", "myq") if k in h)
     steps = max(1, min(args.steps, args.e2e_steps))
 
     # Three streams, layers pipelined: the inputs of layer l+1 go up while layer l computes and
@@ -427,6 +484,8 @@ def bench_e2e(fqvit, layers, tokens_per_step, args, dev, ws):
                 ly["xq"].copy_(h["xq"], non_blocking=True)
                 ly["logits"].copy_(h["logits"], non_blocking=True)
                 ly["v"].copy_(h["v"], non_blocking=True)
+                if "mxq" in h:
+                    ly["merge"]["xq"].copy_(h["mxq"], non_blocking=True)
                 ev_in[i].record(s_in)
             with torch.cuda.stream(s_cmp):
                 s_cmp.wait_event(ev_in[i])
@@ -438,6 +497,8 @@ def bench_e2e(fqvit, layers, tokens_per_step, args, dev, ws):
                 s_out.wait_event(ev_cmp[i])
                 h["yq"].copy_(ly["yq"], non_blocking=True)
                 h["acc"].copy_(ly["acc"], non_blocking=True)
+                if "myq" in h:
+                    h["myq"].copy_(ly["merge"]["yq"], non_blocking=True)
                 ev_out[i].record(s_out)
             started[i] = True
         # the step ends when its last download has landed
@@ -461,7 +522,8 @@ def bench_e2e(fqvit, layers, tokens_per_step, args, dev, ws):
         ms = float(t.item())
     return {"value": round(tokens_per_step * ws * steps / (ms / 1e3), 1), "unit": "tokens/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps,
-            "how": "per layer: pinned H2D of xq, logits, V; LayerNorm + fused attention; D2H of yq and acc; "
+            "how": "per layer: pinned H2D of xq, logits, V (and a patch merging's xq); LayerNorm(s) + fused "
+                   "attention; D2H of yq and acc (and the merging's yq); "
                    "three streams (upload, compute, download), layers pipelined"}
 
 

@@ -26,6 +26,10 @@ S * 1000 + l, draws in this fixed order):
   keys (Sec. 3.3: 98.8 % of ViT-L attention values are below 1/16).
 * V: int8 uniform in [-128, 127], zero point 0.
 * Swin relative-position bias: int8 ``[H, (2w-1)^2]`` uniform in [-16, 16].
+* Swin patch merging (after stages 1-3): the stage's channel model drawn
+  on its side x side map (generator seed S * 1000 + 500 + stage), each 2x2
+  neighbourhood concatenated into one token of 4C channels (``patch_merge``),
+  then gamma, beta and the output quantizer as for a layer.
 * Swin shifted-window mask (odd blocks of a stage whose side exceeds the
   window): region ids ``[n_windows, w*w]`` of the cyclically shifted map
   (three bands per axis: below side - w, below side - shift, the rest;
@@ -145,7 +149,12 @@ def ln_inputs(cfg: Config, layer: int, device="cpu", rows: int | None = None):
     xc = _channel_values(g, st.calib_rows, r, m)
     gamma = (1.0 + 0.1 * torch.randn(st.C, generator=g, device=device)).to(torch.float32)
     beta = (0.1 * torch.randn(st.C, generator=g, device=device)).to(torch.float32)
-    # output quantizer: MinMax of a textbook fp64 LayerNorm of the calibration batch
+    s_out, zp_out = _ln_output_quantizer(xc, gamma, beta)
+    return dict(x=x, x_calib=xc, gamma=gamma, beta=beta, s_out=s_out, zp_out=zp_out, C=st.C, rows=n)
+
+
+def _ln_output_quantizer(xc, gamma, beta):
+    """MinMax (0..255) of a textbook fp64 LayerNorm of the calibration batch: (s_out fp32, zp_out)."""
     xd = xc.double()
     mu = xd.mean(dim=1, keepdim=True)
     var = xd.var(dim=1, unbiased=False, keepdim=True)
@@ -153,8 +162,40 @@ def ln_inputs(cfg: Config, layer: int, device="cpu", rows: int | None = None):
     lo, hi = float(yf.min()), float(yf.max())
     s_out = (hi - lo) / 255.0
     zp_out = int(min(255, max(0, round(-lo / s_out))))
-    return dict(x=x, x_calib=xc, gamma=gamma, beta=beta, s_out=float(torch.tensor(s_out, dtype=torch.float32)),
-                zp_out=zp_out, C=st.C, rows=n)
+    return float(torch.tensor(s_out, dtype=torch.float32)), zp_out
+
+
+def merge_stages(cfg: Config) -> tuple:
+    """Indices of the stages followed by a patch merging (every Swin stage but the last)."""
+    return tuple(i for i, st in enumerate(cfg.stages[:-1]) if st.window and st.side >= 2)
+
+
+def patch_merge(x: torch.Tensor, side: int) -> torch.Tensor:
+    """[images * side^2, C] tokens in raster order -> [images * (side/2)^2, 4C]: each merged token
+    is the concatenation of its 2x2 neighbours (y, x), (y+1, x), (y, x+1), (y+1, x+1)."""
+    C = x.shape[1]
+    g = x.reshape(-1, side // 2, 2, side // 2, 2, C)       # image, y/2, y%2, x/2, x%2, c
+    return g.permute(0, 1, 3, 4, 2, 5).reshape(-1, 4 * C)  # neighbour order: (x%2, y%2) = 00, 01, 10, 11
+
+
+def merge_ln_inputs(cfg: Config, stage: int, device="cpu", images: int | None = None):
+    """Inputs of the LayerNorm of the patch merging after Swin stage ``stage`` (4C channels):
+    tokens of the stage's channel model on its side x side map, gathered 2x2.  ``images``
+    defaults to the batch (the stage's rows / side^2); the calibration batch is 32 images.
+    Generator seeded with seed * 1000 + 500 + stage; draws: channel model, tokens,
+    calibration tokens, gamma, beta."""
+    st = cfg.stages[stage]
+    g = _gen(cfg.seed * 1000 + 500 + stage, device)
+    r, m = _channel_model(g, st.C, cfg.outliers, device)
+    nimg = st.rows // (st.side * st.side) if images is None else images
+    x = patch_merge(_channel_values(g, nimg * st.side * st.side, r, m), st.side)
+    xc = patch_merge(_channel_values(g, 32 * st.side * st.side, r, m), st.side)
+    C4 = 4 * st.C
+    gamma = (1.0 + 0.1 * torch.randn(C4, generator=g, device=device)).to(torch.float32)
+    beta = (0.1 * torch.randn(C4, generator=g, device=device)).to(torch.float32)
+    s_out, zp_out = _ln_output_quantizer(xc, gamma, beta)
+    return dict(x=x.contiguous(), x_calib=xc.contiguous(), gamma=gamma, beta=beta, s_out=s_out, zp_out=zp_out,
+                C=C4, rows=x.shape[0])
 
 
 def attn_inputs(cfg: Config, layer: int, device="cpu", sigma: float = 1.0, bh: int | None = None):
