@@ -66,6 +66,8 @@ def _load():
     lib.or_lis_attn_v.argtypes = [P, i64, P, i64, i32, i64, i32, i32, P, i64]
     lib.or_attn_requant.restype = ctypes.c_int
     lib.or_attn_requant.argtypes = [P, i64, i32, i64, f32, f32, i32, P, i64]
+    lib.or_qk_logits.restype = ctypes.c_int
+    lib.or_qk_logits.argtypes = [P, i64, i32, P, i64, i32, i64, i32, i32, f32, f32, f32, i32, P, i64]
     lib.or_lis_attn_v.restype = ctypes.c_int
     lib.or_num_threads.argtypes = []
     lib.or_num_threads.restype = ctypes.c_int
@@ -236,6 +238,23 @@ def lis_softmax(logits: np.ndarray, L: int, s: float, n: int = 15, bias=None, he
     if rc:
         raise ValueError("or_lis_softmax rejected its arguments")
     return codes, rowsum
+
+
+def qk_logits(q: np.ndarray, k: np.ndarray, zp_q: int, zp_k: int, s_q: float, s_k: float, s_logit: float,
+              zp_l: int, ld: int | None = None) -> np.ndarray:
+    """The MatMul Q K^T and its MinMax 8-bit output quantizer with the dyadic multiplier of the
+    LayerNorm output stage: q, k int8 [BH, L, d] -> int8 logits [BH*L, ld] (ld >= L, zero padding)."""
+    q = _c(q, np.int8)
+    k = _c(k, np.int8)
+    BH, L, d = q.shape
+    assert k.shape == q.shape
+    ld = L if ld is None else ld
+    out = np.zeros((BH * L, ld), np.int8)
+    rc = _load().or_qk_logits(_ptr(q), d, int(zp_q), _ptr(k), d, int(zp_k), BH, L, d, np.float32(s_q),
+                              np.float32(s_k), np.float32(s_logit), int(zp_l), _ptr(out), ld)
+    if rc:
+        raise ValueError("or_qk_logits rejected its arguments")
+    return out
 
 
 def lis_attn_v(codes: np.ndarray, v: np.ndarray, zp_v: int = 0):

@@ -470,6 +470,70 @@ OR_EXPORT int or_attn_requant(const int32_t *acc, int64_t rows, int32_t d, int64
 }
 
 /* ------------------------------------------------------------------ */
+/* The MatMul Q K^T and its 8-bit output quantizer (the logits)        */
+/* ------------------------------------------------------------------ */
+
+/*
+ * Sec. 3 quantizes the MatMul modules with uniform MinMax, and Sec. 4.1 takes
+ * activations asymmetric (a zero point): Q and K arrive as 8-bit codes with
+ * zero points, and the product's output -- the logits fed to Log-Int-Softmax --
+ * is quantized to 8 bits with the logit scale s_logit and zero point zp_l.
+ *   P[bh][i][j] = sum_t (q[bh][i][t] - zp_q) (k[bh][j][t] - zp_k)     (int64)
+ * P s_q s_k / sqrt(d) is the real logit.  Integer-only, the rescaling is the
+ * dyadic multiplier of the supplement's LayerNorm output stage:
+ *   M  = (s_q s_k) / (sqrt(d) s_logit)  in fp32, in this order:
+ *        a = s_q s_k,  r = sqrtf(d),  c = r s_logit,  M = a / c
+ *   N1 = 7 - floor(log2 M)  (at most 31),   N2 = floor(M 2^N1)
+ *   logit = clip(floor((N2 P + 2^(N1-1)) / 2^N1) + zp_l, -128, 127)   N1 > 0
+ *   logit = clip(N2 P 2^min(-N1, 10) + zp_l, -128, 127)                N1 <= 0
+ * Logits are signed: the 8-bit code minus 128, zp_l likewise (the form the
+ * Log-Int-Softmax functions take; the softmax only sees differences).
+ * q [BH][L][ld_q], k [BH][L][ld_k] (d values per row), logits [BH*L][ld_logit]
+ * (row i of head bh at bh*L + i, key j in byte j).
+ */
+OR_EXPORT int or_qk_logits(const int8_t *q, int64_t ld_q, int32_t zp_q, const int8_t *k, int64_t ld_k,
+                           int32_t zp_k, int64_t BH, int32_t L, int32_t d, float s_q, float s_k,
+                           float s_logit, int32_t zp_l, int8_t *logits, int64_t ld_logit)
+{
+    if (!q || !k || !logits || BH < 1 || L < 1 || d < 1 || ld_q < d || ld_k < d || ld_logit < L) return 1;
+    if (!(s_q > 0.0f) || !(s_k > 0.0f) || !(s_logit > 0.0f)) return 1;
+    const float a = s_q * s_k;
+    const float r = sqrtf((float)d);
+    const float c = r * s_logit;
+    const float M = a / c;
+    if (!(M > 0.0f) || !(M < INFINITY)) return 1;
+    int N1 = 7 - ilogbf(M);
+    if (N1 > 31) N1 = 31;
+    const int64_t N2 = (int64_t)floorf(ldexpf(M, N1));
+#ifdef _OPENMP
+#pragma omp parallel for schedule(static)
+#endif
+    for (int64_t bh = 0; bh < BH; ++bh) {
+        for (int32_t i = 0; i < L; ++i) {
+            const int8_t *qi = q + (bh * L + i) * ld_q;
+            for (int32_t j = 0; j < L; ++j) {
+                const int8_t *kj = k + (bh * L + j) * ld_k;
+                int64_t P = 0;
+                for (int32_t t = 0; t < d; ++t) P += ((int64_t)qi[t] - zp_q) * ((int64_t)kj[t] - zp_k);
+                const int64_t num = N2 * P;
+                int64_t R;
+                if (N1 > 0)
+                    R = floor_div_pow2(num + ((int64_t)1 << (N1 - 1)), N1);
+                else if (N1 == 0)
+                    R = num;
+                else {
+                    int sh = -N1;
+                    if (sh > 10) sh = 10;
+                    R = num * ((int64_t)1 << sh);
+                }
+                logits[(bh * L + i) * ld_logit + j] = (int8_t)clamp_i64(R + zp_l, -128, 127);
+            }
+        }
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
 /* Eq. 15 and the supplement's Attn.V: BitShift attention times values */
 /* ------------------------------------------------------------------ */
 
