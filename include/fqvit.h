@@ -304,6 +304,60 @@ FQVIT_API int fqvit_lis_attention_masked_q(const int8_t *logits, int64_t ld_logi
                           uint8_t *out, int64_t ld_out, void *stream);
 
 /* ------------------------------------------------------------------ */
+/* The MatMul Q K^T and its 8-bit output (Sec. 3 MinMax; Sec. 4.1)     */
+/* ------------------------------------------------------------------ */
+
+/*
+ * Logits of attention from 8-bit Q and K codes.  Sec. 3 quantizes MatMul
+ * outputs with uniform MinMax and Sec. 4.1 takes activations asymmetric, so Q
+ * and K come with zero points and the product is quantized to 8 bits:
+ *   P[bh][i][j] = sum_t (q[bh][i][t] - zp_q) (k[bh][j][t] - zp_k)   (exact)
+ *   M  = (s_q s_k) / (sqrt(d) s_logit)  (fp32: a = s_q s_k, r = sqrtf(d),
+ *        c = r s_logit, M = a / c),
+ *   N1 = 7 - floor(log2 M) (at most 31), N2 = floor(M 2^N1)  (the dyadic
+ *        multiplier of the supplement's LayerNorm output stage),
+ *   logit = clip(floor((N2 P + 2^(N1-1)) / 2^N1) + zp_logit, -128, 127)
+ *        (N1 <= 0: clip(N2 P 2^min(-N1, 10) + zp_logit, ...)).
+ * Logits are signed (the 8-bit code minus 128; zp_logit likewise): the form
+ * fqvit_lis_softmax and fqvit_lis_attention take.
+ * q [BH][L][ld_q], k [BH][L][ld_k] int8 (device), d values per row;
+ * logits [BH*L][ld_logit] int8 (device, caller-owned): row i of head bh at
+ * bh*L + i, key j at byte j, bytes L .. ld_logit-1 of a row written as 0.
+ * Supported: 1 <= L <= 640, d <= 64 a multiple of 8, ld_q and ld_k multiples
+ * of 8 with 8-byte aligned bases, ld_logit a multiple of 16 with a 16-byte
+ * aligned base, zero points in -128..127.  Errors: INVALID_ARG (NULL, shapes,
+ * strides, alignment, zero points, scales not positive and finite),
+ * UNSUPPORTED (L, d, or M outside the fp32 range).
+ */
+FQVIT_API int fqvit_qk_logits(const int8_t *q, int64_t ld_q, int32_t zp_q, const int8_t *k, int64_t ld_k,
+                              int32_t zp_k, int64_t BH, int32_t L, int32_t d, float s_q, float s_k,
+                              float s_logit, int32_t zp_logit, int8_t *logits, int64_t ld_logit, void *stream);
+
+/* Bytes of logits workspace fqvit_qk_lis_attention needs for groups of
+ * group_heads heads (<= 0: the library's choice, at most 48 MiB of logits so
+ * that a group's logits stay in the 129 MB L2 between its two kernels):
+ * group x L x ld with ld = L rounded up to 16.  0 for a bad shape. */
+FQVIT_API size_t fqvit_qk_workspace_size(int64_t BH, int32_t L, int64_t group_heads);
+
+/*
+ * Attention from 8-bit Q, K and V: fqvit_qk_logits, then
+ * fqvit_lis_attention_masked on those logits (same arguments, bias and mask
+ * optional), group after group of heads on the caller's stream; the logits of
+ * a group live in `workspace` (device, caller-owned, at least one group:
+ * fqvit_qk_workspace_size) and are overwritten by the next group.  Groups are
+ * multiples of heads (bias) x n_windows (mask), at most group_heads (<= 0: the
+ * library's choice) and what the workspace holds.  acc as in
+ * fqvit_lis_attention.  Errors: those of the two functions; INVALID_ARG when
+ * the workspace holds less than one group.
+ */
+FQVIT_API int fqvit_qk_lis_attention(const int8_t *q, int64_t ld_q, int32_t zp_q, const int8_t *k, int64_t ld_k,
+                              int32_t zp_k, float s_q, float s_k, float s_logit, int32_t zp_logit,
+                              int32_t n_shift, const fqvit_relpos_bias *bias_opt,
+                              const fqvit_window_mask *mask_opt, const int8_t *v, int64_t ld_v,
+                              int32_t zp_v, int64_t BH, int32_t L, int32_t d, int32_t *acc, int64_t ld_acc,
+                              int8_t *workspace, size_t workspace_bytes, int64_t group_heads, void *stream);
+
+/* ------------------------------------------------------------------ */
 /* One layer: norm1 LayerNorm and the attention core (Fig. 4 dataflow) */
 /* ------------------------------------------------------------------ */
 

@@ -403,6 +403,126 @@ int fqvit_lis_attention_masked(const int8_t *logits, int64_t ld_logit, float s_l
     return cuda_status(fqvit::launch_lis_attention(la, a, as_stream(stream)), "lis_attention_masked");
 }
 
+// The logits' dyadic multiplier: M = (s_q s_k) / (sqrt(d) s_logit) in fp32 in this order,
+// N1 = 7 - floor(log2 M) (at most 31), N2 = floor(M 2^N1).
+static int qk_multiplier(float s_q, float s_k, float s_logit, int32_t d, int *n1, int *n2, const char *who)
+{
+    if (!(s_q > 0.0f) || !(s_q < 3.0e38f) || !(s_k > 0.0f) || !(s_k < 3.0e38f) || !(s_logit > 0.0f) ||
+        !(s_logit < 3.0e38f))
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: s_q, s_k and s_logit must be positive and finite", who);
+    const float a = s_q * s_k;
+    const float r = sqrtf((float)d);
+    const float c = r * s_logit;
+    const float M = a / c;
+    if (!(M > 0.0f) || !(M < 1.0e30f))
+        return fail(FQVIT_ERR_UNSUPPORTED, "%s: s_q s_k / (sqrt(d) s_logit) out of range", who);
+    int N1 = 7 - ilogbf(M);
+    if (N1 > 31) N1 = 31;
+    *n1 = N1;
+    *n2 = (int)floorf(ldexpf(M, N1));
+    return FQVIT_OK;
+}
+
+static int check_qk(const fqvit::QkArgs &a, const char *who)
+{
+    if (!a.q || !a.k || !a.logits) return fail(FQVIT_ERR_INVALID_ARG, "%s: NULL pointer", who);
+    if (a.BH < 1 || a.L < 1 || a.d < 1)
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: bad shape BH=%lld L=%d d=%d", who, (long long)a.BH, a.L, a.d);
+    if (a.ld_q < a.d || a.ld_k < a.d || a.ld_logit < a.L)
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: a row stride is below its row", who);
+    if (a.zp_q < -128 || a.zp_q > 127 || a.zp_k < -128 || a.zp_k > 127 || a.zp_l < -128 || a.zp_l > 127)
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: zero points outside -128..127", who);
+    if (a.L > 640 || a.d > 64 || a.d % 8 != 0)
+        return fail(FQVIT_ERR_UNSUPPORTED, "%s: L=%d d=%d (L <= 640, d <= 64 a multiple of 8)", who, a.L, a.d);
+    if (a.ld_q % 8 || a.ld_k % 8 || !aligned(a.q, 8) || !aligned(a.k, 8))
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: Q and K rows must be 8-byte aligned", who);
+    if (a.ld_logit % 16 || !aligned(a.logits, 16))
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: logits rows must be 16-byte aligned", who);
+    if (!fqvit::qk_logits_supported(a)) return fail(FQVIT_ERR_UNSUPPORTED, "%s: shape not supported", who);
+    return FQVIT_OK;
+}
+
+int fqvit_qk_logits(const int8_t *q, int64_t ld_q, int32_t zp_q, const int8_t *k, int64_t ld_k, int32_t zp_k,
+                    int64_t BH, int32_t L, int32_t d, float s_q, float s_k, float s_logit, int32_t zp_logit,
+                    int8_t *logits, int64_t ld_logit, void *stream)
+{
+    fqvit::QkArgs a{q, ld_q, zp_q, k, ld_k, zp_k, BH, L, d, 0, 0, zp_logit, logits, ld_logit};
+    int rc = qk_multiplier(s_q, s_k, s_logit, d, &a.n1, &a.n2, "qk_logits");
+    if (rc) return rc;
+    rc = check_qk(a, "qk_logits");
+    if (rc) return rc;
+    return cuda_status(fqvit::launch_qk_logits(a, as_stream(stream)), "qk_logits");
+}
+
+// Heads per group of the chained attention: at most 48 MiB of logits (they stay in L2 between
+// the two kernels), a multiple of the unit the bias and the mask index by.
+static int64_t qk_group_heads(int64_t BH, int32_t L, int64_t unit, int64_t requested)
+{
+    const int64_t row = (int64_t)L * (((int64_t)L + 15) / 16 * 16);
+    int64_t g = requested > 0 ? requested : ((int64_t)48 << 20) / row;
+    g = g / unit * unit;
+    if (g < unit) g = unit;
+    return g < BH ? g : BH;
+}
+
+size_t fqvit_qk_workspace_size(int64_t BH, int32_t L, int64_t group_heads)
+{
+    if (BH < 1 || L < 1) return 0;
+    const int64_t g = qk_group_heads(BH, L, 1, group_heads);
+    return (size_t)g * L * (((size_t)L + 15) / 16 * 16);
+}
+
+int fqvit_qk_lis_attention(const int8_t *q, int64_t ld_q, int32_t zp_q, const int8_t *k, int64_t ld_k,
+                           int32_t zp_k, float s_q, float s_k, float s_logit, int32_t zp_logit, int32_t n_shift,
+                           const fqvit_relpos_bias *bias_opt, const fqvit_window_mask *mask_opt, const int8_t *v,
+                           int64_t ld_v, int32_t zp_v, int64_t BH, int32_t L, int32_t d, int32_t *acc,
+                           int64_t ld_acc, int8_t *workspace, size_t workspace_bytes, int64_t group_heads,
+                           void *stream)
+{
+    const char *who = "qk_lis_attention";
+    const int64_t ld = ((int64_t)L + 15) / 16 * 16;
+    fqvit::QkArgs qa{q, ld_q, zp_q, k, ld_k, zp_k, BH, L, d, 0, 0, zp_logit, workspace, ld};
+    int rc = qk_multiplier(s_q, s_k, s_logit, d, &qa.n1, &qa.n2, who);
+    if (rc) return rc;
+    rc = check_qk(qa, who);
+    if (rc) return rc;
+    rc = check_attnv(v, ld_v, zp_v, BH, L, d, acc, ld_acc, who);
+    if (rc) return rc;
+    // the Log-Int-Softmax checks on a stand-in for the logits (the workspace, one group's rows)
+    rc = check_lis(workspace, BH * L, L, ld, s_logit, n_shift, bias_opt, who);
+    if (rc) return rc;
+    rc = check_mask(mask_opt, bias_opt, BH * L, L, who);
+    if (rc) return rc;
+    const int64_t unit = (int64_t)(bias_opt ? bias_opt->heads : 1) * (mask_opt ? mask_opt->n_windows : 1);
+    int64_t g = qk_group_heads(BH, L, unit, group_heads);
+    const int64_t fit = (int64_t)(workspace_bytes / (size_t)(L * ld)) / unit * unit;
+    if (fit < unit)
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: workspace of %zu bytes holds fewer than %lld heads", who,
+                    workspace_bytes, (long long)unit);
+    if (g > fit) g = fit;
+    cudaStream_t st = as_stream(stream);
+    for (int64_t h0 = 0; h0 < BH; h0 += g) {
+        const int64_t n = BH - h0 < g ? BH - h0 : g;
+        fqvit::QkArgs a = qa;
+        a.q = q + h0 * L * ld_q;
+        a.k = k + h0 * L * ld_k;
+        a.BH = n;
+        cudaError_t e = fqvit::launch_qk_logits(a, st);
+        if (e != cudaSuccess) return cuda_status(e, who);
+        fqvit::LisArgs la{workspace, n * L, L, ld, s_logit, bias_opt ? bias_opt->table : nullptr,
+                          bias_opt ? bias_opt->heads : 1, bias_opt ? bias_opt->window : 0, nullptr, 0, nullptr};
+        if (mask_opt) {
+            la.region = mask_opt->region;
+            la.n_windows = mask_opt->n_windows;
+            la.mask_value = mask_opt->mask_value;
+        }
+        fqvit::AttnVArgs b{nullptr, 0, v + h0 * L * ld_v, ld_v, zp_v, n, L, d, acc + h0 * L * ld_acc, ld_acc, nullptr};
+        e = fqvit::launch_lis_attention(la, b, st);
+        if (e != cudaSuccess) return cuda_status(e, who);
+    }
+    return ok();
+}
+
 int fqvit_block_int(const fqvit_block_desc *b, void *stream)
 {
     if (!b) return fail(FQVIT_ERR_INVALID_ARG, "block_int: NULL descriptor");

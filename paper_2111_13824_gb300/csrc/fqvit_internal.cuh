@@ -113,6 +113,26 @@ cudaError_t launch_lis_attn_v(const AttnVArgs &a, cudaStream_t st);
 // fused softmax + attn.V; codes written only when a.codes != nullptr
 cudaError_t launch_lis_attention(const LisArgs &a, const AttnVArgs &b, cudaStream_t st);
 
+// Q K^T with its 8-bit output quantizer on the tensor cores (qk_tc.cu):
+// logit = clip(floor((n2 P + 2^(n1-1)) / 2^n1) + zp_l, -128, 127), P = (Q - zp_q)(K - zp_k)^T
+struct QkArgs {
+    const int8_t *q;
+    int64_t ld_q;
+    int zp_q;
+    const int8_t *k;
+    int64_t ld_k;
+    int zp_k;
+    int64_t BH;
+    int L;
+    int d;
+    int n1, n2, zp_l;
+    int8_t *logits;
+    int64_t ld_logit;
+};
+bool qk_logits_supported(const QkArgs &a);
+cudaError_t launch_qk_logits(const QkArgs &a, cudaStream_t st);
+cudaError_t read_clear_qk_status(int *status);
+
 // tensor-core (tcgen05) fused path (lis_tc.cu)
 bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b);
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st);

@@ -618,7 +618,11 @@ cudaError_t read_clear_device_status(int *status, cudaStream_t st)
     if (e != cudaSuccess) return e;
     int wst = 0;
     e = read_clear_win_status(&wst);
+    if (e != cudaSuccess) return e;
     if (*status == 0) *status = wst;
+    int qst = 0;
+    e = read_clear_qk_status(&qst);
+    if (*status == 0) *status = qst;
     return e;
 }
 

@@ -1,0 +1,333 @@
+// qk_tc.cu -- the MatMul Q K^T of attention with its 8-bit output quantizer, on
+// the 5th-generation tensor cores (tcgen05) of sm_103a: int8 Q and K codes with
+// zero points in, int8 logits out (the input of Log-Int-Softmax).
+//
+// P = (Q - zp_q)(K - zp_k)^T is exact on the tensor cores: every shifted code
+// lies in -255 .. 255 (exact in fp16), every product below 2^16, and a sum of
+// at most 64 of them below 2^22, exact in the fp32 accumulators.  The output
+// quantizer is uniform MinMax (Sec. 3) applied with the dyadic multiplier of
+// the supplement's LayerNorm output stage, M = s_q s_k / (sqrt(d) s_logit) as
+// N2 / 2^N1:
+//   logit = clip(floor((N2 P + 2^(N1-1)) / 2^N1) + zp_l, -128, 127).
+// With |P| < 2^22 and N2 < 2^8, N2 P + 2^(N1-1) fits 31 bits, so the epilogue
+// runs in 32-bit integers: the accumulator's bits plus 1.5 2^23 give P, one
+// multiply-add, one arithmetic shift, and a saturating pack of four values.
+//
+// One CTA per SM walks (head, 128-row tile) work items, each CTA a contiguous
+// range, so consecutive tiles share a head.  Per head, K -> fp16 in shared
+// memory (B operand: keys x 64, K-major, 128-byte swizzle, d padded to 64 with
+// zeros); per tile, the 128 query rows of Q likewise (A operand).  The keys go
+// through the tensor cores in chunks of 128 (M = 128, N <= 128, K = 64) into two
+// tensor-memory buffers, one chunk ahead of the epilogue; the 16 warps read a
+// chunk back (warp w: lanes 32 (w % 4) .., columns 32 (w / 4) ..), quantize it
+// and write the bytes into a shared-memory tile of the output, which one bulk
+// copy sends to global memory (a tile's rows are contiguous there).  Every
+// wait is bounded: after two seconds the kernel records a timeout status,
+// drains what it issued and returns.
+#include "fqvit_internal.cuh"
+#include "tc_common.cuh"
+
+#include <cmath>
+#include <cuda_fp16.h>
+
+namespace fqvit {
+
+namespace {
+
+using namespace tc;
+
+constexpr int QM = 128;          // query rows per tile (MMA M)
+constexpr int QNC = 128;         // keys per chunk (MMA N of a full chunk)
+constexpr int QKD = 64;          // the MMA's reduction: d padded to 64
+constexpr int QTHREADS = 512;
+constexpr int QMAXL = 640;       // keys of the longest row
+constexpr int QROW = QKD * 2;    // bytes of an fp16 operand row
+
+struct QkParams {
+    const int8_t *q, *k;
+    int64_t ld_q, ld_k;
+    int zp_q, zp_k;
+    int8_t *out;
+    int64_t ld;
+    int64_t BH;
+    int L, d;
+    int n1;       // N1 >= 1 (the host sends N1 <= 0 to the 64-bit epilogue)
+    uint32_t c1;  // 2^(N1-1) + zp_l 2^N1 - N2 (0x4B400000): the constant of the multiply-add (mod 2^32)
+    int n2;
+    int zp_l;
+};
+
+struct QkShared {
+    uint64_t sfull[2], fin;
+    uint32_t tmem;
+    int abort_flag;
+    int stop;
+};
+
+__device__ __forceinline__ uint32_t pack_sat_s8(int hi, int lo, uint32_t c)
+{
+    uint32_t d;  // bits 31..16: c[15:0], 15..8: sat(hi), 7..0: sat(lo)
+    asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(hi), "r"(lo), "r"(c));
+    return d;
+}
+
+// eight int8 codes minus a zero point -> eight fp16 values (exact: -255 .. 255)
+__device__ __forceinline__ uint4 codes_to_h8(uint2 w, __half2 z)
+{
+    const uint32_t x0 = w.x ^ 0x80808080u, x1 = w.y ^ 0x80808080u;
+    uint32_t h[4] = {i8x2_to_h2(x0, 0x5140), i8x2_to_h2(x0, 0x7362), i8x2_to_h2(x1, 0x5140), i8x2_to_h2(x1, 0x7362)};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        __half2 t = __hsub2(*reinterpret_cast<const __half2 *>(&h[i]), z);
+        h[i] = *reinterpret_cast<const uint32_t *>(&t);
+    }
+    return make_uint4(h[0], h[1], h[2], h[3]);
+}
+
+// The logit of one accumulator (an exact integer P in fp32, |P| < 2^22).
+//   FOLD: (N2 P + 2^(N1-1) + zp_l 2^N1) >> N1 in 32 bits (the host checked that it fits)
+//   else: the 64-bit formula, N1 of any sign
+template <bool FOLD>
+__device__ __forceinline__ int logit_of(uint32_t acc_bits, const QkParams &p)
+{
+    if (FOLD) {
+        const uint32_t x = __float_as_uint(__fadd_rn(__uint_as_float(acc_bits), 12582912.0f));
+        return (int)(x * (uint32_t)p.n2 + p.c1) >> p.n1;
+    } else {
+        const int P = __float2int_rn(__uint_as_float(acc_bits));
+        const long long num = (long long)p.n2 * P;
+        long long R;
+        if (p.n1 > 0)
+            R = (num + (1ll << (p.n1 - 1))) >> p.n1;
+        else
+            R = num * (1ll << min(-p.n1, 10));
+        R += p.zp_l;
+        return (int)(R < -128 ? -128 : R > 127 ? 127 : R);
+    }
+}
+
+template <bool FOLD>
+__global__ void __launch_bounds__(QTHREADS, 1) qk_logits_tc_kernel(QkParams p)
+{
+    extern __shared__ unsigned char dsm_raw[];
+    __shared__ QkShared sh;
+    unsigned char *base = dsm_raw + ((1024u - (sa(dsm_raw) & 1023u)) & 1023u);
+    unsigned char *KS = base;                            // QMAXL x 128 B (keys, fp16, swizzled)
+    unsigned char *QS = KS + QMAXL * QROW;               // QM x 128 B
+    unsigned char *OS = QS + QM * QROW;                  // QM x ld bytes: the output tile
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    volatile int *abort_flag = &sh.abort_flag;
+    volatile int *stop = &sh.stop;
+    if (tid == 0) {
+        mbar_init(&sh.sfull[0], 1);
+        mbar_init(&sh.sfull[1], 1);
+        mbar_init(&sh.fin, 1);
+        sh.abort_flag = 0;
+        sh.stop = 0;
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(&sh.tmem)),
+                     "r"(2 * QNC));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    const int L = p.L, d = p.d;
+    const int L16 = (L + 15) & ~15;                     // keys that go through the MMAs
+    const int nch = (L + QNC - 1) / QNC;
+    // bytes of each output row past the MMA'd keys (up to ld) stay zero for the whole launch
+    for (int x = tid; x < QM * (int)(p.ld - L16); x += QTHREADS) {
+        const int r = x / (int)(p.ld - L16), j = x - r * (int)(p.ld - L16);
+        OS[(size_t)r * p.ld + L16 + j] = 0;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sh.tmem;
+
+    const int tpb = (L + QM - 1) / QM;
+    const int64_t ntiles = p.BH * tpb;
+    const int64_t t_begin = (int64_t)blockIdx.x * ntiles / gridDim.x;
+    const int64_t t_end = (int64_t)(blockIdx.x + 1) * ntiles / gridDim.x;
+    // instruction descriptor: D f32, A/B f16 K-major, M = 128, N = n
+    auto idesc = [](int n) -> uint32_t { return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(QM >> 4) << 24); };
+    const __half2 zq2 = __half2half2(__int2half_rn(p.zp_q)), zk2 = __half2half2(__int2half_rn(p.zp_k));
+
+    uint32_t use[2] = {0, 0};  // completed phases of each tensor-memory buffer
+    uint32_t issued = 0;       // MMA commits issued (thread 0)
+    int cur_bh = -1;
+    bool stores = false;       // a bulk store is in flight (thread 0)
+    for (int64_t t = t_begin; t < t_end; ++t) {
+        const int bh = (int)(t / tpb);
+        const int r0 = (int)(t - (int64_t)bh * tpb) * QM;
+        // ---- operands: K of a new head, the tile's Q rows (8 values = 16 bytes of fp16 per item)
+        if (bh != cur_bh) {
+            for (int x = tid; x < L16 * 8; x += QTHREADS) {
+                const int key = x >> 3, c = x & 7;
+                uint4 h = make_uint4(0, 0, 0, 0);
+                if (key < L && 8 * c < d)
+                    h = codes_to_h8(
+                        __ldg(reinterpret_cast<const uint2 *>(p.k + ((size_t)bh * L + key) * p.ld_k + 8 * c)), zk2);
+                *reinterpret_cast<uint4 *>(KS + key * QROW + ((c ^ (key & 7)) << 4)) = h;
+            }
+            cur_bh = bh;
+        }
+        for (int x = tid; x < QM * 8; x += QTHREADS) {
+            const int r = x >> 3, c = x & 7;
+            uint4 h = make_uint4(0, 0, 0, 0);
+            if (r0 + r < L && 8 * c < d)
+                h = codes_to_h8(
+                    __ldg(reinterpret_cast<const uint2 *>(p.q + ((size_t)bh * L + r0 + r) * p.ld_q + 8 * c)), zq2);
+            *reinterpret_cast<uint4 *>(QS + r * QROW + ((c ^ (r & 7)) << 4)) = h;
+        }
+        fence_async_smem();  // the operands are read by the MMAs
+        if (tid == 0 && stores) {  // the previous tile's bulk store has read the output tile
+            asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+            stores = false;
+        }
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+        if (*stop) break;
+        // ---- the first two chunks
+        auto issue = [&](int c) {
+            const int n = min(QNC, L16 - c * QNC);
+            const uint32_t a0 = sa(QS), b0 = sa(KS) + (uint32_t)(c * QNC * QROW);
+#pragma unroll
+            for (int s = 0; s < QKD / 16; ++s)
+                mma_f16_ss(tmem + (uint32_t)((c & 1) * QNC), smem_desc(a0 + 32 * s, 16, 1024),
+                           smem_desc(b0 + 32 * s, 16, 1024), idesc(n), s != 0);
+            mma_commit(&sh.sfull[c & 1]);
+            ++issued;
+        };
+        if (tid == 0) {
+            issue(0);
+            if (nch > 1) issue(1);
+        }
+        // ---- chunks: read back, quantize, into the output tile
+        const int qr = 32 * (warp & 3) + lane;  // tile row of this thread
+        const int g = warp >> 2;                // 32-column group of a chunk
+        bool bad = false;
+        for (int c = 0; c < nch; ++c) {
+            const int b = c & 1;
+            if (!mbar_wait_warp(&sh.sfull[b], use[b] & 1, abort_flag)) {
+                bad = true;
+                *stop = 1;
+            }
+            ++use[b];
+            tc_fence_after();
+            const int col0 = c * QNC + 32 * g;  // first key of this warp's 32 columns
+            if (!bad && col0 < L16) {
+                uint32_t v[32];
+                tmem_ld32(tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(b * QNC + 32 * g), v);
+                tmem_wait_ld();
+                uint32_t w[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int l0 = logit_of<FOLD>(v[4 * i], p), l1 = logit_of<FOLD>(v[4 * i + 1], p);
+                    const int l2 = logit_of<FOLD>(v[4 * i + 2], p), l3 = logit_of<FOLD>(v[4 * i + 3], p);
+                    w[i] = pack_sat_s8(l1, l0, pack_sat_s8(l3, l2, 0u));
+                    const int k0 = col0 + 4 * i;  // keys at or past L: zero bytes
+                    if (k0 + 4 > L) w[i] &= k0 >= L ? 0u : (0xFFFFFFFFu >> (32 - 8 * (L - k0)));
+                }
+                unsigned char *dst = OS + (size_t)qr * p.ld + col0;
+                *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+                if (col0 + 16 < L16) *reinterpret_cast<uint4 *>(dst + 16) = make_uint4(w[4], w[5], w[6], w[7]);
+            }
+            tc_fence_before();
+            __syncthreads();  // buffer b is read: chunk c + 2 may overwrite it
+            tc_fence_after();
+            if (*stop) break;
+            if (tid == 0 && c + 2 < nch) issue(c + 2);
+        }
+        if (*stop) break;
+        // ---- the tile's rows to global memory: one bulk copy (rows r0 .. of head bh are contiguous)
+        fence_async_smem();
+        __syncthreads();
+        if (tid == 0) {
+            const uint32_t bytes = (uint32_t)(min(QM, L - r0) * p.ld);
+            asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(
+                             p.out + ((size_t)bh * L + r0) * p.ld),
+                         "r"(sa(OS)), "r"(bytes)
+                         : "memory");
+            asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+            stores = true;
+        }
+    }
+    // every store and every MMA issued has completed before shared and tensor memory are released
+    if (tid == 0) {
+        if (stores) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        if (issued > 0) {
+            mma_commit(&sh.fin);
+            mbar_wait(&sh.fin, 0, abort_flag, false);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * QNC));
+}
+
+size_t qk_smem_bytes(int64_t ld) { return 1024 + (size_t)QMAXL * QROW + (size_t)QM * QROW + (size_t)QM * ld; }
+
+constexpr size_t kQkStaticSmem = sizeof(QkShared) + 64;
+
+template <bool FOLD>
+cudaError_t qk_launch(const QkParams &p, size_t smem, int grid, cudaStream_t st)
+{
+    cudaError_t e = cudaFuncSetAttribute(qk_logits_tc_kernel<FOLD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    qk_logits_tc_kernel<FOLD><<<grid, QTHREADS, smem, st>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool qk_logits_supported(const QkArgs &a)
+{
+    return a.L >= 1 && a.L <= QMAXL && a.d >= 1 && a.d <= QKD && a.d % 8 == 0 && a.ld_q % 8 == 0 &&
+           a.ld_k % 8 == 0 && a.ld_logit % 16 == 0 && ((uintptr_t)a.q % 8) == 0 && ((uintptr_t)a.k % 8) == 0 &&
+           ((uintptr_t)a.logits % 16) == 0 && qk_smem_bytes(a.ld_logit) + kQkStaticSmem <= 232448;
+}
+
+cudaError_t launch_qk_logits(const QkArgs &a, cudaStream_t st)
+{
+    QkParams p{};
+    p.q = a.q;
+    p.k = a.k;
+    p.ld_q = a.ld_q;
+    p.ld_k = a.ld_k;
+    p.zp_q = a.zp_q;
+    p.zp_k = a.zp_k;
+    p.out = a.logits;
+    p.ld = a.ld_logit;
+    p.BH = a.BH;
+    p.L = a.L;
+    p.d = a.d;
+    p.n1 = a.n1;
+    p.n2 = a.n2;
+    p.zp_l = a.zp_l;
+    // 32-bit epilogue: N1 >= 1 and |N2 P| + 2^(N1-1) + |zp_l| 2^N1 < 2^31 for every P the codes allow
+    const double pmax = (double)a.d * (128.0 + std::fabs((double)a.zp_q)) * (128.0 + std::fabs((double)a.zp_k));
+    const bool fold = a.n1 >= 1 && a.n1 <= 31 &&
+                      (double)a.n2 * pmax + std::ldexp(1.0, a.n1 - 1) + std::fabs((double)a.zp_l) * std::ldexp(1.0, a.n1) <
+                          2147483648.0;
+    if (fold)
+        p.c1 = (uint32_t)((1ull << (a.n1 - 1)) + ((uint64_t)(int64_t)a.zp_l << a.n1) -
+                          (uint64_t)a.n2 * 0x4B400000ull);
+    const size_t smem = qk_smem_bytes(a.ld_logit);
+    const int64_t ntiles = a.BH * ((a.L + QM - 1) / QM);
+    const int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());
+    return fold ? qk_launch<true>(p, smem, grid, st) : qk_launch<false>(p, smem, grid, st);
+}
+
+cudaError_t read_clear_qk_status(int *status)
+{
+    int zero = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(status, g_status, sizeof(int));
+    if (e != cudaSuccess) return e;
+    return cudaMemcpyToSymbol(g_status, &zero, sizeof(int));
+}
+
+}  // namespace fqvit

@@ -235,6 +235,15 @@ __device__ __forceinline__ void mma_f16_ta(uint32_t dt, uint32_t at, uint64_t bd
         : "memory");
 }
 
+// D (tensor memory) (+)= A B with both operands in shared memory (descriptors)
+__device__ __forceinline__ void mma_f16_ss(uint32_t dt, uint64_t ad, uint64_t bd, uint32_t idesc, bool accumulate)
+{
+    asm volatile(
+        "{ .reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p; }" ::"r"(dt),
+        "l"(ad), "l"(bd), "r"(idesc), "r"((uint32_t)accumulate)
+        : "memory");
+}
+
 // shared-memory matrix descriptor without swizzle
 __device__ __forceinline__ uint64_t smem_desc_plain(uint32_t addr, uint32_t lbo, uint32_t sbo)
 {

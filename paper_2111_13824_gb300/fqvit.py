@@ -50,6 +50,7 @@ EXPORTS = (
     "fqvit_calibrate_ptf_noalloc",
     "fqvit_calibrate_minmax", "fqvit_calibrate_sse_partial", "fqvit_calibrate_combine",
     "fqvit_lis_softmax_masked", "fqvit_lis_attention_masked", "fqvit_lis_attention_masked_q",
+    "fqvit_qk_logits", "fqvit_qk_workspace_size", "fqvit_qk_lis_attention",
 )
 
 
@@ -85,6 +86,10 @@ def load(path: str | Path | None = None):
                                        ctypes.c_int),
         "fqvit_lis_attention_masked_q": ([P, i64, f32, i32, P, P, P, i64, i32, i64, i32, i32, f32, f32, i32, P,
                                           i64, P], ctypes.c_int),
+        "fqvit_qk_logits": ([P, i64, i32, P, i64, i32, i64, i32, i32, f32, f32, f32, i32, P, i64, P], ctypes.c_int),
+        "fqvit_qk_workspace_size": ([i64, i32, i64], sz),
+        "fqvit_qk_lis_attention": ([P, i64, i32, P, i64, i32, f32, f32, f32, i32, i32, P, P, P, i64, i32, i64, i32,
+                                    i32, P, i64, P, sz, i64, P], ctypes.c_int),
         "fqvit_block_int": ([P, P], ctypes.c_int),
         "fqvit_sync_status": ([P], ctypes.c_int),
         "fqvit_calibrate_ptf_noalloc": ([P, i64, i32, i64, i32, i32, P, P, P, P, P], ctypes.c_int),
@@ -362,6 +367,45 @@ def lis_attention_masked_q(logits: torch.Tensor, s_logit: float, v: torch.Tensor
                                                int(zp_v), BH, L, d, float(s_v), float(s_out), int(zp_out), _p(out),
                                                out.stride(1), _stream(stream)))
     return out
+
+
+def qk_logits(q: torch.Tensor, k: torch.Tensor, zp_q: int, zp_k: int, s_q: float, s_k: float, s_logit: float,
+              zp_logit: int, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Q K^T and its 8-bit output quantizer (fqvit_qk_logits): int8 [BH, L, d] x 2 -> int8 [BH*L, ld]."""
+    BH, L, d = q.shape
+    if out is None:
+        out = torch.empty(BH * L, (L + 15) // 16 * 16, dtype=torch.int8, device=q.device)
+    _check(load().fqvit_qk_logits(_p(q), q.stride(1), int(zp_q), _p(k), k.stride(1), int(zp_k), BH, L, d,
+                                  float(s_q), float(s_k), float(s_logit), int(zp_logit), _p(out), _ld(out),
+                                  _stream(stream)))
+    return out
+
+
+def qk_workspace_size(BH: int, L: int, group_heads: int = 0) -> int:
+    return int(load().fqvit_qk_workspace_size(BH, L, group_heads))
+
+
+def qk_lis_attention(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, zp_q: int, zp_k: int, s_q: float, s_k: float,
+                     s_logit: float, zp_logit: int, zp_v: int = 0, acc: torch.Tensor | None = None,
+                     workspace: torch.Tensor | None = None, group_heads: int = 0, bias: torch.Tensor | None = None,
+                     heads: int = 1, window: int = 0, region: torch.Tensor | None = None, mask_value: int = 0,
+                     n_shift: int = 15, stream=None) -> torch.Tensor:
+    """Attention from int8 Q, K, V (fqvit_qk_lis_attention): int32 [BH, L, d]."""
+    BH, L, d = v.shape
+    if acc is None:
+        acc = torch.empty(BH, L, d, dtype=torch.int32, device=v.device)
+    if workspace is None:
+        workspace = torch.empty(qk_workspace_size(BH, L, group_heads), dtype=torch.int8, device=v.device)
+    b = _bias(bias, heads, window)
+    m = _mask(region, mask_value)
+    _check(load().fqvit_qk_lis_attention(_p(q), q.stride(1), int(zp_q), _p(k), k.stride(1), int(zp_k), float(s_q),
+                                         float(s_k), float(s_logit), int(zp_logit), n_shift,
+                                         ctypes.byref(b) if b is not None else None,
+                                         ctypes.byref(m) if m is not None else None, _p(v), v.stride(1), int(zp_v),
+                                         BH, L, d, _p(acc), acc.stride(1), _p(workspace),
+                                         workspace.numel() * workspace.element_size(), int(group_heads),
+                                         _stream(stream)))
+    return acc
 
 
 def block_int(xq, zp_in, alpha, gamma, beta, s_out, zp_out, yq, logits, ld_logit, s_logit, v, zp_v, acc,

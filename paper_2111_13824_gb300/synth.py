@@ -24,6 +24,9 @@ S * 1000 + l, draws in this fixed order):
   int8 range by its min / max (``s_logit``).  sigma = 1 is the literal
   config, sigma = 2 the "peaked" variant whose rows put most mass on a few
   keys (Sec. 3.3: 98.8 % of ViT-L attention values are below 1/16).
+  The int8 codes of Q and K, their scales and the logits' zero point
+  (round(-min / s_logit) - 128, signed) are returned too: the inputs of the
+  Q K^T path.
 * V: int8 uniform in [-128, 127], zero point 0.
 * Swin relative-position bias: int8 ``[H, (2w-1)^2]`` uniform in [-16, 16].
 * Swin patch merging (after stages 1-3): the stage's channel model drawn
@@ -228,8 +231,14 @@ def attn_inputs(cfg: Config, layer: int, device="cpu", sigma: float = 1.0, bh: i
     ld = ld_pad(L)
     logits = torch.zeros(BH * L, ld, dtype=torch.int8, device=device)
     logits[:, :L] = qq.reshape(BH * L, L).to(torch.int8)
+    # the int8 Q and K codes (symmetric MinMax) and the logits' MinMax zero point, signed
+    # (the 8-bit zero point round(-lo / s_logit) minus 128): the inputs of the Q K^T path
+    zp_logit = int(min(255, max(0, round(-lo / s_logit)))) - 128
     return dict(logits=logits, ld_logit=ld, s_logit=s_logit, v=v.contiguous(), bias=bias,
-                heads=st.H, window=st.window, BH=BH, L=L, d=d)
+                heads=st.H, window=st.window, BH=BH, L=L, d=d,
+                q=qi.to(torch.int8).contiguous(), k=ki.to(torch.int8).contiguous(),
+                s_q=float(torch.tensor(sq, dtype=torch.float32)), s_k=float(torch.tensor(sk, dtype=torch.float32)),
+                zp_logit=zp_logit)
 
 
 def layer_window_mask(cfg: Config, layer: int, device="cpu"):

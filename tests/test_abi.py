@@ -116,3 +116,31 @@ def test_window_mask_checks(lib):
     assert attq(ctypes.byref(fqvit.WindowMask(fake, 4, -100))) == 1
     assert attq(ctypes.byref(fqvit.WindowMask(fake, 2, -100)), zp=300) == 1
     assert "zp_out" in _err(lib)
+
+
+def test_qk_checks(lib):
+    """fqvit_qk_logits / fqvit_qk_lis_attention reject bad arguments before any launch."""
+    fake = ctypes.c_void_p(4096)
+    f = lambda *a: lib.fqvit_qk_logits(*a)  # noqa: E731
+    ok = [fake, 64, 0, fake, 64, 0, 2, 197, 64, 0.03, 0.03, 0.04, 0, fake, 208, None]
+    assert f(*[None] + ok[1:]) == 1                                     # NULL q
+    bad = list(ok); bad[7] = 641; bad[14] = 656
+    assert f(*bad) == 2 and "L=641" in _err(lib)                        # L > 640
+    bad = list(ok); bad[8] = 12; bad[1] = 12; bad[4] = 12
+    assert f(*bad) == 2                                                 # d not a multiple of 8
+    bad = list(ok); bad[14] = 200
+    assert f(*bad) == 1                                                 # ld_logit not a multiple of 16
+    bad = list(ok); bad[2] = 128
+    assert f(*bad) == 1 and "zero points" in _err(lib)                  # zp_q outside -128..127
+    bad = list(ok); bad[11] = 0.0
+    assert f(*bad) == 1                                                 # s_logit not positive
+    bad = list(ok); bad[9] = 1e30; bad[10] = 1e30; bad[11] = 1e-30
+    assert f(*bad) == 2                                                 # M leaves the fp32 range
+    assert lib.fqvit_qk_workspace_size(4, 49, 3) == 3 * 49 * 64
+    assert lib.fqvit_qk_workspace_size(0, 49, 3) == 0
+    assert lib.fqvit_qk_workspace_size(10 ** 6, 577, 0) <= 48 << 20
+    g = lambda ws_bytes, v=fake: lib.fqvit_qk_lis_attention(  # noqa: E731
+        fake, 64, 0, fake, 64, 0, 0.03, 0.03, 0.04, 0, 15, None, None, v, 64, 0, 4, 197, 64, fake, 64, fake,
+        ws_bytes, 0, None)
+    assert g(197 * 208 - 1) == 1 and "workspace" in _err(lib)          # less than one head
+    assert g(10 ** 8, v=None) == 1                                      # NULL V
