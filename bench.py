@@ -66,10 +66,17 @@ def ln_bytes(rows, C):
 OUT8_SV = 1.0 / 127.0  # V's scale for the 8-bit output option (any value: the work is the same)
 
 
-def attn_bytes(BH, L, d, out_bytes=4):
+def metric_name(args):
+    if args.config == "vit_l384" and not args.qk:
+        return METRIC
+    return f"tokens/s, PTF-LN + {'Q K^T + ' if args.qk else ''}LIS attention, {args.config}"
+
+
+def attn_bytes(BH, L, d, out_bytes=4, qk=False):
     """Algorithmic bytes of one fused attention launch: 1 B / logit + 1 B / V element + 4 B / acc element
-    (1 B / output element with the 8-bit requantized output)."""
-    return BH * (L * L + L * d + out_bytes * L * d)
+    (1 B / output element with the 8-bit requantized output).  From Q and K (--qk): 1 B per Q and per K
+    element instead of the logits, which stay on chip and in L2."""
+    return BH * ((2 * L * d if qk else L * L) + L * d + out_bytes * L * d)
 
 
 def recorded_traffic(config, kernel):
@@ -93,10 +100,11 @@ def recorded_traffic(config, kernel):
 
 # ------------------------------------------------------------------ workload
 
-def make_layers(cfg, device, sigma=1.0, limit=0):
+def make_layers(cfg, device, sigma=1.0, limit=0, qk=False):
     from paper_2111_13824_gb300 import fqvit
 
     layers = []
+    ws = None  # --qk: one logits workspace, reused group after group and layer after layer
     for l in range(cfg.layers if limit <= 0 else min(limit, cfg.layers)):
         st = synth.layer_stage(cfg, l)
         d = synth.ln_inputs(cfg, l, device=device)
@@ -104,9 +112,14 @@ def make_layers(cfg, device, sigma=1.0, limit=0):
         zp_i, s_f = int(zp.item()), float(s.item())
         xq = fqvit.ptf_quantize(d["x"], s_f, zp_i, alpha)
         a = synth.attn_inputs(cfg, l, device=device, sigma=sigma)
+        if qk and ws is None:
+            ws = torch.empty(fqvit.qk_workspace_size(a["BH"], a["L"]), dtype=torch.int8, device=device)
         layers.append(dict(
+            qk=qk, q=a["q"] if qk else None, k=a["k"] if qk else None, s_q=a["s_q"], s_k=a["s_k"],
+            zp_logit=a["zp_logit"], workspace=ws,
             xq=xq, zp=zp_i, alpha=alpha, gamma=d["gamma"], beta=d["beta"], s_out=d["s_out"], zp_out=d["zp_out"],
-            yq=torch.empty_like(xq), logits=a["logits"], s_logit=a["s_logit"], v=a["v"], bias=a["bias"],
+            yq=torch.empty_like(xq), logits=None if qk else a["logits"], s_logit=a["s_logit"], v=a["v"],
+            bias=a["bias"],
             heads=a["heads"], window=a["window"],
             region=synth.layer_window_mask(cfg, l, device=device), mask_value=synth.swin_mask_value(a["s_logit"]),
             acc=torch.empty(a["BH"], a["L"], a["d"], dtype=torch.int32, device=device),
@@ -134,14 +147,26 @@ def make_merge(cfg, stage, device):
                 yq=torch.empty_like(xq), rows=d["rows"], C=d["C"])
 
 
+def qk_group(ly):
+    """Heads per group of the chained --qk attention (the library's choice for the layer's shape)."""
+    from paper_2111_13824_gb300 import fqvit
+
+    return max(1, fqvit.qk_workspace_size(ly["BH"], ly["L"]) // (ly["L"] * synth.ld_pad(ly["L"])))
+
+
 def layernorm(fq, m):
     fq.ptf_layernorm(m["xq"], m["zp"], m["alpha"], m["gamma"], m["beta"], m["s_out"], m["zp_out"], out=m["yq"])
 
 
 def attention(fq, ly, out8=False):
-    """The layer's fused attention; Swin's shifted blocks take their window mask."""
+    """The layer's fused attention; Swin's shifted blocks take their window mask.  --qk: from the
+    int8 Q, K and V (Q K^T on the tensor cores, then the fused attention, head group by group)."""
     kw = dict(bias=ly["bias"], heads=ly["heads"], window=ly["window"])
-    if ly["region"] is not None:
+    if ly["qk"]:
+        fq.qk_lis_attention(ly["q"], ly["k"], ly["v"], 0, 0, ly["s_q"], ly["s_k"], ly["s_logit"], ly["zp_logit"],
+                            acc=ly["acc"], workspace=ly["workspace"], region=ly["region"],
+                            mask_value=ly["mask_value"], **kw)
+    elif ly["region"] is not None:
         if out8:  # the output requantized to 8 bits (output scale = V's: M = 2^-15)
             fq.lis_attention_masked_q(ly["logits"], ly["s_logit"], ly["v"], ly["region"], ly["mask_value"], 0,
                                       OUT8_SV, OUT8_SV, 128, out=ly["out8"], **kw)
@@ -217,10 +242,11 @@ class OracleSample:
     the LayerNorm elements of the whole step (every layer, and Swin's patch
     mergings) and the second by the step's attention logits."""
 
-    def __init__(self, cfg, heads=1, ln_rows=512, layer=0):
+    def __init__(self, cfg, heads=1, ln_rows=512, layer=0, qk=False):
         import oracle
 
         self.oracle = oracle
+        self.qk = qk
         self.cfg, self.heads, self.ln_rows = cfg, heads, ln_rows
         self.st = synth.layer_stage(cfg, layer)
         d = synth.ln_inputs(cfg, layer, rows=ln_rows)
@@ -238,7 +264,11 @@ class OracleSample:
         t0 = time.perf_counter()
         o.ptf_layernorm(*self.ln)
         t1 = time.perf_counter()
-        co, _ = o.lis_softmax(self.x, a["L"], a["s_logit"], bias=self.bias, heads=a["heads"],
+        x = self.x
+        if self.qk:  # the logits from Q and K first
+            x = o.qk_logits(a["q"].numpy(), a["k"].numpy(), 0, 0, a["s_q"], a["s_k"], a["s_logit"], a["zp_logit"],
+                            ld=synth.ld_pad(a["L"]))
+        co, _ = o.lis_softmax(x, a["L"], a["s_logit"], bias=self.bias, heads=a["heads"],
                               window=a["window"] or 7)
         o.lis_attn_v(co, self.v, 0)
         t2 = time.perf_counter()
@@ -248,7 +278,8 @@ class OracleSample:
         return step, t2 - t0
 
     def describe(self):
-        return (f"layer 0: LayerNorm of {self.ln_rows} of {self.st.rows} rows and LIS + BitShift attn.V of "
+        return (f"layer 0: LayerNorm of {self.ln_rows} of {self.st.rows} rows and "
+                f"{'Q K^T logits + ' if self.qk else ''}LIS + BitShift attn.V of "
                 f"{self.heads} of {self.st.BH} heads, scaled to the step's LayerNorm elements and attention "
                 f"logits ({self.cfg.layers} layers" + (", patch mergings)" if synth.merge_stages(self.cfg) else ")"))
 
@@ -280,7 +311,9 @@ def bench_gpu(args):
         torch.distributed.barrier()
     fqvit.load()
     cfg = synth.CONFIGS[args.config]
-    layers = make_layers(cfg, dev, sigma=args.sigma, limit=args.layers)
+    if args.qk and args.out8:
+        raise SystemExit("--qk and --out8 together are not a bench mode")
+    layers = make_layers(cfg, dev, sigma=args.sigma, limit=args.layers, qk=args.qk)
     tokens_per_step = cfg.first_tokens
 
     for _ in range(args.warmup):
@@ -369,7 +402,7 @@ def bench_gpu(args):
     ln_ms = [a.elapsed_time(b) for a, b in ln_events]
     peak, peak_kind = peaks()
     # per-launch algorithmic bytes (averaged over the stack's layer shapes)
-    ab = [attn_bytes(ly["BH"], ly["L"], ly["d"], 1 if args.out8 else 4) for ly in layers]
+    ab = [attn_bytes(ly["BH"], ly["L"], ly["d"], 1 if args.out8 else 4, qk=args.qk) for ly in layers]
     lb = [ln_bytes(ly["rows"], ly["C"]) for ly in layers]
     attn_gbs = sum(ab) * args.steps / (sum(attn_ms) / 1e3) / 1e9
     ln_gbs = sum(lb) * args.steps / (sum(ln_ms) / 1e3) / 1e9
@@ -379,9 +412,29 @@ def bench_gpu(args):
     stack_gbs = step_bytes / (ms_per_step / 1e3) / 1e9
     dominant = "attention" if sum(attn_ms) >= sum(ln_ms) else "layernorm"
     dom_gbs = attn_gbs if dominant == "attention" else ln_gbs
-    traffic = None if args.out8 else recorded_traffic(args.config, dominant)  # the record is of the int32 output
+    # the records are of the int32 output from logits, or (key "<config>:qk") of the --qk step
+    traffic = None if args.out8 else recorded_traffic(args.config + (":qk" if args.qk else ""), dominant)
     if args.traffic:
         traffic = json.loads(args.traffic).get(dominant)
+
+    if args.qk:  # the Q K^T kernel alone on layer 0, all heads in one launch, outside the step
+        ly = layers[0]
+        full = torch.empty(ly["BH"] * ly["L"], synth.ld_pad(ly["L"]), dtype=torch.int8, device=dev)
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(10)]
+        for i in range(13):
+            if i >= 3:
+                evs[i - 3][0].record()
+            fqvit.qk_logits(ly["q"], ly["k"], 0, 0, ly["s_q"], ly["s_k"], ly["s_logit"], ly["zp_logit"], out=full)
+            if i >= 3:
+                evs[i - 3][1].record()
+        torch.cuda.synchronize()
+        qk_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
+        qk_b = ly["BH"] * (2 * ly["L"] * ly["d"] + ly["L"] * full.shape[1])
+        qk_stats = {"gbs": round(qk_b / (qk_ms / 1e3) / 1e9, 1), "ms_per_launch": round(qk_ms, 5),
+                    "bytes_per_launch": qk_b, "frac": round(qk_b / (qk_ms / 1e3) / 1e9 / peak, 4),
+                    "how": "fqvit_qk_logits on layer 0, all heads in one launch (Q, K read, logits written "
+                           "to HBM), 10 launches after 3, outside the timed step"}
+        del full
 
     e2e = None
     if not args.no_e2e:
@@ -392,7 +445,7 @@ def bench_gpu(args):
         cpu = cpu_baseline(cfg, args)
 
     line = {
-        "metric": METRIC if args.config == "vit_l384" else f"tokens/s, PTF-LN + LIS attention, {args.config}",
+        "metric": metric_name(args),
         "value": round(value, 1),
         "unit": "tokens/s",
         "n_gpus": ws,
@@ -405,7 +458,8 @@ def bench_gpu(args):
         "dtype": "int8",
         "data": "synthetic (seeded generator of the paper's layer shapes and statistics)",
         "config": {
-            "workload": f"{cfg.name}: {cfg.note}, {cfg.layers} layers of PTF LayerNorm + fused LIS attention",
+            "workload": f"{cfg.name}: {cfg.note}, {cfg.layers} layers of PTF LayerNorm + "
+                        f"{'Q K^T + ' if args.qk else ''}fused LIS attention",
             "tokens_per_step_per_gpu": tokens_per_step,
             "layers": len(layers),
             "step_bytes": step_bytes,
@@ -414,6 +468,8 @@ def bench_gpu(args):
             "parallelism": f"replicas x{ws} (independent batches, no collective)",
             "launch": "cuda_graph" if graph is not None else "eager",
             "attention_output": "uint8 (requantized)" if args.out8 else "int32 accumulators",
+            "attention_input": (f"int8 Q, K, V: fqvit_qk_lis_attention, head groups of {qk_group(layers[0])}"
+                                if args.qk else "int8 logits, int8 V"),
             "shifted_window_layers": sum(ly["region"] is not None for ly in layers),
             "patch_merges": len(merges),
         },
@@ -424,6 +480,7 @@ def bench_gpu(args):
                           "bytes_per_launch": round(sum(ab) / len(ab))},
             "layernorm": {"gbs": round(ln_gbs, 1), "ms_per_launch": round(sum(ln_ms) / len(ln_ms), 5),
                           "bytes_per_launch": round(sum(lb) / len(lb))},
+            **({"qk_logits": qk_stats} if args.qk else {}),
             **({"patch_merge_layernorm": {
                 "gbs": round(sum(mb) * args.steps / (sum(merge_ms) / 1e3) / 1e9, 1),
                 "ms_per_launch": round(sum(merge_ms) / len(merge_ms), 5),
@@ -434,7 +491,8 @@ def bench_gpu(args):
                      "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
                      else "fallback"},
         "clocks": clk,
-        "gpu_launches": (2 * len(layers) + len(merges)) * args.steps,
+        "gpu_launches": (sum(1 + (2 * -(-ly["BH"] // qk_group(ly)) if args.qk else 1) for ly in layers)
+                         + len(merges)) * args.steps,
     }
     if e2e is not None:
         line["e2e"] = e2e
@@ -451,14 +509,16 @@ def bench_e2e(fqvit, layers, tokens_per_step, args, dev, ws):
     layer's inputs from pinned host memory to the device and its outputs back."""
     host = []
     for ly in layers:
-        h = {k: ly[k].cpu().pin_memory() for k in ("xq", "logits", "v")}
+        ins = ("xq", "q", "k", "v") if ly["qk"] else ("xq", "logits", "v")
+        h = {k: ly[k].cpu().pin_memory() for k in ins}
         h["yq"] = torch.empty_like(ly["yq"], device="cpu").pin_memory()
         h["acc"] = torch.empty_like(ly["acc"], device="cpu").pin_memory()
         if ly["merge"] is not None:  # the patch merging's LayerNorm input and output
             h["mxq"] = ly["merge"]["xq"].cpu().pin_memory()
             h["myq"] = torch.empty_like(ly["merge"]["yq"], device="cpu").pin_memory()
         host.append(h)
-    h2d = sum(h[k].numel() * h[k].element_size() for h in host for k in ("xq", "logits", "v", "mxq") if k in h)
+    h2d = sum(h[k].numel() * h[k].element_size() for h in host for k in ("xq", "logits", "q", "k", "v", "mxq")
+              if k in h)
     d2h = sum(h[k].numel() * h[k].element_size() for h in host for k in ("yq", "acc", "myq") if k in h)
     steps = max(1, min(args.steps, args.e2e_steps))
 
@@ -482,8 +542,9 @@ def bench_e2e(fqvit, layers, tokens_per_step, args, dev, ws):
                 if started[i]:
                     s_in.wait_event(ev_cmp[i])
                 ly["xq"].copy_(h["xq"], non_blocking=True)
-                ly["logits"].copy_(h["logits"], non_blocking=True)
-                ly["v"].copy_(h["v"], non_blocking=True)
+                for key in ("logits", "q", "k", "v"):
+                    if key in h:
+                        ly[key].copy_(h[key], non_blocking=True)
                 if "mxq" in h:
                     ly["merge"]["xq"].copy_(h["mxq"], non_blocking=True)
                 ev_in[i].record(s_in)
@@ -522,7 +583,8 @@ def bench_e2e(fqvit, layers, tokens_per_step, args, dev, ws):
         ms = float(t.item())
     return {"value": round(tokens_per_step * ws * steps / (ms / 1e3), 1), "unit": "tokens/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps,
-            "how": "per layer: pinned H2D of xq, logits, V (and a patch merging's xq); LayerNorm(s) + fused "
+            "how": "per layer: pinned H2D of xq, logits (--qk: Q and K), V (and a patch merging's xq); "
+                   "LayerNorm(s) + fused "
                    "attention; D2H of yq and acc (and the merging's yq); "
                    "three streams (upload, compute, download), layers pipelined"}
 
@@ -532,11 +594,11 @@ def cpu_baseline(cfg, args):
     (grown toward --cpu-seconds of work), repeated until the budget is spent."""
     import oracle
 
-    probe = OracleSample(cfg, heads=1, ln_rows=256)
+    probe = OracleSample(cfg, heads=1, ln_rows=256, qk=args.qk)
     _, spent = probe.run()
     scale = max(1, int(args.cpu_seconds / max(spent, 1e-3)))
     st = cfg.stages[0]
-    smp = OracleSample(cfg, heads=min(st.BH, scale), ln_rows=min(st.rows, 256 * scale))
+    smp = OracleSample(cfg, heads=min(st.BH, scale), ln_rows=min(st.rows, 256 * scale), qk=args.qk)
     ests, total = [], 0.0
     while total < args.cpu_seconds or not ests:
         est, spent = smp.run()
@@ -557,7 +619,7 @@ def bench_reference(args):
     import oracle
 
     oracle.build()
-    smp = OracleSample(cfg, heads=4, ln_rows=2048)
+    smp = OracleSample(cfg, heads=4, ln_rows=2048, qk=args.qk)
     for _ in range(args.warmup):
         smp.run()
     ests = []
@@ -570,11 +632,12 @@ def bench_reference(args):
     sample = f"per step: {smp.describe()}"
     line = {
         "impl": "reference",
-        "metric": METRIC if args.config == "vit_l384" else f"tokens/s, PTF-LN + LIS attention, {args.config}",
+        "metric": metric_name(args),
         "value": round(value, 3), "unit": "tokens/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(step * 1e3, 3), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "int8", "data": "synthetic (seeded generator of the paper's layer shapes and statistics)",
-        "config": {"workload": f"{cfg.name}: {cfg.note}, {cfg.layers} layers of PTF LayerNorm + LIS attention",
+        "config": {"workload": f"{cfg.name}: {cfg.note}, {cfg.layers} layers of PTF LayerNorm + "
+                               f"{'Q K^T + ' if args.qk else ''}LIS attention",
                    "tokens_per_step_per_gpu": cfg.first_tokens, "layers": cfg.layers},
         "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": oracle.num_threads(),
                          "kind": "oracle", "sample": sample},
@@ -599,6 +662,8 @@ def main():
     ap.add_argument("--traffic", default=None, help="JSON {kernel: dram bytes per launch} from an ncu capture")
     ap.add_argument("--layers", type=int, default=0, help="time only the first N layers (profiling cases)")
     ap.add_argument("--no-graph", action="store_true", help="launch the timed steps eagerly instead of as one CUDA graph")
+    ap.add_argument("--qk", action="store_true",
+                    help="attention from int8 Q, K, V (fqvit_qk_lis_attention) instead of int8 logits")
     ap.add_argument("--out8", action="store_true",
                     help="the attention output requantized to 8 bits (fqvit_lis_attention_q) instead of int32")
     args = ap.parse_args()

@@ -17,18 +17,24 @@
 // range, so consecutive tiles share a head.  Per head, K -> fp16 in shared
 // memory (B operand: keys x 64, K-major, 128-byte swizzle, d padded to 64 with
 // zeros); per tile, the 128 query rows of Q likewise (A operand).  The keys go
-// through the tensor cores in chunks of 128 (M = 128, N <= 128, K = 64) into two
-// tensor-memory buffers, one chunk ahead of the epilogue; the 16 warps read a
+// through the tensor cores in chunks of 128 (M = 128, N <= 128, K = 64) into four
+// tensor-memory buffers, up to four chunks ahead of the epilogue; the 16 warps read a
 // chunk back (warp w: lanes 32 (w % 4) .., columns 32 (w / 4) ..), quantize it
-// and write the bytes into a shared-memory tile of the output, which one bulk
-// copy sends to global memory (a tile's rows are contiguous there).  Every
-// wait is bounded: after two seconds the kernel records a timeout status,
-// drains what it issued and returns.
+// and write the bytes into a shared-memory tile of the output; all threads then
+// copy the tile out with coalesced 16-byte stores (its rows are contiguous in
+// global memory).  A bulk copy of the tile drained at a fraction of the SM's
+// share of the write bandwidth and held up the next tile; per-thread stores of
+// each row's pieces scattered the writes.  Every wait is bounded: after two
+// seconds the kernel records a timeout status, drains what it issued and
+// returns.
 #include "fqvit_internal.cuh"
 #include "tc_common.cuh"
 
 #include <cmath>
+#include <cstring>
+#include <cuda.h>
 #include <cuda_fp16.h>
+#include <cudaTypedefs.h>
 
 namespace fqvit {
 
@@ -38,10 +44,13 @@ using namespace tc;
 
 constexpr int QM = 128;          // query rows per tile (MMA M)
 constexpr int QNC = 128;         // keys per chunk (MMA N of a full chunk)
+constexpr int QNBUF = 4;         // tensor-memory buffers of a chunk (all 512 columns)
 constexpr int QKD = 64;          // the MMA's reduction: d padded to 64
 constexpr int QTHREADS = 512;
 constexpr int QMAXL = 640;       // keys of the longest row
 constexpr int QROW = QKD * 2;    // bytes of an fp16 operand row
+constexpr int QNST = 3;          // BULK: staging buffers of a chunk's output (128 x 128 bytes each)
+constexpr int QST_BYTES = QM * QNC;
 
 struct QkParams {
     const int8_t *q, *k;
@@ -58,7 +67,7 @@ struct QkParams {
 };
 
 struct QkShared {
-    uint64_t sfull[2], fin;
+    uint64_t sfull[QNBUF], fin, qload, kload;
     uint32_t tmem;
     int abort_flag;
     int stop;
@@ -106,36 +115,46 @@ __device__ __forceinline__ int logit_of(uint32_t acc_bits, const QkParams &p)
     }
 }
 
-template <bool FOLD>
-__global__ void __launch_bounds__(QTHREADS, 1) qk_logits_tc_kernel(QkParams p)
+// BULK: Q and K rows reach shared memory as int8 by bulk copies one tile (one head) ahead of
+// their conversion (strides of at most 64 bytes, multiples of 16), and each chunk's 128 x 128
+// output bytes leave through one of QNST staging buffers (128-byte swizzle) by a tensor store
+// of the logits viewed as [BH][L][ld] (rows past L and bytes past ld clipped), so the drain of
+// one chunk overlaps the work on the next.  Else each thread loads its codes from global
+// memory as it converts them, and the tile's output is copied out from a shared-memory tile.
+template <bool FOLD, bool BULK>
+__global__ void __launch_bounds__(QTHREADS, 1)
+    qk_logits_tc_kernel(const __grid_constant__ QkParams p, const __grid_constant__ CUtensorMap tmap)
 {
     extern __shared__ unsigned char dsm_raw[];
     __shared__ QkShared sh;
     unsigned char *base = dsm_raw + ((1024u - (sa(dsm_raw) & 1023u)) & 1023u);
     unsigned char *KS = base;                            // QMAXL x 128 B (keys, fp16, swizzled)
     unsigned char *QS = KS + QMAXL * QROW;               // QM x 128 B
-    unsigned char *OS = QS + QM * QROW;                  // QM x ld bytes: the output tile
+    unsigned char *OS = QS + QM * QROW;                  // BULK: QNST x 16 KB staging; else QM x ld bytes
+    unsigned char *KST = OS + (BULK ? (size_t)QNST * QST_BYTES : (size_t)QM * p.ld);  // BULK: L x ld_k int8
+    unsigned char *QST = KST + (size_t)QMAXL * 64;       // BULK: QM x ld_q int8 of the next tile
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile int *abort_flag = &sh.abort_flag;
     volatile int *stop = &sh.stop;
     if (tid == 0) {
-        mbar_init(&sh.sfull[0], 1);
-        mbar_init(&sh.sfull[1], 1);
+        for (int b = 0; b < QNBUF; ++b) mbar_init(&sh.sfull[b], 1);
         mbar_init(&sh.fin, 1);
+        mbar_init(&sh.qload, 1);
+        mbar_init(&sh.kload, 1);
         sh.abort_flag = 0;
         sh.stop = 0;
     }
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(&sh.tmem)),
-                     "r"(2 * QNC));
+                     "r"(QNBUF * QNC));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     const int L = p.L, d = p.d;
     const int L16 = (L + 15) & ~15;                     // keys that go through the MMAs
     const int nch = (L + QNC - 1) / QNC;
     // bytes of each output row past the MMA'd keys (up to ld) stay zero for the whole launch
-    for (int x = tid; x < QM * (int)(p.ld - L16); x += QTHREADS) {
+    for (int x = tid; !BULK && x < QM * (int)(p.ld - L16); x += QTHREADS) {
         const int r = x / (int)(p.ld - L16), j = x - r * (int)(p.ld - L16);
         OS[(size_t)r * p.ld + L16 + j] = 0;
     }
@@ -152,70 +171,114 @@ __global__ void __launch_bounds__(QTHREADS, 1) qk_logits_tc_kernel(QkParams p)
     auto idesc = [](int n) -> uint32_t { return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(QM >> 4) << 24); };
     const __half2 zq2 = __half2half2(__int2half_rn(p.zp_q)), zk2 = __half2half2(__int2half_rn(p.zp_k));
 
-    uint32_t use[2] = {0, 0};  // completed phases of each tensor-memory buffer
+    // BULK: the copies of a tile's Q rows and of a head's K rows
+    auto copy_q = [&](int64_t tt) {
+        const int bq = (int)(tt / tpb), rq = (int)(tt - (int64_t)bq * tpb) * QM;
+        const uint32_t bytes = (uint32_t)(min(QM, L - rq) * p.ld_q);
+        mbar_expect_tx(&sh.qload, bytes);
+        bulk_g2s(QST, p.q + ((size_t)bq * L + rq) * p.ld_q, bytes, &sh.qload);
+    };
+    auto copy_k = [&](int bk) {
+        const uint32_t bytes = (uint32_t)(L * p.ld_k);
+        mbar_expect_tx(&sh.kload, bytes);
+        bulk_g2s(KST, p.k + (size_t)bk * L * p.ld_k, bytes, &sh.kload);
+    };
+    // BULK: phases waited for and copies issued (thread 0) on the two copy barriers; a copy is
+    // issued only after the previous one on its barrier was waited for, so at most one is in flight
+    uint32_t qph = 0, kph = 0, qiss = 0, kiss = 0;
+    if (BULK && tid == 0 && t_begin < t_end) {
+        copy_q(t_begin);
+        copy_k((int)(t_begin / tpb));
+        qiss = kiss = 1;
+    }
+
+    // chunks are numbered across the CTA's tiles: chunk gc uses buffer gc % QNBUF, whose barrier
+    // then completes its phase gc / QNBUF
+    uint32_t g0 = 0;  // number of the tile's first chunk
     uint32_t issued = 0;       // MMA commits issued (thread 0)
     int cur_bh = -1;
-    bool stores = false;       // a bulk store is in flight (thread 0)
     for (int64_t t = t_begin; t < t_end; ++t) {
         const int bh = (int)(t / tpb);
         const int r0 = (int)(t - (int64_t)bh * tpb) * QM;
         // ---- operands: K of a new head, the tile's Q rows (8 values = 16 bytes of fp16 per item)
+        bool cbad = false;
         if (bh != cur_bh) {
-            for (int x = tid; x < L16 * 8; x += QTHREADS) {
+            if (BULK) {
+                cbad = !mbar_wait_warp(&sh.kload, kph & 1, abort_flag);
+                ++kph;
+            }
+            for (int x = tid; x < L16 * 8 && !cbad; x += QTHREADS) {
                 const int key = x >> 3, c = x & 7;
                 uint4 h = make_uint4(0, 0, 0, 0);
-                if (key < L && 8 * c < d)
-                    h = codes_to_h8(
-                        __ldg(reinterpret_cast<const uint2 *>(p.k + ((size_t)bh * L + key) * p.ld_k + 8 * c)), zk2);
+                if (key < L && 8 * c < d) {
+                    const uint2 w = BULK ? *reinterpret_cast<const uint2 *>(KST + key * p.ld_k + 8 * c)
+                                         : __ldg(reinterpret_cast<const uint2 *>(p.k + ((size_t)bh * L + key) * p.ld_k + 8 * c));
+                    h = codes_to_h8(w, zk2);
+                }
                 *reinterpret_cast<uint4 *>(KS + key * QROW + ((c ^ (key & 7)) << 4)) = h;
             }
             cur_bh = bh;
         }
-        for (int x = tid; x < QM * 8; x += QTHREADS) {
+        if (BULK && !cbad) {
+            cbad = !mbar_wait_warp(&sh.qload, qph & 1, abort_flag);
+            ++qph;
+        }
+        for (int x = tid; x < QM * 8 && !cbad; x += QTHREADS) {
             const int r = x >> 3, c = x & 7;
             uint4 h = make_uint4(0, 0, 0, 0);
-            if (r0 + r < L && 8 * c < d)
-                h = codes_to_h8(
-                    __ldg(reinterpret_cast<const uint2 *>(p.q + ((size_t)bh * L + r0 + r) * p.ld_q + 8 * c)), zq2);
+            if (r0 + r < L && 8 * c < d) {
+                const uint2 w = BULK ? *reinterpret_cast<const uint2 *>(QST + r * p.ld_q + 8 * c)
+                                     : __ldg(reinterpret_cast<const uint2 *>(p.q + ((size_t)bh * L + r0 + r) * p.ld_q + 8 * c));
+                h = codes_to_h8(w, zq2);
+            }
             *reinterpret_cast<uint4 *>(QS + r * QROW + ((c ^ (r & 7)) << 4)) = h;
         }
+        if (cbad) *stop = 1;
         fence_async_smem();  // the operands are read by the MMAs
-        if (tid == 0 && stores) {  // the previous tile's bulk store has read the output tile
-            asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-            stores = false;
-        }
         tc_fence_before();
         __syncthreads();
         tc_fence_after();
         if (*stop) break;
-        // ---- the first two chunks
+        // ---- the staging buffers are converted: the next tile's Q (and the next head's K) may land
+        if (BULK && tid == 0 && t + 1 < t_end) {
+            copy_q(t + 1);
+            ++qiss;
+            if ((int)((t + 1) / tpb) != bh) {
+                copy_k((int)((t + 1) / tpb));
+                ++kiss;
+            }
+        }
+        // ---- the first chunks (up to one per buffer)
         auto issue = [&](int c) {
             const int n = min(QNC, L16 - c * QNC);
             const uint32_t a0 = sa(QS), b0 = sa(KS) + (uint32_t)(c * QNC * QROW);
 #pragma unroll
             for (int s = 0; s < QKD / 16; ++s)
-                mma_f16_ss(tmem + (uint32_t)((c & 1) * QNC), smem_desc(a0 + 32 * s, 16, 1024),
+                mma_f16_ss(tmem + (uint32_t)(((g0 + c) % QNBUF) * QNC), smem_desc(a0 + 32 * s, 16, 1024),
                            smem_desc(b0 + 32 * s, 16, 1024), idesc(n), s != 0);
-            mma_commit(&sh.sfull[c & 1]);
+            mma_commit(&sh.sfull[(g0 + c) % QNBUF]);
             ++issued;
         };
-        if (tid == 0) {
-            issue(0);
-            if (nch > 1) issue(1);
-        }
+        if (tid == 0)
+            for (int c = 0; c < nch && c < QNBUF; ++c) issue(c);
         // ---- chunks: read back, quantize, into the output tile
         const int qr = 32 * (warp & 3) + lane;  // tile row of this thread
         const int g = warp >> 2;                // 32-column group of a chunk
         bool bad = false;
         for (int c = 0; c < nch; ++c) {
-            const int b = c & 1;
-            if (!mbar_wait_warp(&sh.sfull[b], use[b] & 1, abort_flag)) {
+            const uint32_t b = (g0 + c) % QNBUF;
+            if (!mbar_wait_warp(&sh.sfull[b], ((g0 + c) / QNBUF) & 1, abort_flag)) {
                 bad = true;
                 *stop = 1;
             }
-            ++use[b];
             tc_fence_after();
             const int col0 = c * QNC + 32 * g;  // first key of this warp's 32 columns
+            // BULK: this chunk's staging buffer, 16-byte unit u of tile row qr at u ^ (qr % 8)
+            unsigned char *srow = OS + (size_t)((g0 + c) % QNST) * QST_BYTES + qr * QNC;
+            if (BULK && !bad && col0 >= L16 && col0 < p.ld) {  // bytes past the keys, inside the row
+                *reinterpret_cast<uint4 *>(srow + (((2 * g) ^ (qr & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+                *reinterpret_cast<uint4 *>(srow + (((2 * g + 1) ^ (qr & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+            }
             if (!bad && col0 < L16) {
                 uint32_t v[32];
                 tmem_ld32(tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(b * QNC + 32 * g), v);
@@ -226,36 +289,62 @@ __global__ void __launch_bounds__(QTHREADS, 1) qk_logits_tc_kernel(QkParams p)
                     const int l0 = logit_of<FOLD>(v[4 * i], p), l1 = logit_of<FOLD>(v[4 * i + 1], p);
                     const int l2 = logit_of<FOLD>(v[4 * i + 2], p), l3 = logit_of<FOLD>(v[4 * i + 3], p);
                     w[i] = pack_sat_s8(l1, l0, pack_sat_s8(l3, l2, 0u));
-                    const int k0 = col0 + 4 * i;  // keys at or past L: zero bytes
-                    if (k0 + 4 > L) w[i] &= k0 >= L ? 0u : (0xFFFFFFFFu >> (32 - 8 * (L - k0)));
                 }
-                unsigned char *dst = OS + (size_t)qr * p.ld + col0;
-                *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
-                if (col0 + 16 < L16) *reinterpret_cast<uint4 *>(dst + 16) = make_uint4(w[4], w[5], w[6], w[7]);
+                if (col0 + 32 > L) {  // keys at or past L: zero bytes (the last chunk only)
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const int k0 = col0 + 4 * i;
+                        if (k0 + 4 > L) w[i] &= k0 >= L ? 0u : (0xFFFFFFFFu >> (32 - 8 * (L - k0)));
+                    }
+                }
+                if (BULK) {  // units past L16 hold zeros (w is masked past L) or lie past ld (clipped)
+                    *reinterpret_cast<uint4 *>(srow + (((2 * g) ^ (qr & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+                    *reinterpret_cast<uint4 *>(srow + (((2 * g + 1) ^ (qr & 7)) << 4)) =
+                        col0 + 16 < L16 ? make_uint4(w[4], w[5], w[6], w[7]) : make_uint4(0, 0, 0, 0);
+                } else {
+                    unsigned char *dst = OS + (size_t)qr * p.ld + col0;
+                    *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+                    if (col0 + 16 < L16) *reinterpret_cast<uint4 *>(dst + 16) = make_uint4(w[4], w[5], w[6], w[7]);
+                }
+            }
+            if (BULK) {
+                fence_async_smem();  // the staging bytes are read by the tensor store
+                // the store of chunk gc - 2 has read its buffer, which chunk gc + 1 writes next
+                if (tid == 0) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
             }
             tc_fence_before();
-            __syncthreads();  // buffer b is read: chunk c + 2 may overwrite it
+            __syncthreads();  // buffer b is read: chunk c + QNBUF may overwrite it
             tc_fence_after();
             if (*stop) break;
-            if (tid == 0 && c + 2 < nch) issue(c + 2);
+            if (BULK && tid == 0) {  // chunk c of the tile: columns c 128 .., rows r0 .., head bh
+                asm volatile(
+                    "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(&tmap),
+                    "r"(c * QNC), "r"(r0), "r"(bh), "r"(sa(OS + (size_t)((g0 + c) % QNST) * QST_BYTES))
+                    : "memory");
+                asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+            }
+            if (tid == 0 && c + QNBUF < nch) issue(c + QNBUF);
         }
         if (*stop) break;
-        // ---- the tile's rows to global memory: one bulk copy (rows r0 .. of head bh are contiguous)
-        fence_async_smem();
-        __syncthreads();
-        if (tid == 0) {
-            const uint32_t bytes = (uint32_t)(min(QM, L - r0) * p.ld);
-            asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(
-                             p.out + ((size_t)bh * L + r0) * p.ld),
-                         "r"(sa(OS)), "r"(bytes)
-                         : "memory");
-            asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-            stores = true;
+        g0 += (uint32_t)nch;
+        // ---- (without BULK) the tile's rows to global memory (contiguous there): 16 bytes per
+        //      thread and step, each warp's stores one contiguous 512-byte run; the next tile's
+        //      epilogue writes the tile again only after its first barrier
+        if (!BULK) {
+            __syncthreads();
+            const int64_t bytes = (int64_t)min(QM, L - r0) * p.ld;
+            int8_t *gdst = p.out + ((size_t)bh * L + r0) * p.ld;
+            for (int64_t x = 16 * (int64_t)tid; x < bytes; x += 16 * QTHREADS)
+                *reinterpret_cast<uint4 *>(gdst + x) = *reinterpret_cast<const uint4 *>(OS + x);
         }
     }
     // every store and every MMA issued has completed before shared and tensor memory are released
     if (tid == 0) {
-        if (stores) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        if (BULK) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");  // the tensor stores
+        if (BULK) {  // a copy issued ahead and never waited for (the loop stopped early)
+            if (qph < qiss) mbar_wait(&sh.qload, qph & 1, abort_flag, false);
+            if (kph < kiss) mbar_wait(&sh.kload, kph & 1, abort_flag, false);
+        }
         if (issued > 0) {
             mma_commit(&sh.fin);
             mbar_wait(&sh.fin, 0, abort_flag, false);
@@ -265,21 +354,59 @@ __global__ void __launch_bounds__(QTHREADS, 1) qk_logits_tc_kernel(QkParams p)
     __syncthreads();
     tc_fence_after();
     if (warp == 0)
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * QNC));
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(QNBUF * QNC));
 }
 
-size_t qk_smem_bytes(int64_t ld) { return 1024 + (size_t)QMAXL * QROW + (size_t)QM * QROW + (size_t)QM * ld; }
+size_t qk_smem_bytes(int64_t ld, bool bulk)
+{
+    return 1024 + (size_t)QMAXL * QROW + (size_t)QM * QROW +
+           (bulk ? (size_t)QNST * QST_BYTES + (size_t)QMAXL * 64 + QM * 64 : (size_t)QM * ld);
+}
 
 constexpr size_t kQkStaticSmem = sizeof(QkShared) + 64;
 
-template <bool FOLD>
-cudaError_t qk_launch(const QkParams &p, size_t smem, int grid, cudaStream_t st)
+template <bool FOLD, bool BULK>
+cudaError_t qk_launch(const QkParams &p, const CUtensorMap &tm, size_t smem, int grid, cudaStream_t st)
 {
-    cudaError_t e = cudaFuncSetAttribute(qk_logits_tc_kernel<FOLD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+    cudaError_t e = cudaFuncSetAttribute(qk_logits_tc_kernel<FOLD, BULK>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    qk_logits_tc_kernel<FOLD><<<grid, QTHREADS, smem, st>>>(p);
+    qk_logits_tc_kernel<FOLD, BULK><<<grid, QTHREADS, smem, st>>>(p, tm);
     return cudaGetLastError();
+}
+
+// The logits as a 3-d tensor [BH][L][ld] of bytes for the tensor stores: boxes of 128 x 128 x 1,
+// 128-byte swizzle.  False when the driver's encoder is unavailable or rejects the shape.
+bool logits_tensor_map(CUtensorMap *tm, int8_t *out, int64_t BH, int L, int64_t ld)
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    if (!encode) return false;
+    const cuuint64_t dims[3] = {(cuuint64_t)ld, (cuuint64_t)L, (cuuint64_t)BH};
+    const cuuint64_t strides[2] = {(cuuint64_t)ld, (cuuint64_t)ld * (cuuint64_t)L};
+    const cuuint32_t box[3] = {(cuuint32_t)QNC, (cuuint32_t)QM, 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return encode(tm, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, out, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Bulk copies of the operands (16-byte aligned rows of at most 64 bytes) and tensor stores of the
+// output (rows and row strides of at least one 128 x 128 box)
+bool qk_bulk(const QkArgs &a)
+{
+    return a.ld_q % 16 == 0 && a.ld_k % 16 == 0 && a.ld_q <= 64 && a.ld_k <= 64 && ((uintptr_t)a.q % 16) == 0 &&
+           ((uintptr_t)a.k % 16) == 0 && a.L >= QM && a.ld_logit >= QNC &&
+           qk_smem_bytes(a.ld_logit, true) + kQkStaticSmem <= 232448;
 }
 
 }  // namespace
@@ -288,7 +415,7 @@ bool qk_logits_supported(const QkArgs &a)
 {
     return a.L >= 1 && a.L <= QMAXL && a.d >= 1 && a.d <= QKD && a.d % 8 == 0 && a.ld_q % 8 == 0 &&
            a.ld_k % 8 == 0 && a.ld_logit % 16 == 0 && ((uintptr_t)a.q % 8) == 0 && ((uintptr_t)a.k % 8) == 0 &&
-           ((uintptr_t)a.logits % 16) == 0 && qk_smem_bytes(a.ld_logit) + kQkStaticSmem <= 232448;
+           ((uintptr_t)a.logits % 16) == 0 && qk_smem_bytes(a.ld_logit, false) + kQkStaticSmem <= 232448;
 }
 
 cudaError_t launch_qk_logits(const QkArgs &a, cudaStream_t st)
@@ -316,10 +443,15 @@ cudaError_t launch_qk_logits(const QkArgs &a, cudaStream_t st)
     if (fold)
         p.c1 = (uint32_t)((1ull << (a.n1 - 1)) + ((uint64_t)(int64_t)a.zp_l << a.n1) -
                           (uint64_t)a.n2 * 0x4B400000ull);
-    const size_t smem = qk_smem_bytes(a.ld_logit);
+    CUtensorMap tm;
+    memset(&tm, 0, sizeof(tm));
+    const bool bulk = qk_bulk(a) && logits_tensor_map(&tm, a.logits, a.BH, a.L, a.ld_logit);
+    const size_t smem = qk_smem_bytes(a.ld_logit, bulk);
     const int64_t ntiles = a.BH * ((a.L + QM - 1) / QM);
     const int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());
-    return fold ? qk_launch<true>(p, smem, grid, st) : qk_launch<false>(p, smem, grid, st);
+    if (bulk)
+        return fold ? qk_launch<true, true>(p, tm, smem, grid, st) : qk_launch<false, true>(p, tm, smem, grid, st);
+    return fold ? qk_launch<true, false>(p, tm, smem, grid, st) : qk_launch<false, false>(p, tm, smem, grid, st);
 }
 
 cudaError_t read_clear_qk_status(int *status)
