@@ -96,12 +96,13 @@ __device__ __forceinline__ uint4 codes_to_h8(uint2 w, __half2 z)
 // The logit of one accumulator (an exact integer P in fp32, |P| < 2^22).
 //   FOLD: (N2 P + 2^(N1-1) + zp_l 2^N1) >> N1 in 32 bits (the host checked that it fits)
 //   else: the 64-bit formula, N1 of any sign
+// (n2, c1, n1: the launch's constants, held in registers by the caller)
 template <bool FOLD>
-__device__ __forceinline__ int logit_of(uint32_t acc_bits, const QkParams &p)
+__device__ __forceinline__ int logit_of(uint32_t acc_bits, const QkParams &p, uint32_t n2, uint32_t c1, int n1)
 {
     if (FOLD) {
         const uint32_t x = __float_as_uint(__fadd_rn(__uint_as_float(acc_bits), 12582912.0f));
-        return (int)(x * (uint32_t)p.n2 + p.c1) >> p.n1;
+        return (int)(x * n2 + c1) >> n1;
     } else {
         const int P = __float2int_rn(__uint_as_float(acc_bits));
         const long long num = (long long)p.n2 * P;
@@ -170,6 +171,10 @@ __global__ void __launch_bounds__(QTHREADS, 1)
     // instruction descriptor: D f32, A/B f16 K-major, M = 128, N = n
     auto idesc = [](int n) -> uint32_t { return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(QM >> 4) << 24); };
     const __half2 zq2 = __half2half2(__int2half_rn(p.zp_q)), zk2 = __half2half2(__int2half_rn(p.zp_k));
+    // the requantization's constants in registers (an integer multiply-add takes one constant-bank operand)
+    uint32_t rn2 = (uint32_t)p.n2, rc1 = p.c1;
+    int rn1 = p.n1;
+    asm volatile("" : "+r"(rn2), "+r"(rc1), "+r"(rn1));
 
     // BULK: the copies of a tile's Q rows and of a head's K rows
     auto copy_q = [&](int64_t tt) {
@@ -286,8 +291,10 @@ __global__ void __launch_bounds__(QTHREADS, 1)
                 uint32_t w[8];
 #pragma unroll
                 for (int i = 0; i < 8; ++i) {
-                    const int l0 = logit_of<FOLD>(v[4 * i], p), l1 = logit_of<FOLD>(v[4 * i + 1], p);
-                    const int l2 = logit_of<FOLD>(v[4 * i + 2], p), l3 = logit_of<FOLD>(v[4 * i + 3], p);
+                    const int l0 = logit_of<FOLD>(v[4 * i], p, rn2, rc1, rn1);
+                    const int l1 = logit_of<FOLD>(v[4 * i + 1], p, rn2, rc1, rn1);
+                    const int l2 = logit_of<FOLD>(v[4 * i + 2], p, rn2, rc1, rn1);
+                    const int l3 = logit_of<FOLD>(v[4 * i + 3], p, rn2, rc1, rn1);
                     w[i] = pack_sat_s8(l1, l0, pack_sat_s8(l3, l2, 0u));
                 }
                 if (col0 + 32 > L) {  // keys at or past L: zero bytes (the last chunk only)
