@@ -587,6 +587,7 @@ bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
 
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
 {
+    if (lis_attention_tc_packed(a.L)) return launch_lis_attention_tc_packed(a, b, st);  // lis_tc_pack.cu
     TcParams p{a.logits, a.ld_logit, a.s_logit, b.v, b.acc, b.BH, a.L, b.zp_v, iexp_consts_host(a.s_logit),
                b.out8, b.ld_out8, b.rq_n1, b.rq_n2, b.rq_zp};
     const size_t smem = tc_smem_bytes(a.L, a.ld_logit);
@@ -622,7 +623,11 @@ cudaError_t read_clear_device_status(int *status, cudaStream_t st)
     if (*status == 0) *status = wst;
     int qst = 0;
     e = read_clear_qk_status(&qst);
+    if (e != cudaSuccess) return e;
     if (*status == 0) *status = qst;
+    int pst = 0;
+    e = read_clear_tcp_status(&pst);
+    if (*status == 0) *status = pst;
     return e;
 }
 

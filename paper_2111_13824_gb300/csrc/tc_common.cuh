@@ -68,15 +68,13 @@ __device__ __forceinline__ bool mbar_try_for(uint64_t *b, uint32_t parity, uint3
 }
 
 // Bounded wait: the thread sleeps in the barrier (woken when the phase completes) in slices of
-// at most 50 us, and between slices for 32 ns doubling to 256 ns (a waiter that waits out a
-// whole tile then takes few issue slots from the warps that work); false on timeout or
-// (honor_abort) when another role gave up.
+// at most 50 us; false on timeout or (honor_abort) when another role gave up.  (Sleeps growing
+// to 256 ns between slices were tried: no gain for long rows, 5-8 % slower for short ones.)
 static __device__ __noinline__ bool mbar_wait(uint64_t *b, uint32_t parity, volatile int *abort_flag,
                                        bool honor_abort = true)
 {
     if (mbar_try(b, parity)) return true;
     const uint64_t t0 = gtimer();
-    uint32_t ns = 32;
     for (;;) {
         if (mbar_try_for(b, parity, 50000)) return true;
         if (honor_abort && *abort_flag) return false;
@@ -85,8 +83,7 @@ static __device__ __noinline__ bool mbar_wait(uint64_t *b, uint32_t parity, vola
             atomicExch(&g_status, 5);
             return false;
         }
-        __nanosleep(ns);
-        if (ns < 256) ns <<= 1;
+        __nanosleep(64);
     }
 }
 
