@@ -12,7 +12,10 @@ input are offline (setup), as in post-training quantization.
 Algorithmic bytes per layer: LayerNorm 2 bytes per element (int8 in and out)
 plus 9 bytes of per-channel parameters; attention 1 byte per logit, 1 per V
 element and 4 per int32 accumulator (the 4-bit codes stay on chip).  The K
-timed steps run as one CUDA graph (--no-graph: eager launches).
+timed steps run as one CUDA graph holding only the kernels, which are
+launched with programmatic dependent launch (a kernel's set-up overlaps the
+previous kernel's tail); the per-kernel times come from a second graph of up to
+three steps with timing events around each kernel (--no-graph: eager launches).
 
 Prints ONE JSON line (rank 0).
 
@@ -332,49 +335,59 @@ def bench_gpu(args):
             ev_kw["external"] = True
         except TypeError:
             use_graph = False
-    attn_events = [(torch.cuda.Event(**ev_kw), torch.cuda.Event(**ev_kw)) for _ in range(args.steps * len(layers))]
-    ln_events = [(torch.cuda.Event(**ev_kw), torch.cuda.Event(**ev_kw)) for _ in range(args.steps * len(layers))]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-
     merges = [ly["merge"] for ly in layers if ly["merge"] is not None]
-    merge_events = [(torch.cuda.Event(**ev_kw), torch.cuda.Event(**ev_kw)) for _ in range(args.steps * len(merges))]
+    ev_steps = min(args.steps, 3)  # steps of the per-kernel timing pass
+    ev = {}
 
-    def enqueue_steps():
+    def new_events(kw):
+        ev["attn"] = [(torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(ev_steps * len(layers))]
+        ev["ln"] = [(torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(ev_steps * len(layers))]
+        ev["merge"] = [(torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(ev_steps * len(merges))]
+
+    new_events(ev_kw)
+
+    def enqueue_steps(steps, events):
+        """The step's launches; with events, each kernel between a pair of timing events (which
+        serialise the kernels: the timed step runs without them)."""
         k = km = 0
-        for _ in range(args.steps):
+
+        def mark(name, idx, j):
+            if events:
+                ev[name][idx][j].record()
+
+        for _ in range(steps):
             for ly in layers:
                 if ly["merge"] is not None:
-                    merge_events[km][0].record()
+                    mark("merge", km, 0)
                     layernorm(fqvit, ly["merge"])
-                    merge_events[km][1].record()
+                    mark("merge", km, 1)
                     km += 1
-                ln_events[k][0].record()
+                mark("ln", k, 0)
                 fqvit.ptf_layernorm(ly["xq"], ly["zp"], ly["alpha"], ly["gamma"], ly["beta"], ly["s_out"],
                                     ly["zp_out"], out=ly["yq"])
-                ln_events[k][1].record()
-                attn_events[k][0].record()
+                mark("ln", k, 1)
+                mark("attn", k, 0)
                 attention(fqvit, ly, args.out8)
-                attn_events[k][1].record()
+                mark("attn", k, 1)
                 k += 1
 
-    graph = None
+    graph = ev_graph = None
     if use_graph:
         try:
             graph = torch.cuda.CUDAGraph()
             with torch.cuda.graph(graph):
-                enqueue_steps()
+                enqueue_steps(args.steps, False)
+            ev_graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(ev_graph):
+                enqueue_steps(ev_steps, True)
             graph.replay()  # upload and one untimed pass
             torch.cuda.synchronize()
         except Exception as exc:  # noqa: BLE001 - any capture failure falls back to eager launches
             print(f"bench: CUDA graph unavailable ({type(exc).__name__}: {exc}); eager launches", file=sys.stderr)
-            graph = None
+            graph = ev_graph = None
             torch.cuda.synchronize()
-            attn_events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                           for _ in range(args.steps * len(layers))]
-            ln_events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                         for _ in range(args.steps * len(layers))]
-            merge_events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                            for _ in range(args.steps * len(merges))]
+            new_events(dict(enable_timing=True))
     clocks = ClockSampler(local)
     if ws > 1:
         torch.distributed.barrier()
@@ -385,7 +398,7 @@ def bench_gpu(args):
     if graph is not None:
         graph.replay()
     else:
-        enqueue_steps()
+        enqueue_steps(args.steps, False)
     end.record()
     torch.cuda.synchronize()
     clk = clocks.stop()
@@ -398,14 +411,22 @@ def bench_gpu(args):
     ms_per_step = elapsed_ms / args.steps
     value = tokens_per_step * ws * args.steps / (elapsed_ms / 1e3)
 
+    # per-kernel durations: a separate pass of the same launches with timing events around each
+    if ev_graph is not None:
+        ev_graph.replay()
+    else:
+        enqueue_steps(ev_steps, True)
+    torch.cuda.synchronize()
+    attn_events, ln_events, merge_events = ev["attn"], ev["ln"], ev["merge"]
+
     attn_ms = [a.elapsed_time(b) for a, b in attn_events]
     ln_ms = [a.elapsed_time(b) for a, b in ln_events]
     peak, peak_kind = peaks()
     # per-launch algorithmic bytes (averaged over the stack's layer shapes)
     ab = [attn_bytes(ly["BH"], ly["L"], ly["d"], 1 if args.out8 else 4, qk=args.qk) for ly in layers]
     lb = [ln_bytes(ly["rows"], ly["C"]) for ly in layers]
-    attn_gbs = sum(ab) * args.steps / (sum(attn_ms) / 1e3) / 1e9
-    ln_gbs = sum(lb) * args.steps / (sum(ln_ms) / 1e3) / 1e9
+    attn_gbs = sum(ab) * ev_steps / (sum(attn_ms) / 1e3) / 1e9
+    ln_gbs = sum(lb) * ev_steps / (sum(ln_ms) / 1e3) / 1e9
     mb = [ln_bytes(m["rows"], m["C"]) for m in merges]
     merge_ms = [a.elapsed_time(b) for a, b in merge_events]
     step_bytes = sum(ab) + sum(lb) + sum(mb)
@@ -482,7 +503,7 @@ def bench_gpu(args):
                           "bytes_per_launch": round(sum(lb) / len(lb))},
             **({"qk_logits": qk_stats} if args.qk else {}),
             **({"patch_merge_layernorm": {
-                "gbs": round(sum(mb) * args.steps / (sum(merge_ms) / 1e3) / 1e9, 1),
+                "gbs": round(sum(mb) * ev_steps / (sum(merge_ms) / 1e3) / 1e9, 1),
                 "ms_per_launch": round(sum(merge_ms) / len(merge_ms), 5),
                 "bytes_per_launch": round(sum(mb) / len(mb))}} if merges else {}),
         },

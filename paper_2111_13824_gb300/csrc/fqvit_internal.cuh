@@ -10,6 +10,33 @@ namespace fqvit {
 // Number of SMs of the current device (cached per device).
 int sm_count();
 
+// Programmatic dependent launch.  The step's kernels are launched with programmatic stream
+// serialization: the next kernel's CTAs may start (and run their set-up: barriers, tensor
+// memory, tables computed from arguments) while the previous kernel's last CTAs finish.  Every
+// such kernel calls pdl_release() at entry and pdl_wait() before its first access to global
+// memory (read or write): the wait returns once the previous grid has completed and its writes
+// are visible, so the data dependencies of the stream stay as in a plain launch.  Without the
+// launch attribute both are no-ops.
+__device__ __forceinline__ void pdl_release() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... Params, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args &&...args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
+
 // Sets the thread's fqvit_last_error message (empty for FQVIT_OK); returns code.
 int record_error(int code, const char *msg);
 

@@ -149,6 +149,8 @@ __global__ void __launch_bounds__(kWarps * 32)
     float *bs_s = gs_s + a.C;
     uint8_t *al_s = reinterpret_cast<uint8_t *>(bs_s + a.C);
     __shared__ LnShared sh;
+    pdl_release();
+    pdl_wait();  // everything below reads or writes global memory
     ln_prologue(a, gs_s, bs_s, al_s, sh, true);
 
     constexpr int RPW = 32 / S;  // rows per warp
@@ -356,8 +358,8 @@ cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st)
 #define FQ_LN_LAUNCH(SS, N)                                                                      \
     {                                                                                           \
         cudaFuncSetAttribute(ln_vec_kernel<SS, N>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
-        ln_vec_kernel<SS, N><<<blocks_for((const void *)ln_vec_kernel<SS, N>), kWarps * 32, smem, st>>>(a); \
-        return cudaGetLastError();                                                              \
+        return launch_pdl(ln_vec_kernel<SS, N>, dim3(blocks_for((const void *)ln_vec_kernel<SS, N>)), \
+                          dim3(kWarps * 32), smem, st, a);                                      \
     }
         if (S < 32) {
             switch (S) {

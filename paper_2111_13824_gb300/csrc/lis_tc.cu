@@ -161,6 +161,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile int *abort_flag = &sh.abort_flag;
     volatile int *stop_flag = &sh.stop;
+    pdl_release();
     if (tid == 0) {
         mbar_init(&sh.lload, 1);
         mbar_init(&sh.lfree, TSOFT);
@@ -192,6 +193,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = sh.tmem;
+    pdl_wait();  // the set-up above touched no global memory
 
     const int L = p.L;
     const int tpb = (L + TM - 1) / TM;
@@ -561,8 +563,7 @@ cudaError_t tc_launch(const TcParams &p, size_t smem, int grid, cudaStream_t st)
     cudaError_t e = cudaFuncSetAttribute(lis_attn_tc_kernel<NKB, SMALL_E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
-    lis_attn_tc_kernel<NKB, SMALL_E><<<grid, TTHREADS, smem, st>>>(p);
-    return cudaGetLastError();
+    return launch_pdl(lis_attn_tc_kernel<NKB, SMALL_E>, dim3(grid), dim3(TTHREADS), smem, st, p);
 }
 
 template <int NKB>

@@ -235,6 +235,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tcp_kernel(TcParams p)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile int *abort_flag = &sh.abort_flag;
     volatile int *stop_flag = &sh.stop;
+    pdl_release();
     if (tid == 0) {
         mbar_init(&sh.lload, 1);
         mbar_init(&sh.lfree, TSOFT);
@@ -268,6 +269,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tcp_kernel(TcParams p)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = sh.tmem;
+    pdl_wait();  // the set-up above touched no global memory
 
     const int L = p.L;
     const int tpb = (L + TM - 1) / TM;
@@ -661,8 +663,7 @@ cudaError_t tc_launch(const TcParams &p, size_t smem, int grid, cudaStream_t st)
     cudaError_t e = cudaFuncSetAttribute(lis_attn_tcp_kernel<NKB, SMALL_E, PACK>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    lis_attn_tcp_kernel<NKB, SMALL_E, PACK><<<grid, TTHREADS, smem, st>>>(p);
-    return cudaGetLastError();
+    return launch_pdl(lis_attn_tcp_kernel<NKB, SMALL_E, PACK>, dim3(grid), dim3(TTHREADS), smem, st, p);
 }
 
 // whether a launch packs tiles across heads (L >= 128: a tile then holds rows of at most two heads)

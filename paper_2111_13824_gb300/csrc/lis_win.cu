@@ -132,6 +132,7 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
     const int h = r >> 6, i = r & 63;
     const int L = p.L;
     volatile int *abort_flag = &sh.abort_flag;
+    pdl_release();
 
     if (tid == 0) {
         for (int k = 0; k < p.ng; ++k) {
@@ -153,6 +154,7 @@ __global__ void __launch_bounds__(WMAXG * 128, 1) lis_attn_win_kernel(WinParams 
     for (int k = tid; k < 64; k += blockDim.x)  // D_1 = 3, D_k = 3 2^(k-1) - 1 (exact up to k = 24)
         dk[k] = k <= 1 ? 3.0f : __fsub_rn(__int_as_float(((k + 127) << 23) | 0x400000), 1.0f);
     const int nb = 2 * p.window - 1;
+    pdl_wait();  // the first access to global memory follows
     if (BIAS) {
         for (int x = tid; x < p.heads * nb * nb; x += blockDim.x) Bs_all[x] = (unsigned char)p.bias[x];
         // entry of (query i, key j) = qbase[i] - koff[j]: (y_i - y_j + w - 1) nb + (x_i - x_j + w - 1)
@@ -523,8 +525,7 @@ cudaError_t win_launch_q(const WinParams &p, size_t smem, int grid, cudaStream_t
     cudaError_t e = cudaFuncSetAttribute(lis_attn_win_kernel<D, BIAS, SMALL_E, NQ, MASK>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    lis_attn_win_kernel<D, BIAS, SMALL_E, NQ, MASK><<<grid, 128 * p.ng, smem, st>>>(p);
-    return cudaGetLastError();
+    return launch_pdl(lis_attn_win_kernel<D, BIAS, SMALL_E, NQ, MASK>, dim3(grid), dim3(128 * p.ng), smem, st, p);
 }
 
 template <int D, bool BIAS, bool SMALL_E, bool MASK>

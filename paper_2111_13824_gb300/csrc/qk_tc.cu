@@ -138,6 +138,7 @@ __global__ void __launch_bounds__(QTHREADS, 1)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile int *abort_flag = &sh.abort_flag;
     volatile int *stop = &sh.stop;
+    pdl_release();
     if (tid == 0) {
         for (int b = 0; b < QNBUF; ++b) mbar_init(&sh.sfull[b], 1);
         mbar_init(&sh.fin, 1);
@@ -191,6 +192,7 @@ __global__ void __launch_bounds__(QTHREADS, 1)
     // BULK: phases waited for and copies issued (thread 0) on the two copy barriers; a copy is
     // issued only after the previous one on its barrier was waited for, so at most one is in flight
     uint32_t qph = 0, kph = 0, qiss = 0, kiss = 0;
+    pdl_wait();  // the set-up above touched no global memory
     if (BULK && tid == 0 && t_begin < t_end) {
         copy_q(t_begin);
         copy_k((int)(t_begin / tpb));
@@ -378,8 +380,7 @@ cudaError_t qk_launch(const QkParams &p, const CUtensorMap &tm, size_t smem, int
     cudaError_t e = cudaFuncSetAttribute(qk_logits_tc_kernel<FOLD, BULK>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    qk_logits_tc_kernel<FOLD, BULK><<<grid, QTHREADS, smem, st>>>(p, tm);
-    return cudaGetLastError();
+    return launch_pdl(qk_logits_tc_kernel<FOLD, BULK>, dim3(grid), dim3(QTHREADS), smem, st, p, tm);
 }
 
 // The logits as a 3-d tensor [BH][L][ld] of bytes for the tensor stores: boxes of 128 x 128 x 1,
