@@ -69,6 +69,8 @@ def _load():
     lib.or_qk_logits.restype = ctypes.c_int
     lib.or_qk_logits.argtypes = [P, i64, i32, P, i64, i32, i64, i32, i32, f32, f32, f32, i32, P, i64]
     lib.or_lis_attn_v.restype = ctypes.c_int
+    lib.or_linear_q.restype = ctypes.c_int
+    lib.or_linear_q.argtypes = [P, i64, i32, i64, i32, f32, P, i32, i64, P, P, f32, i32, P, i64, P, i64]
     lib.or_num_threads.argtypes = []
     lib.or_num_threads.restype = ctypes.c_int
     lib.or_set_num_threads.argtypes = [ctypes.c_int]
@@ -283,3 +285,26 @@ def attn_requant(acc: np.ndarray, s_v: float, s_out: float, zp_out: int) -> np.n
     if rc != 0:
         raise ValueError("or_attn_requant rejected its arguments")
     return y
+
+
+def linear_q(x: np.ndarray, zp_x: int, s_x: float, w: np.ndarray, s_w: np.ndarray, bias: np.ndarray | None,
+             s_y: float, zp_y: int):
+    """A MinMax Linear layer (Sec. 3; Sec. 4.1: symmetric channel-wise weights, asymmetric
+    layer-wise activations) with its dyadic output multipliers: x uint8 [M, K], w int8 [N, K],
+    s_w float32 [N], bias int32 [N] or None -> (y uint8 [M, N], acc int32 [M, N])."""
+    x = _c(x, np.uint8)
+    w = _c(w, np.int8)
+    s_w = _c(s_w, np.float32)
+    b = None if bias is None else _c(bias, np.int32)
+    M, K = x.shape
+    N = w.shape[0]
+    assert w.shape[1] == K and s_w.shape == (N,)
+    y = np.zeros((M, N), np.uint8)
+    acc = np.zeros((M, N), np.int32)
+    rc = _load().or_linear_q(_ptr(x), M, K, K, int(zp_x), np.float32(s_x), _ptr(w), N, K, _ptr(s_w), _ptr(b),
+                             np.float32(s_y), int(zp_y), _ptr(y), N, _ptr(acc), N)
+    if rc == 1:
+        raise ValueError("or_linear_q rejected its arguments")
+    if rc == 3:
+        raise OverflowError("or_linear_q: an accumulator does not fit int32")
+    return y, acc

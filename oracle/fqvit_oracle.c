@@ -1,6 +1,7 @@
 /*
  * fqvit_oracle.c -- plain, slow CPU oracle for the FQ-ViT integer inference
- * path (PTF LayerNorm and Log-Int-Softmax attention).
+ * path (PTF LayerNorm, Log-Int-Softmax attention and the MinMax Linear
+ * layers of the block).
  *
  * TEST INFRASTRUCTURE ONLY.  This file is the checker the CUDA library is
  * compared against.  Only tests, the package smoke check and the bench's CPU
@@ -15,7 +16,8 @@
  * Parity status: every function below is pinned by tests under tests/
  * (worked example of Find_First_One, hand-computed i-exp points, closed-form
  * softmax rows, MinMax special cases of PTF, textbook LayerNorm agreement,
- * matmul form of the BitShift product).
+ * matmul form of the BitShift product, permutation-weight and unit-multiplier
+ * closed forms of the Linear layer).
  */
 #include <math.h>
 #include <stdint.h>
@@ -576,5 +578,95 @@ OR_EXPORT int or_lis_attn_v(const uint8_t *codes, int64_t ld_codes, const int8_t
         }
         free(a);
     }
+    return overflow ? 3 : 0;
+}
+
+/* ------------------------------------------------------------------ */
+/* MinMax Linear layer (Sec. 3, Sec. 4.1)                              */
+/* ------------------------------------------------------------------ */
+
+/*
+ * A Linear layer of the fully quantized block.  Sec. 3 quantizes Linear
+ * layers with uniform MinMax; Sec. 4.1 makes the weights symmetric and
+ * channel-wise and the activations asymmetric and layer-wise:
+ *   x  uint8 [M][ld_x]   real value (x - zp_x) s_x
+ *   w  int8  [N][ld_w]   real value  w s_w[n]       (output channel n)
+ *   b  int32 [N]         real value  b s_x s_w[n]   (NULL: no bias)
+ * The integer product, in int64:
+ *   acc[m][n] = sum_k (x[m][k] - zp_x) w[n][k] + b[n]
+ * and the output quantizer, uniform MinMax with scale s_y and zero point
+ * zp_y, applied with the dyadic multiplier of the supplement's LayerNorm
+ * output stage, one per output channel:
+ *   M_n = (s_x s_w[n]) / s_y   in fp32, in this order
+ *   N1  = 7 - floor(log2 M_n)  (at most 31),   N2 = floor(M_n 2^N1)
+ *   y   = clip(floor((N2 acc + 2^(N1-1)) / 2^N1) + zp_y, 0, 255)   N1 > 0
+ *   y   = clip(N2 acc 2^min(-N1, 10) + zp_y, 0, 255)                N1 <= 0
+ * y [M][ld_y]; acc_opt [M][ld_acc] (may be NULL) receives acc.
+ * Returns 1 for invalid arguments (a scale that is not positive and finite,
+ * or an M_n outside (0, 1e30)), 3 if an acc does not fit int32 (its stored
+ * value is then saturated).
+ */
+OR_EXPORT int or_linear_q(const uint8_t *x, int64_t M, int32_t K, int64_t ld_x, int32_t zp_x, float s_x,
+                          const int8_t *w, int32_t N, int64_t ld_w, const float *s_w, const int32_t *bias,
+                          float s_y, int32_t zp_y, uint8_t *y, int64_t ld_y, int32_t *acc_opt, int64_t ld_acc)
+{
+    if (!x || !w || !s_w || !y || M < 1 || K < 1 || N < 1 || ld_x < K || ld_w < K || ld_y < N) return 1;
+    if (acc_opt && ld_acc < N) return 1;
+    if (zp_x < 0 || zp_x > 255 || zp_y < 0 || zp_y > 255) return 1;
+    if (!(s_x > 0.0f) || !(s_x < INFINITY) || !(s_y > 0.0f) || !(s_y < INFINITY)) return 1;
+    int32_t *n1 = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
+    int64_t *n2 = (int64_t *)malloc(sizeof(int64_t) * (size_t)N);
+    int bad = 0;
+    for (int32_t n = 0; n < N; ++n) {
+        const float a = s_x * s_w[n];
+        const float Mn = a / s_y;
+        if (!(s_w[n] > 0.0f) || !(Mn > 0.0f) || !(Mn < 1.0e30f)) {
+            bad = 1;
+            n1[n] = 0;
+            n2[n] = 0;
+            continue;
+        }
+        int e = 7 - ilogbf(Mn);
+        if (e > 31) e = 31;
+        n1[n] = e;
+        n2[n] = (int64_t)floorf(ldexpf(Mn, e));
+    }
+    if (bad) {
+        free(n1);
+        free(n2);
+        return 1;
+    }
+    int overflow = 0;
+#ifdef _OPENMP
+#pragma omp parallel for schedule(static) reduction(| : overflow)
+#endif
+    for (int64_t m = 0; m < M; ++m) {
+        const uint8_t *xm = x + m * ld_x;
+        for (int32_t n = 0; n < N; ++n) {
+            const int8_t *wn = w + (int64_t)n * ld_w;
+            int64_t s = 0;
+            for (int32_t k = 0; k < K; ++k) s += ((int64_t)xm[k] - zp_x) * (int64_t)wn[k];
+            if (bias) s += bias[n];
+            if (s > INT32_MAX || s < INT32_MIN) {
+                overflow = 1;
+                s = clamp_i64(s, INT32_MIN, INT32_MAX);
+            }
+            if (acc_opt) acc_opt[m * ld_acc + n] = (int32_t)s;
+            const int64_t num = n2[n] * s;
+            int64_t R;
+            if (n1[n] > 0)
+                R = floor_div_pow2(num + ((int64_t)1 << (n1[n] - 1)), n1[n]);
+            else if (n1[n] == 0)
+                R = num;
+            else {
+                int sh = -n1[n];
+                if (sh > 10) sh = 10;
+                R = num * ((int64_t)1 << sh);
+            }
+            y[m * ld_y + n] = (uint8_t)clamp_i64(R + zp_y, 0, 255);
+        }
+    }
+    free(n1);
+    free(n2);
     return overflow ? 3 : 0;
 }
