@@ -59,6 +59,56 @@ def peaks():
     return 6800.0, "fallback"
 
 
+def tensor_peak():
+    """Dense fp16 / bf16 tensor-core TFLOP/s for a kernel timed alone (the burst figure; the two
+    types have the same dense rate on this GPU)."""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        if "bf16_tflops" in d:
+            return float(d["bf16_tflops"]), "measured"
+    return 1900.0, "fallback"
+
+
+def bench_linear(fqvit, cfg, dev):
+    """The block's four MinMax Linear layers (QKV, projection, fc1, fc2) of layer 0 at the
+    config's token count, each call (the fp16 copy of X, then the tensor-core product and its
+    requantization) timed alone with CUDA events: 10 calls after 3."""
+    peak, kind = tensor_peak()
+    out, tot_ms, tot_flop = {}, 0.0, 0
+    for k in synth.LINEAR_KINDS:
+        a = synth.linear_inputs(cfg, 0, k, device=dev)
+        wh = fqvit.linear_pack_weight(a["w"])
+        ws = torch.empty(fqvit.linear_workspace_size(a["M"], a["K"]), dtype=torch.uint8, device=dev)
+        y = torch.empty(a["M"], a["N"], dtype=torch.uint8, device=dev)
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(10)]
+        for i in range(13):
+            if i >= 3:
+                evs[i - 3][0].record()
+            fqvit.linear_q(a["x"], a["zp_x"], a["s_x"], wh, a["s_w"], a["bias"], a["s_y"], a["zp_y"], out=y,
+                           workspace=ws)
+            if i >= 3:
+                evs[i - 3][1].record()
+        torch.cuda.synchronize()
+        fqvit.sync_status()
+        ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in evs)
+        flop = 2 * a["M"] * a["N"] * a["K"]
+        tf = flop / (ms / 1e3) / 1e12
+        out[k] = {"M": a["M"], "N": a["N"], "K": a["K"], "ms_per_call": round(ms, 5), "tflops": round(tf, 1),
+                  "frac": round(tf / peak, 4)}
+        tot_ms += ms
+        tot_flop += flop
+        del a, wh, ws, y
+    tf = tot_flop / (tot_ms / 1e3) / 1e12
+    out["block"] = {"ms": round(tot_ms, 5), "tflops": round(tf, 1), "frac": round(tf / peak, 4),
+                    "peak_tflops": peak, "peak_source": f"{kind} (MEASURED_PEAKS.json bf16_tflops)"
+                    if kind == "measured" else "fallback"}
+    out["how"] = ("fqvit_linear_q per layer of block 0 (fp16 copy of X + tcgen05 product + per-channel "
+                  "requantization), 10 calls after 3, outside the timed step; FLOP = 2 M N K")
+    return out
+
+
 # ------------------------------------------------------------------ byte model
 
 def ln_bytes(rows, C):
@@ -457,6 +507,8 @@ def bench_gpu(args):
                            "to HBM), 10 launches after 3, outside the timed step"}
         del full
 
+    lin_stats = bench_linear(fqvit, cfg, dev) if args.linear else None
+
     e2e = None
     if not args.no_e2e:
         e2e = bench_e2e(fqvit, layers, tokens_per_step, args, dev, ws)
@@ -502,6 +554,7 @@ def bench_gpu(args):
             "layernorm": {"gbs": round(ln_gbs, 1), "ms_per_launch": round(sum(ln_ms) / len(ln_ms), 5),
                           "bytes_per_launch": round(sum(lb) / len(lb))},
             **({"qk_logits": qk_stats} if args.qk else {}),
+            **({"linear": lin_stats} if lin_stats else {}),
             **({"patch_merge_layernorm": {
                 "gbs": round(sum(mb) * ev_steps / (sum(merge_ms) / 1e3) / 1e9, 1),
                 "ms_per_launch": round(sum(merge_ms) / len(merge_ms), 5),
@@ -687,6 +740,8 @@ def main():
                     help="attention from int8 Q, K, V (fqvit_qk_lis_attention) instead of int8 logits")
     ap.add_argument("--out8", action="store_true",
                     help="the attention output requantized to 8 bits (fqvit_lis_attention_q) instead of int32")
+    ap.add_argument("--linear", action="store_true",
+                    help="also time the block's MinMax Linear layers (fqvit_linear_q) alone, outside the step")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

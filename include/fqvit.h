@@ -52,6 +52,8 @@ FQVIT_API const char *fqvit_last_error(void);
  * FQVIT_ERR_TIMEOUT if a kernel of this library abandoned a bounded wait
  * (every wait on an asynchronous copy or tensor-core operation gives up after
  * two seconds, drains what it issued and returns) since the last call,
+ * FQVIT_ERR_INVALID_ARG if fqvit_linear_q met a per-channel weight scale that
+ * is not positive and finite (device data the host does not see),
  * FQVIT_ERR_CUDA if the stream reports an error, else FQVIT_OK.  The word is
  * cleared.  Not part of the paper; a diagnostic of this implementation. */
 FQVIT_API int fqvit_sync_status(void *stream);
@@ -356,6 +358,56 @@ FQVIT_API int fqvit_qk_lis_attention(const int8_t *q, int64_t ld_q, int32_t zp_q
                               const fqvit_window_mask *mask_opt, const int8_t *v, int64_t ld_v,
                               int32_t zp_v, int64_t BH, int32_t L, int32_t d, int32_t *acc, int64_t ld_acc,
                               int8_t *workspace, size_t workspace_bytes, int64_t group_heads, void *stream);
+
+/* ------------------------------------------------------------------ */
+/* MinMax Linear layers of the block (Sec. 3; Sec. 4.1)                */
+/* ------------------------------------------------------------------ */
+
+/*
+ * Weights of a Linear layer in the form fqvit_linear_q takes: int8 codes
+ * w [N][ld_w] (symmetric, channel-wise; device) -> fp16 w_h [N][K] (device,
+ * caller-owned, written once and kept with the model).  Every code is exact
+ * in fp16.  Supported: K a multiple of 8, ld_w a multiple of 8 with an 8-byte
+ * aligned base, w_h 16-byte aligned.  Errors: INVALID_ARG (NULL, shapes,
+ * alignment), UNSUPPORTED (K).
+ */
+FQVIT_API int fqvit_linear_pack_weight(const int8_t *w, int32_t N, int32_t K, int64_t ld_w, uint16_t *w_h,
+                                       void *stream);
+
+/* Bytes of workspace fqvit_linear_q needs: the fp16 copy of the activations,
+ * M x K x 2.  0 for a bad shape. */
+FQVIT_API size_t fqvit_linear_workspace_size(int64_t M, int32_t K);
+
+/*
+ * A Linear layer of the fully quantized block.  Sec. 3 quantizes Linear
+ * layers with uniform MinMax; Sec. 4.1 takes the weights symmetric and
+ * channel-wise, the activations asymmetric and layer-wise:
+ *   acc[m][n] = sum_k (x[m][k] - zp_x) w[n][k] + bias[n]        (exact, int32)
+ *   M_n = (s_x s_w[n]) / s_y     (fp32, in this order)
+ *   N1 = 7 - floor(log2 M_n) (at most 31), N2 = floor(M_n 2^N1)  (the dyadic
+ *        multiplier of the supplement's LayerNorm output stage, per channel)
+ *   y[m][n] = clip(floor((N2 acc + 2^(N1-1)) / 2^N1) + zp_y, 0, 255)
+ *        (N1 <= 0: clip(N2 acc 2^min(-N1, 10) + zp_y, 0, 255)).
+ * The bias is the integer bias at scale s_x s_w[n] (|bias[n]| <= 2^30).
+ * x [M][ld_x] uint8 (device); w_h [N][K] from fqvit_linear_pack_weight;
+ * s_w [N] float and bias_opt [N] int32 (device; bias NULL = none);
+ * y [M][ld_y] uint8 (device, caller-owned); acc_opt [M][ld_acc] int32
+ * (device, may be NULL) receives acc; workspace (device, caller-owned, at
+ * least fqvit_linear_workspace_size(M, K) bytes, 16-byte aligned) is
+ * overwritten.  Two launches on `stream` (the fp16 copy of x, then the
+ * tensor-core product and its requantization).
+ * Supported: K <= 16384 a multiple of 8, N <= 4096 a multiple of 16,
+ * ld_x a multiple of 8 with an 8-byte aligned base, ld_y a multiple of 16 and
+ * ld_acc of 4 with 16-byte aligned bases, zero points in 0..255.  Errors:
+ * INVALID_ARG (NULL, shapes, strides, alignment, zero points, s_x or s_y not
+ * positive and finite, a small workspace), UNSUPPORTED (K, N, M >= 2^31).  A
+ * weight scale that is not positive and finite is device data: its channel
+ * holds zp_y and fqvit_sync_status reports INVALID_ARG.
+ */
+FQVIT_API int fqvit_linear_q(const uint8_t *x, int64_t M, int32_t K, int64_t ld_x, int32_t zp_x, float s_x,
+                             const uint16_t *w_h, int32_t N, const float *s_w, const int32_t *bias_opt, float s_y,
+                             int32_t zp_y, uint8_t *y, int64_t ld_y, int32_t *acc_opt, int64_t ld_acc,
+                             void *workspace, size_t workspace_bytes, void *stream);
 
 /* ------------------------------------------------------------------ */
 /* One layer: norm1 LayerNorm and the attention core (Fig. 4 dataflow) */

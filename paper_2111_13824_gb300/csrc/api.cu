@@ -78,6 +78,10 @@ int fqvit_sync_status(void *stream)
     if (e != cudaSuccess) return fail(FQVIT_ERR_CUDA, "sync_status: %s", cudaGetErrorString(e));
     if (status == FQVIT_ERR_TIMEOUT)
         return fail(FQVIT_ERR_TIMEOUT, "a kernel abandoned a bounded wait (results of that launch are invalid)");
+    if (status == FQVIT_ERR_INVALID_ARG)
+        return fail(FQVIT_ERR_INVALID_ARG,
+                    "a Linear layer met a weight scale s_w[n] that is not positive and finite, or a multiplier "
+                    "s_x s_w[n] / s_y outside (0, 1e30) (those channels hold zp_y)");
     return ok();
 }
 
@@ -521,6 +525,55 @@ int fqvit_qk_lis_attention(const int8_t *q, int64_t ld_q, int32_t zp_q, const in
         if (e != cudaSuccess) return cuda_status(e, who);
     }
     return ok();
+}
+
+// ---- MinMax Linear layers -------------------------------------------------
+
+size_t fqvit_linear_workspace_size(int64_t M, int32_t K)
+{
+    if (M < 1 || K < 1) return 0;
+    return (size_t)M * (size_t)K * 2;
+}
+
+int fqvit_linear_pack_weight(const int8_t *w, int32_t N, int32_t K, int64_t ld_w, uint16_t *w_h, void *stream)
+{
+    const char *who = "linear_pack_weight";
+    if (!w || !w_h) return fail(FQVIT_ERR_INVALID_ARG, "%s: NULL pointer", who);
+    if (N < 1 || K < 1 || ld_w < K)
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: bad shape N=%d K=%d ld_w=%lld", who, N, K, (long long)ld_w);
+    if (K % 8) return fail(FQVIT_ERR_UNSUPPORTED, "%s: K=%d (a multiple of 8)", who, K);
+    if (ld_w % 8 || !aligned(w, 8) || !aligned(w_h, 16))
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: w rows must be 8-byte aligned and w_h 16-byte aligned", who);
+    return cuda_status(fqvit::launch_linear_pack_weight(w, N, K, ld_w, w_h, as_stream(stream)), who);
+}
+
+int fqvit_linear_q(const uint8_t *x, int64_t M, int32_t K, int64_t ld_x, int32_t zp_x, float s_x,
+                   const uint16_t *w_h, int32_t N, const float *s_w, const int32_t *bias_opt, float s_y,
+                   int32_t zp_y, uint8_t *y, int64_t ld_y, int32_t *acc_opt, int64_t ld_acc, void *workspace,
+                   size_t workspace_bytes, void *stream)
+{
+    const char *who = "linear_q";
+    if (!x || !w_h || !s_w || !y || !workspace) return fail(FQVIT_ERR_INVALID_ARG, "%s: NULL pointer", who);
+    if (M < 1 || K < 1 || N < 1 || ld_x < K || ld_y < N || (acc_opt && ld_acc < N))
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: bad shape M=%lld K=%d N=%d", who, (long long)M, K, N);
+    if (zp_x < 0 || zp_x > 255 || zp_y < 0 || zp_y > 255)
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: zero points outside 0..255", who);
+    if (!(s_x > 0.0f) || !(s_x < 3.0e38f) || !(s_y > 0.0f) || !(s_y < 3.0e38f))
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: s_x and s_y must be positive and finite", who);
+    if (K % 8 || K > 16384 || N % 16 || N > 4096 || M > ((int64_t)1 << 31) - 1)
+        return fail(FQVIT_ERR_UNSUPPORTED, "%s: K=%d N=%d M=%lld (K <= 16384 a multiple of 8, N <= 4096 a "
+                    "multiple of 16, M < 2^31)", who, K, N, (long long)M);
+    if (ld_x % 8 || !aligned(x, 8) || !aligned(w_h, 16) || ld_y % 16 || !aligned(y, 16) || !aligned(s_w, 4) ||
+        !aligned(bias_opt, 4) || (acc_opt && (ld_acc % 4 || !aligned(acc_opt, 16))) || !aligned(workspace, 16))
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: misaligned pointer or row stride", who);
+    if (workspace_bytes < fqvit_linear_workspace_size(M, K))
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: workspace of %zu bytes, %zu needed", who, workspace_bytes,
+                    fqvit_linear_workspace_size(M, K));
+    fqvit::LinearArgs a{x,    M,        ld_x, K,    zp_x,    s_x,    w_h,    N,
+                        s_w,  bias_opt, s_y,  zp_y, y,       ld_y,   acc_opt, ld_acc,
+                        static_cast<uint16_t *>(workspace)};
+    if (!fqvit::linear_supported(a)) return fail(FQVIT_ERR_UNSUPPORTED, "%s: N=%d needs too much shared memory", who, N);
+    return cuda_status(fqvit::launch_linear(a, as_stream(stream)), who);
 }
 
 int fqvit_block_int(const fqvit_block_desc *b, void *stream)

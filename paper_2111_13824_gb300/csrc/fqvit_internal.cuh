@@ -175,8 +175,31 @@ bool lis_attention_win_eligible(const LisArgs &a, const AttnVArgs &b);
 cudaError_t launch_lis_attention_win(const LisArgs &a, const AttnVArgs &b, cudaStream_t st);
 cudaError_t read_clear_win_status(int *status);
 
-// Synchronizes st, returns the device status word (0 ok, 5 a bounded wait
-// timed out) and clears it.
+// ---- MinMax Linear layer on the tensor cores (linear_tc.cu) ----------------
+struct LinearArgs {
+    const uint8_t *x;
+    int64_t M, ld_x;
+    int K, zp_x;
+    float s_x;
+    const uint16_t *w_h;  // fp16 [N][K]
+    int N;
+    const float *s_w;
+    const int32_t *bias;  // may be NULL
+    float s_y;
+    int zp_y;
+    uint8_t *y;
+    int64_t ld_y;
+    int32_t *acc;  // may be NULL
+    int64_t ld_acc;
+    uint16_t *xh;  // workspace: fp16 [M][K]
+};
+bool linear_supported(const LinearArgs &a);
+cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st);
+cudaError_t launch_linear_pack_weight(const int8_t *w, int N, int K, int64_t ld_w, uint16_t *w_h, cudaStream_t st);
+cudaError_t read_clear_linear_status(int *status);
+
+// Synchronizes st, returns the device status word (0 ok, 1 a device-side argument was
+// invalid, 5 a bounded wait timed out) and clears it.
 cudaError_t read_clear_device_status(int *status, cudaStream_t st);
 
 // Attention implementation choice: 0 automatic, 1 CUDA cores only (FQVIT_ATTN_PATH=cuda_core),

@@ -1,0 +1,436 @@
+// linear_tc.cu -- the MinMax Linear layers of the fully quantized block on the
+// 5th-generation tensor cores (tcgen05) of sm_103a.  Sec. 3 quantizes Linear
+// layers with uniform MinMax; Sec. 4.1 makes the weights symmetric and
+// channel-wise and the activations asymmetric and layer-wise:
+//   acc[m][n] = sum_k (x[m][k] - zp_x) w[n][k] + b[n]
+//   y[m][n]   = clip(floor((N2_n acc + 2^(N1_n - 1)) / 2^N1_n) + zp_y, 0, 255)
+// with N1_n, N2_n the dyadic form of M_n = s_x s_w[n] / s_y (the output stage of
+// the supplement's LayerNorm; N1_n <= 0 is a product by N2_n 2^min(-N1_n, 10)).
+//
+// Exactness.  x - zp_x lies in -255 .. 255 and w in -128 .. 127, both exact in
+// fp16, every product exact in fp32.  A sum of such integers is exact in fp32
+// while its partial sums stay within 2^24; the reduction runs in chunks of kc
+// steps of 64 with 64 kc max|x - zp_x| 128 <= 2^22 (kc = 2 for zp_x at 0 or
+// 255, 4 for zp_x = 128), the scale at which the attention's BitShift product
+// (sums near 2^22 with unit terms) is exact on these tensor cores.  Each chunk
+// is accumulated afresh in tensor memory and added in int32 by the epilogue.
+//
+// Layout.  The weights are converted once to fp16 [N][K] (fqvit_linear_pack_weight);
+// the activations per call to fp16 (x - zp_x) [M][K] in a workspace by an
+// elementwise kernel.  Both reach shared memory by TMA tensor loads with the
+// 128-byte swizzle: per stage a box of 64 (K) x 128 rows of X and 64 x 256 rows
+// of W, four stages.
+//
+// Roles (320 threads): warps 0-7 are the epilogue (warp w reads tensor-memory
+// lanes 32 (w % 4) .. and columns 128 (w / 4) .. of a tile), warp 8 lane 0
+// issues the TMA loads, warp 9 lane 0 the MMAs (M = 128, N <= 256, K = 16).
+// Tiles of 128 x 256 outputs; each CTA (one per SM) takes a contiguous range
+// of tiles, N-tiles fastest, so consecutive tiles share their X rows in L2.
+// Two accumulators of 256 tensor-memory columns: the MMAs of the next chunk
+// run while the epilogue reads the last.  Every wait is bounded: after two
+// seconds the kernel records a timeout status, drains the copies and MMAs it
+// issued and returns.
+#include "fqvit_internal.cuh"
+#include "tc_common.cuh"
+
+#include <cstring>
+#include <cuda.h>
+#include <cuda_fp16.h>
+#include <cudaTypedefs.h>
+
+namespace fqvit {
+
+namespace {
+
+using namespace tc;
+
+constexpr int LM = 128;                   // output rows per tile (MMA M)
+constexpr int LN = 256;                   // output columns per tile (MMA N at most)
+constexpr int LK = 64;                    // reduction per stage: one 128-byte swizzle row of fp16
+constexpr int LST = 4;                    // stages
+constexpr int LA_BYTES = LM * LK * 2;     // 16 KB
+constexpr int LB_BYTES = LN * LK * 2;     // 32 KB
+constexpr int LSTAGE = LA_BYTES + LB_BYTES;
+constexpr int LTHREADS = 320;
+constexpr int LEPI_WARPS = 8;
+constexpr int LMAXN = 4096;               // channels of the shared-memory table
+
+struct LinParams {
+    int64_t M;
+    int N, K;
+    int ksteps;    // ceil(K / 64)
+    int kc;        // steps per exact chunk
+    int zp_y;
+    float s_x, s_y;
+    const float *s_w;
+    const int32_t *bias;
+    uint8_t *y;
+    int64_t ld_y;
+    int32_t *acc;
+    int64_t ld_acc;
+    int64_t mtiles;
+    int ntiles;
+};
+
+struct LinShared {
+    uint64_t full[LST], empty[LST], cfull[2], cempty[2], fin;
+    uint32_t tmem;
+    int abort_flag;
+};
+
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int x, int y, uint64_t *bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], "
+        "[%4];" ::"r"(sa(dst)),
+        "l"(map), "r"(x), "r"(y), "r"(sa(bar))
+        : "memory");
+}
+
+// Per output channel: the multiplier and the shift of the requantization (mult < 2^18 in
+// bits 0..17, shift 0..31 in bits 24..28) and the bias.  N1 <= 0 folds 2^min(-N1, 10) into
+// the multiplier with shift 0.  The fp32 operations are single IEEE round-to-nearest ones,
+// as on the host.
+__device__ __forceinline__ int2 channel_constants(const LinParams &p, int n, bool &bad)
+{
+    const float sw = p.s_w[n];
+    const float Mn = __fdiv_rn(__fmul_rn(p.s_x, sw), p.s_y);
+    int mult = 0, shift = 0;
+    if (sw > 0.0f && Mn > 0.0f && Mn < 1.0e30f) {
+        int n1 = 7 - ilogbf(Mn);
+        if (n1 > 31) n1 = 31;
+        const int n2 = (int)floorf(ldexpf(Mn, n1));
+        if (n1 >= 0) {
+            mult = n2;
+            shift = n1;
+        } else {
+            mult = n2 << min(-n1, 10);
+        }
+    } else {
+        bad = true;
+    }
+    return make_int2(mult | (shift << 24), p.bias ? p.bias[n] : 0);
+}
+
+// y code of one accumulator (the bias added): (mult acc + 2^(shift-1)) >> shift, + zp_y, clipped
+__device__ __forceinline__ uint32_t y_code(int acc, int2 ch, int zp_y)
+{
+    const int mult = ch.x & 0xFFFFFF, shift = ch.x >> 24;
+    const long long num = (long long)mult * acc + (long long)((1u << shift) >> 1);
+    const long long R = (num >> shift) + zp_y;
+    return (uint32_t)(R < 0 ? 0 : R > 255 ? 255 : R);
+}
+
+template <bool ACC>
+__global__ void __launch_bounds__(LTHREADS, 1)
+    linear_tc_kernel(const __grid_constant__ LinParams p, const __grid_constant__ CUtensorMap tmx,
+                     const __grid_constant__ CUtensorMap tmw)
+{
+    extern __shared__ unsigned char dsm_raw[];
+    __shared__ LinShared sh;
+    unsigned char *base = dsm_raw + ((1024u - (sa(dsm_raw) & 1023u)) & 1023u);
+    int2 *CH = reinterpret_cast<int2 *>(base + (size_t)LST * LSTAGE);  // [N] channel constants
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    volatile int *abort_flag = &sh.abort_flag;
+    pdl_release();
+    if (tid == 0) {
+        for (int s = 0; s < LST; ++s) {
+            mbar_init(&sh.full[s], 1);
+            mbar_init(&sh.empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&sh.cfull[b], 1);
+            mbar_init(&sh.cempty[b], LEPI_WARPS);
+        }
+        mbar_init(&sh.fin, 1);
+        sh.abort_flag = 0;
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(&sh.tmem)),
+                     "r"(2 * LN));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    pdl_wait();  // the set-up above touched no global memory
+    bool bad = false;
+    for (int n = tid; n < p.N; n += LTHREADS) CH[n] = channel_constants(p, n, bad);
+    if (bad) atomicExch(&g_status, 1);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sh.tmem;
+
+    const int64_t ntiles = p.mtiles * p.ntiles;
+    const int64_t t_begin = (int64_t)blockIdx.x * ntiles / gridDim.x;
+    const int64_t t_end = (int64_t)(blockIdx.x + 1) * ntiles / gridDim.x;
+
+    if (warp == LEPI_WARPS) {
+        // ---- TMA producer: stage it % LST holds step it; it is issued once step it - LST was consumed
+        if (lane == 0) {
+            uint32_t it = 0;
+            bool ok = true;
+            for (int64_t t = t_begin; t < t_end && ok; ++t) {
+                const int mt = (int)(t / p.ntiles), nt = (int)(t - (int64_t)mt * p.ntiles);
+                for (int ks = 0; ks < p.ksteps; ++ks, ++it) {
+                    const uint32_t st = it % LST;
+                    if (it >= LST && !mbar_wait(&sh.empty[st], ((it / LST) - 1) & 1, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    unsigned char *sA = base + (size_t)st * LSTAGE;
+                    mbar_expect_tx(&sh.full[st], LSTAGE);
+                    tma_load_2d(sA, &tmx, ks * LK, mt * LM, &sh.full[st]);
+                    tma_load_2d(sA + LA_BYTES, &tmw, ks * LK, nt * LN, &sh.full[st]);
+                }
+            }
+            // the last (up to LST) loads may still be in flight if the consumer stopped early
+            for (uint32_t j = it > LST ? it - LST : 0; j < it; ++j)
+                mbar_wait(&sh.full[j % LST], (j / LST) & 1, abort_flag, false);
+        }
+        __syncwarp();
+    } else if (warp == LEPI_WARPS + 1) {
+        // ---- MMA issuer: chunk gc accumulates in tensor-memory buffer gc % 2
+        if (lane == 0) {
+            uint32_t it = 0, gc = 0, commits = 0;
+            bool ok = true;
+            for (int64_t t = t_begin; t < t_end && ok; ++t) {
+                const int mt = (int)(t / p.ntiles), nt = (int)(t - (int64_t)mt * p.ntiles);
+                (void)mt;
+                const int n_mma = min(LN, p.N - nt * LN);  // a multiple of 16 (N is)
+                const uint32_t idesc = (1u << 4) | ((uint32_t)(n_mma >> 3) << 17) | ((uint32_t)(LM >> 4) << 24);
+                for (int c0 = 0; c0 < p.ksteps && ok; c0 += p.kc, ++gc) {
+                    const uint32_t b = gc & 1;
+                    if (gc >= 2 && !mbar_wait(&sh.cempty[b], ((gc >> 1) - 1) & 1, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const int c1 = min(p.ksteps, c0 + p.kc);
+                    for (int ks = c0; ks < c1; ++ks, ++it) {
+                        const uint32_t st = it % LST;
+                        if (!mbar_wait(&sh.full[st], (it / LST) & 1, abort_flag)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t a0 = sa(base + (size_t)st * LSTAGE), b0 = a0 + LA_BYTES;
+#pragma unroll
+                        for (int s = 0; s < LK / 16; ++s)
+                            mma_f16_ss(tmem + b * LN, smem_desc(a0 + 32 * s, 16, 1024),
+                                       smem_desc(b0 + 32 * s, 16, 1024), idesc, ks > c0 || s > 0);
+                        mma_commit(&sh.empty[st]);  // the stage is free once these MMAs completed
+                        ++commits;
+                    }
+                    if (!ok) break;
+                    mma_commit(&sh.cfull[b]);
+                    ++commits;
+                }
+            }
+            if (commits > 0) {  // every MMA issued has completed before tensor memory is released
+                mma_commit(&sh.fin);
+                mbar_wait(&sh.fin, 0, abort_flag, false);
+            }
+        }
+        __syncwarp();
+    } else {
+        // ---- epilogue: warp w, lanes 32 (w % 4) .. (tile rows), columns 128 (w / 4) ..
+        const int q = warp & 3, h = warp >> 2;
+        const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(128 * h);
+        const int nch = (p.ksteps + p.kc - 1) / p.kc;
+        uint32_t gc = 0;
+        bool ok = true;
+        for (int64_t t = t_begin; t < t_end && ok; ++t) {
+            const int mt = (int)(t / p.ntiles), nt = (int)(t - (int64_t)mt * p.ntiles);
+            int sum[128];
+            for (int c = 0; c < nch; ++c, ++gc) {
+                const uint32_t b = gc & 1;
+                if (!mbar_wait_warp(&sh.cfull[b], (gc >> 1) & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {  // 16 columns at a time (registers: sum holds 128)
+                    uint32_t v[16];
+                    tmem_ld16(tl + b * LN + 16 * j, v);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const int a = __float2int_rn(__uint_as_float(v[i]));  // an exact integer
+                        sum[16 * j + i] = c == 0 ? a : sum[16 * j + i] + a;
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sh.cempty[b]);
+            }
+            if (!ok) break;
+            const int64_t row = (int64_t)mt * LM + 32 * q + lane;
+            const int col0 = nt * LN + 128 * h;
+#pragma unroll
+            for (int g = 0; g < 8; ++g) {
+                const int col = col0 + 16 * g;
+                if (col >= p.N) break;  // N is a multiple of 16: whole groups
+                int a[16];
+                uint32_t w[4];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int2 ch = CH[col + i];
+                    a[i] = sum[16 * g + i] + ch.y;
+                    const uint32_t yc = y_code(a[i], ch, p.zp_y);
+                    if ((i & 3) == 0)
+                        w[i >> 2] = yc;
+                    else
+                        w[i >> 2] |= yc << (8 * (i & 3));
+                }
+                if (row < p.M) {
+                    *reinterpret_cast<uint4 *>(p.y + row * p.ld_y + col) = make_uint4(w[0], w[1], w[2], w[3]);
+                    if (ACC) {
+                        int4 *dst = reinterpret_cast<int4 *>(p.acc + row * p.ld_acc + col);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) dst[i] = make_int4(a[4 * i], a[4 * i + 1], a[4 * i + 2], a[4 * i + 3]);
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * LN));
+}
+
+// Eight bytes to eight fp16 values minus a zero point z (exact): byte b becomes the fp16
+// 1024 + b (exponent of 1024, b in the mantissa), then 1024 + zp is subtracted.  Signed codes
+// arrive with their sign bit flipped (b = w + 128) and zp = 128.
+__device__ __forceinline__ uint4 bytes_to_h8(uint2 w, __half2 z)
+{
+    uint32_t h[4] = {__byte_perm(w.x, 0x64u, 0x4140), __byte_perm(w.x, 0x64u, 0x4342),
+                     __byte_perm(w.y, 0x64u, 0x4140), __byte_perm(w.y, 0x64u, 0x4342)};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        __half2 t = __hsub2(*reinterpret_cast<const __half2 *>(&h[i]), z);
+        h[i] = *reinterpret_cast<const uint32_t *>(&t);
+    }
+    return make_uint4(h[0], h[1], h[2], h[3]);
+}
+
+// src [rows][ld] bytes (K a multiple of 8) -> dst [rows][K] fp16 of (byte ^ flip) - zp
+__global__ void __launch_bounds__(256) bytes_to_half_kernel(const uint8_t *src, int64_t rows, int K, int64_t ld,
+                                                            uint32_t flip, int zp, uint16_t *dst)
+{
+    pdl_release();
+    pdl_wait();
+    const int kv = K >> 3;
+    const int64_t items = rows * kv;
+    const __half2 z = __half2half2(__int2half_rn(1024 + zp));
+    for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < items; x += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = x / kv;
+        const int c = (int)(x - r * kv);
+        uint2 w = __ldg(reinterpret_cast<const uint2 *>(src + r * ld + 8 * c));
+        w.x ^= flip;
+        w.y ^= flip;
+        *reinterpret_cast<uint4 *>(dst + r * K + 8 * c) = bytes_to_h8(w, z);
+    }
+}
+
+size_t linear_smem_bytes(int N) { return 1024 + (size_t)LST * LSTAGE + (size_t)N * sizeof(int2); }
+
+// fp16 [rows][K] row-major as a 2-d tensor for the TMA loads: boxes of 64 x box_rows, 128-byte
+// swizzle, zeros outside.  False when the driver's encoder is unavailable or rejects the shape.
+bool half_tensor_map(CUtensorMap *tm, const uint16_t *ptr, int64_t rows, int K, int box_rows)
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    if (!encode) return false;
+    const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)LK, (cuuint32_t)box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return encode(tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<uint16_t *>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <bool ACC>
+cudaError_t linear_launch(const LinParams &p, const CUtensorMap &tx, const CUtensorMap &tw, size_t smem, int grid,
+                          cudaStream_t st)
+{
+    cudaError_t e = cudaFuncSetAttribute(linear_tc_kernel<ACC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(linear_tc_kernel<ACC>, dim3(grid), dim3(LTHREADS), smem, st, p, tx, tw);
+}
+
+cudaError_t launch_bytes_to_half(const uint8_t *src, int64_t rows, int K, int64_t ld, uint32_t flip, int zp,
+                                 uint16_t *dst, cudaStream_t st)
+{
+    const int64_t items = rows * (K / 8);
+    int64_t blocks = (items + 255) / 256;
+    const int64_t cap = (int64_t)sm_count() * 8;
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    return launch_pdl(bytes_to_half_kernel, dim3((unsigned)blocks), dim3(256), 0, st, src, rows, K, ld, flip, zp,
+                      dst);
+}
+
+}  // namespace
+
+bool linear_supported(const LinearArgs &a) { return a.N <= LMAXN && linear_smem_bytes(a.N) + sizeof(LinShared) + 64 <= 232448; }
+
+cudaError_t launch_linear_pack_weight(const int8_t *w, int N, int K, int64_t ld_w, uint16_t *w_h, cudaStream_t st)
+{
+    return launch_bytes_to_half(reinterpret_cast<const uint8_t *>(w), N, K, ld_w, 0x80808080u, 128, w_h, st);
+}
+
+cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st)
+{
+    cudaError_t e = launch_bytes_to_half(a.x, a.M, a.K, a.ld_x, 0u, a.zp_x, a.xh, st);
+    if (e != cudaSuccess) return e;
+    CUtensorMap tx, tw;
+    memset(&tx, 0, sizeof(tx));
+    memset(&tw, 0, sizeof(tw));
+    if (!half_tensor_map(&tx, a.xh, a.M, a.K, LM) || !half_tensor_map(&tw, a.w_h, a.N, a.K, LN))
+        return cudaErrorInvalidValue;
+    LinParams p{};
+    p.M = a.M;
+    p.N = a.N;
+    p.K = a.K;
+    p.ksteps = (a.K + LK - 1) / LK;
+    const int maxabs = a.zp_x > 255 - a.zp_x ? a.zp_x : 255 - a.zp_x;  // 128 .. 255
+    p.kc = 512 / maxabs;  // 64 kc maxabs 128 <= 2^22
+    p.zp_y = a.zp_y;
+    p.s_x = a.s_x;
+    p.s_y = a.s_y;
+    p.s_w = a.s_w;
+    p.bias = a.bias;
+    p.y = a.y;
+    p.ld_y = a.ld_y;
+    p.acc = a.acc;
+    p.ld_acc = a.ld_acc;
+    p.mtiles = (a.M + LM - 1) / LM;
+    p.ntiles = (a.N + LN - 1) / LN;
+    const int64_t tiles = p.mtiles * p.ntiles;
+    const int grid = (int)(tiles < sm_count() ? tiles : sm_count());
+    const size_t smem = linear_smem_bytes(a.N);
+    return a.acc ? linear_launch<true>(p, tx, tw, smem, grid, st) : linear_launch<false>(p, tx, tw, smem, grid, st);
+}
+
+cudaError_t read_clear_linear_status(int *status)
+{
+    int zero = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(status, g_status, sizeof(int));
+    if (e != cudaSuccess) return e;
+    return cudaMemcpyToSymbol(g_status, &zero, sizeof(int));
+}
+
+}  // namespace fqvit

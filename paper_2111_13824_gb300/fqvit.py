@@ -51,6 +51,7 @@ EXPORTS = (
     "fqvit_calibrate_minmax", "fqvit_calibrate_sse_partial", "fqvit_calibrate_combine",
     "fqvit_lis_softmax_masked", "fqvit_lis_attention_masked", "fqvit_lis_attention_masked_q",
     "fqvit_qk_logits", "fqvit_qk_workspace_size", "fqvit_qk_lis_attention",
+    "fqvit_linear_pack_weight", "fqvit_linear_workspace_size", "fqvit_linear_q",
 )
 
 
@@ -90,6 +91,10 @@ def load(path: str | Path | None = None):
         "fqvit_qk_workspace_size": ([i64, i32, i64], sz),
         "fqvit_qk_lis_attention": ([P, i64, i32, P, i64, i32, f32, f32, f32, i32, i32, P, P, P, i64, i32, i64, i32,
                                     i32, P, i64, P, sz, i64, P], ctypes.c_int),
+        "fqvit_linear_pack_weight": ([P, i32, i32, i64, P, P], ctypes.c_int),
+        "fqvit_linear_workspace_size": ([i64, i32], sz),
+        "fqvit_linear_q": ([P, i64, i32, i64, i32, f32, P, i32, P, P, f32, i32, P, i64, P, i64, P, sz, P],
+                           ctypes.c_int),
         "fqvit_block_int": ([P, P], ctypes.c_int),
         "fqvit_sync_status": ([P], ctypes.c_int),
         "fqvit_calibrate_ptf_noalloc": ([P, i64, i32, i64, i32, i32, P, P, P, P, P], ctypes.c_int),
@@ -406,6 +411,40 @@ def qk_lis_attention(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, zp_q: in
                                          workspace.numel() * workspace.element_size(), int(group_heads),
                                          _stream(stream)))
     return acc
+
+
+def linear_pack_weight(w: torch.Tensor, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """int8 weight codes [N, K] -> the fp16 copy [N, K] fqvit_linear_q takes (fqvit_linear_pack_weight)."""
+    N, K = w.shape
+    if out is None:
+        out = torch.empty(N, K, dtype=torch.float16, device=w.device)
+    _check(load().fqvit_linear_pack_weight(_p(w), N, K, _ld(w), _p(out), _stream(stream)))
+    return out
+
+
+def linear_workspace_size(M: int, K: int) -> int:
+    return int(load().fqvit_linear_workspace_size(int(M), int(K)))
+
+
+def linear_q(x: torch.Tensor, zp_x: int, s_x: float, w_h: torch.Tensor, s_w: torch.Tensor,
+             bias: torch.Tensor | None, s_y: float, zp_y: int, out: torch.Tensor | None = None,
+             acc: torch.Tensor | None = None, workspace: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """A MinMax Linear layer (fqvit_linear_q): uint8 x [M, K] (zp_x, s_x), packed fp16 weights
+    [N, K] with per-channel scales s_w [N] and int32 bias [N] -> uint8 y [M, N] (s_y, zp_y);
+    acc, if given, receives the int32 accumulators."""
+    M, K = x.shape
+    N = w_h.shape[0]
+    if w_h.dtype != torch.float16 or w_h.shape[1] != K or not w_h.is_contiguous():
+        raise ValueError("w_h must be the contiguous fp16 [N, K] array of linear_pack_weight")
+    if out is None:
+        out = torch.empty(M, N, dtype=torch.uint8, device=x.device)
+    if workspace is None:
+        workspace = torch.empty(linear_workspace_size(M, K), dtype=torch.uint8, device=x.device)
+    _check(load().fqvit_linear_q(_p(x), M, K, _ld(x), int(zp_x), float(s_x), _p(w_h), N, _p(s_w), _p(bias),
+                                 float(s_y), int(zp_y), _p(out), _ld(out), _p(acc),
+                                 _ld(acc) if acc is not None else 0, _p(workspace), workspace.numel(),
+                                 _stream(stream)))
+    return out
 
 
 def block_int(xq, zp_in, alpha, gamma, beta, s_out, zp_out, yq, logits, ld_logit, s_logit, v, zp_v, acc,

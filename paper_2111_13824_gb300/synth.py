@@ -279,3 +279,54 @@ def shifted_window_regions(side: int, window: int, shift: int | None = None) -> 
 def swin_mask_value(s_logit: float, real: float = -100.0) -> int:
     """The Swin mask (-100 in real units) in logit units, kept inside -32768 .. 0."""
     return max(-32768, min(0, int(round(real / s_logit))))
+
+
+# ---- MinMax Linear layers of the block -------------------------------------
+
+LINEAR_KINDS = ("qkv", "proj", "fc1", "fc2")
+
+
+def linear_shape(C: int, kind: str) -> tuple[int, int]:
+    """(N, K) of a block's Linear layer: QKV C -> 3C, projection C -> C, MLP C -> 4C -> C."""
+    return {"qkv": (3 * C, C), "proj": (C, C), "fc1": (4 * C, C), "fc2": (C, 4 * C)}[kind]
+
+
+def linear_inputs(cfg: Config, layer: int, kind: str, device="cpu", rows: int | None = None,
+                  calib_rows: int = 512):
+    """Inputs of one MinMax Linear layer (generator seed S * 1000 + 700 + 4 layer + kind index).
+
+    * activations, real ``[rows, K]``: N(0, 1) for the LayerNorm outputs (QKV, fc1) and the
+      attention output (projection); GELU of N(0, 1) for the MLP's hidden layer (fc2), so its
+      zero point sits near the bottom of the range.  Quantized asymmetric, layer-wise, by the
+      min / max of the draw (Sec. 4.1).
+    * weights ``[N, K]``: N(0, 0.02^2) times a per-channel factor U(0.5, 2), quantized
+      symmetric, channel-wise (s_w = max |w_n| / 127, codes in -127 .. 127).
+    * bias: N(0, 0.02^2), as an integer at scale s_x s_w[n].
+    * output quantizer: min / max of the real-valued layer over the first ``calib_rows`` rows,
+      mapped to 0 .. 255 (MinMax).
+    """
+    st = layer_stage(cfg, layer)
+    N, K = linear_shape(st.C, kind)
+    M = st.rows if rows is None else rows
+    g = _gen(cfg.seed * 1000 + 700 + 4 * layer + LINEAR_KINDS.index(kind), device)
+    xr = torch.randn(M, K, generator=g, device=device, dtype=torch.float32)
+    if kind == "fc2":
+        xr = torch.nn.functional.gelu(xr)
+    lo, hi = float(xr.min()), float(xr.max())
+    s_x = float(torch.tensor((hi - lo) / 255.0, dtype=torch.float32))
+    zp_x = int(min(255, max(0, round(-lo / s_x))))
+    x = torch.clamp(torch.round(xr / s_x) + zp_x, 0, 255).to(torch.uint8)
+    del xr
+    wr = 0.02 * torch.randn(N, K, generator=g, device=device, dtype=torch.float32)
+    wr *= 0.5 + 1.5 * torch.rand(N, 1, generator=g, device=device)
+    s_w = (wr.abs().amax(dim=1) / 127.0).to(torch.float32)
+    w = torch.clamp(torch.round(wr / s_w[:, None]), -127, 127).to(torch.int8)
+    br = 0.02 * torch.randn(N, generator=g, device=device, dtype=torch.float64)
+    bias = torch.round(br / (s_x * s_w.double())).to(torch.int32)
+    c = min(M, calib_rows)
+    real = ((x[:c].double() - zp_x) * s_x) @ (w.double() * s_w.double()[:, None]).T + bias.double() * (s_x * s_w.double())
+    ylo, yhi = float(real.min()), float(real.max())
+    s_y = float(torch.tensor((yhi - ylo) / 255.0, dtype=torch.float32))
+    zp_y = int(min(255, max(0, round(-ylo / s_y))))
+    return dict(x=x.contiguous(), zp_x=zp_x, s_x=s_x, w=w.contiguous(), s_w=s_w.contiguous(),
+                bias=bias.contiguous(), s_y=s_y, zp_y=zp_y, M=M, N=N, K=K)

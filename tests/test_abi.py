@@ -144,3 +144,40 @@ def test_qk_checks(lib):
         ws_bytes, 0, None)
     assert g(197 * 208 - 1) == 1 and "workspace" in _err(lib)          # less than one head
     assert g(10 ** 8, v=None) == 1                                      # NULL V
+
+
+def test_linear_checks(lib):
+    """fqvit_linear_q / fqvit_linear_pack_weight reject bad arguments before any launch."""
+    fake = ctypes.c_void_p(4096)
+    M, K, N = 300, 384, 1152
+    ws = lib.fqvit_linear_workspace_size(M, K)
+    assert ws == M * K * 2 and lib.fqvit_linear_workspace_size(0, K) == 0
+    f = lambda *a: lib.fqvit_linear_q(*a)  # noqa: E731
+    ok = [fake, M, K, K, 128, 0.04, fake, N, fake, None, 0.03, 120, fake, N, None, 0, fake, ws, None]
+    assert f(*[None] + ok[1:]) == 1                                     # NULL x
+    bad = list(ok); bad[8] = None
+    assert f(*bad) == 1                                                 # NULL s_w
+    bad = list(ok); bad[2] = 100; bad[3] = 100
+    assert f(*bad) == 2 and "K=100" in _err(lib)                        # K not a multiple of 8
+    bad = list(ok); bad[7] = 1160; bad[13] = 1168
+    assert f(*bad) == 2                                                 # N not a multiple of 16
+    bad = list(ok); bad[7] = 4112; bad[13] = 4112
+    assert f(*bad) == 2                                                 # N > 4096
+    bad = list(ok); bad[2] = 16392; bad[3] = 16392
+    assert f(*bad) == 2                                                 # K > 16384
+    bad = list(ok); bad[4] = 256
+    assert f(*bad) == 1 and "zero points" in _err(lib)                  # zp_x outside 0..255
+    bad = list(ok); bad[10] = float("inf")
+    assert f(*bad) == 1                                                 # s_y not finite
+    bad = list(ok); bad[13] = N + 8
+    assert f(*bad) == 1                                                 # ld_y not a multiple of 16
+    bad = list(ok); bad[3] = K + 4
+    assert f(*bad) == 1                                                 # ld_x not a multiple of 8
+    bad = list(ok); bad[14] = fake; bad[15] = N - 4
+    assert f(*bad) == 1                                                 # ld_acc below N
+    bad = list(ok); bad[17] = ws - 1
+    assert f(*bad) == 1 and "workspace" in _err(lib)                    # small workspace
+    p = lambda *a: lib.fqvit_linear_pack_weight(*a)  # noqa: E731
+    assert p(None, N, K, K, fake, None) == 1
+    assert p(fake, N, 100, 100, fake, None) == 2
+    assert p(fake, N, K, K, ctypes.c_void_p(4104), None) == 1           # w_h not 16-byte aligned
