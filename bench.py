@@ -740,8 +740,9 @@ def main():
                     help="attention from int8 Q, K, V (fqvit_qk_lis_attention) instead of int8 logits")
     ap.add_argument("--out8", action="store_true",
                     help="the attention output requantized to 8 bits (fqvit_lis_attention_q) instead of int32")
-    ap.add_argument("--linear", action="store_true",
-                    help="also time the block's MinMax Linear layers (fqvit_linear_q) alone, outside the step")
+    ap.add_argument("--no-linear", dest="linear", action="store_false",
+                    help="skip the separate timing of the block's MinMax Linear layers (fqvit_linear_q), "
+                         "which runs after the timed step and is reported under kernels.linear")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
