@@ -507,7 +507,12 @@ def bench_gpu(args):
                            "to HBM), 10 launches after 3, outside the timed step"}
         del full
 
-    lin_stats = bench_linear(fqvit, cfg, dev) if args.linear else None
+    lin_stats = None
+    if args.linear:  # outside the timed step; a failure here is reported, not fatal to the line
+        try:
+            lin_stats = bench_linear(fqvit, cfg, dev)
+        except Exception as e:  # noqa: BLE001
+            lin_stats = {"error": f"{type(e).__name__}: {e}"[:300]}
 
     e2e = None
     if not args.no_e2e:
