@@ -114,3 +114,28 @@ def test_qk_inputs_are_codes_and_scales(name):
     assert a["q"].dtype == torch.int8 and a["k"].dtype == torch.int8 and a["q"].shape == (2, a["L"], a["d"])
     assert int(a["q"].abs().max()) <= 127 and a["s_q"] > 0 and a["s_k"] > 0
     assert -128 <= a["zp_logit"] <= 127
+
+
+@pytest.mark.parametrize("name,kind", [("deit_t", "qkv"), ("deit_t", "fc2"), ("swin_s", "fc1"), ("vit_b", "proj")])
+def test_linear_inputs_structure(name, kind):
+    """The Linear generator: shapes of the block's layers, symmetric per-channel weight codes,
+    asymmetric activation codes, an int32 bias and a MinMax output quantizer."""
+    cfg = synth.CONFIGS[name]
+    a = synth.linear_inputs(cfg, 0, kind, rows=300)
+    C = synth.layer_stage(cfg, 0).C
+    N, K = {"qkv": (3 * C, C), "proj": (C, C), "fc1": (4 * C, C), "fc2": (C, 4 * C)}[kind]
+    assert (a["M"], a["N"], a["K"]) == (300, N, K)
+    assert a["x"].dtype == torch.uint8 and a["x"].shape == (300, K)
+    assert a["w"].dtype == torch.int8 and a["w"].shape == (N, K) and int(a["w"].abs().max()) <= 127
+    # every channel reaches its own maximum code (symmetric MinMax per channel)
+    assert torch.all(a["w"].abs().amax(dim=1) == 127)
+    assert a["s_w"].dtype == torch.float32 and bool(torch.all(a["s_w"] > 0))
+    assert a["bias"].dtype == torch.int32 and a["bias"].shape == (N,)
+    assert 0 <= a["zp_x"] <= 255 and 0 <= a["zp_y"] <= 255 and a["s_x"] > 0 and a["s_y"] > 0
+    # GELU's input to fc2 sits above -0.17: its zero point is near the bottom of the range
+    if kind == "fc2":
+        assert a["zp_x"] < 32
+    else:
+        assert 96 < a["zp_x"] < 160
+    # the activation codes span the range (MinMax of the draw)
+    assert int(a["x"].min()) == 0 and int(a["x"].max()) == 255
