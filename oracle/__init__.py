@@ -38,7 +38,13 @@ def _load():
     if _lib is not None:
         return _lib
     build()
-    lib = ctypes.CDLL(str(_LIB))
+    _lib = _declare(ctypes.CDLL(str(_LIB)))
+    return _lib
+
+
+def _declare(lib):
+    """Declare the C signatures on a loaded copy of the oracle (also used by the tests' planted
+    mistakes, which compile altered copies of the source)."""
     P = ctypes.c_void_p
     i64, i32, f32 = ctypes.c_int64, ctypes.c_int32, ctypes.c_float
     lib.or_calibrate_ptf.argtypes = [P, i64, i32, i64, i32, P, P, P, P]
@@ -75,7 +81,6 @@ def _load():
     lib.or_num_threads.restype = ctypes.c_int
     lib.or_set_num_threads.argtypes = [ctypes.c_int]
     lib.or_set_num_threads.restype = None
-    _lib = lib
     return lib
 
 

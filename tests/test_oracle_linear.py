@@ -5,8 +5,10 @@ quantizer applied with the dyadic multiplier of the supplement's LayerNorm outpu
 Each pin checks or_linear_q against something other than itself:
 - closed forms of the integer product: permutation weights (N != K, so a transposed weight
   matrix or a swapped index fails), all-ones weights, and an input equal to its zero point;
-- exact multipliers (M_n = 1, 2^-3, 2^-30 at the N1 cap, 300 and 4096 for N1 <= 0), where the
-  dyadic requantization reduces to a rounded shift or a product;
+- exact multipliers (M_n = 1, 2^-3, 2^-30 and 3 2^-32 at the N1 cap, 300 and 4096 for
+  N1 <= 0, 1 + 2^-8 and 255 2^-10 for the 8-bit truncation of M_n), where the dyadic
+  requantization reduces to a rounded shift or a product;
+- the one-sided bounds of a truncated multiplier for scales of many significant bits;
 - the real-valued layer in fp64, within the 8-bit multiplier's error bound;
 - the int32 overflow report and the argument checks.
 """
@@ -164,3 +166,54 @@ def test_overflow_and_argument_checks():
         oracle.linear_q(x, 0, 0.0, w, np.ones(3, np.float32), None, 1.0, 0)
     with pytest.raises(ValueError):  # M_n >= 1e30
         oracle.linear_q(x, 0, 1e20, w, np.full(3, 1e20, np.float32), None, 1.0, 0)
+
+
+def test_eight_bit_truncation_of_the_multiplier():
+    """The reading keeps 8 significant bits of M_n.  M = 1 + 2^-8: N1 = 7, N2 = floor(128.5) = 128,
+    so the multiplier is exactly 1 and y = acc for acc in 0 .. 254 (where M itself would round
+    acc >= 128 up by one).  M = 255 2^-10 (8 bits): N1 = 10, N2 = 255,
+    y = floor(255 acc / 1024 + 1/2) + zp_y."""
+    vals = list(range(0, 128))
+    x, w = _one_hot(len(vals), 128, vals)
+    w[0, 0] = 2  # acc = 2 v, 0 .. 254
+    y, _ = oracle.linear_q(x, 128, 1.0, w, np.array([1.0 + 2.0 ** -8], np.float32), None, 1.0, 0)
+    assert y[:, 0].tolist() == [2 * v for v in vals]
+    vals = list(range(-128, 128))
+    x, w = _one_hot(len(vals), 128, vals)
+    w[0, 0] = 127  # acc = 127 v, up to 16129 in magnitude
+    acc_v = [127 * v for v in vals]
+    y, _ = oracle.linear_q(x, 128, 1.0, w, np.array([255 * 2.0 ** -10], np.float32), None, 1.0, 128)
+    assert y[:, 0].tolist() == [min(255, max(0, (255 * a + 512) // 1024 + 128)) for a in acc_v]
+
+
+def test_shift_cap_truncates_the_multiplier():
+    """M = 3 2^-32: N1 = 38 is capped at 31, N2 = floor(1.5) = 1: y = floor((acc + 2^30) / 2^31) + zp_y."""
+    x = np.full((1, 3), 9, np.uint8)  # x = zp_x: acc is the bias alone
+    w = np.ones((1, 3), np.int8)
+    for b, want in ((3 * 2 ** 29, 1), (2 ** 30 - 1, 0), (-(2 ** 30), 0), (-(2 ** 30) - 1, -1)):
+        y, acc = oracle.linear_q(x, 9, 2.0 ** -15, w, np.array([3 * 2.0 ** -17], np.float32),
+                                 np.array([b], np.int32), 1.0, 20)
+        assert int(acc[0, 0]) == b and int(y[0, 0]) == 20 + want, b
+
+
+def test_multiplier_truncates():
+    """N2 / 2^N1 lies in (M (1 - 2^-7), M]: for acc >= 0 and scales of many significant bits,
+    floor(M acc (1 - 2^-7) + 1/2) <= y - zp_y <= floor(M acc + 1/2), with M the fp32 value of
+    (s_x s_w[n]) / s_y in exact rational arithmetic."""
+    from fractions import Fraction
+    import math
+    rng = _rng(7)
+    M_, K, N = 40, 16, 24
+    x = rng.integers(100, 256, size=(M_, K)).astype(np.uint8)      # x - zp_x >= 0
+    w = rng.integers(0, 128, size=(N, K)).astype(np.int8)           # w >= 0
+    s_x, s_y = np.float32(0.0173), np.float32(0.91)
+    s_w = (rng.uniform(0.5, 2.0, size=N) * 2.9e-3).astype(np.float32)
+    y, acc = oracle.linear_q(x, 100, float(s_x), w, s_w, None, float(s_y), 0)
+    assert acc.min() >= 0
+    for n in range(N):
+        Mn = Fraction(float(np.float32(np.float32(s_x * s_w[n]) / s_y)))
+        for m in range(M_):
+            a = int(acc[m, n])
+            hi = math.floor(Mn * a + Fraction(1, 2))
+            lo = math.floor(Mn * a * (1 - Fraction(1, 128)) + Fraction(1, 2))
+            assert hi <= 255 and lo <= int(y[m, n]) <= hi, (m, n)

@@ -7,7 +7,7 @@ dyadic multiplier of the LayerNorm output stage).
   dropped term shows up, the products are not symmetric).
 * Where M has at most 8 significant bits (including N1 <= 0 and the N1 = 31
   cap) the result is the exactly rounded product floor(P M + 1/2), computed
-  with rational arithmetic.
+  with rational arithmetic; M = 1 + 2^-8 keeps 8 bits (the multiplier is 1).
 * For any scales it stays within the truncation bound of an 8-bit multiplier
   of the exact real logit, and it is monotone in P.
 * Log-Int-Softmax only sees differences: moving the zero point leaves the
@@ -78,6 +78,21 @@ def test_exact_rounding_for_multipliers_of_eight_bits(kk, e):
         assert np.array_equal(got.astype(np.int64), _exact(P, M, zp_l)), (kk, e, zp_l)
 
 
+def test_multiplier_keeps_eight_bits():
+    """M = 1 + 2^-8 (nine significant bits): N1 = 7 and N2 = floor(128.5) = 128, so the
+    multiplier is exactly 1 and every unclipped logit is P + zp_l; most P here are at least 128,
+    where M itself would round P up by one."""
+    rng = np.random.default_rng(21)
+    q = rng.integers(1, 3, size=(2, 17, 64)).astype(np.int8)
+    k = rng.integers(1, 3, size=(2, 17, 64)).astype(np.int8)
+    s_q = (1 + 2.0 ** -8) * 2.0 ** -3
+    assert np.float32(np.float32(s_q) * np.float32(2.0 ** -4)) / np.float32(2.0 ** -7) == 1 + 2.0 ** -8
+    got = oracle.qk_logits(q, k, 0, 0, s_q, 2.0 ** -4, 2.0 ** -10, -100)
+    P = _product(q, k, 0, 0).reshape(-1, 17)
+    assert P.min() >= 100 and (P >= 128).mean() > 0.5
+    assert np.array_equal(got.astype(np.int64), np.clip(P - 100, -128, 127))
+
+
 @pytest.mark.parametrize("d,s_q,s_k,s_logit", [(64, 0.031, 0.027, 0.0441), (32, 0.5, 0.011, 0.37),
                                                (64, 0.0123, 0.0456, 0.0031), (16, 1.7, 0.9, 13.0)])
 def test_within_the_bound_of_an_eight_bit_multiplier(d, s_q, s_k, s_logit):
@@ -98,7 +113,7 @@ def test_softmax_codes_ignore_the_zero_point():
     q, k = _qk(5, 2, 49, 32, lo=-40, hi=40)
     a = oracle.qk_logits(q, k, 0, 0, 0.05, 0.05, 0.06, -20, ld=64)
     b = oracle.qk_logits(q, k, 0, 0, 0.05, 0.05, 0.06, 7, ld=64)
-    assert a[:, :49].max() + 27 <= 127 and a[:, :49].min() >= -128  # no clipping either way
+    assert int(a[:, :49].max()) + 27 <= 127 and int(a[:, :49].min()) >= -128  # no clipping either way
     assert np.array_equal(b[:, :49].astype(np.int64), a[:, :49].astype(np.int64) + 27)
     ca, _ = oracle.lis_softmax(a, 49, 0.06)
     cb, _ = oracle.lis_softmax(b, 49, 0.06)
