@@ -295,6 +295,23 @@ def test_ptf_factor_follows_channel_range():
     assert np.array_equal(alpha, np.argmin(sse, axis=1))
 
 
+def test_ptf_ties_take_the_smallest_factor():
+    # a channel of zeros and a channel on the coarsest grid (values -s0, 0, s0 with s0 = 2^K s)
+    # quantize without error for every factor: Eq. 10's minimum is attained by every alpha, and
+    # the reading breaks the tie toward the smallest
+    rng = np.random.default_rng(9)
+    K, rows = 3, 500
+    x = rng.uniform(-5.0, 5.0, (rows, 3)).astype(np.float32)
+    x[0, 0], x[1, 0] = -5.0, 5.0
+    s0 = np.float32(np.float32(10.0) / np.float32(255.0))
+    x[:, 1] = 0.0
+    x[:, 2] = rng.integers(-1, 2, rows).astype(np.float32) * s0
+    s, zp, alpha, sse = oracle.calibrate_ptf(x, K=K)
+    assert np.float32(s) * np.float32(2 ** K) == s0
+    assert np.all(sse[1] == 0.0) and np.all(sse[2] == 0.0)
+    assert alpha[1] == 0 and alpha[2] == 0
+
+
 def test_ptf_sse_definition():
     x = _channels(4, rows=200, C=8)
     K = 3
@@ -358,6 +375,26 @@ def test_ln_gamma_zero_and_constant_row():
     beta_q = np.clip(np.rint((beta.astype(np.float64) / s_out).astype(np.float32)) + zp_out, 0, 255)
     assert np.all(y[:, 5] == beta_q[5])
     assert np.array_equal(y[3], beta_q.astype(np.uint8))
+
+
+def test_ln_exact_row_by_hand():
+    # A row whose statistics are exact: x - zp_in = +-64 on 8 channels (alpha = 0), so M1 = 0,
+    # D = 8 * 8 * 64^2 = 2^18, sqrt(D) = 512, C / sqrt(D) = 2^-6, and the mean term vanishes.
+    # With s_out = 2^-6, gamma = +-129.5 2^-6 and beta = 0: A = +-2.0234375 (nine significant
+    # bits), and the supplement's output stage gives N1 = 7 - floor(log2 |A|) = 6 and
+    # N2 = floor(129.5) = 129 (eight bits), Y = floor((sign(A) 129 X + 32) / 64) + zp_out:
+    # the quotient is +-129.5 or +-128.5 and rounds to +-129, the sign that of A X, so
+    # Y = clip(+-129 + zp_out).
+    C = 8
+    xq = np.array([[192, 64] * 4], np.uint8)
+    alpha = np.zeros(C, np.uint8)
+    beta = np.zeros(C, np.float32)
+    s_out = 2.0 ** -6
+    for sign, zp_out, want in ((1, 0, [129, 0]), (1, 126, [255, 0]), (-1, 200, [71, 255]), (-1, 129, [0, 255])):
+        gamma = np.full(C, sign * 129.5 * 2.0 ** -6, np.float32)
+        y, m1, m2 = oracle.ptf_layernorm(xq, 128, alpha, gamma, beta, s_out, zp_out)
+        assert int(m1[0]) == 0 and int(m2[0]) == 8 * 64 * 64
+        assert y[0].tolist() == want * 4, (sign, zp_out)
 
 
 def test_ln_shift_by_factor_equals_minmax_path():

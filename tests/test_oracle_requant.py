@@ -51,6 +51,17 @@ def test_exact_for_multipliers_of_eight_bits(k, e):
         assert np.array_equal(got.astype(np.int64), _exact(acc, M, zp)), (k, e, zp)
 
 
+def test_multiplier_keeps_eight_bits():
+    # M = 1 + 2^-8 (nine significant bits): N1 = 7, N2 = floor(128.5) = 128, so the multiplier is
+    # exactly 1 and y = acc + zp_out for acc in 0 .. 254, where M itself would round acc >= 128 up
+    s_out = 2.0 ** -10
+    s_v = (1 + 2.0 ** -8) * 32.0
+    assert float(np.float32(np.float32(s_v) / np.float32(s_out))) * 2.0 ** -15 == 1 + 2.0 ** -8
+    acc = np.arange(0, 255, dtype=np.int32).reshape(-1, 5)
+    got = oracle.attn_requant(acc, s_v, s_out, 0)
+    assert np.array_equal(got.astype(np.int64), acc.astype(np.int64))
+
+
 def test_cap_of_the_shift_for_tiny_multipliers():
     # M = 2^-30: N1 = 37 capped at 31, N2 = 2: still the exactly rounded product
     s_out = 1.0
