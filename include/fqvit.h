@@ -58,6 +58,14 @@ FQVIT_API const char *fqvit_last_error(void);
  * cleared.  Not part of the paper; a diagnostic of this implementation. */
 FQVIT_API int fqvit_sync_status(void *stream);
 
+/* Exercises the failure path of the bounded waits without a fault: launches
+ * one CTA on `stream` whose thread waits, through the same bounded wait the
+ * kernels use, on an mbarrier that nothing completes.  The wait gives up
+ * after two seconds and records the timeout; the next fqvit_sync_status
+ * returns FQVIT_ERR_TIMEOUT and the context stays usable.  Returns
+ * FQVIT_ERR_CUDA if the launch fails.  Not part of the paper. */
+FQVIT_API int fqvit_selftest_bounded_wait(void *stream);
+
 /* ------------------------------------------------------------------ */
 /* Power-of-Two Factor calibration (Sec. 3.2, Eqs. 8-10)              */
 /* ------------------------------------------------------------------ */

@@ -76,6 +76,10 @@ int fqvit_sync_status(void *stream)
     int status = 0;
     cudaError_t e = fqvit::read_clear_device_status(&status, as_stream(stream));
     if (e != cudaSuccess) return fail(FQVIT_ERR_CUDA, "sync_status: %s", cudaGetErrorString(e));
+    int lst = 0;  // the Linear layers' status word (linear_tc.cu)
+    e = fqvit::read_clear_linear_status(&lst);
+    if (e != cudaSuccess) return fail(FQVIT_ERR_CUDA, "sync_status: %s", cudaGetErrorString(e));
+    if (status == 0 || (status == FQVIT_ERR_INVALID_ARG && lst == FQVIT_ERR_TIMEOUT)) status = lst;
     if (status == FQVIT_ERR_TIMEOUT)
         return fail(FQVIT_ERR_TIMEOUT, "a kernel abandoned a bounded wait (results of that launch are invalid)");
     if (status == FQVIT_ERR_INVALID_ARG)
@@ -525,6 +529,11 @@ int fqvit_qk_lis_attention(const int8_t *q, int64_t ld_q, int32_t zp_q, const in
         if (e != cudaSuccess) return cuda_status(e, who);
     }
     return ok();
+}
+
+int fqvit_selftest_bounded_wait(void *stream)
+{
+    return cuda_status(fqvit::launch_bounded_wait_probe(as_stream(stream)), "selftest_bounded_wait");
 }
 
 // ---- MinMax Linear layers -------------------------------------------------

@@ -197,9 +197,12 @@ bool linear_supported(const LinearArgs &a);
 cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st);
 cudaError_t launch_linear_pack_weight(const int8_t *w, int N, int K, int64_t ld_w, uint16_t *w_h, cudaStream_t st);
 cudaError_t read_clear_linear_status(int *status);
+// one CTA whose wait on an mbarrier that nothing completes gives up (the bounded wait's timeout)
+cudaError_t launch_bounded_wait_probe(cudaStream_t st);
 
-// Synchronizes st, returns the device status word (0 ok, 1 a device-side argument was
-// invalid, 5 a bounded wait timed out) and clears it.
+// Synchronizes st, returns the device status word of the attention and LayerNorm kernels
+// (0 ok, 5 a bounded wait timed out) and clears it; the Linear layers' word is read by
+// read_clear_linear_status.
 cudaError_t read_clear_device_status(int *status, cudaStream_t st);
 
 // Attention implementation choice: 0 automatic, 1 CUDA cores only (FQVIT_ATTN_PATH=cuda_core),

@@ -383,7 +383,28 @@ cudaError_t launch_bytes_to_half(const uint8_t *src, int64_t rows, int K, int64_
                       dst);
 }
 
+// The bounded wait on a barrier that nothing completes: one thread of one CTA waits on phase 0
+// of a fresh mbarrier of count 1, with the same two-second wait the kernels use; it gives up,
+// records the timeout status and returns (the failure path, without a fault).
+__global__ void bounded_wait_probe_kernel()
+{
+    __shared__ uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        abort_flag = 0;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) (void)mbar_wait(&bar, 0, &abort_flag);
+}
+
 }  // namespace
+
+cudaError_t launch_bounded_wait_probe(cudaStream_t st)
+{
+    bounded_wait_probe_kernel<<<1, 32, 0, st>>>();
+    return cudaGetLastError();
+}
 
 bool linear_supported(const LinearArgs &a) { return a.N <= LMAXN && linear_smem_bytes(a.N) + sizeof(LinShared) + 64 <= 232448; }
 

@@ -628,11 +628,7 @@ cudaError_t read_clear_device_status(int *status, cudaStream_t st)
     if (*status == 0) *status = qst;
     int pst = 0;
     e = read_clear_tcp_status(&pst);
-    if (e != cudaSuccess) return e;
     if (*status == 0) *status = pst;
-    int lst = 0;
-    e = read_clear_linear_status(&lst);
-    if (*status == 0) *status = lst;
     return e;
 }
 

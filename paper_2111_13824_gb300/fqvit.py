@@ -52,6 +52,7 @@ EXPORTS = (
     "fqvit_lis_softmax_masked", "fqvit_lis_attention_masked", "fqvit_lis_attention_masked_q",
     "fqvit_qk_logits", "fqvit_qk_workspace_size", "fqvit_qk_lis_attention",
     "fqvit_linear_pack_weight", "fqvit_linear_workspace_size", "fqvit_linear_q",
+    "fqvit_selftest_bounded_wait",
 )
 
 
@@ -91,6 +92,7 @@ def load(path: str | Path | None = None):
         "fqvit_qk_workspace_size": ([i64, i32, i64], sz),
         "fqvit_qk_lis_attention": ([P, i64, i32, P, i64, i32, f32, f32, f32, i32, i32, P, P, P, i64, i32, i64, i32,
                                     i32, P, i64, P, sz, i64, P], ctypes.c_int),
+        "fqvit_selftest_bounded_wait": ([P], ctypes.c_int),
         "fqvit_linear_pack_weight": ([P, i32, i32, i64, P, P], ctypes.c_int),
         "fqvit_linear_workspace_size": ([i64, i32], sz),
         "fqvit_linear_q": ([P, i64, i32, i64, i32, f32, P, i32, P, P, f32, i32, P, i64, P, i64, P, sz, P],
@@ -145,6 +147,12 @@ def _bias(bias, heads, window):
 def sync_status(stream=None) -> None:
     """Synchronize the stream; raise FqvitError if a kernel abandoned a bounded wait."""
     _check(load().fqvit_sync_status(_stream(stream)))
+
+
+def selftest_bounded_wait(stream=None) -> None:
+    """One CTA waits on a barrier nothing completes (fqvit_selftest_bounded_wait); the next
+    sync_status raises FqvitError with ERR_TIMEOUT."""
+    _check(load().fqvit_selftest_bounded_wait(_stream(stream)))
 
 
 def version() -> int:
