@@ -37,6 +37,12 @@ MUTANTS = [
     (PINS, "or_calibrate_sse", "err += (double)d * (double)d;", "err += fabs((double)d);", "absolute, not squared error"),
     (PINS, "or_calibrate_ptf", "if (e[a] < e[best_a]) best_a = a;", "if (e[a] <= e[best_a]) best_a = a;",
      "ties to the largest factor"),
+    (PINS, "or_calibrate_minmax", "float mn = x[0], mx = x[0];", "float mn = 0.0f, mx = x[0];",
+     "minimum started at zero"),
+    (PINS, "or_calibrate_minmax", "for (int64_t r = 0; r < rows; ++r)", "for (int64_t r = 1; r < rows; ++r)",
+     "first row skipped"),
+    (PINS, "or_ptf_quantize", "float q = rintf(x[r * ld_x + c] / sa);", "float q = truncf(x[r * ld_x + c] / sa);",
+     "codes truncated, not rounded"),
     (PINS, "or_ptf_quantize", "float sa = ldexpf(s, alpha[c]);", "float sa = s;", "factor ignored"),
     (PINS, "or_ptf_quantize", "xq[r * ld_q + c] = (uint8_t)((int32_t)q + zp);", "xq[r * ld_q + c] = (uint8_t)((int32_t)q);",
      "zero point dropped"),
@@ -55,6 +61,8 @@ MUTANTS = [
      "int64_t xh = ((int64_t)xr[c] - zp_in);\n            float gs", "PTF shift missing in the output"),
     (PINS, "or_ptf_layernorm", "clamp_i64(R + zp_out, 0, 255)", "clamp_i64(R - zp_out, 0, 255)",
      "output zero point subtracted"),
+    (PINS, "or_ptf_layernorm", "float bqf = clamp_f32(rintf(bsc),", "float bqf = clamp_f32(floorf(bsc),",
+     "B 2^N1 floored, not rounded"),
     # i-exp (Algorithm 1) and I-Log2 (Algorithm 2)
     (PINS, "or_iexp_consts", "*q_ln2 = (int64_t)floor(-OR_LN2 / sd);", "*q_ln2 = (int64_t)ceil(-OR_LN2 / sd);",
      "q_ln2 rounded up"),
@@ -74,6 +82,7 @@ MUTANTS = [
     (LIS_PINS, "or_lis_softmax_masked", "uint64_t qrev = (2 * S + ev[j]) / (2 * ev[j]);",
      "uint64_t qrev = S / ev[j];", "reciprocal truncated, not rounded"),
     (LIS_PINS, "or_lis_softmax_masked", "if (code > 15) code = 15;", "if (code > 14) code = 14;", "clip at 14"),
+    (LIS_PINS, "or_lis_softmax_masked", "S += ev[j];", "if (j + 1 < L) S += ev[j];", "last key left out of the sum"),
     (LIS_PINS, "or_lis_softmax_masked", "ev[j] = or_iexp((int64_t)qv[j] - m, n, q_ln2, q_b, q_c);",
      "ev[j] = or_iexp((int64_t)qv[j] - m - 1, n, q_ln2, q_b, q_c);", "maximum off by one"),
     (LIS_PINS, "or_lis_softmax_masked", "relpos_index(i, j, window)", "relpos_index(j, i, window)",
@@ -89,6 +98,8 @@ MUTANTS = [
      "shift by the code, not 15 - code"),
     (PINS, "or_lis_attn_v", "a[t] += ((int64_t)vh[(int64_t)j * ld_v + t] - zp_v) * w;",
      "a[t] += ((int64_t)vh[(int64_t)t * 0 + j] - zp_v) * w;", "V read along the wrong axis"),
+    (PINS, "or_lis_attn_v", "a[t] += ((int64_t)vh[(int64_t)j * ld_v + t] - zp_v) * w;",
+     "a[t] += ((int64_t)vh[(int64_t)j * ld_v + t]) * w;", "V zero point dropped"),
     # 8-bit attention output (Eq. 3 with the dyadic multiplier)
     ("test_oracle_requant", "or_attn_requant", "const float M = ldexpf(s_v / s_out, -15);",
      "const float M = ldexpf(s_v / s_out, -14);", "2^15 of the BitShift scale off by one"),

@@ -258,6 +258,22 @@ def _channels(seed, rows=300, C=40):
     return (m + r / 6 * rng.normal(0, 1, (rows, C))).astype(np.float32)
 
 
+def test_minmax_range_is_the_data_range():
+    # Eqs. 4-5 over all calibration elements, the range not widened to include 0: all-positive
+    # data keeps its own minimum, and extremes anywhere (the first row away from its first
+    # element, the last row) are found; K = 0 then gives s = (7 - 3) / 255 and zp = clip(-191) = 0
+    rng = np.random.default_rng(12)
+    x = rng.uniform(3.5, 6.5, (50, 7)).astype(np.float32)
+    x[0, 5] = 7.0
+    x[49, 6] = 3.0
+    assert oracle.calibrate_minmax(x) == (3.0, 7.0)
+    x2 = x.copy()
+    x2[0, 3] = 2.5
+    assert oracle.calibrate_minmax(x2) == (2.5, 7.0)
+    s, zp, _, _ = oracle.calibrate_ptf(x, K=0)
+    assert np.float32(s) == np.float32(np.float32(4.0) / np.float32(255.0)) and zp == 0
+
+
 def test_ptf_k0_is_minmax():
     x = _channels(1)
     s, zp, alpha, sse = oracle.calibrate_ptf(x, K=0)
