@@ -160,12 +160,8 @@ bool qk_logits_supported(const QkArgs &a);
 cudaError_t launch_qk_logits(const QkArgs &a, cudaStream_t st);
 cudaError_t read_clear_qk_status(int *status);
 
-// the same with tiles packed across heads, for 128 <= L <= 384 (lis_tc_pack.cu)
-bool lis_attention_tc_packed(int L);
-cudaError_t launch_lis_attention_tc_packed(const LisArgs &a, const AttnVArgs &b, cudaStream_t st);
-cudaError_t read_clear_tcp_status(int *status);
-
-// tensor-core (tcgen05) fused path (lis_tc.cu)
+// tensor-core (tcgen05) fused path for rows of 65 .. 640 keys (lis_tc.cu); rows of 128 .. 384 keys
+// take tiles packed across heads
 bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b);
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st);
 

@@ -1,5 +1,6 @@
 // lis_tc.cu -- fused Log-Int-Softmax + BitShift attention times values on
-// the 5th-generation tensor cores (tcgen05) of sm_103a.
+// the 5th-generation tensor cores (tcgen05) of sm_103a, for rows of 65 .. 640
+// keys (head dimension 64).
 //
 // Eq. 15 is a matrix product: acc = P (V - zp_V) with P[i][j] = 2^(15 - code_ij),
 // computed as P V - zp_V (P 1).  Every P entry and every int8 value of V is exact
@@ -8,26 +9,54 @@
 // partial sum of P V is an integer below 2^24, and the row sums P 1 (a second,
 // N = 16 product against a block of ones, only when zp_V != 0) stay below 2^17:
 // fp16 operands with fp32 accumulation give the integers exactly, and
-// zp_V (P 1) is subtracted in int32.  The kernel evaluates the products as
+// zp_V (P 1) is subtracted in int32.  The products run as
 // tcgen05.mma.kind::f16 (M = 128 query rows, N = 64 = d, K = 16 keys per
-// instruction) with the accumulators in tensor memory.
+// instruction) with the operand P and the accumulators in tensor memory.
 //
-// One CTA per SM walks (head, 128-row tile) work items.  Roles:
-//   warps 0-15 (four threads per query row; warp w serves rows 32 (w % 4) ..
-//     and the keys 16 (w / 4) .. +15 of every block of 64 keys): the tile's
-//     logits go from shared memory into registers, the row maximum and the
-//     i-exp row sum are combined over the four threads of a row through
-//     shared memory, the row's 256 possible operands are tabulated, and every
-//     4-bit code is written, as the fp16 operand 2^(15-code) looked up in that
-//     table, straight into tensor memory (the A operand: row = lane, K-major
-//     pairs per column).  The same threads convert a head's V rows to fp16
-//     (128B-swizzled, MN-major shared-memory tile, the B operand).
-//   warps 16-19 (one per tensor-memory lane quarter): read each tile's
-//     accumulators out of tensor memory as soon as its MMAs complete and store
-//     the int32 rows (32-byte stores) while the softmax warps work on the next
-//     tile; warp 16, lane 0 also issues the tile's MMAs (four per key block)
-//     once every operand is written, warp 17, lane 0 the bulk copy of the next
-//     tile's logits into shared memory, plus L2 prefetches.
+// One CTA per SM walks a contiguous range of 128-row tiles.  Without PACK a
+// tile holds rows of one head (the last tile of a head is partly empty); with
+// PACK (128 <= L <= 384) tile t holds rows 128 t .. 128 t + 127 of all BH L
+// rows, so it may hold the end of one head and the start of the next: those
+// run two sets of MMAs, one per head, against two V buffers into two
+// accumulators.
+//
+// Roles:
+//   warps 0-15, the softmax threads, four per query row (thread (r, q): warp
+//     4 q + r / 32, lane r % 32, so that lanes are rows are tensor-memory
+//     lanes; part q takes keys 64 kb + 16 q .. +15 of every 64-key block kb).
+//     Per tile: the row's logits from the bulk-copied tile into registers, the
+//     row maximum, then every logit byte becomes its distance d = m - q to the
+//     maximum (four at once: a borrow-free 32-bit subtraction of the biased
+//     bytes from the replicated maximum), the i-exp row sum from a table
+//     indexed by d, the row's 15 code thresholds, the row's operand table (the
+//     fp16 operand 2^(15 - code) of every d), and the operands of the row's
+//     keys, looked up by d, straight into tensor memory.
+//   warps 16-19, one per tensor-memory lane quarter: the accumulators of the
+//     previous tile out of tensor memory into global memory, V of a new head
+//     into the fp16 B operand in shared memory, the tile's MMAs (warp 16, lane
+//     0) and the bulk copy of the next tile's logits (warp 17, lane 0).
+//
+// The combined table (64 KB at the start of dynamic shared memory): line d
+// (d = 0 .. 255) is 256 bytes.  Bytes 0 .. 127 hold the high byte 4 (30 - code)
+// of the operand of distance d for the 128 rows of the tile, row r at byte
+// 4 (r % 32) + r / 32, so that the 32 rows of a warp read 32 different banks;
+// bytes 128 .. 255 hold 32 copies of the i-exp value e(d), copy c at byte
+// 128 + 4 c (lane c reads its own copy: no bank conflicts for random d).  One
+// byte permute turns a distance byte and a per-thread byte into an address
+// (d << 8 | offset), so a table lookup costs one permute and one load.
+//
+// The operand table from thresholds: code(d) = #{k <= 15 : d >= delta_k} with
+// delta_k the first d at which e(d) D_k <= 2S (D_1 = 3, D_k = 3 2^(k-1) - 1,
+// an exact FMA test against 2S = hi + lo), where the i-exp values never rise
+// with d.  The four parts of a row find its thresholds by binary search and
+// add one, in byte r / 32 of the table word (line delta_k, lane r % 32), with a
+// shared-memory atomic; then thread (lane l, warp g) turns lines 16 g .. 16 g +
+// 15 of column l into codes by a running sum (four rows per word, counts
+// below 16 per byte: no carries), the carry-in from the lines below taken from
+// per-group totals counted at the same time.  The floored constants of a few
+// scales make e(d) rise at band edges; those scales evaluate every entry
+// directly with the code test.
+//
 // Every wait is bounded: after two seconds the kernel records a timeout
 // status, drains what it issued and returns (the host reads the status with
 // fqvit_sync_status).
@@ -45,71 +74,138 @@ namespace {
 using namespace lis;
 using namespace tc;
 
-constexpr int TM = 128;        // query rows per tile (MMA M)
-constexpr int TKB = 64;        // keys per key block
-constexpr int TD = 64;         // head dimension (MMA N)
-constexpr int TCOPIES = 32;    // replicas of the i-exp table (one per lane)
-constexpr int B_SLOT = TKB * TD * 2;
+constexpr int TM = 128;                    // query rows per tile (MMA M)
+constexpr int TKB = 64;                    // keys per key block
+constexpr int TD = 64;                     // head dimension (MMA N)
+constexpr int KSTEP_B = 16 * TD * 2;       // bytes of B per 16 keys (one MMA K step)
+constexpr int TPARTS = 4;                  // threads per query row
+constexpr int TSOFT = TM * TPARTS;         // softmax threads (16 warps)
+constexpr int TEPI_WARP = TSOFT / 32;      // warps 16..19: read-out, one per lane quarter
+constexpr int TMMA_WARP = TEPI_WARP;       //   warp 16 lane 0 also issues the MMAs
+constexpr int TCOPY_WARP = TEPI_WARP + 1;  //   warp 17 lane 0 also copies the logits tiles
+constexpr int TTHREADS = TSOFT + 128;
+constexpr int TMAXKB = 10;                 // key blocks of the longest row (L <= 640)
+constexpr int kPackMaxBlocks = 6;          // PACK for 128 <= L <= 384
+
+// dynamic shared memory
+constexpr uint32_t TAB_OFF = 0;                       // 256 lines x 256 B
+constexpr uint32_t LUT_BYTE = 128;                    // i-exp copies in a line
+constexpr uint32_t RMAX_OFF = 65536;                  // int [4][128]: row maxima of the parts
+constexpr uint32_t RSUM_OFF = RMAX_OFF + 2048;        // u64 [4][128]: row sums of the parts
+constexpr uint32_t GT_OFF = RSUM_OFF + 4096;          // u32 [32][20]: thresholds per (lane, 16-line group)
+constexpr int GT_LD = 20;                             //   (row stride 20 words: 16-byte loads without conflicts)
+constexpr uint32_t BK_OFF = GT_OFF + 32 * GT_LD * 4;  // u16 [1024] threshold buckets, or {hi, lo, hibits} [128]
+                                                      //   of the rows (scales whose i-exp values rise)
+constexpr uint32_t LG_OFF = BK_OFF + 2048;            // logits tile TM x ld, then B (1024-aligned)
+
+// Threshold buckets.  delta_k = #{d : e(d) > T} with T = 2S / D_k (i-exp values never rising with d).
+// T is approximated by T' = fp32(fp32(2S) * fp32(1 / D_k)), within 2^-22 of T; the bucket of T' (its
+// fp32 bits without the low 17, 64 buckets per octave) gives delta_k within [lo, lo + span]: lo counts
+// the values above the bucket's upper edge (raised by 2^-20), lo + span those above its lower edge
+// (lowered by 2^-20).  The exact test e(d) D_k <= 2S then settles the span by binary search (one probe
+// at usual scales).  Buckets cover 16 octaves below e(0); above them delta_k = 0, below them (T under
+// the smallest value e(0) 2^-15) delta_k = 256.
+constexpr int BK_SHIFT = 17;
+constexpr int BK_N = 1024;
+
+// fp32 1 / D_k for k = 1 .. 15 (D_1 = 3, D_k = 3 2^(k-1) - 1)
+__constant__ float kRcpD[16] = {0.0f,          1.0f / 3.0f,     1.0f / 5.0f,     1.0f / 11.0f,
+                                1.0f / 23.0f,  1.0f / 47.0f,    1.0f / 95.0f,    1.0f / 191.0f,
+                                1.0f / 383.0f, 1.0f / 767.0f,   1.0f / 1535.0f,  1.0f / 3071.0f,
+                                1.0f / 6143.0f, 1.0f / 12287.0f, 1.0f / 24575.0f, 1.0f / 49151.0f};
+
+// tensor memory: D at 0 (PACK: the second head's D at 64), the operands P from ta_col on (8 columns
+// per 16 keys), then the row sums of P (zp_V != 0), 16 columns
+__host__ __device__ constexpr int ta_col(bool pack) { return pack ? 2 * TD : TD; }
+__host__ __device__ constexpr int tr_col(int nkb, bool pack) { return ta_col(pack) + 32 * nkb; }
+__host__ __device__ constexpr int tmem_cols(int nkb, bool pack)
+{
+    return tr_col(nkb, pack) + 16 <= 128 ? 128 : tr_col(nkb, pack) + 16 <= 256 ? 256 : 512;
+}
 
 struct TcParams {
     const int8_t *logits;
     int64_t ld;
-    float s;
     const int8_t *v;
     int32_t *acc;
     int64_t BH;
     int L;
-    int zp;  // zero point of V (acc = sum_j 2^(15-code) (V - zp))
+    int zp;    // zero point of V (acc = sum_j 2^(15-code) (V - zp))
     IexpC ic;  // Algorithm 1 constants of the scale
     uint8_t *out8;  // when not null: 8-bit outputs (requant8 with n1, n2, zp8) instead of acc
     int64_t ld_out8;
     int n1, n2, zp8;
 };
 
-constexpr int TPARTS = 4;                         // threads per query row
-constexpr int TSOFT = TM * TPARTS;                // softmax threads (16 warps)
-constexpr int TEPI_WARP = TSOFT / 32;             // warps 16..19: accumulator read-out, one per lane quarter
-constexpr int TMMA_WARP = TEPI_WARP;              //   warp 16 lane 0 also issues the MMAs
-constexpr int TCOPY_WARP = TEPI_WARP + 1;         //   warp 17 lane 0 also copies the logits tiles
-constexpr int TTHREADS = TSOFT + 128;
-constexpr int TMAXKB = 10;                        // key blocks of the longest row (L <= 640)
-constexpr int TA_COL = TD;                        // D: columns 0..63; A of key block kb: 64 + 32 kb ..
-// row sums of P (only when zp_V != 0): 16 columns after A
-__host__ __device__ constexpr int tr_col(int nkb) { return TA_COL + 32 * nkb; }
-constexpr int SCR_THR = 0;                        // the logits tile doubles as threshold scratch: int32 [16][TM]
-constexpr int SCR_BYTES = 16 * TM * 4;
+// A tile: rows g0 .. g0 + rows - 1 of the [BH * L] logit rows; the first nsplit belong to head h0,
+// the rest (PACK only) to head h0 + 1.
+struct TileInfo {
+    int64_t g0;
+    int rows, h0, nsplit;
+};
 
-// tensor-memory columns for NKB key blocks (a power of two >= 32)
-__host__ __device__ constexpr int tmem_cols(int nkb)
+template <bool PACK>
+__device__ __forceinline__ TileInfo tile_info(int64_t t, int L, int64_t BH, int tpb)
 {
-    return tr_col(nkb) + 16 <= 128 ? 128 : tr_col(nkb) + 16 <= 256 ? 256 : 512;
+    TileInfo ti;
+    if (PACK) {
+        ti.g0 = t * TM;
+        ti.rows = (int)min((int64_t)TM, BH * L - ti.g0);
+        ti.h0 = (int)(ti.g0 / L);
+        ti.nsplit = (int)min((int64_t)ti.rows, (int64_t)(ti.h0 + 1) * L - ti.g0);
+    } else {
+        ti.h0 = (int)(t / tpb);
+        const int r0 = (int)(t - (int64_t)ti.h0 * tpb) * TM;
+        ti.g0 = (int64_t)ti.h0 * L + r0;
+        ti.rows = min(TM, L - r0);
+        ti.nsplit = ti.rows;
+    }
+    return ti;
+}
+
+// the tile after ti, without a division (PACK: a step of TM <= L rows crosses at most one head boundary)
+template <bool PACK>
+__device__ __forceinline__ TileInfo next_tile(TileInfo ti, int L, int64_t total)
+{
+    if (PACK) {
+        ti.g0 += TM;
+        if (ti.g0 >= (int64_t)(ti.h0 + 1) * L) ++ti.h0;
+        ti.rows = (int)min((int64_t)TM, total - ti.g0);
+        ti.nsplit = (int)min((int64_t)ti.rows, (int64_t)(ti.h0 + 1) * L - ti.g0);
+    } else {
+        int r0 = (int)(ti.g0 - (int64_t)ti.h0 * L) + TM;
+        if (r0 >= L) {
+            ++ti.h0;
+            r0 = 0;
+        }
+        ti.g0 = (int64_t)ti.h0 * L + r0;
+        ti.rows = min(TM, L - r0);
+        ti.nsplit = ti.rows;
+    }
+    return ti;
 }
 
 struct TcShared {
     uint64_t lload, lfree, afull, mmadone, fin;
     IexpC c;
     uint32_t tmem;
+    uint32_t b_off;  // offset of the B operand in dynamic shared memory (1024-aligned address)
+    int bk0, bkmax;  // bucket number of table entry 0, and of the last entry
     int abort_flag;
-    int rising;  // some i-exp value exceeds the one before it (floored constants)
-    int stop;    // set (never cleared) by a softmax thread whose wait gave up
-    int ew_stop; // the same for the read-out warps
+    int rising;   // some i-exp value exceeds the one before it (floored constants)
+    int stop;     // set (never cleared) by a softmax thread whose wait gave up
+    int ew_stop;  // the same for the read-out warps
 };
 
-// Named barrier 1 over the TSOFT softmax threads.  Every softmax thread reaches every one of
-// these barriers (the waits before them are bounded), so they end.  bar.sync is warp-aligned:
-// lanes of a row-dependent branch meet first.
+// Named barrier 1 over the TSOFT softmax threads.  Every softmax thread reaches every one of these
+// barriers (the waits before them are bounded), so they end.  bar.sync is warp-aligned: lanes of a
+// row-dependent branch meet first.
 __device__ __forceinline__ void soft_bar()
 {
     __syncwarp();
     asm volatile("bar.sync 1, %0;" ::"n"(TSOFT) : "memory");
 }
 
-// i-exp value of byte J of w: table entry m - q of this lane's replica (lutq points at entry m)
-template <int J>
-__device__ __forceinline__ uint32_t iexp_at(const uint32_t *lutq, uint32_t w)
-{
-    return lutq[-TCOPIES * sbyte<J>(w)];
-}
 // Named barrier 2 over the 128 read-out threads
 __device__ __forceinline__ void epi_bar()
 {
@@ -117,50 +213,133 @@ __device__ __forceinline__ void epi_bar()
     asm volatile("bar.sync 2, 128;" ::: "memory");
 }
 
-// Per tile (128 query rows of one head):
-//   copy (warp 17, lane 0): logits tile -> shared memory (bulk copy) once the previous tile's
-//               table is built, L2 prefetch of the tile after it (and of the next head's V)
-//   softmax:    thread (row r, part q) takes keys 64 kb + 16 q .. +15 of every key block into
-//               registers; the row maximum and the i-exp row sum are combined over the four parts
-//               through shared memory.  The row's operands go into a table indexed by the raw
-//               logit byte: word j of row r (OT[j][r], so that the 32 rows of a warp sit in 32
-//               different banks) holds, in byte b, 4 (30 - code) for the logit byte 4 j + b.
-//               Codes only depend on the row maximum, the row sum and the logit, so one table
-//               serves the whole row.  Where the i-exp values never rise with the distance d to
-//               the maximum, code(d) = #{k <= 15 : d >= delta_k} for the row's thresholds delta_k
-//               (the first d with e(d) D_k <= 2S): the four parts find them by binary search,
-//               histogram them into the table words and turn each word into its codes with a
-//               byte prefix sum (a multiply by 0x01010101); the floored constants of a few scales
-//               break the monotony, and those evaluate every entry.  Every logit then costs one
-//               table load; two loads and one byte permute give the fp16 pair 2^(15-code) that
-//               goes to tensor memory (A, K-major rows = lanes) once the previous tile's MMAs are
-//               done.  V of a head -> fp16 in shared memory (B, MN-major) whenever the head
-//               changes.
-//   MMA (warp 16, lane 0): after all operands of the tile are written, 4 MMAs per key block,
-//               one commit
-//   read-out (warps 16-19): the tile's accumulators, while the softmax warps work on the next
-// Each CTA takes a contiguous range of tiles, so that consecutive tiles share a head.
-// SMALL_E: every i-exp value is below 2^28 (decided on the host from the scale), so 16 of them
-// sum exactly in 32 bits
-template <int NKB, bool SMALL_E>
+// byte J of the distance word v in bits 8..15, byte 0 of the offset register o in bits 0..7: the
+// table address (d << 8) | offset.  o < 256, so its bytes 1..3 are the zero bytes of the result.
+template <int J>
+__device__ __forceinline__ uint32_t tab_addr(uint32_t v, uint32_t o)
+{
+    uint32_t y;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(y) : "r"(v), "r"(o), "n"(0x5504 | (J << 4)));
+    return y;
+}
+
+// word of the table at byte offset a (a multiple of 4)
+__device__ __forceinline__ uint32_t tab32(const unsigned char *tab, uint32_t a)
+{
+    return *reinterpret_cast<const uint32_t *>(tab + TAB_OFF + a);
+}
+
+// the fp16 pair (high bytes b0 of t0 and b1 of t1; low bytes zero) for two keys
+__device__ __forceinline__ uint32_t pack_ops(uint32_t t0, uint32_t t1)
+{
+    uint32_t y;
+    asm("prmt.b32 %0, %1, %2, 0x4101;" : "=r"(y) : "r"(t0), "r"(t1));
+    return y;
+}
+
+// V rows of one head (int8, L x 64) -> fp16 B (MN-major, 128-byte swizzled rows), rows of keys at
+// or past L up to the last 16-key step zero.  The 128 read-out threads: thread t takes 16 values
+// (16 (t % 4) ..) of keys t / 4, t / 4 + 32, ...
+__device__ __forceinline__ void convert_v(const int8_t *vh, int L, int nkeys, unsigned char *Bs, int t)
+{
+    const int c4 = t & 3;
+    for (int j0 = t >> 2; j0 < nkeys; j0 += 4 * 32) {
+        uint4 x[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int j = j0 + 32 * u;
+            x[u] = (j < L) ? __ldg(reinterpret_cast<const uint4 *>(vh + (size_t)j * TD + 16 * c4))
+                           : make_uint4(0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int j = j0 + 32 * u;
+            if (j >= nkeys) break;
+            uint4 a = make_uint4(0, 0, 0, 0), b = make_uint4(0, 0, 0, 0);
+            if (j < L) {
+                const uint32_t x0 = x[u].x ^ 0x80808080u, x1 = x[u].y ^ 0x80808080u;
+                const uint32_t x2 = x[u].z ^ 0x80808080u, x3 = x[u].w ^ 0x80808080u;
+                a = make_uint4(i8x2_to_h2(x0, 0x5140), i8x2_to_h2(x0, 0x7362), i8x2_to_h2(x1, 0x5140),
+                               i8x2_to_h2(x1, 0x7362));
+                b = make_uint4(i8x2_to_h2(x2, 0x5140), i8x2_to_h2(x2, 0x7362), i8x2_to_h2(x3, 0x5140),
+                               i8x2_to_h2(x3, 0x7362));
+            }
+            unsigned char *row = Bs + (size_t)j * 128;
+            *reinterpret_cast<uint4 *>(row + (((2 * c4) ^ (j & 7)) << 4)) = a;
+            *reinterpret_cast<uint4 *>(row + (((2 * c4 + 1) ^ (j & 7)) << 4)) = b;
+        }
+    }
+}
+
+// One row of the accumulators (32 lanes = 32 rows of a lane quarter) out of tensor memory: columns
+// dcol .. dcol + 63 of lane quarter etl, or, for lanes with use2, dcol2 .. (the second head's D).
+__device__ __forceinline__ void read_out_row(const TcParams &p, uint32_t etl, uint32_t dcol, uint32_t dcol2,
+                                             bool any2, bool use2, int64_t grow, bool ok_row, int zsum)
+{
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        uint32_t va[32];
+        tmem_ld32(etl + dcol + 32 * h, va);
+        tmem_wait_ld();
+        if (any2) {
+            uint32_t vb[32];
+            tmem_ld32(etl + dcol2 + 32 * h, vb);
+            tmem_wait_ld();
+            if (use2) {
+#pragma unroll
+                for (int c = 0; c < 32; ++c) va[c] = vb[c];
+            }
+        }
+        if (!ok_row) continue;
+        if (p.out8) {  // 8-bit outputs: 32 bytes of this half of the row
+            uint32_t wq[8];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                wq[c] = 0;
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                    wq[c] |= requant8(__float2int_rn(__uint_as_float(va[4 * c + k])) - zsum, p.n1, p.n2, p.zp8)
+                             << (8 * k);
+            }
+            uint4 *d8 = reinterpret_cast<uint4 *>(p.out8 + (size_t)grow * p.ld_out8 + 32 * h);
+            d8[0] = make_uint4(wq[0], wq[1], wq[2], wq[3]);
+            d8[1] = make_uint4(wq[4], wq[5], wq[6], wq[7]);
+        } else {
+            int32_t *dst = p.acc + (size_t)grow * TD + 32 * h;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                int v8[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) v8[j] = __float2int_rn(__uint_as_float(va[8 * c + j])) - zsum;
+                stg256(dst + 8 * c, v8);
+            }
+        }
+    }
+}
+
+// SMALL_E: every i-exp value is below 2^28 (decided on the host from the scale), so 16 of them sum
+// exactly in 32 bits
+template <int NKB, bool SMALL_E, bool PACK>
 __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
 {
-    extern __shared__ unsigned char dsm_raw[];
+    extern __shared__ __align__(1024) unsigned char dsm[];
     __shared__ TcShared sh;
-    __shared__ __align__(16) uint32_t OT[64 * TM];              // operand table: word j of row r at [j][r]
-    __shared__ float LUTF[256];                                 // fp32 of the i-exp values (exact: <= 16 bits)
-    __shared__ __align__(128) uint32_t ONES[128];               // 16 x 16 fp16 ones: B of the row sums of P
-    unsigned char *base = dsm_raw + ((1024u - (sa(dsm_raw) & 1023u)) & 1023u);
-    unsigned char *Bs = base;                                   // NKB x 8 KB
-    uint32_t *LUT = (uint32_t *)(Bs + NKB * B_SLOT);            // 256 x TCOPIES
-    int *red_max = (int *)(LUT + 256 * TCOPIES);                // TPARTS x TM
-    unsigned long long *red_sum = (unsigned long long *)(red_max + TPARTS * TM);
-    unsigned char *LG = (unsigned char *)(red_sum + TPARTS * TM);  // TM x ld logits, then scratch
-    int *thr = (int *)(LG + SCR_THR);                           // 16 x TM: delta_k of each row
+    __shared__ float LUTF[256];                    // fp32 of the i-exp values (exact: <= 16 bits)
+    __shared__ __align__(128) uint32_t ONES[128];  // 16 x 16 fp16 ones: B of the row sums of P
+    int *red_max = reinterpret_cast<int *>(dsm + RMAX_OFF);
+    unsigned long long *red_sum = reinterpret_cast<unsigned long long *>(dsm + RSUM_OFF);
+    uint32_t *GT = reinterpret_cast<uint32_t *>(dsm + GT_OFF);
+    uint16_t *BK = reinterpret_cast<uint16_t *>(dsm + BK_OFF);
+    float *rs_hi = reinterpret_cast<float *>(dsm + BK_OFF);
+    float *rs_lo = rs_hi + TM;
+    int *rs_bits = reinterpret_cast<int *>(rs_lo + TM);
+    unsigned char *LG = dsm + LG_OFF;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile int *abort_flag = &sh.abort_flag;
     volatile int *stop_flag = &sh.stop;
+    const int L = p.L;
+    const int nsteps = (L + 15) >> 4;  // MMA K steps of 16 keys
     pdl_release();
     if (tid == 0) {
         mbar_init(&sh.lload, 1);
@@ -173,368 +352,420 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
         sh.stop = 0;
         sh.ew_stop = 0;
         sh.c = p.ic;
+        const uint32_t lg_end = sa(dsm) + LG_OFF + (uint32_t)(TM * p.ld);
+        sh.b_off = ((lg_end + 1023u) & ~1023u) - sa(dsm);
     }
     if (warp == TMMA_WARP) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(&sh.tmem)),
-                     "r"(tmem_cols(NKB)));
+                     "r"(tmem_cols(NKB, PACK)));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     __syncthreads();
     {
         const IexpC c = sh.c;
-        for (int i = tid; i < 256 * TCOPIES; i += blockDim.x) LUT[i] = iexp_neg(i / TCOPIES, c);
+        for (int i = tid; i < 256 * 32; i += blockDim.x)
+            *reinterpret_cast<uint32_t *>(dsm + TAB_OFF + (uint32_t)(i >> 5) * 256u + LUT_BYTE + 4u * (i & 31)) =
+                iexp_neg(i >> 5, c);
         for (int d = tid; d < 256; d += blockDim.x) LUTF[d] = __uint2float_rn(iexp_neg(d, c));
         for (int i = tid; i < 128; i += blockDim.x) ONES[i] = 0x3C003C00u;
         for (int d = tid; d < 255; d += blockDim.x)
             if (iexp_neg(d, c) < iexp_neg(d + 1, c)) sh.rising = 1;
+    }
+    if (tid == 0) {
+        const int bkmax = (int)(__float_as_uint(__uint2float_rn(iexp_neg(0, sh.c)) * (1.0f + 0x1p-20f)) >> BK_SHIFT);
+        sh.bkmax = bkmax;
+        sh.bk0 = bkmax - (BK_N - 1);
+    }
+    __syncthreads();  // LUTF, rising, the bucket range
+    if (!sh.rising) {
+        // #{d : e(d) > x} by binary search (the values never rise with d)
+        auto count_above = [&](float x) -> int {
+            int lo = 0;
+            for (int step = 128; step >= 1; step >>= 1)
+                if (LUTF[lo + step - 1] > x) lo += step;
+            if (lo == 255 && LUTF[255] > x) lo = 256;
+            return lo;
+        };
+        for (int i = tid; i < BK_N; i += blockDim.x) {
+            const uint32_t b = (uint32_t)(sh.bk0 + i);
+            const float e_lo = __uint_as_float(b << BK_SHIFT) * (1.0f - 0x1p-20f);
+            const float e_hi = __uint_as_float((b + 1) << BK_SHIFT) * (1.0f + 0x1p-20f);
+            const int lo = count_above(e_hi), hi = count_above(e_lo);
+            BK[i] = (uint16_t)(lo | (min(hi - lo, 127) << 9));  // 127: the search runs on to 256
+        }
     }
     fence_async_smem();  // ONES is read by the MMAs
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = sh.tmem;
+    unsigned char *Bs = dsm + sh.b_off;
+    const uint32_t b_bytes = (uint32_t)nsteps * KSTEP_B;  // one V buffer
     pdl_wait();  // the set-up above touched no global memory
 
-    const int L = p.L;
     const int tpb = (L + TM - 1) / TM;
-    const int64_t ntiles = p.BH * tpb;
+    const int64_t total = p.BH * L;
+    const int64_t ntiles = PACK ? (total + TM - 1) / TM : p.BH * tpb;
     const int64_t t_begin = (int64_t)blockIdx.x * ntiles / gridDim.x;
     const int ncta_tiles = (int)((int64_t)(blockIdx.x + 1) * ntiles / gridDim.x - t_begin);
-    // (head, first row) of tile t_begin; every role steps it by one tile per iteration
-    const int bh_begin = (int)(t_begin / tpb);
-    const int r0_begin = (int)(t_begin - (int64_t)bh_begin * tpb) * TM;
+    constexpr int TA = ta_col(PACK);
+    constexpr int TR = tr_col(NKB, PACK);
 
     if (tid < TSOFT) {
-        const int r = tid & (TM - 1), q = tid >> 7;   // warp (q, r / 32): lanes = rows = TMEM lanes
-        const int kk = tid >> 3, ci = tid & 7;        // V conversion: key kk of a block, values 8 ci .. +7
-        const uint32_t lut_lane = sa(LUT) + 4u * (uint32_t)lane;
-        const uint32_t r4 = 4u * (uint32_t)r;
-        const unsigned char *otb = reinterpret_cast<const unsigned char *>(OT);
-        const uint32_t tlane = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-        const bool monotone = !sh.rising;            // codes never fall as d grows
-        const int xs = (int)(int8_t)(uint8_t)(64 * q);  // part q's table words 16 q .. +15: logits xs .. xs + 63
-        int npad = 0;  // keys at or past L inside this part's last partial block (summed as -128, then removed)
-#pragma unroll
-        for (int kb = 0; kb < NKB; ++kb) {
-            const int k0 = kb * TKB + 16 * q;
-            if (k0 < L && k0 + 16 > L) npad = k0 + 16 - L;
-        }
-        int it = 0;
+        const int k4 = warp & 3, q = warp >> 2;
+        const int r = 32 * k4 + lane;                    // row of the tile = tensor-memory lane
+        const uint32_t rowb = 4u * (uint32_t)lane + (uint32_t)k4;  // this row's byte in a table line
+        const uint32_t lutb = LUT_BYTE + 4u * (uint32_t)lane;      // this lane's i-exp copy in a line
+        const uint32_t tlane = tmem + ((uint32_t)(k4 * 32) << 16);
+        const bool monotone = !sh.rising;  // codes never fall as d grows
+        const uint32_t inc = 1u << (8 * k4);  // this row's byte of a table word
+        // keys of this part in the last 64-key block (0 .. 16; every other block holds 16)
+        const int last_keys = min(16, max(0, L - ((NKB - 1) * TKB + 16 * q)));
+        // keys at or past L inside this part's last partial block (summed as -128, then removed)
+        const int npad = last_keys > 0 ? 16 - last_keys : 0;
         bool wait_bad = false;
-        int conv_bh = -1;
-        int bh = bh_begin;
-        int r0 = r0_begin;
-        for (; it < ncta_tiles; ++it, r0 = r0 + TM < L ? r0 + TM : (++bh, 0)) {
-            const int row = r0 + r;
-            const bool valid = row < L;
+        TileInfo ti = tile_info<PACK>(t_begin, L, p.BH, tpb);
+        for (int it = 0; it < ncta_tiles; ++it, ti = next_tile<PACK>(ti, L, total)) {
+            const bool valid = r < ti.rows;
             const bool lbad = !mbar_wait_warp(&sh.lload, it & 1, abort_flag);
-            const unsigned char *lr = LG + (size_t)r * p.ld + 16 * q;
+            // ---- this part's logits into registers; keys at or past L become -128 (no effect on the
+            //      maximum; their i-exp values are removed from the sum, their operands are zero)
+            // (every part has 16 keys in each block but the last: L > 64 (NKB - 1))
             uint4 w[NKB];
 #pragma unroll
-            for (int kb = 0; kb < NKB; ++kb) {
-                const int k0 = kb * TKB + 16 * q;
-                w[kb] = (valid && k0 < L) ? *reinterpret_cast<const uint4 *>(lr + kb * TKB)
-                                          : make_uint4(0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u);
-                if (valid && k0 < L && k0 + 16 > L) {  // keys at or past L: -128 (no effect on the max)
-                    const int n = L - k0;
-                    uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
+            for (int kb = 0; kb < NKB; ++kb) w[kb] = make_uint4(0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u);
+            if (valid) {
+                const unsigned char *lr = LG + (size_t)r * p.ld + 16 * q;
 #pragma unroll
-                    for (int b = 0; b < 4; ++b) {
-                        const int keep = n - 4 * b;
-                        if (keep <= 0)
-                            ww[b] = 0x80808080u;
-                        else if (keep < 4)
-                            ww[b] = (ww[b] & (0xFFFFFFFFu >> (32 - 8 * keep))) |
-                                    (0x80808080u & ~(0xFFFFFFFFu >> (32 - 8 * keep)));
+                for (int kb = 0; kb < NKB - 1; ++kb) w[kb] = *reinterpret_cast<const uint4 *>(lr + kb * TKB);
+                if (last_keys > 0) {
+                    uint4 x = *reinterpret_cast<const uint4 *>(lr + (NKB - 1) * TKB);
+                    if (last_keys < 16) {
+                        uint32_t ww[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+                        for (int b = 0; b < 4; ++b) {
+                            const int keep = last_keys - 4 * b;
+                            if (keep <= 0)
+                                ww[b] = 0x80808080u;
+                            else if (keep < 4)
+                                ww[b] = (ww[b] & (0xFFFFFFFFu >> (32 - 8 * keep))) |
+                                        (0x80808080u & ~(0xFFFFFFFFu >> (32 - 8 * keep)));
+                        }
+                        x = make_uint4(ww[0], ww[1], ww[2], ww[3]);
                     }
-                    w[kb] = make_uint4(ww[0], ww[1], ww[2], ww[3]);
+                    w[NKB - 1] = x;
                 }
             }
-            // ---- row maximum over the four parts
-            // signed 16-bit lanes: the high byte of the larger lane is the larger byte, so lanes of w
-            // carry bytes 1 and 3 and lanes of w << 8 bytes 0 and 2
-            uint32_t mo = 0x80008000u, me = 0x80008000u;
+            mbar_arrive(&sh.lfree);  // the logits tile may be refilled
+            // ---- row maximum: odd bytes as the high bytes of signed 16-bit lanes, even bytes biased
+            //      to 0 .. 255 in unsigned 16-bit lanes
+            uint32_t mo = 0x80008000u, me = 0u;
 #pragma unroll
             for (int kb = 0; kb < NKB; ++kb) {
-                mo = vmax16x2(vmax16x2(mo, w[kb].x), vmax16x2(w[kb].y, vmax16x2(w[kb].z, w[kb].w)));
-                me = vmax16x2(vmax16x2(me, w[kb].x << 8), vmax16x2(w[kb].y << 8, vmax16x2(w[kb].z << 8, w[kb].w << 8)));
+                const uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
+#pragma unroll
+                for (int b = 0; b < 4; ++b) {
+                    mo = vmax16x2(mo, ww[b]);
+                    me = vmax16x2u(me, (ww[b] ^ 0x00800080u) & 0x00FF00FFu);
+                }
             }
-            int m = max(max(sbyte<1>(mo), sbyte<3>(mo)), max(sbyte<1>(me), sbyte<3>(me)));
+            int m = max(max(sbyte<1>(mo), sbyte<3>(mo)), max((int)(me & 0xFFFFu), (int)(me >> 16)) - 128);
             red_max[q * TM + r] = m;
             if (lbad || wait_bad) *stop_flag = 1;
-            soft_bar();
+            soft_bar();  // A
             if (*stop_flag) break;  // every softmax thread leaves here together
             m = max(max(red_max[r], red_max[TM + r]), max(red_max[2 * TM + r], red_max[3 * TM + r]));
-            // ---- i-exp row sum over the four parts
-            const uint32_t *lutq = LUT + lane + m * TCOPIES;
-            unsigned long long S = 0;
-            if (valid) {
+            // the previous tile's operand table is dead (every thread has passed its lookups): clear
+            // its bytes and the group totals for this tile's thresholds
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t c = (uint32_t)(tid + TSOFT * i);
+                *reinterpret_cast<uint4 *>(dsm + TAB_OFF + (c >> 3) * 256u + (c & 7u) * 16u) = make_uint4(0, 0, 0, 0);
+            }
+            GT[tid] = 0u;
+            if (tid < 32 * GT_LD - TSOFT) GT[TSOFT + tid] = 0u;
+            // ---- distances: byte d = m - q = (m + 128) - (q + 128), four per word, no borrows
+            {
+                const uint32_t mrep = (uint32_t)(m + 128) * 0x01010101u;
 #pragma unroll
                 for (int kb = 0; kb < NKB; ++kb) {
-                    if (kb * TKB + 16 * q < L) {
-                        const uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
-                        if (SMALL_E) {  // 16 values below 2^28: a 32-bit partial sum is exact
-                            uint32_t a = 0;
+                    w[kb].x = mrep - (w[kb].x ^ 0x80808080u);
+                    w[kb].y = mrep - (w[kb].y ^ 0x80808080u);
+                    w[kb].z = mrep - (w[kb].z ^ 0x80808080u);
+                    w[kb].w = mrep - (w[kb].w ^ 0x80808080u);
+                }
+            }
+            // ---- i-exp row sum over the four parts
+            unsigned long long S = 0;
+            if (valid) {
+                auto sum16 = [&](const uint4 &x) {
+                    const uint32_t ww[4] = {x.x, x.y, x.z, x.w};
+                    if (SMALL_E) {  // 16 values below 2^28: a 32-bit partial sum is exact
+                        uint32_t a = 0;
 #pragma unroll
-                            for (int b = 0; b < 4; ++b) {
-                                a += iexp_at<0>(lutq, ww[b]) + iexp_at<1>(lutq, ww[b]);
-                                a += iexp_at<2>(lutq, ww[b]) + iexp_at<3>(lutq, ww[b]);
-                            }
-                            S += a;
+                        for (int b = 0; b < 4; ++b) {
+                            const uint32_t e0 = tab32(dsm, tab_addr<0>(ww[b], lutb));
+                            const uint32_t e1 = tab32(dsm, tab_addr<1>(ww[b], lutb));
+                            const uint32_t e2 = tab32(dsm, tab_addr<2>(ww[b], lutb));
+                            const uint32_t e3 = tab32(dsm, tab_addr<3>(ww[b], lutb));
+                            a += e0 + e1;
+                            a += e2 + e3;
+                        }
+                        S += a;
+                    } else {
+#pragma unroll
+                        for (int b = 0; b < 4; ++b) {
+                            const uint32_t e0 = tab32(dsm, tab_addr<0>(ww[b], lutb));
+                            const uint32_t e1 = tab32(dsm, tab_addr<1>(ww[b], lutb));
+                            const uint32_t e2 = tab32(dsm, tab_addr<2>(ww[b], lutb));
+                            const uint32_t e3 = tab32(dsm, tab_addr<3>(ww[b], lutb));
+                            S += (unsigned long long)(e0 + e1) + (unsigned long long)(e2 + e3);  // e < 2^31
+                        }
+                    }
+                };
+#pragma unroll
+                for (int kb = 0; kb < NKB - 1; ++kb) sum16(w[kb]);
+                if (last_keys > 0) sum16(w[NKB - 1]);
+                // the padding bytes (-128, distance m + 128)
+                S -= (unsigned long long)npad * tab32(dsm, ((uint32_t)(m + 128) << 8) + lutb);
+            }
+            red_sum[q * TM + r] = S;
+            soft_bar();  // B
+            S = red_sum[r] + red_sum[TM + r] + red_sum[2 * TM + r] + red_sum[3 * TM + r];
+            const RowSum rs = split_2s(S);
+            if (monotone) {
+                // ---- this row's thresholds: part q finds delta_k for k = q + 1, q + 5, q + 9, q + 13
+                //      from the buckets and adds them to the table words
+                if (valid) {
+                    // e(d) D_k <= 2S, exact: one rounding of an exact product minus hi, against lo
+                    auto hit = [&](int d, float D) -> bool { return __fmaf_rn(LUTF[d], D, -rs.hi) <= rs.lo; };
+                    const int bk0 = sh.bk0, bkmax = sh.bkmax;
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const int k = q + 1 + 4 * i;
+                        if (k > 15) break;
+                        const float D = k == 1 ? 3.0f : (float)(3 * (1 << (k - 1)) - 1);
+                        const int b = (int)(__float_as_uint(rs.hi * kRcpD[k]) >> BK_SHIFT);
+                        int lo, n;  // delta_k in [lo, lo + n]
+                        if (b > bkmax) {
+                            lo = 0, n = 0;
+                        } else if (b < bk0) {
+                            lo = 256, n = 0;
                         } else {
-#pragma unroll
-                            for (int b = 0; b < 4; ++b) {
-                                const uint32_t e0 = iexp_at<0>(lutq, ww[b]), e1 = iexp_at<1>(lutq, ww[b]);
-                                const uint32_t e2 = iexp_at<2>(lutq, ww[b]), e3 = iexp_at<3>(lutq, ww[b]);
-                                S += (unsigned long long)(e0 + e1) + (unsigned long long)(e2 + e3);  // e < 2^31
+                            const uint32_t v = BK[b - bk0];
+                            lo = (int)(v & 511u);
+                            n = (int)(v >> 9);
+                            if (n == 127) n = 256 - lo;
+                        }
+                        while (n > 0) {  // the first d in [lo, lo + n) that hits, else lo + n
+                            const int h = n >> 1;
+                            if (hit(lo + h, D)) {
+                                n = h;
+                            } else {
+                                lo += h + 1;
+                                n -= h + 1;
                             }
+                        }
+                        if (lo < 256) {
+                            atomicAdd(reinterpret_cast<unsigned int *>(dsm + TAB_OFF + ((uint32_t)lo << 8) +
+                                                                       4u * (uint32_t)lane),
+                                      inc);
+                            atomicAdd(&GT[lane * GT_LD + (lo >> 4)], inc);
                         }
                     }
                 }
-                S -= (unsigned long long)npad * lutq[128 * TCOPIES];  // the padding bytes, -128 each
+            } else if (q == 0) {
+                rs_hi[r] = rs.hi;
+                rs_lo[r] = rs.lo;
+                rs_bits[r] = rs.hibits;
             }
-            red_sum[q * TM + r] = S;
-            // the table words of the previous tile are dead: clear this part's words for the histogram
-            if (valid && monotone) {
-#pragma unroll
-                for (int i = 0; i < 16; ++i) OT[(16 * q + i) * TM + r] = 0u;
-            }
-            soft_bar();
-            S = red_sum[r] + red_sum[TM + r] + red_sum[2 * TM + r] + red_sum[3 * TM + r];
-            const RowSum rs = split_2s(S);
-            // ---- this row's thresholds: part q finds delta_k for k = q + 1, q + 5, q + 9, q + 13,
-            //      the four binary searches interleaved
-            if (valid && monotone) {
-                float Dk[4];
-                int lo[4];
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const int k = q + 1 + 4 * i;
-                    Dk[i] = k == 1 ? 3.0f : (float)(3 * (1 << (min(k, 15) - 1)) - 1);
-                    lo[i] = 0;
-                }
-                // e(d) D_k <= 2S, exact: one rounding of an exact product minus hi, against lo
-                auto hit = [&](int d, float D) -> bool { return __fmaf_rn(LUTF[d], D, -rs.hi) <= rs.lo; };
-#pragma unroll
-                for (int step = 128; step >= 1; step >>= 1)
-#pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                        if (!hit(lo[i] + step - 1, Dk[i])) lo[i] += step;
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const int k = q + 1 + 4 * i;
-                    if (lo[i] == 255 && !hit(255, Dk[i])) lo[i] = 256;
-                    if (k <= 15) thr[(k - 1) * TM + r] = lo[i];
-                }
-            }
-            soft_bar();
-            // ---- this row's operand table
-            if (valid) {
+            soft_bar();  // C
+            // ---- the operand table: thread (lane, warp g) builds lines 16 g .. 16 g + 15 of column
+            //      lane (rows lane, 32 + lane, 64 + lane, 96 + lane)
+            {
+                const int g = warp;
                 if (monotone) {
-                    // E(x) = 30 - code(x) = 15 + #{k : m - delta_k < x}.  Histogram of the thresholds
-                    // m - delta_k over this part's logits (byte x - xs of the words), counting those
-                    // below xs, then per word the exclusive byte prefix sum.
-                    int n = 0;
+                    uint32_t carry = 0;  // thresholds below line 16 g, per row byte
+                    {
+                        const uint4 *gt = reinterpret_cast<const uint4 *>(GT + lane * GT_LD);
+                        const uint4 g0 = gt[0], g1 = gt[1], g2 = gt[2], g3 = gt[3];
+                        const uint32_t gv[16] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w,
+                                                 g2.x, g2.y, g2.z, g2.w, g3.x, g3.y, g3.z, g3.w};
 #pragma unroll
-                    for (int k = 0; k < 15; ++k) {
-                        const int t = m - thr[k * TM + r] - xs;
-                        n += t < 0 ? 1 : 0;
-                        if ((unsigned)t < 64u) OT[(16 * q + (t >> 2)) * TM + r] += 1u << (8 * (t & 3));
+                        for (int j = 0; j < 15; ++j) carry += j < g ? gv[j] : 0u;
                     }
 #pragma unroll
                     for (int i = 0; i < 16; ++i) {
-                        uint32_t *wp = &OT[(16 * q + i) * TM + r];
-                        const uint32_t h = *wp;
-                        *wp = 0x3C3C3C3Cu + 4u * ((uint32_t)n * 0x01010101u + (h << 8) * 0x01010101u);
-                        n += (int)((h * 0x01010101u) >> 24);
+                        uint32_t *wp = reinterpret_cast<uint32_t *>(dsm + TAB_OFF + (uint32_t)(16 * g + i) * 256u +
+                                                                    4u * (uint32_t)lane);
+                        carry += *wp;
+                        *wp = 0x78787878u - 4u * carry;  // 4 (30 - code) per byte
                     }
                 } else {
-                    auto E_at = [&](int x) -> uint32_t {
-                        return operand_exp(lds32(lut_lane + (uint32_t)((m - x) * (TCOPIES * 4))), rs.hibits, rs.hi, rs.lo);
-                    };
-#pragma unroll 2
+#pragma unroll 1
                     for (int i = 0; i < 16; ++i) {
-                        const int j = q + 4 * i;
-                        const int xlo = (int)(int8_t)(uint8_t)(4 * j);  // logits of word j: xlo .. xlo + 3
-                        if (xlo > m) continue;                          // no key of this row reads it
-                        const int hb = min(3, m - xlo);                 // bytes above hb exceed the maximum
-                        const uint32_t E0 = E_at(xlo);
-                        const uint32_t E1 = hb >= 1 ? E_at(xlo + 1) : E0;
-                        const uint32_t E2 = hb >= 2 ? E_at(xlo + 2) : E1;
-                        const uint32_t E3 = hb >= 3 ? E_at(xlo + 3) : E2;
-                        OT[j * TM + r] = 4u * (E0 | (E1 << 8) | (E2 << 16) | (E3 << 24));
+                        const int d = 16 * g + i;
+                        const float ef = LUTF[d];
+                        uint32_t word = 0;
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const int rr = 32 * k + lane;
+                            const uint32_t E = operand_exp_f(ef, rs_bits[rr], rs_hi[rr], rs_lo[rr]);
+                            word |= (4u * E) << (8 * k);
+                        }
+                        *reinterpret_cast<uint32_t *>(dsm + TAB_OFF + (uint32_t)d * 256u + 4u * (uint32_t)lane) = word;
                     }
                 }
             }
-            soft_bar();
-            mbar_arrive(&sh.lfree);  // the logits tile and its scratch are free: the next tile may load
-            // the previous tile's MMAs have read A and B: they may be rewritten
+            soft_bar();  // D
+            // the previous tile's MMAs have read the operands in tensor memory: they may be rewritten
             if (it > 0 && !mbar_wait_warp(&sh.mmadone, (it - 1) & 1, abort_flag)) {
                 wait_bad = true;  // the next tile's first barrier ends the loop for all
                 continue;
             }
-            // ---- V of a new head -> fp16 B
-            if (bh != conv_bh) {
-#pragma unroll
-                for (int kb = 0; kb < NKB; ++kb) {
-                    const int key = kb * TKB + kk;
-                    uint4 v4 = make_uint4(0, 0, 0, 0);
-                    if (key < L) {
-                        const uint2 vw = __ldg(reinterpret_cast<const uint2 *>(p.v + ((size_t)bh * L + key) * TD + 8 * ci));
-                        const uint32_t x0 = vw.x ^ 0x80808080u, x1 = vw.y ^ 0x80808080u;
-                        v4.x = i8x2_to_h2(x0, 0x5140);
-                        v4.y = i8x2_to_h2(x0, 0x7362);
-                        v4.z = i8x2_to_h2(x1, 0x5140);
-                        v4.w = i8x2_to_h2(x1, 0x7362);
-                    }
-                    *reinterpret_cast<uint4 *>(Bs + kb * B_SLOT + kk * 128 + ((ci ^ (kk & 7)) << 4)) = v4;
-                }
-                conv_bh = bh;
-            }
             // ---- operands of this row's keys -> tensor memory
-#pragma unroll
-            for (int kb = 0; kb < NKB; ++kb) {
-                const int k0 = kb * TKB + 16 * q;
-                uint32_t o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                if (valid && k0 < L) {
-                    const uint32_t ww[4] = {w[kb].x, w[kb].y, w[kb].z, w[kb].w};
+            {
+                auto ops16 = [&](const uint4 &x, uint32_t (&o)[8]) {
+                    const uint32_t ww[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
                     for (int b = 0; b < 4; ++b) {
-                        const uint32_t v = ww[b];
-                        // word (byte >> 2) of this row, then byte (byte & 3) of it into the high byte
-                        // of each fp16 half; the low bytes copy the sign of a table byte (zero)
-                        const uint32_t t0 = *reinterpret_cast<const uint32_t *>(otb + (((v << 7) & 0x7E00u) | r4));
-                        const uint32_t t1 = *reinterpret_cast<const uint32_t *>(otb + (((v >> 1) & 0x7E00u) | r4));
-                        const uint32_t t2 = *reinterpret_cast<const uint32_t *>(otb + (((v >> 9) & 0x7E00u) | r4));
-                        const uint32_t t3 = *reinterpret_cast<const uint32_t *>(otb + (((v >> 17) & 0x7E00u) | r4));
-                        o[2 * b] = prmt(t0, t1, ((v << 4) & 0x3030u) | 0x4808u);
-                        o[2 * b + 1] = prmt(t2, t3, ((v >> 12) & 0x3030u) | 0x4808u);
+                        const uint32_t t0 = dsm[TAB_OFF + tab_addr<0>(ww[b], rowb)];
+                        const uint32_t t1 = dsm[TAB_OFF + tab_addr<1>(ww[b], rowb)];
+                        const uint32_t t2 = dsm[TAB_OFF + tab_addr<2>(ww[b], rowb)];
+                        const uint32_t t3 = dsm[TAB_OFF + tab_addr<3>(ww[b], rowb)];
+                        o[2 * b] = pack_ops(t0, t1);
+                        o[2 * b + 1] = pack_ops(t2, t3);
                     }
-                    if (k0 + 16 > L) {  // keys at or past L get a zero operand
-                        const int n = L - k0;
+                };
 #pragma unroll
-                        for (int c = 0; c < 8; ++c) {
-                            if (2 * c >= n)
+                for (int kb = 0; kb < NKB - 1; ++kb) {
+                    uint32_t o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                    if (valid) ops16(w[kb], o);
+                    tmem_st8(tlane + TA + 32 * kb + 8 * q, o);
+                }
+                if (last_keys > 0) {  // warp-uniform
+                    uint32_t o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                    if (valid) {
+                        ops16(w[NKB - 1], o);
+#pragma unroll
+                        for (int c = 0; c < 8; ++c) {  // keys at or past L get a zero operand
+                            if (2 * c >= last_keys)
                                 o[c] = 0;
-                            else if (2 * c + 1 == n)
+                            else if (2 * c + 1 == last_keys)
                                 o[c] &= 0xFFFFu;
                         }
                     }
+                    tmem_st8(tlane + TA + 32 * (NKB - 1) + 8 * q, o);
                 }
-                tmem_st8(tlane + TA_COL + 32 * kb + 8 * q, o);
             }
             __syncwarp();
-            asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+            tmem_wait_st();
             tc_fence_before();
-            fence_async_smem();
             mbar_arrive(&sh.afull);
         }
     } else {
-        // ---------------- read-out warps (lane quarter eq), with the MMA issue and the logits copies
+        // ---------------- read-out warps (lane quarter eq), with V, the MMA issue and the logits copies
         const int eq = warp & 3;
+        const int et = tid - TSOFT;  // 0 .. 127
         const uint32_t etl = tmem + ((uint32_t)(eq * 32) << 16);
         volatile int *ew_stop = &sh.ew_stop;
-        const int nkb = (L + TKB - 1) / TKB;
-        int bh = bh_begin;
-        int r0 = r0_begin;
-        if (warp == TCOPY_WARP && lane == 0) {
-            prefetch_l2(p.v + (size_t)bh * L * TD, (uint32_t)(L * TD));
-            const uint32_t bl = (uint32_t)(min(TM, L - r0) * p.ld);
+        int conv_hi = -1;  // the last head whose V went into its B buffer
+        int ncopies = 0;
+        auto bbuf = [&](int h) -> unsigned char * { return Bs + (PACK ? (uint32_t)(h & 1) * b_bytes : 0u); };
+        auto last_head = [](const TileInfo &t) { return t.nsplit < t.rows ? t.h0 + 1 : t.h0; };
+        TileInfo ti = tile_info<PACK>(t_begin, L, p.BH, tpb);
+        TileInfo tp = ti;  // the previous tile
+        if (warp == TCOPY_WARP && lane == 0 && ncta_tiles > 0) {
+            prefetch_l2(p.v + (size_t)ti.h0 * L * TD, (uint32_t)(L * TD));
+            if (last_head(ti) != ti.h0) prefetch_l2(p.v + (size_t)last_head(ti) * L * TD, (uint32_t)(L * TD));
+            const uint32_t bl = (uint32_t)(ti.rows * p.ld);
             mbar_expect_tx(&sh.lload, bl);
-            bulk_g2s(LG, p.logits + ((size_t)bh * L + r0) * p.ld, bl, &sh.lload);
+            bulk_g2s(LG, p.logits + (size_t)ti.g0 * p.ld, bl, &sh.lload);
+            ++ncopies;
         }
-        for (int it = 0; it < ncta_tiles; ++it, r0 = r0 + TM < L ? r0 + TM : (++bh, 0)) {
+        auto read_out = [&](const TileInfo &t) {
+            const int i = 32 * eq + lane;  // row of the tile
+            const bool any2 = PACK && t.nsplit < 32 * eq + 32 && t.nsplit < t.rows;
+            const bool use2 = PACK && i >= t.nsplit;
+            int zsum = 0;  // zp (sum_j 2^(15-code_j)), an exact integer below 2^24 times |zp| <= 255
+            if (p.zp != 0) {
+                uint32_t rsv;
+                tmem_ld1(etl + TR, rsv);
+                tmem_wait_ld();
+                zsum = p.zp * __float2int_rn(__uint_as_float(rsv));
+            }
+            read_out_row(p, etl, 0, TD, any2, use2, t.g0 + i, i < t.rows, zsum);
+        };
+        int it = 0;
+        for (; it < ncta_tiles; ++it) {
+            if (it > 0) {
+                tp = ti;
+                ti = next_tile<PACK>(ti, L, total);
+            }
             if (warp == TCOPY_WARP && lane == 0 && it + 1 < ncta_tiles) {
-                // the next tile's logits as soon as this tile's table is built
-                const int bhn = r0 + TM < L ? bh : bh + 1;
-                const int r0n = r0 + TM < L ? r0 + TM : 0;
+                // the next tile's logits as soon as every softmax thread holds this tile's
+                const TileInfo tn = next_tile<PACK>(ti, L, total);
                 if (mbar_wait(&sh.lfree, it & 1, abort_flag)) {
-                    const uint32_t bl = (uint32_t)(min(TM, L - r0n) * p.ld);
+                    const uint32_t bl = (uint32_t)(tn.rows * p.ld);
                     mbar_expect_tx(&sh.lload, bl);
-                    bulk_g2s(LG, p.logits + ((size_t)bhn * L + r0n) * p.ld, bl, &sh.lload);
-                    if (bhn != bh) prefetch_l2(p.v + (size_t)bhn * L * TD, (uint32_t)(L * TD));
+                    bulk_g2s(LG, p.logits + (size_t)tn.g0 * p.ld, bl, &sh.lload);
+                    ++ncopies;
+                    if (last_head(tn) != last_head(ti))
+                        prefetch_l2(p.v + (size_t)last_head(tn) * L * TD, (uint32_t)(L * TD));
                     if (it + 2 < ncta_tiles) {
-                        const int r0m = r0n + TM < L ? r0n + TM : 0;
-                        const int bhm = r0n + TM < L ? bhn : bhn + 1;
-                        prefetch_l2(p.logits + ((size_t)bhm * L + r0m) * p.ld, (uint32_t)(min(TM, L - r0m) * p.ld));
+                        const TileInfo tm = next_tile<PACK>(tn, L, total);
+                        prefetch_l2(p.logits + (size_t)tm.g0 * p.ld, (uint32_t)(tm.rows * p.ld));
                     }
                 }
             }
-            if (warp == TMMA_WARP && lane == 0) {
-                // this tile's MMAs once its operands are in place
-                if (mbar_wait(&sh.afull, it & 1, abort_flag)) {
+            bool ok = true;
+            if (it > 0) {  // the previous tile's accumulators; then D and the B buffers are free
+                ok = mbar_wait_warp(&sh.mmadone, (it - 1) & 1, abort_flag);
+                if (ok) {
                     tc_fence_after();
-                    const uint32_t b0 = sa(Bs);
-                    const uint64_t ones = smem_desc_plain(sa(ONES), 128, 256);
-                    if (p.zp == 0) {
-                        for (int kb = 0; kb < nkb; ++kb)
-#pragma unroll
-                            for (int s = 0; s < TKB / 16; ++s)
-                                mma_f16_ta(tmem, tmem + TA_COL + 32 * kb + 8 * s,
-                                           smem_desc(b0 + kb * B_SLOT + 2048 * s, 1024, 1024), (kb | s) != 0);
-                    } else {
-                        for (int kb = 0; kb < nkb; ++kb)
-#pragma unroll
-                            for (int s = 0; s < TKB / 16; ++s) {
-                                mma_f16_ta(tmem, tmem + TA_COL + 32 * kb + 8 * s,
-                                           smem_desc(b0 + kb * B_SLOT + 2048 * s, 1024, 1024), (kb | s) != 0);
-                                mma_f16_ta(tmem + tr_col(NKB), tmem + TA_COL + 32 * kb + 8 * s, ones,
-                                           (kb | s) != 0, kIdescOnes);
-                            }
-                    }
-                    mma_commit(&sh.mmadone);
+                    read_out(tp);
                 }
             }
-            // this tile's accumulators: row 32 eq + lane of the tile, 64 columns in two halves
-            const bool ok = mbar_wait_warp(&sh.mmadone, it & 1, abort_flag);
+            // V of this tile's head(s) not yet in B
             if (ok) {
-                tc_fence_after();
-                const int row = r0 + 32 * eq + lane;
-                int32_t *dst = p.out8 ? nullptr : p.acc + ((size_t)bh * L + row) * TD;
-                // zp (sum_j 2^(15-code_j)), an exact integer below 2^24 times |zp| <= 255
-                int zsum = 0;
-                if (p.zp != 0) {
-                    uint32_t rs;
-                    tmem_ld1(etl + tr_col(NKB), rs);
-                    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-                    zsum = p.zp * __float2int_rn(__uint_as_float(rs));
-                }
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    uint32_t va[32];
-                    tmem_ld32(etl + 32 * h, va);
-                    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-                    if (row < L && p.out8) {  // 8-bit outputs: 32 bytes of this half of the row
-                        uint32_t wq[8];
-#pragma unroll
-                        for (int c = 0; c < 8; ++c) {
-                            wq[c] = 0;
-#pragma unroll
-                            for (int k = 0; k < 4; ++k)
-                                wq[c] |= requant8(__float2int_rn(__uint_as_float(va[4 * c + k])) - zsum, p.n1, p.n2,
-                                                  p.zp8) << (8 * k);
-                        }
-                        uint4 *d8 = reinterpret_cast<uint4 *>(p.out8 + ((size_t)bh * L + row) * p.ld_out8 + 32 * h);
-                        d8[0] = make_uint4(wq[0], wq[1], wq[2], wq[3]);
-                        d8[1] = make_uint4(wq[4], wq[5], wq[6], wq[7]);
-                    } else if (row < L) {
-#pragma unroll
-                        for (int c = 0; c < 4; ++c) {
-                            int v8[8];
-#pragma unroll
-                            for (int j = 0; j < 8; ++j)
-                                v8[j] = __float2int_rn(__uint_as_float(va[8 * c + j])) - zsum;
-                            stg256(dst + 32 * h + 8 * c, v8);
-                        }
-                    }
+                for (int h = max(conv_hi + 1, ti.h0); h <= last_head(ti); ++h) {
+                    convert_v(p.v + (size_t)h * L * TD, L, 16 * nsteps, bbuf(h), et);
+                    conv_hi = h;
                 }
             }
+            fence_async_smem();
             tc_fence_before();
             if (!ok) *ew_stop = 1;
-            epi_bar();  // all four quarters have read D: the next tile's MMAs may overwrite it
+            epi_bar();  // D read, B written: this tile's MMAs may run
             if (*ew_stop) break;
+            if (warp == TMMA_WARP && lane == 0) {
+                if (mbar_wait(&sh.afull, it & 1, abort_flag)) {
+                    tc_fence_after();
+                    const uint64_t ones = smem_desc_plain(sa(ONES), 128, 256);
+                    const int nh = (PACK && ti.nsplit < ti.rows) ? 2 : 1;
+                    for (int hh = 0; hh < nh; ++hh) {
+                        const uint32_t b0 = sa(bbuf(ti.h0 + hh));
+                        const uint32_t dcol = tmem + (uint32_t)(hh * TD);
+                        for (int s = 0; s < nsteps; ++s)
+                            mma_f16_ta(dcol, tmem + TA + 8 * s, smem_desc(b0 + KSTEP_B * s, 1024, 1024), s != 0);
+                    }
+                    if (p.zp != 0)
+                        for (int s = 0; s < nsteps; ++s)
+                            mma_f16_ta(tmem + TR, tmem + TA + 8 * s, ones, s != 0, kIdescOnes);
+                    mma_commit(&sh.mmadone);
+                } else {
+                    *ew_stop = 1;
+                }
+            }
         }
-        if (warp == TCOPY_WARP && lane == 0) mbar_wait(&sh.lload, (ncta_tiles - 1) & 1, abort_flag, false);
+        if (it == ncta_tiles && ncta_tiles > 0 && !*ew_stop) {  // the last tile's accumulators
+            if (mbar_wait_warp(&sh.mmadone, (ncta_tiles - 1) & 1, abort_flag)) {
+                tc_fence_after();
+                read_out(ti);
+            }
+        }
+        if (warp == TCOPY_WARP && lane == 0 && ncopies > 0)  // no copy may land after the CTA exits
+            mbar_wait(&sh.lload, (ncopies - 1) & 1, abort_flag, false);
         if (warp == TMMA_WARP && lane == 0) {  // every MMA issued has completed before tensor memory is freed
             mma_commit(&sh.fin);
             mbar_wait(&sh.fin, 0, abort_flag, false);
@@ -544,32 +775,41 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     __syncthreads();
     tc_fence_after();
     if (warp == TMMA_WARP)
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tmem_cols(NKB)));
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tmem_cols(NKB, PACK)));
 }
 
-size_t tc_smem_bytes(int L, int64_t ld)
+// dynamic shared memory of a launch (the B buffers after the logits tile, 1024-aligned; up to 1008
+// bytes of alignment slack when the dynamic window itself is only 16-byte aligned)
+size_t tc_smem_bytes(int L, int64_t ld, bool pack)
 {
-    const int nkb = (L + TKB - 1) / TKB;
-    const size_t lg = (size_t)TM * ld > (size_t)SCR_BYTES ? (size_t)TM * ld : (size_t)SCR_BYTES;
-    return 1024 + (size_t)nkb * B_SLOT + (size_t)256 * TCOPIES * 4 + (size_t)TPARTS * TM * (4 + 8) + lg;
+    const size_t nsteps = (size_t)(L + 15) / 16;
+    const size_t lg_end = LG_OFF + (size_t)TM * ld;
+    return ((lg_end + 1023) & ~(size_t)1023) + 1008 + (pack ? 2 : 1) * nsteps * KSTEP_B;
 }
 
-// static shared memory of the kernel: the operand table, the fp32 i-exp table, the control block
-constexpr size_t kTcStaticSmem = (size_t)64 * TM * 4 + 1024 + 512 + 256;
+// static shared memory of the kernel: the control block, the fp32 i-exp table, the ones block
+constexpr size_t kTcStaticSmem = 2048;
 
-template <int NKB, bool SMALL_E>
+bool use_pack(int L) { return L >= TM && L <= kPackMaxBlocks * TKB; }
+
+template <int NKB, bool SMALL_E, bool PACK>
 cudaError_t tc_launch(const TcParams &p, size_t smem, int grid, cudaStream_t st)
 {
-    cudaError_t e = cudaFuncSetAttribute(lis_attn_tc_kernel<NKB, SMALL_E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+    cudaError_t e = cudaFuncSetAttribute(lis_attn_tc_kernel<NKB, SMALL_E, PACK>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(lis_attn_tc_kernel<NKB, SMALL_E>, dim3(grid), dim3(TTHREADS), smem, st, p);
+    return launch_pdl(lis_attn_tc_kernel<NKB, SMALL_E, PACK>, dim3(grid), dim3(TTHREADS), smem, st, p);
 }
 
 template <int NKB>
-cudaError_t tc_launch_e(bool small_e, const TcParams &p, size_t smem, int grid, cudaStream_t st)
+cudaError_t tc_launch_e(bool small_e, bool pack, const TcParams &p, size_t smem, int grid, cudaStream_t st)
 {
-    return small_e ? tc_launch<NKB, true>(p, smem, grid, st) : tc_launch<NKB, false>(p, smem, grid, st);
+    if constexpr (NKB <= kPackMaxBlocks && NKB >= 2) {
+        if (pack)
+            return small_e ? tc_launch<NKB, true, true>(p, smem, grid, st)
+                           : tc_launch<NKB, false, true>(p, smem, grid, st);
+    }
+    return small_e ? tc_launch<NKB, true, false>(p, smem, grid, st) : tc_launch<NKB, false, false>(p, smem, grid, st);
 }
 
 // Whether every i-exp value of the scale is below 2^28: the largest is e(0) = (q_b^2 + q_c) 2^15.
@@ -583,29 +823,29 @@ bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
                                : (b.ld_acc == TD && ((uintptr_t)b.acc % 32) == 0);
     return b.d == TD && a.bias == nullptr && a.region == nullptr && a.codes == nullptr && a.L <= TMAXKB * TKB &&
            a.ld_logit % 16 == 0 && b.ld_v == TD && out_ok && ((uintptr_t)a.logits % 16) == 0 &&
-           ((uintptr_t)b.v % 16) == 0 && tc_smem_bytes(a.L, a.ld_logit) + kTcStaticSmem <= 232448;
+           ((uintptr_t)b.v % 16) == 0 && tc_smem_bytes(a.L, a.ld_logit, use_pack(a.L)) + kTcStaticSmem <= 232448;
 }
 
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
 {
-    if (lis_attention_tc_packed(a.L)) return launch_lis_attention_tc_packed(a, b, st);  // lis_tc_pack.cu
-    TcParams p{a.logits, a.ld_logit, a.s_logit, b.v, b.acc, b.BH, a.L, b.zp_v, iexp_consts_host(a.s_logit),
+    TcParams p{a.logits, a.ld_logit, b.v, b.acc, b.BH, a.L, b.zp_v, iexp_consts_host(a.s_logit),
                b.out8, b.ld_out8, b.rq_n1, b.rq_n2, b.rq_zp};
-    const size_t smem = tc_smem_bytes(a.L, a.ld_logit);
-    const int64_t ntiles = b.BH * ((a.L + TM - 1) / TM);
+    const bool pack = use_pack(a.L);
+    const size_t smem = tc_smem_bytes(a.L, a.ld_logit, pack);
+    const int64_t ntiles = pack ? (b.BH * a.L + TM - 1) / TM : b.BH * ((a.L + TM - 1) / TM);
     const int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());
     const bool se = small_iexp(p.ic);
     switch ((a.L + TKB - 1) / TKB) {
-    case 1: return tc_launch_e<1>(se, p, smem, grid, st);
-    case 2: return tc_launch_e<2>(se, p, smem, grid, st);
-    case 3: return tc_launch_e<3>(se, p, smem, grid, st);
-    case 4: return tc_launch_e<4>(se, p, smem, grid, st);
-    case 5: return tc_launch_e<5>(se, p, smem, grid, st);
-    case 6: return tc_launch_e<6>(se, p, smem, grid, st);
-    case 7: return tc_launch_e<7>(se, p, smem, grid, st);
-    case 8: return tc_launch_e<8>(se, p, smem, grid, st);
-    case 9: return tc_launch_e<9>(se, p, smem, grid, st);
-    default: return tc_launch_e<10>(se, p, smem, grid, st);
+    case 1: return tc_launch_e<1>(se, pack, p, smem, grid, st);
+    case 2: return tc_launch_e<2>(se, pack, p, smem, grid, st);
+    case 3: return tc_launch_e<3>(se, pack, p, smem, grid, st);
+    case 4: return tc_launch_e<4>(se, pack, p, smem, grid, st);
+    case 5: return tc_launch_e<5>(se, pack, p, smem, grid, st);
+    case 6: return tc_launch_e<6>(se, pack, p, smem, grid, st);
+    case 7: return tc_launch_e<7>(se, pack, p, smem, grid, st);
+    case 8: return tc_launch_e<8>(se, pack, p, smem, grid, st);
+    case 9: return tc_launch_e<9>(se, pack, p, smem, grid, st);
+    default: return tc_launch_e<10>(se, pack, p, smem, grid, st);
     }
 }
 
@@ -624,11 +864,7 @@ cudaError_t read_clear_device_status(int *status, cudaStream_t st)
     if (*status == 0) *status = wst;
     int qst = 0;
     e = read_clear_qk_status(&qst);
-    if (e != cudaSuccess) return e;
     if (*status == 0) *status = qst;
-    int pst = 0;
-    e = read_clear_tcp_status(&pst);
-    if (*status == 0) *status = pst;
     return e;
 }
 
