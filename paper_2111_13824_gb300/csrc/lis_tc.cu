@@ -1,6 +1,6 @@
 // lis_tc.cu -- fused Log-Int-Softmax + BitShift attention times values on
-// the 5th-generation tensor cores (tcgen05) of sm_103a, for rows of 65 .. 640
-// keys (head dimension 64).
+// the 5th-generation tensor cores (tcgen05) of sm_103a, for rows of 65 .. 592
+// keys (head dimension 64; the longest rows its shared-memory layout holds).
 //
 // Eq. 15 is a matrix product: acc = P (V - zp_V) with P[i][j] = 2^(15 - code_ij),
 // computed as P V - zp_V (P 1).  Every P entry and every int8 value of V is exact
@@ -36,14 +36,15 @@
 //     into the fp16 B operand in shared memory, the tile's MMAs (warp 16, lane
 //     0) and the bulk copy of the next tile's logits (warp 17, lane 0).
 //
-// The combined table (64 KB at the start of dynamic shared memory): line d
+// The combined table (64 KB at the absolute shared-memory address 64 K): line d
 // (d = 0 .. 255) is 256 bytes.  Bytes 0 .. 127 hold the high byte 4 (30 - code)
 // of the operand of distance d for the 128 rows of the tile, row r at byte
 // 4 (r % 32) + r / 32, so that the 32 rows of a warp read 32 different banks;
 // bytes 128 .. 255 hold 32 copies of the i-exp value e(d), copy c at byte
 // 128 + 4 c (lane c reads its own copy: no bank conflicts for random d).  One
-// byte permute turns a distance byte and a per-thread byte into an address
-// (d << 8 | offset), so a table lookup costs one permute and one load.
+// byte permute turns a distance byte and a per-thread register into the full
+// address 64 K | d << 8 | offset, so a table lookup costs one permute and one
+// load.
 //
 // The operand table from thresholds: code(d) = #{k <= 15 : d >= delta_k} with
 // delta_k the first d at which e(d) D_k <= 2S (D_1 = 3, D_k = 3 2^(k-1) - 1,
@@ -77,26 +78,64 @@ using namespace tc;
 constexpr int TM = 128;                    // query rows per tile (MMA M)
 constexpr int TKB = 64;                    // keys per key block
 constexpr int TD = 64;                     // head dimension (MMA N)
-constexpr int KSTEP_B = 16 * TD * 2;       // bytes of B per 16 keys (one MMA K step)
 constexpr int TPARTS = 4;                  // threads per query row
 constexpr int TSOFT = TM * TPARTS;         // softmax threads (16 warps)
 constexpr int TEPI_WARP = TSOFT / 32;      // warps 16..19: read-out, one per lane quarter
 constexpr int TMMA_WARP = TEPI_WARP;       //   warp 16 lane 0 also issues the MMAs
 constexpr int TCOPY_WARP = TEPI_WARP + 1;  //   warp 17 lane 0 also copies the logits tiles
 constexpr int TTHREADS = TSOFT + 128;
-constexpr int TMAXKB = 10;                 // key blocks of the longest row (L <= 640)
+constexpr int TMAXKB = 10;                 // key blocks of the longest row
 constexpr int kPackMaxBlocks = 6;          // PACK for 128 <= L <= 384
 
-// dynamic shared memory
-constexpr uint32_t TAB_OFF = 0;                       // 256 lines x 256 B
-constexpr uint32_t LUT_BYTE = 128;                    // i-exp copies in a line
-constexpr uint32_t RMAX_OFF = 65536;                  // int [4][128]: row maxima of the parts
-constexpr uint32_t RSUM_OFF = RMAX_OFF + 2048;        // u64 [4][128]: row sums of the parts
-constexpr uint32_t GT_OFF = RSUM_OFF + 4096;          // u32 [32][20]: thresholds per (lane, 16-line group)
+// Shared memory.  The kernel has no static shared memory, so its dynamic shared memory starts at
+// the first address after the 1 KB the driver reserves (1024; the kernel checks it).  The combined
+// table sits at the absolute address 64 K, so that one byte permute of a distance byte and a per-thread
+// register holding (1 << 16 | byte offset) gives the full shared-memory address of a lookup (no add).
+// Region A, from the start up to 64 K: the control area, then as many 2 KB B blocks (16 keys of V in
+// fp16 each) as fit; region C, from 128 K on: the remaining B blocks, then the logits tile.
+constexpr uint32_t kTabAbs = 0x10000;
+constexpr uint32_t LUT_BYTE = 128;                    // i-exp copies in a table line
+// control area (offsets from the start of dynamic shared memory)
+constexpr uint32_t C_SH = 0;                          // TcShared
+constexpr uint32_t C_ONES = 256;                      // 16 x 16 fp16 ones: B of the row sums of P
+constexpr uint32_t C_LUTF = 1024;                     // fp32 of the i-exp values (exact: <= 16 bits)
+constexpr uint32_t C_RMAX = 2048;                     // int [4][128]: row maxima of the parts
+constexpr uint32_t C_RSUM = 4096;                     // u64 [4][128]: row sums of the parts
+constexpr uint32_t C_GT = 8192;                       // u32 [32][20]: thresholds per (lane, 16-line group)
 constexpr int GT_LD = 20;                             //   (row stride 20 words: 16-byte loads without conflicts)
-constexpr uint32_t BK_OFF = GT_OFF + 32 * GT_LD * 4;  // u16 [1024] threshold buckets, or {hi, lo, hibits} [128]
+constexpr uint32_t C_BK = C_GT + 32 * GT_LD * 4;      // u16 [1024] threshold buckets, or {hi, lo, hibits} [128]
                                                       //   of the rows (scales whose i-exp values rise)
-constexpr uint32_t LG_OFF = BK_OFF + 2048;            // logits tile TM x ld, then B (1024-aligned)
+constexpr uint32_t C_END = C_BK + 2048;
+constexpr uint32_t kBlk = 16 * 64 * 2;                // one B block: 16 keys x 64 values, fp16
+constexpr uint32_t kSmemOptin = 232448;               // dynamic shared memory a CTA may have
+
+struct TcLayout {
+    uint32_t tab;  // offset of the table (absolute kTabAbs)
+    uint32_t bA;   // offset of the first B block of region A (1024-aligned address)
+    int nA;        // B blocks in region A
+    uint32_t bC;   // offset of region C (absolute 2 kTabAbs)
+    uint32_t lg;   // offset of the logits tile
+    uint32_t need; // dynamic bytes the layout spans
+    bool fits;
+};
+
+// Layout for dynamic shared memory at absolute address base (a multiple of 1024), nblocks B blocks and a
+// logits tile of lg_bytes
+__host__ __device__ inline TcLayout tc_layout(uint32_t base, int nblocks, uint32_t lg_bytes)
+{
+    TcLayout l;
+    l.fits = base + C_END <= kTabAbs;
+    l.tab = kTabAbs - base;
+    const uint32_t a0 = (base + C_END + 1023u) & ~1023u;
+    const int navail = a0 < kTabAbs ? (int)((kTabAbs - a0) / kBlk) : 0;
+    l.nA = navail < nblocks ? navail : nblocks;
+    l.bA = a0 - base;
+    l.bC = 2 * kTabAbs - base;
+    l.lg = l.bC + (uint32_t)(nblocks - l.nA) * kBlk;
+    l.need = l.lg + lg_bytes;
+    l.fits = l.fits && l.need <= kSmemOptin;
+    return l;
+}
 
 // Threshold buckets.  delta_k = #{d : e(d) > T} with T = 2S / D_k (i-exp values never rising with d).
 // T is approximated by T' = fp32(fp32(2S) * fp32(1 / D_k)), within 2^-22 of T; the bucket of T' (its
@@ -108,7 +147,9 @@ constexpr uint32_t LG_OFF = BK_OFF + 2048;            // logits tile TM x ld, th
 constexpr int BK_SHIFT = 17;
 constexpr int BK_N = 1024;
 
-// fp32 1 / D_k for k = 1 .. 15 (D_1 = 3, D_k = 3 2^(k-1) - 1)
+// D_k and fp32 1 / D_k for k = 1 .. 15 (D_1 = 3, D_k = 3 2^(k-1) - 1)
+__constant__ float kD[16] = {0.0f,    3.0f,    5.0f,    11.0f,   23.0f,   47.0f,    95.0f,    191.0f,
+                             383.0f,  767.0f,  1535.0f, 3071.0f, 6143.0f, 12287.0f, 24575.0f, 49151.0f};
 __constant__ float kRcpD[16] = {0.0f,          1.0f / 3.0f,     1.0f / 5.0f,     1.0f / 11.0f,
                                 1.0f / 23.0f,  1.0f / 47.0f,    1.0f / 95.0f,    1.0f / 191.0f,
                                 1.0f / 383.0f, 1.0f / 767.0f,   1.0f / 1535.0f,  1.0f / 3071.0f,
@@ -135,6 +176,7 @@ struct TcParams {
     uint8_t *out8;  // when not null: 8-bit outputs (requant8 with n1, n2, zp8) instead of acc
     int64_t ld_out8;
     int n1, n2, zp8;
+    uint32_t smem;  // dynamic shared memory of the launch
 };
 
 // A tile: rows g0 .. g0 + rows - 1 of the [BH * L] logit rows; the first nsplit belong to head h0,
@@ -187,9 +229,9 @@ __device__ __forceinline__ TileInfo next_tile(TileInfo ti, int L, int64_t total)
 
 struct TcShared {
     uint64_t lload, lfree, afull, mmadone, fin;
+    TcLayout ly;
     IexpC c;
     uint32_t tmem;
-    uint32_t b_off;  // offset of the B operand in dynamic shared memory (1024-aligned address)
     int bk0, bkmax;  // bucket number of table entry 0, and of the last entry
     int abort_flag;
     int rising;   // some i-exp value exceeds the one before it (floored constants)
@@ -213,20 +255,38 @@ __device__ __forceinline__ void epi_bar()
     asm volatile("bar.sync 2, 128;" ::: "memory");
 }
 
-// byte J of the distance word v in bits 8..15, byte 0 of the offset register o in bits 0..7: the
-// table address (d << 8) | offset.  o < 256, so its bytes 1..3 are the zero bytes of the result.
+// byte J of the distance word v in bits 8..15, bytes 0 and 2 of the offset register o = (1 << 16) |
+// offset in bits 0..7 and 16..23: the absolute table address kTabAbs | d << 8 | offset
 template <int J>
 __device__ __forceinline__ uint32_t tab_addr(uint32_t v, uint32_t o)
 {
     uint32_t y;
-    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(y) : "r"(v), "r"(o), "n"(0x5504 | (J << 4)));
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(y) : "r"(v), "r"(o), "n"(0x7604 | (J << 4)));
     return y;
 }
 
-// word of the table at byte offset a (a multiple of 4)
-__device__ __forceinline__ uint32_t tab32(const unsigned char *tab, uint32_t a)
+// shared-memory accesses at absolute addresses
+// (volatile: the compiler keeps them between the barriers that order the table's writes and reads)
+__device__ __forceinline__ uint32_t lds_u32(uint32_t a)
 {
-    return *reinterpret_cast<const uint32_t *>(tab + TAB_OFF + a);
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ uint32_t lds_u8(uint32_t a)
+{
+    uint32_t v;
+    asm volatile("ld.shared.u8 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ void sts_u32(uint32_t a, uint32_t v) { asm volatile("st.shared.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory"); }
+__device__ __forceinline__ void sts_zero16(uint32_t a)
+{
+    asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" ::"r"(a), "r"(0u) : "memory");
+}
+__device__ __forceinline__ void red_add_u32(uint32_t a, uint32_t v)
+{
+    asm volatile("red.shared.add.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
 }
 
 // the fp16 pair (high bytes b0 of t0 and b1 of t1; low bytes zero) for two keys
@@ -237,22 +297,35 @@ __device__ __forceinline__ uint32_t pack_ops(uint32_t t0, uint32_t t1)
     return y;
 }
 
-// V rows of one head (int8, L x 64) -> fp16 B (MN-major, 128-byte swizzled rows), rows of keys at
-// or past L up to the last 16-key step zero.  The 128 read-out threads: thread t takes 16 values
-// (16 (t % 4) ..) of keys t / 4, t / 4 + 32, ...
-__device__ __forceinline__ void convert_v(const int8_t *vh, int L, int nkeys, unsigned char *Bs, int t)
+// Where the B blocks are: the first nA at offset bA of dynamic shared memory, the rest at bC
+struct BlkMap {
+    uint32_t bA, bC;
+    int nA;
+};
+
+// Offset of B block blk (16 keys of one V buffer) in dynamic shared memory
+__device__ __forceinline__ uint32_t blk_off(const BlkMap &bm, int blk)
+{
+    return blk < bm.nA ? bm.bA + (uint32_t)blk * kBlk : bm.bC + (uint32_t)(blk - bm.nA) * kBlk;
+}
+
+// V rows of one head (int8, L x 64) -> fp16 B (MN-major, 128-byte swizzled rows) in the B blocks
+// blk0 .., rows of keys at or past L up to the last 16-key step zero.  The 128 read-out threads:
+// thread t takes 16 values (16 (t % 4) ..) of keys t / 4, t / 4 + 32, ...
+__device__ __forceinline__ void convert_v(const int8_t *vh, int L, int nkeys, unsigned char *dsm, const BlkMap &bm,
+                                          int blk0, int t)
 {
     const int c4 = t & 3;
-    for (int j0 = t >> 2; j0 < nkeys; j0 += 4 * 32) {
-        uint4 x[4];
+    for (int j0 = t >> 2; j0 < nkeys; j0 += 8 * 32) {
+        uint4 x[8];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < 8; ++u) {
             const int j = j0 + 32 * u;
             x[u] = (j < L) ? __ldg(reinterpret_cast<const uint4 *>(vh + (size_t)j * TD + 16 * c4))
                            : make_uint4(0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u);
         }
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < 8; ++u) {
             const int j = j0 + 32 * u;
             if (j >= nkeys) break;
             uint4 a = make_uint4(0, 0, 0, 0), b = make_uint4(0, 0, 0, 0);
@@ -264,7 +337,7 @@ __device__ __forceinline__ void convert_v(const int8_t *vh, int L, int nkeys, un
                 b = make_uint4(i8x2_to_h2(x2, 0x5140), i8x2_to_h2(x2, 0x7362), i8x2_to_h2(x3, 0x5140),
                                i8x2_to_h2(x3, 0x7362));
             }
-            unsigned char *row = Bs + (size_t)j * 128;
+            unsigned char *row = dsm + blk_off(bm, blk0 + (j >> 4)) + (uint32_t)(j & 15) * 128;
             *reinterpret_cast<uint4 *>(row + (((2 * c4) ^ (j & 7)) << 4)) = a;
             *reinterpret_cast<uint4 *>(row + (((2 * c4 + 1) ^ (j & 7)) << 4)) = b;
         }
@@ -323,17 +396,16 @@ template <int NKB, bool SMALL_E, bool PACK>
 __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
 {
     extern __shared__ __align__(1024) unsigned char dsm[];
-    __shared__ TcShared sh;
-    __shared__ float LUTF[256];                    // fp32 of the i-exp values (exact: <= 16 bits)
-    __shared__ __align__(128) uint32_t ONES[128];  // 16 x 16 fp16 ones: B of the row sums of P
-    int *red_max = reinterpret_cast<int *>(dsm + RMAX_OFF);
-    unsigned long long *red_sum = reinterpret_cast<unsigned long long *>(dsm + RSUM_OFF);
-    uint32_t *GT = reinterpret_cast<uint32_t *>(dsm + GT_OFF);
-    uint16_t *BK = reinterpret_cast<uint16_t *>(dsm + BK_OFF);
-    float *rs_hi = reinterpret_cast<float *>(dsm + BK_OFF);
+    TcShared &sh = *reinterpret_cast<TcShared *>(dsm + C_SH);
+    uint32_t *ONES = reinterpret_cast<uint32_t *>(dsm + C_ONES);
+    float *LUTF = reinterpret_cast<float *>(dsm + C_LUTF);
+    int *red_max = reinterpret_cast<int *>(dsm + C_RMAX);
+    unsigned long long *red_sum = reinterpret_cast<unsigned long long *>(dsm + C_RSUM);
+    uint32_t *GT = reinterpret_cast<uint32_t *>(dsm + C_GT);
+    uint16_t *BK = reinterpret_cast<uint16_t *>(dsm + C_BK);
+    float *rs_hi = reinterpret_cast<float *>(dsm + C_BK);
     float *rs_lo = rs_hi + TM;
     int *rs_bits = reinterpret_cast<int *>(rs_lo + TM);
-    unsigned char *LG = dsm + LG_OFF;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile int *abort_flag = &sh.abort_flag;
@@ -341,6 +413,16 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     const int L = p.L;
     const int nsteps = (L + 15) >> 4;  // MMA K steps of 16 keys
     pdl_release();
+    {
+        // the layout for this CTA's shared-memory window; a window other than the expected one, or too
+        // small, is reported (FQVIT_ERR_UNSUPPORTED) instead of run
+        const TcLayout ly = tc_layout(sa(dsm), (PACK ? 2 : 1) * nsteps, (uint32_t)(TM * p.ld));
+        if (!ly.fits || ly.need > p.smem || (sa(dsm) & 1023u) != 0) {
+            if (tid == 0) atomicCAS(&g_status, 0, 2);
+            return;
+        }
+        if (tid == 0) sh.ly = ly;
+    }
     if (tid == 0) {
         mbar_init(&sh.lload, 1);
         mbar_init(&sh.lfree, TSOFT);
@@ -352,8 +434,6 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
         sh.stop = 0;
         sh.ew_stop = 0;
         sh.c = p.ic;
-        const uint32_t lg_end = sa(dsm) + LG_OFF + (uint32_t)(TM * p.ld);
-        sh.b_off = ((lg_end + 1023u) & ~1023u) - sa(dsm);
     }
     if (warp == TMMA_WARP) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(&sh.tmem)),
@@ -364,8 +444,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     {
         const IexpC c = sh.c;
         for (int i = tid; i < 256 * 32; i += blockDim.x)
-            *reinterpret_cast<uint32_t *>(dsm + TAB_OFF + (uint32_t)(i >> 5) * 256u + LUT_BYTE + 4u * (i & 31)) =
-                iexp_neg(i >> 5, c);
+            sts_u32(kTabAbs + (uint32_t)(i >> 5) * 256u + LUT_BYTE + 4u * (i & 31), iexp_neg(i >> 5, c));
         for (int d = tid; d < 256; d += blockDim.x) LUTF[d] = __uint2float_rn(iexp_neg(d, c));
         for (int i = tid; i < 128; i += blockDim.x) ONES[i] = 0x3C003C00u;
         for (int d = tid; d < 255; d += blockDim.x)
@@ -399,8 +478,6 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = sh.tmem;
-    unsigned char *Bs = dsm + sh.b_off;
-    const uint32_t b_bytes = (uint32_t)nsteps * KSTEP_B;  // one V buffer
     pdl_wait();  // the set-up above touched no global memory
 
     const int tpb = (L + TM - 1) / TM;
@@ -414,15 +491,21 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     if (tid < TSOFT) {
         const int k4 = warp & 3, q = warp >> 2;
         const int r = 32 * k4 + lane;                    // row of the tile = tensor-memory lane
-        const uint32_t rowb = 4u * (uint32_t)lane + (uint32_t)k4;  // this row's byte in a table line
-        const uint32_t lutb = LUT_BYTE + 4u * (uint32_t)lane;      // this lane's i-exp copy in a line
+        // offset registers of the table lookups (1 << 16 selects the table's 64 K page): this row's byte
+        // in a line, and this lane's i-exp copy in a line
+        const uint32_t rowb = 0x10000u | (4u * (uint32_t)lane + (uint32_t)k4);
+        const uint32_t lutb = 0x10000u | (LUT_BYTE + 4u * (uint32_t)lane);
         const uint32_t tlane = tmem + ((uint32_t)(k4 * 32) << 16);
         const bool monotone = !sh.rising;  // codes never fall as d grows
         const uint32_t inc = 1u << (8 * k4);  // this row's byte of a table word
-        // keys of this part in the last 64-key block (0 .. 16; every other block holds 16)
-        const int last_keys = min(16, max(0, L - ((NKB - 1) * TKB + 16 * q)));
-        // keys at or past L inside this part's last partial block (summed as -128, then removed)
-        const int npad = last_keys > 0 ? 16 - last_keys : 0;
+        // The last 64-key block holds R = 1 .. 64 keys (every other block holds 16 per part).  With R > 16
+        // part q takes keys 16 q .. 16 q + 15 of it; with R <= 16 (one 16-key MMA step) the four parts
+        // take 4 keys each, 4 q .. 4 q + 3, so that no part does a whole extra chunk for a few keys.
+        const int R = L - (NKB - 1) * TKB;
+        const bool quarter = R <= 16;
+        const int last_keys = quarter ? min(4, max(0, R - 4 * q)) : min(16, max(0, R - 16 * q));
+        // keys at or past L inside this part's last slice (summed as -128, then removed)
+        const int npad = last_keys > 0 ? (quarter ? 4 : 16) - last_keys : 0;
         bool wait_bad = false;
         TileInfo ti = tile_info<PACK>(t_begin, L, p.BH, tpb);
         for (int it = 0; it < ncta_tiles; ++it, ti = next_tile<PACK>(ti, L, total)) {
@@ -435,10 +518,18 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
 #pragma unroll
             for (int kb = 0; kb < NKB; ++kb) w[kb] = make_uint4(0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u);
             if (valid) {
-                const unsigned char *lr = LG + (size_t)r * p.ld + 16 * q;
+                const unsigned char *lr = dsm + sh.ly.lg + (size_t)r * p.ld + 16 * q;
 #pragma unroll
                 for (int kb = 0; kb < NKB - 1; ++kb) w[kb] = *reinterpret_cast<const uint4 *>(lr + kb * TKB);
-                if (last_keys > 0) {
+                if (quarter) {
+                    if (last_keys > 0) {
+                        uint32_t x = *reinterpret_cast<const uint32_t *>(lr - 16 * q + (NKB - 1) * TKB + 4 * q);
+                        if (last_keys < 4)
+                            x = (x & (0xFFFFFFFFu >> (32 - 8 * last_keys))) |
+                                (0x80808080u & ~(0xFFFFFFFFu >> (32 - 8 * last_keys)));
+                        w[NKB - 1].x = x;
+                    }
+                } else if (last_keys > 0) {
                     uint4 x = *reinterpret_cast<const uint4 *>(lr + (NKB - 1) * TKB);
                     if (last_keys < 16) {
                         uint32_t ww[4] = {x.x, x.y, x.z, x.w};
@@ -480,7 +571,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const uint32_t c = (uint32_t)(tid + TSOFT * i);
-                *reinterpret_cast<uint4 *>(dsm + TAB_OFF + (c >> 3) * 256u + (c & 7u) * 16u) = make_uint4(0, 0, 0, 0);
+                sts_zero16(kTabAbs + (c >> 3) * 256u + (c & 7u) * 16u);
             }
             GT[tid] = 0u;
             if (tid < 32 * GT_LD - TSOFT) GT[TSOFT + tid] = 0u;
@@ -504,10 +595,10 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                         uint32_t a = 0;
 #pragma unroll
                         for (int b = 0; b < 4; ++b) {
-                            const uint32_t e0 = tab32(dsm, tab_addr<0>(ww[b], lutb));
-                            const uint32_t e1 = tab32(dsm, tab_addr<1>(ww[b], lutb));
-                            const uint32_t e2 = tab32(dsm, tab_addr<2>(ww[b], lutb));
-                            const uint32_t e3 = tab32(dsm, tab_addr<3>(ww[b], lutb));
+                            const uint32_t e0 = lds_u32(tab_addr<0>(ww[b], lutb));
+                            const uint32_t e1 = lds_u32(tab_addr<1>(ww[b], lutb));
+                            const uint32_t e2 = lds_u32(tab_addr<2>(ww[b], lutb));
+                            const uint32_t e3 = lds_u32(tab_addr<3>(ww[b], lutb));
                             a += e0 + e1;
                             a += e2 + e3;
                         }
@@ -515,19 +606,27 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                     } else {
 #pragma unroll
                         for (int b = 0; b < 4; ++b) {
-                            const uint32_t e0 = tab32(dsm, tab_addr<0>(ww[b], lutb));
-                            const uint32_t e1 = tab32(dsm, tab_addr<1>(ww[b], lutb));
-                            const uint32_t e2 = tab32(dsm, tab_addr<2>(ww[b], lutb));
-                            const uint32_t e3 = tab32(dsm, tab_addr<3>(ww[b], lutb));
+                            const uint32_t e0 = lds_u32(tab_addr<0>(ww[b], lutb));
+                            const uint32_t e1 = lds_u32(tab_addr<1>(ww[b], lutb));
+                            const uint32_t e2 = lds_u32(tab_addr<2>(ww[b], lutb));
+                            const uint32_t e3 = lds_u32(tab_addr<3>(ww[b], lutb));
                             S += (unsigned long long)(e0 + e1) + (unsigned long long)(e2 + e3);  // e < 2^31
                         }
                     }
                 };
 #pragma unroll
                 for (int kb = 0; kb < NKB - 1; ++kb) sum16(w[kb]);
-                if (last_keys > 0) sum16(w[NKB - 1]);
+                if (quarter) {
+                    if (last_keys > 0) {
+                        const uint32_t x = w[NKB - 1].x;
+                        S += (unsigned long long)(lds_u32(tab_addr<0>(x, lutb)) + lds_u32(tab_addr<1>(x, lutb))) +
+                             (unsigned long long)(lds_u32(tab_addr<2>(x, lutb)) + lds_u32(tab_addr<3>(x, lutb)));
+                    }
+                } else if (last_keys > 0) {
+                    sum16(w[NKB - 1]);
+                }
                 // the padding bytes (-128, distance m + 128)
-                S -= (unsigned long long)npad * tab32(dsm, ((uint32_t)(m + 128) << 8) + lutb);
+                S -= (unsigned long long)npad * lds_u32(((uint32_t)(m + 128) << 8) + lutb);
             }
             red_sum[q * TM + r] = S;
             soft_bar();  // B
@@ -540,37 +639,48 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                     // e(d) D_k <= 2S, exact: one rounding of an exact product minus hi, against lo
                     auto hit = [&](int d, float D) -> bool { return __fmaf_rn(LUTF[d], D, -rs.hi) <= rs.lo; };
                     const int bk0 = sh.bk0, bkmax = sh.bkmax;
+                    // the four searches run side by side (independent chains)
+                    float D[4];
+                    int lo[4], n[4];  // delta_k in [lo, lo + n]
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
-                        const int k = q + 1 + 4 * i;
-                        if (k > 15) break;
-                        const float D = k == 1 ? 3.0f : (float)(3 * (1 << (k - 1)) - 1);
-                        const int b = (int)(__float_as_uint(rs.hi * kRcpD[k]) >> BK_SHIFT);
-                        int lo, n;  // delta_k in [lo, lo + n]
-                        if (b > bkmax) {
-                            lo = 0, n = 0;
-                        } else if (b < bk0) {
-                            lo = 256, n = 0;
+                        const int k = min(q + 1 + 4 * i, 15);
+                        D[i] = kD[k];
+                        const int b = (int)(__float_as_uint(rs.hi * kRcpD[k]) >> BK_SHIFT) - bk0;
+                        if ((unsigned)b < (unsigned)BK_N) {
+                            const uint32_t v = BK[b];
+                            lo[i] = (int)(v & 511u);
+                            n[i] = (int)(v >> 9);
+                            if (n[i] == 127) n[i] = 256 - lo[i];
                         } else {
-                            const uint32_t v = BK[b - bk0];
-                            lo = (int)(v & 511u);
-                            n = (int)(v >> 9);
-                            if (n == 127) n = 256 - lo;
+                            lo[i] = b < 0 ? 256 : 0;  // below the buckets: every value lies above T
+                            n[i] = 0;
                         }
-                        while (n > 0) {  // the first d in [lo, lo + n) that hits, else lo + n
-                            const int h = n >> 1;
-                            if (hit(lo + h, D)) {
-                                n = h;
-                            } else {
-                                lo += h + 1;
-                                n -= h + 1;
+                    }
+                    (void)bkmax;
+                    // the first d in [lo, lo + n) that hits, else lo + n (binary search)
+                    for (int step = 0; step < 9; ++step) {
+                        bool more = false;
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            if (n[i] > 0) {
+                                const int h = n[i] >> 1;
+                                if (hit(lo[i] + h, D[i])) {
+                                    n[i] = h;
+                                } else {
+                                    lo[i] += h + 1;
+                                    n[i] -= h + 1;
+                                }
+                                more |= n[i] > 0;
                             }
                         }
-                        if (lo < 256) {
-                            atomicAdd(reinterpret_cast<unsigned int *>(dsm + TAB_OFF + ((uint32_t)lo << 8) +
-                                                                       4u * (uint32_t)lane),
-                                      inc);
-                            atomicAdd(&GT[lane * GT_LD + (lo >> 4)], inc);
+                        if (!more) break;
+                    }
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        if (q + 1 + 4 * i <= 15 && lo[i] < 256) {
+                            red_add_u32(kTabAbs + ((uint32_t)lo[i] << 8) + 4u * (uint32_t)lane, inc);
+                            atomicAdd(&GT[lane * GT_LD + (lo[i] >> 4)], inc);
                         }
                     }
                 }
@@ -594,12 +704,14 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
 #pragma unroll
                         for (int j = 0; j < 15; ++j) carry += j < g ? gv[j] : 0u;
                     }
+                    const uint32_t a0 = kTabAbs + (uint32_t)(16 * g) * 256u + 4u * (uint32_t)lane;
+                    uint32_t h[16];  // the 16 loads first: the running sum then has no load in its chain
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) h[i] = lds_u32(a0 + 256u * i);
 #pragma unroll
                     for (int i = 0; i < 16; ++i) {
-                        uint32_t *wp = reinterpret_cast<uint32_t *>(dsm + TAB_OFF + (uint32_t)(16 * g + i) * 256u +
-                                                                    4u * (uint32_t)lane);
-                        carry += *wp;
-                        *wp = 0x78787878u - 4u * carry;  // 4 (30 - code) per byte
+                        carry += h[i];
+                        sts_u32(a0 + 256u * i, 0x78787878u - 4u * carry);  // 4 (30 - code) per byte
                     }
                 } else {
 #pragma unroll 1
@@ -613,7 +725,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                             const uint32_t E = operand_exp_f(ef, rs_bits[rr], rs_hi[rr], rs_lo[rr]);
                             word |= (4u * E) << (8 * k);
                         }
-                        *reinterpret_cast<uint32_t *>(dsm + TAB_OFF + (uint32_t)d * 256u + 4u * (uint32_t)lane) = word;
+                        sts_u32(kTabAbs + (uint32_t)d * 256u + 4u * (uint32_t)lane, word);
                     }
                 }
             }
@@ -629,31 +741,40 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                     const uint32_t ww[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
                     for (int b = 0; b < 4; ++b) {
-                        const uint32_t t0 = dsm[TAB_OFF + tab_addr<0>(ww[b], rowb)];
-                        const uint32_t t1 = dsm[TAB_OFF + tab_addr<1>(ww[b], rowb)];
-                        const uint32_t t2 = dsm[TAB_OFF + tab_addr<2>(ww[b], rowb)];
-                        const uint32_t t3 = dsm[TAB_OFF + tab_addr<3>(ww[b], rowb)];
+                        const uint32_t t0 = lds_u8(tab_addr<0>(ww[b], rowb));
+                        const uint32_t t1 = lds_u8(tab_addr<1>(ww[b], rowb));
+                        const uint32_t t2 = lds_u8(tab_addr<2>(ww[b], rowb));
+                        const uint32_t t3 = lds_u8(tab_addr<3>(ww[b], rowb));
                         o[2 * b] = pack_ops(t0, t1);
                         o[2 * b + 1] = pack_ops(t2, t3);
                     }
                 };
+                // (rows past the tile's end take whatever their padding bytes give: their accumulator rows
+                // are never read, and a row of D depends only on its own row of operands)
 #pragma unroll
                 for (int kb = 0; kb < NKB - 1; ++kb) {
-                    uint32_t o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                    if (valid) ops16(w[kb], o);
+                    uint32_t o[8];
+                    ops16(w[kb], o);
                     tmem_st8(tlane + TA + 32 * kb + 8 * q, o);
                 }
-                if (last_keys > 0) {  // warp-uniform
-                    uint32_t o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                    if (valid) {
-                        ops16(w[NKB - 1], o);
+                if (quarter) {  // every part writes its 2 columns of the last MMA step (zeros past L)
+                    const uint32_t x = w[NKB - 1].x;
+                    uint32_t o0 = pack_ops(lds_u8(tab_addr<0>(x, rowb)), lds_u8(tab_addr<1>(x, rowb)));
+                    uint32_t o1 = pack_ops(lds_u8(tab_addr<2>(x, rowb)), lds_u8(tab_addr<3>(x, rowb)));
+                    if (last_keys < 4) {
+                        o1 = last_keys <= 2 ? 0u : (o1 & 0xFFFFu);
+                        if (last_keys < 2) o0 = last_keys == 1 ? (o0 & 0xFFFFu) : 0u;
+                    }
+                    tmem_st2(tlane + TA + 32 * (NKB - 1) + 2 * q, o0, o1);
+                } else if (last_keys > 0) {  // warp-uniform
+                    uint32_t o[8];
+                    ops16(w[NKB - 1], o);
 #pragma unroll
-                        for (int c = 0; c < 8; ++c) {  // keys at or past L get a zero operand
-                            if (2 * c >= last_keys)
-                                o[c] = 0;
-                            else if (2 * c + 1 == last_keys)
-                                o[c] &= 0xFFFFu;
-                        }
+                    for (int c = 0; c < 8; ++c) {  // keys at or past L get a zero operand
+                        if (2 * c >= last_keys)
+                            o[c] = 0;
+                        else if (2 * c + 1 == last_keys)
+                            o[c] &= 0xFFFFu;
                     }
                     tmem_st8(tlane + TA + 32 * (NKB - 1) + 8 * q, o);
                 }
@@ -671,7 +792,9 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
         volatile int *ew_stop = &sh.ew_stop;
         int conv_hi = -1;  // the last head whose V went into its B buffer
         int ncopies = 0;
-        auto bbuf = [&](int h) -> unsigned char * { return Bs + (PACK ? (uint32_t)(h & 1) * b_bytes : 0u); };
+        auto blk0 = [&](int h) -> int { return PACK ? (h & 1) * nsteps : 0; };  // first B block of head h's V
+        const BlkMap bm{sh.ly.bA, sh.ly.bC, sh.ly.nA};
+        unsigned char *LG = dsm + sh.ly.lg;
         auto last_head = [](const TileInfo &t) { return t.nsplit < t.rows ? t.h0 + 1 : t.h0; };
         TileInfo ti = tile_info<PACK>(t_begin, L, p.BH, tpb);
         TileInfo tp = ti;  // the previous tile
@@ -729,7 +852,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
             // V of this tile's head(s) not yet in B
             if (ok) {
                 for (int h = max(conv_hi + 1, ti.h0); h <= last_head(ti); ++h) {
-                    convert_v(p.v + (size_t)h * L * TD, L, 16 * nsteps, bbuf(h), et);
+                    convert_v(p.v + (size_t)h * L * TD, L, 16 * nsteps, dsm, bm, blk0(h), et);
                     conv_hi = h;
                 }
             }
@@ -744,10 +867,18 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                     const uint64_t ones = smem_desc_plain(sa(ONES), 128, 256);
                     const int nh = (PACK && ti.nsplit < ti.rows) ? 2 : 1;
                     for (int hh = 0; hh < nh; ++hh) {
-                        const uint32_t b0 = sa(bbuf(ti.h0 + hh));
+                        const int bb = blk0(ti.h0 + hh);
                         const uint32_t dcol = tmem + (uint32_t)(hh * TD);
-                        for (int s = 0; s < nsteps; ++s)
-                            mma_f16_ta(dcol, tmem + TA + 8 * s, smem_desc(b0 + KSTEP_B * s, 1024, 1024), s != 0);
+                        // the blocks in order, region A's then region C's: a descriptor's address field
+                        // (address / 16) grows by kBlk / 16 per block
+                        uint64_t da = smem_desc(sa(dsm) + blk_off(bm, bb), 1024, 1024);
+                        const uint64_t dc = smem_desc(sa(dsm) + bm.bC, 1024, 1024);
+                        uint32_t at = tmem + TA;
+                        for (int s = 0; s < nsteps; ++s) {
+                            mma_f16_ta(dcol, at, da, s != 0);
+                            at += 8;
+                            da = (bb + s + 1 == bm.nA) ? dc : da + (kBlk >> 4);
+                        }
                     }
                     if (p.zp != 0)
                         for (int s = 0; s < nsteps; ++s)
@@ -778,17 +909,13 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tmem_cols(NKB, PACK)));
 }
 
-// dynamic shared memory of a launch (the B buffers after the logits tile, 1024-aligned; up to 1008
-// bytes of alignment slack when the dynamic window itself is only 16-byte aligned)
-size_t tc_smem_bytes(int L, int64_t ld, bool pack)
+// Dynamic shared memory of a launch: the layout's extent with the window at its expected start (1024:
+// the kernel has no static shared memory), or 0 when it does not fit.
+uint32_t tc_smem_bytes(int L, int64_t ld, bool pack)
 {
-    const size_t nsteps = (size_t)(L + 15) / 16;
-    const size_t lg_end = LG_OFF + (size_t)TM * ld;
-    return ((lg_end + 1023) & ~(size_t)1023) + 1008 + (pack ? 2 : 1) * nsteps * KSTEP_B;
+    const TcLayout l = tc_layout(1024u, (pack ? 2 : 1) * ((L + 15) / 16), (uint32_t)(TM * ld));
+    return l.fits ? l.need : 0u;
 }
-
-// static shared memory of the kernel: the control block, the fp32 i-exp table, the ones block
-constexpr size_t kTcStaticSmem = 2048;
 
 bool use_pack(int L) { return L >= TM && L <= kPackMaxBlocks * TKB; }
 
@@ -823,15 +950,15 @@ bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b)
                                : (b.ld_acc == TD && ((uintptr_t)b.acc % 32) == 0);
     return b.d == TD && a.bias == nullptr && a.region == nullptr && a.codes == nullptr && a.L <= TMAXKB * TKB &&
            a.ld_logit % 16 == 0 && b.ld_v == TD && out_ok && ((uintptr_t)a.logits % 16) == 0 &&
-           ((uintptr_t)b.v % 16) == 0 && tc_smem_bytes(a.L, a.ld_logit, use_pack(a.L)) + kTcStaticSmem <= 232448;
+           ((uintptr_t)b.v % 16) == 0 && a.ld_logit <= 1024 && tc_smem_bytes(a.L, a.ld_logit, use_pack(a.L)) > 0;
 }
 
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st)
 {
-    TcParams p{a.logits, a.ld_logit, b.v, b.acc, b.BH, a.L, b.zp_v, iexp_consts_host(a.s_logit),
-               b.out8, b.ld_out8, b.rq_n1, b.rq_n2, b.rq_zp};
     const bool pack = use_pack(a.L);
-    const size_t smem = tc_smem_bytes(a.L, a.ld_logit, pack);
+    const uint32_t smem = tc_smem_bytes(a.L, a.ld_logit, pack);
+    TcParams p{a.logits, a.ld_logit, b.v, b.acc, b.BH, a.L, b.zp_v, iexp_consts_host(a.s_logit),
+               b.out8, b.ld_out8, b.rq_n1, b.rq_n2, b.rq_zp, smem};
     const int64_t ntiles = pack ? (b.BH * a.L + TM - 1) / TM : b.BH * ((a.L + TM - 1) / TM);
     const int grid = (int)(ntiles < sm_count() ? ntiles : sm_count());
     const bool se = small_iexp(p.ic);

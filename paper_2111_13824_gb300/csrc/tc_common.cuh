@@ -209,6 +209,13 @@ __device__ __forceinline__ int sbyte(uint32_t w)
     return (int)y;
 }
 
+// warp-collective (.sync.aligned): the whole warp, converged, writes its 32 lanes (2 columns)
+__device__ __forceinline__ void tmem_st2(uint32_t taddr, uint32_t r0, uint32_t r1)
+{
+    __syncwarp();
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x2.b32 [%0], {%1,%2};" ::"r"(taddr), "r"(r0), "r"(r1) : "memory");
+}
+
 // warp-collective (.sync.aligned): the whole warp, converged, writes its 32 lanes (4 columns)
 __device__ __forceinline__ void tmem_st4(uint32_t taddr, const uint32_t (&r)[4])
 {
