@@ -33,6 +33,7 @@ import subprocess
 import sys
 import time
 
+import numpy as np
 import torch
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -287,56 +288,6 @@ class ClockSampler:
 
 # ------------------------------------------------------------------ CPU oracle baseline
 
-class OracleSample:
-    """A bounded sample of one layer for the CPU oracle, scaled to the whole step.
-
-    Sample: the LayerNorm of `ln_rows` rows and the Log-Int-Softmax + BitShift
-    attn.V of `heads` attention heads of layer 0; the estimate scales the first by
-    the LayerNorm elements of the whole step (every layer, and Swin's patch
-    mergings) and the second by the step's attention logits."""
-
-    def __init__(self, cfg, heads=1, ln_rows=512, layer=0, qk=False):
-        import oracle
-
-        self.oracle = oracle
-        self.qk = qk
-        self.cfg, self.heads, self.ln_rows = cfg, heads, ln_rows
-        self.st = synth.layer_stage(cfg, layer)
-        d = synth.ln_inputs(cfg, layer, rows=ln_rows)
-        a = synth.attn_inputs(cfg, layer, bh=heads)
-        s, zp, alpha, _ = oracle.calibrate_ptf(d["x_calib"].numpy(), K=cfg.K)
-        self.ln = (oracle.ptf_quantize(d["x"].numpy(), s, zp, alpha), zp, alpha, d["gamma"].numpy(),
-                   d["beta"].numpy(), d["s_out"], d["zp_out"])
-        self.a = a
-        self.x, self.v = a["logits"].numpy(), a["v"].numpy()
-        self.bias = a["bias"].numpy() if a["bias"] is not None else None
-
-    def run(self):
-        """Returns (estimated seconds per step, seconds of CPU work spent)."""
-        o, a = self.oracle, self.a
-        t0 = time.perf_counter()
-        o.ptf_layernorm(*self.ln)
-        t1 = time.perf_counter()
-        x = self.x
-        if self.qk:  # the logits from Q and K first
-            x = o.qk_logits(a["q"].numpy(), a["k"].numpy(), 0, 0, a["s_q"], a["s_k"], a["s_logit"], a["zp_logit"],
-                            ld=synth.ld_pad(a["L"]))
-        co, _ = o.lis_softmax(x, a["L"], a["s_logit"], bias=self.bias, heads=a["heads"],
-                              window=a["window"] or 7)
-        o.lis_attn_v(co, self.v, 0)
-        t2 = time.perf_counter()
-        ln_elems, logits = step_elements(self.cfg)
-        step = ((t1 - t0) * ln_elems / (self.ln_rows * self.st.C)
-                + (t2 - t1) * logits / (self.heads * self.st.L * self.st.L))
-        return step, t2 - t0
-
-    def describe(self):
-        return (f"layer 0: LayerNorm of {self.ln_rows} of {self.st.rows} rows and "
-                f"{'Q K^T logits + ' if self.qk else ''}LIS + BitShift attn.V of "
-                f"{self.heads} of {self.st.BH} heads, scaled to the step's LayerNorm elements and attention "
-                f"logits ({self.cfg.layers} layers" + (", patch mergings)" if synth.merge_stages(self.cfg) else ")"))
-
-
 def step_elements(cfg):
     """(LayerNorm elements, attention logits) of one step over the whole config."""
     ln = sum(st.layers * st.rows * st.C for st in cfg.stages)
@@ -346,7 +297,270 @@ def step_elements(cfg):
     return ln, sum(st.layers * st.BH * st.L * st.L for st in cfg.stages)
 
 
+def _host(t):
+    return t.detach().cpu().numpy()
+
+
+class OracleLeg:
+    """The oracle, as it stands, on this host's cores, fed the GPU step's own resident inputs.
+
+    Timing: all of layer 0 (every LayerNorm row and every attention head) on all cores, and a
+    bounded part of it (256 rows, 2 heads; Swin: one image) on one core; each is scaled by the
+    step's LayerNorm elements and attention logits to the whole step.  Parity: the same layer-0
+    outputs, and sampled LayerNorm rows and heads of every other layer, compared element by
+    element with what the GPU step wrote."""
+
+    def __init__(self, cfg, layers, args):
+        import oracle
+
+        self.o, self.cfg, self.layers, self.args = oracle, cfg, layers, args
+        self.mismatch = []
+        self.checked_rows = self.checked_heads = 0
+
+    # -- the oracle on part of one layer, from that layer's resident inputs
+    def _ln(self, m, rows):
+        xq = _host(m["xq"][rows])
+        return self.o.ptf_layernorm(xq, m["zp"], _host(m["alpha"]), _host(m["gamma"]), _host(m["beta"]), m["s_out"],
+                                    m["zp_out"])[0]
+
+    def _attn(self, ly, h0, h1):
+        """Outputs of heads h0 .. h1 - 1 (Swin: whole images, so that bias and mask line up)."""
+        o, L = self.o, ly["L"]
+        if ly["qk"]:
+            x = o.qk_logits(_host(ly["q"][h0:h1]), _host(ly["k"][h0:h1]), 0, 0, ly["s_q"], ly["s_k"], ly["s_logit"],
+                            ly["zp_logit"], ld=synth.ld_pad(L))
+        else:
+            x = _host(ly["logits"][h0 * L:h1 * L])
+        bias = _host(ly["bias"]) if ly["bias"] is not None else None
+        reg = _host(ly["region"]) if ly["region"] is not None else None
+        co, _ = o.lis_softmax(x, L, ly["s_logit"], bias=bias, heads=ly["heads"], window=ly["window"] or 7, region=reg,
+                              mask_value=ly["mask_value"] if reg is not None else 0)
+        acc, _ = o.lis_attn_v(co, _host(ly["v"][h0:h1]), 0)
+        if self.args.out8:
+            return o.attn_requant(acc, OUT8_SV, OUT8_SV, 128)
+        return acc
+
+    def _gpu_attn(self, ly, h0, h1):
+        return _host((ly["out8"] if self.args.out8 else ly["acc"])[h0:h1])
+
+    def _head_unit(self, ly):
+        """Heads per independent unit: one head, or (windowed attention) one image's heads."""
+        return ly["BH"] // 64 if ly["window"] else 1
+
+    def _compare(self, what, got, want):
+        if not np.array_equal(got, want):
+            self.mismatch.append(f"{what}: {int((got != want).sum())} elements differ")
+
+    # -- the legs
+    def layer0_all_cores(self):
+        """Seconds of the LayerNorm and of the attention of all of layer 0, all cores; checks them."""
+        o, ly = self.o, self.layers[0]
+        o.set_num_threads(os.cpu_count() or 1)
+        t0 = time.perf_counter()
+        yo = self._ln(ly, slice(None))
+        t1 = time.perf_counter()
+        ao = self._attn(ly, 0, ly["BH"])
+        t2 = time.perf_counter()
+        self._compare("layer 0 LayerNorm", _host(ly["yq"]), yo)
+        self._compare("layer 0 attention", self._gpu_attn(ly, 0, ly["BH"]), ao)
+        self.checked_rows += ly["rows"]
+        self.checked_heads += ly["BH"]
+        return t1 - t0, t2 - t1
+
+    def layer0_one_core(self, rows=256, units=2):
+        o, ly = self.o, self.layers[0]
+        o.set_num_threads(1)
+        hu = self._head_unit(ly)
+        t0 = time.perf_counter()
+        self._ln(ly, slice(0, rows))
+        t1 = time.perf_counter()
+        self._attn(ly, 0, units * hu)
+        t2 = time.perf_counter()
+        o.set_num_threads(os.cpu_count() or 1)
+        return (t1 - t0) * ly["rows"] / rows, (t2 - t1) * ly["BH"] / (units * hu)
+
+    def other_layers(self, rows=64, units=2):
+        """Sampled rows and heads of every layer but 0 (and of every patch merging's LayerNorm)."""
+        for i, ly in enumerate(self.layers):
+            for m, tag in ((ly, f"layer {i}"), (ly["merge"], f"merge before layer {i}")):
+                if m is None or (i == 0 and m is ly):
+                    continue
+                sel = np.linspace(0, m["rows"] - 1, rows).astype(np.int64)
+                self._compare(f"{tag} LayerNorm", _host(m["yq"][torch.from_numpy(sel).to(m["yq"].device)]),
+                              self._ln(m, torch.from_numpy(sel).to(m["xq"].device)))
+                self.checked_rows += rows
+            if i == 0:
+                continue
+            hu = self._head_unit(ly)
+            nunit = ly["BH"] // hu
+            for u in sorted({(i * 7919) % nunit, nunit - 1 - (i * 104729) % nunit})[:units]:
+                self._compare(f"layer {i} attention unit {u}", self._gpu_attn(ly, u * hu, (u + 1) * hu),
+                              self._attn(ly, u * hu, (u + 1) * hu))
+                self.checked_heads += hu
+
+    def verdict(self):
+        n = len(self.layers)
+        if self.mismatch:
+            return "MISMATCH: " + "; ".join(self.mismatch[:4])
+        return (f"bit-exact against the oracle: all of layer 0, sampled rows and heads of the other {n - 1} "
+                f"layer(s) ({self.checked_rows} LayerNorm rows, {self.checked_heads} attention heads)")
+
+
 # ------------------------------------------------------------------ main arms
+
+def time_config(fqvit, cfg, layers, args, steps, warmup, dev, ws, sample_clocks=False):
+    """Times `steps` steps of the config's stack (one CUDA graph of the kernels, launched with
+    programmatic dependent launch), then a second pass with timing events around each kernel.
+    Returns the step time, the per-kernel times and byte rates, and the clock record."""
+    for _ in range(warmup):
+        for ly in layers:
+            run_layer(fqvit, ly)
+    torch.cuda.synchronize()
+
+    use_graph = not args.no_graph
+    ev_kw = dict(enable_timing=True)
+    if use_graph:
+        try:
+            torch.cuda.Event(enable_timing=True, external=True)
+            ev_kw["external"] = True
+        except TypeError:
+            use_graph = False
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    merges = [ly["merge"] for ly in layers if ly["merge"] is not None]
+    ev_steps = min(steps, 3)  # steps of the per-kernel timing pass
+    ev = {}
+
+    def new_events(kw):
+        ev["attn"] = [(torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(ev_steps * len(layers))]
+        ev["ln"] = [(torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(ev_steps * len(layers))]
+        ev["merge"] = [(torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(ev_steps * len(merges))]
+
+    new_events(ev_kw)
+
+    def enqueue_steps(n, events):
+        """The step's launches; with events, each kernel between a pair of timing events (which
+        serialise the kernels: the timed step runs without them)."""
+        k = km = 0
+
+        def mark(name, idx, j):
+            if events:
+                ev[name][idx][j].record()
+
+        for _ in range(n):
+            for ly in layers:
+                if ly["merge"] is not None:
+                    mark("merge", km, 0)
+                    layernorm(fqvit, ly["merge"])
+                    mark("merge", km, 1)
+                    km += 1
+                mark("ln", k, 0)
+                layernorm(fqvit, ly)
+                mark("ln", k, 1)
+                mark("attn", k, 0)
+                attention(fqvit, ly, args.out8)
+                mark("attn", k, 1)
+                k += 1
+
+    graph = ev_graph = None
+    if use_graph:
+        try:
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph):
+                enqueue_steps(steps, False)
+            ev_graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(ev_graph):
+                enqueue_steps(ev_steps, True)
+            graph.replay()  # upload and one untimed pass
+            torch.cuda.synchronize()
+        except Exception as exc:  # noqa: BLE001 - any capture failure falls back to eager launches
+            print(f"bench: CUDA graph unavailable ({type(exc).__name__}: {exc}); eager launches", file=sys.stderr)
+            graph = ev_graph = None
+            torch.cuda.synchronize()
+            new_events(dict(enable_timing=True))
+    clocks = ClockSampler(torch.cuda.current_device()) if sample_clocks else None
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)  # let the sampler start before the timed region
+    start.record()
+    if graph is not None:
+        graph.replay()
+    else:
+        enqueue_steps(steps, False)
+    end.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop() if clocks else None
+    elapsed_ms = start.elapsed_time(end)
+    if ws > 1:
+        t = torch.tensor([elapsed_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+        torch.distributed.barrier()
+
+    # per-kernel durations: a separate pass of the same launches with timing events around each
+    if ev_graph is not None:
+        ev_graph.replay()
+    else:
+        enqueue_steps(ev_steps, True)
+    torch.cuda.synchronize()
+    fqvit.sync_status()
+    attn_ms = [a.elapsed_time(b) for a, b in ev["attn"]]
+    ln_ms = [a.elapsed_time(b) for a, b in ev["ln"]]
+    merge_ms = [a.elapsed_time(b) for a, b in ev["merge"]]
+    ab = [attn_bytes(ly["BH"], ly["L"], ly["d"], 1 if args.out8 else 4, qk=args.qk) for ly in layers]
+    lb = [ln_bytes(ly["rows"], ly["C"]) for ly in layers]
+    mb = [ln_bytes(m["rows"], m["C"]) for m in merges]
+    return dict(elapsed_ms=elapsed_ms, ms_per_step=elapsed_ms / steps, graph=graph is not None, clocks=clk,
+                ev_steps=ev_steps, attn_ms=attn_ms, ln_ms=ln_ms, merge_ms=merge_ms, ab=ab, lb=lb, mb=mb,
+                merges=merges, step_bytes=sum(ab) + sum(lb) + sum(mb))
+
+
+def kernel_stats(t, peak, ev_steps):
+    """Per-kernel byte rates (algorithmic bytes over CUDA-event durations) of a time_config result."""
+    attn_gbs = sum(t["ab"]) * ev_steps / (sum(t["attn_ms"]) / 1e3) / 1e9
+    ln_gbs = sum(t["lb"]) * ev_steps / (sum(t["ln_ms"]) / 1e3) / 1e9
+    out = {
+        "attention": {"gbs": round(attn_gbs, 1), "frac": round(attn_gbs / peak, 4),
+                      "ms_per_launch": round(sum(t["attn_ms"]) / len(t["attn_ms"]), 5),
+                      "bytes_per_launch": round(sum(t["ab"]) / len(t["ab"]))},
+        "layernorm": {"gbs": round(ln_gbs, 1), "frac": round(ln_gbs / peak, 4),
+                      "ms_per_launch": round(sum(t["ln_ms"]) / len(t["ln_ms"]), 5),
+                      "bytes_per_launch": round(sum(t["lb"]) / len(t["lb"]))},
+    }
+    if t["merges"]:
+        mg = sum(t["mb"]) * ev_steps / (sum(t["merge_ms"]) / 1e3) / 1e9
+        out["patch_merge_layernorm"] = {"gbs": round(mg, 1), "frac": round(mg / peak, 4),
+                                        "ms_per_launch": round(sum(t["merge_ms"]) / len(t["merge_ms"]), 5),
+                                        "bytes_per_launch": round(sum(t["mb"]) / len(t["mb"]))}
+    return out, attn_gbs, ln_gbs
+
+
+def other_configs(fqvit, args, dev, ws, peak):
+    """The other four configs of the workload list, each timed like the headline step (fewer steps,
+    no host-copy or CPU legs): tokens/s, HBM GB/s and the fraction of the measured peak."""
+    out = {}
+    for name in ("deit_t", "deit_s", "vit_b", "swin_s"):
+        if name == args.config:
+            continue
+        cfg = synth.CONFIGS[name]
+        try:
+            layers = make_layers(cfg, dev, sigma=args.sigma, qk=args.qk)
+            steps = max(3, min(args.steps, 10))
+            t = time_config(fqvit, cfg, layers, args, steps, 3, dev, ws)
+            ks, _, _ = kernel_stats(t, peak, t["ev_steps"])
+            gbs = t["step_bytes"] / (t["ms_per_step"] / 1e3) / 1e9
+            out[name] = {"value": round(cfg.first_tokens * ws * steps / (t["elapsed_ms"] / 1e3), 1),
+                         "unit": "tokens/s", "ms_per_step": round(t["ms_per_step"], 5), "steps": steps,
+                         "layers": len(layers), "hbm_gbs": round(gbs, 1), "hbm_frac": round(gbs / peak, 4),
+                         "kernels": ks, "workload": f"{cfg.name}: {cfg.note}"}
+            del layers
+            torch.cuda.empty_cache()
+        except Exception as e:  # noqa: BLE001 - one config failing is reported, not fatal to the line
+            out[name] = {"error": f"{type(e).__name__}: {e}"[:300]}
+    return out
+
 
 def bench_gpu(args):
     from paper_2111_13824_gb300 import build as fbuild
@@ -368,120 +582,15 @@ def bench_gpu(args):
         raise SystemExit("--qk and --out8 together are not a bench mode")
     layers = make_layers(cfg, dev, sigma=args.sigma, limit=args.layers, qk=args.qk)
     tokens_per_step = cfg.first_tokens
-
-    for _ in range(args.warmup):
-        for ly in layers:
-            run_layer(fqvit, ly)
-    torch.cuda.synchronize()
-
-    # The K timed steps go into one CUDA graph (launches and their timing events), so that
-    # the host's per-call enqueue cost stays out of the timed region; eager launches when the
-    # graph cannot be built (a PyTorch without external events, or a capture error).
-    use_graph = not args.no_graph
-    ev_kw = dict(enable_timing=True)
-    if use_graph:
-        try:
-            torch.cuda.Event(enable_timing=True, external=True)
-            ev_kw["external"] = True
-        except TypeError:
-            use_graph = False
-    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    merges = [ly["merge"] for ly in layers if ly["merge"] is not None]
-    ev_steps = min(args.steps, 3)  # steps of the per-kernel timing pass
-    ev = {}
-
-    def new_events(kw):
-        ev["attn"] = [(torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(ev_steps * len(layers))]
-        ev["ln"] = [(torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(ev_steps * len(layers))]
-        ev["merge"] = [(torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(ev_steps * len(merges))]
-
-    new_events(ev_kw)
-
-    def enqueue_steps(steps, events):
-        """The step's launches; with events, each kernel between a pair of timing events (which
-        serialise the kernels: the timed step runs without them)."""
-        k = km = 0
-
-        def mark(name, idx, j):
-            if events:
-                ev[name][idx][j].record()
-
-        for _ in range(steps):
-            for ly in layers:
-                if ly["merge"] is not None:
-                    mark("merge", km, 0)
-                    layernorm(fqvit, ly["merge"])
-                    mark("merge", km, 1)
-                    km += 1
-                mark("ln", k, 0)
-                fqvit.ptf_layernorm(ly["xq"], ly["zp"], ly["alpha"], ly["gamma"], ly["beta"], ly["s_out"],
-                                    ly["zp_out"], out=ly["yq"])
-                mark("ln", k, 1)
-                mark("attn", k, 0)
-                attention(fqvit, ly, args.out8)
-                mark("attn", k, 1)
-                k += 1
-
-    graph = ev_graph = None
-    if use_graph:
-        try:
-            graph = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(graph):
-                enqueue_steps(args.steps, False)
-            ev_graph = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(ev_graph):
-                enqueue_steps(ev_steps, True)
-            graph.replay()  # upload and one untimed pass
-            torch.cuda.synchronize()
-        except Exception as exc:  # noqa: BLE001 - any capture failure falls back to eager launches
-            print(f"bench: CUDA graph unavailable ({type(exc).__name__}: {exc}); eager launches", file=sys.stderr)
-            graph = ev_graph = None
-            torch.cuda.synchronize()
-            new_events(dict(enable_timing=True))
-    clocks = ClockSampler(local)
-    if ws > 1:
-        torch.distributed.barrier()
-    torch.cuda.synchronize()
-    clocks.start()
-    time.sleep(0.3)  # let the sampler start before the timed region
-    start.record()
-    if graph is not None:
-        graph.replay()
-    else:
-        enqueue_steps(args.steps, False)
-    end.record()
-    torch.cuda.synchronize()
-    clk = clocks.stop()
-    elapsed_ms = start.elapsed_time(end)
-    if ws > 1:
-        t = torch.tensor([elapsed_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
-        torch.distributed.barrier()
-    ms_per_step = elapsed_ms / args.steps
-    value = tokens_per_step * ws * args.steps / (elapsed_ms / 1e3)
-
-    # per-kernel durations: a separate pass of the same launches with timing events around each
-    if ev_graph is not None:
-        ev_graph.replay()
-    else:
-        enqueue_steps(ev_steps, True)
-    torch.cuda.synchronize()
-    attn_events, ln_events, merge_events = ev["attn"], ev["ln"], ev["merge"]
-
-    attn_ms = [a.elapsed_time(b) for a, b in attn_events]
-    ln_ms = [a.elapsed_time(b) for a, b in ln_events]
     peak, peak_kind = peaks()
-    # per-launch algorithmic bytes (averaged over the stack's layer shapes)
-    ab = [attn_bytes(ly["BH"], ly["L"], ly["d"], 1 if args.out8 else 4, qk=args.qk) for ly in layers]
-    lb = [ln_bytes(ly["rows"], ly["C"]) for ly in layers]
-    attn_gbs = sum(ab) * ev_steps / (sum(attn_ms) / 1e3) / 1e9
-    ln_gbs = sum(lb) * ev_steps / (sum(ln_ms) / 1e3) / 1e9
-    mb = [ln_bytes(m["rows"], m["C"]) for m in merges]
-    merge_ms = [a.elapsed_time(b) for a, b in merge_events]
-    step_bytes = sum(ab) + sum(lb) + sum(mb)
+
+    t = time_config(fqvit, cfg, layers, args, args.steps, args.warmup, dev, ws, sample_clocks=True)
+    elapsed_ms, ms_per_step = t["elapsed_ms"], t["ms_per_step"]
+    value = tokens_per_step * ws * args.steps / (elapsed_ms / 1e3)
+    ks, attn_gbs, ln_gbs = kernel_stats(t, peak, t["ev_steps"])
+    step_bytes = t["step_bytes"]
     stack_gbs = step_bytes / (ms_per_step / 1e3) / 1e9
-    dominant = "attention" if sum(attn_ms) >= sum(ln_ms) else "layernorm"
+    dominant = "attention" if sum(t["attn_ms"]) >= sum(t["ln_ms"]) else "layernorm"
     dom_gbs = attn_gbs if dominant == "attention" else ln_gbs
     # the records are of the int32 output from logits, or (key "<config>:qk") of the --qk step
     traffic = None if args.out8 else recorded_traffic(args.config + (":qk" if args.qk else ""), dominant)
@@ -501,26 +610,25 @@ def bench_gpu(args):
         torch.cuda.synchronize()
         qk_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
         qk_b = ly["BH"] * (2 * ly["L"] * ly["d"] + ly["L"] * full.shape[1])
-        qk_stats = {"gbs": round(qk_b / (qk_ms / 1e3) / 1e9, 1), "ms_per_launch": round(qk_ms, 5),
-                    "bytes_per_launch": qk_b, "frac": round(qk_b / (qk_ms / 1e3) / 1e9 / peak, 4),
-                    "how": "fqvit_qk_logits on layer 0, all heads in one launch (Q, K read, logits written "
-                           "to HBM), 10 launches after 3, outside the timed step"}
+        ks["qk_logits"] = {"gbs": round(qk_b / (qk_ms / 1e3) / 1e9, 1), "ms_per_launch": round(qk_ms, 5),
+                           "bytes_per_launch": qk_b, "frac": round(qk_b / (qk_ms / 1e3) / 1e9 / peak, 4),
+                           "how": "fqvit_qk_logits on layer 0, all heads in one launch (Q, K read, logits written "
+                                  "to HBM), 10 launches after 3, outside the timed step"}
         del full
 
-    lin_stats = None
     if args.linear:  # outside the timed step; a failure here is reported, not fatal to the line
         try:
-            lin_stats = bench_linear(fqvit, cfg, dev)
+            ks["linear"] = bench_linear(fqvit, cfg, dev)
         except Exception as e:  # noqa: BLE001
-            lin_stats = {"error": f"{type(e).__name__}: {e}"[:300]}
+            ks["linear"] = {"error": f"{type(e).__name__}: {e}"[:300]}
 
     e2e = None
     if not args.no_e2e:
         e2e = bench_e2e(fqvit, layers, tokens_per_step, args, dev, ws)
 
-    cpu = None
+    cpu = parity = None
     if rank == 0 and ws == 1 and not args.no_cpu:
-        cpu = cpu_baseline(cfg, args)
+        cpu, parity = cpu_baseline(cfg, layers, args)
 
     line = {
         "metric": metric_name(args),
@@ -544,39 +652,33 @@ def bench_gpu(args):
             "l2": f"inputs {step_bytes / 1e9:.2f} GB per step, larger than the 129 MB L2 (no flush)",
             "logit_sigma": args.sigma,
             "parallelism": f"replicas x{ws} (independent batches, no collective)",
-            "launch": "cuda_graph" if graph is not None else "eager",
+            "launch": "cuda_graph" if t["graph"] else "eager",
             "attention_output": "uint8 (requantized)" if args.out8 else "int32 accumulators",
             "attention_input": (f"int8 Q, K, V: fqvit_qk_lis_attention, head groups of {qk_group(layers[0])}"
                                 if args.qk else "int8 logits, int8 V"),
             "shifted_window_layers": sum(ly["region"] is not None for ly in layers),
-            "patch_merges": len(merges),
+            "patch_merges": len(t["merges"]),
         },
         "hbm_gbs": round(stack_gbs, 1),
         "hbm_frac": round(stack_gbs / peak, 4),
-        "kernels": {
-            "attention": {"gbs": round(attn_gbs, 1), "ms_per_launch": round(sum(attn_ms) / len(attn_ms), 5),
-                          "bytes_per_launch": round(sum(ab) / len(ab))},
-            "layernorm": {"gbs": round(ln_gbs, 1), "ms_per_launch": round(sum(ln_ms) / len(ln_ms), 5),
-                          "bytes_per_launch": round(sum(lb) / len(lb))},
-            **({"qk_logits": qk_stats} if args.qk else {}),
-            **({"linear": lin_stats} if lin_stats else {}),
-            **({"patch_merge_layernorm": {
-                "gbs": round(sum(mb) * ev_steps / (sum(merge_ms) / 1e3) / 1e9, 1),
-                "ms_per_launch": round(sum(merge_ms) / len(merge_ms), 5),
-                "bytes_per_launch": round(sum(mb) / len(mb))}} if merges else {}),
-        },
+        "kernels": ks,
         "roofline": {"kernel": dominant, "bound": "hbm", "achieved": round(dom_gbs, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(dom_gbs / peak, 4), "traffic": traffic,
                      "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
                      else "fallback"},
-        "clocks": clk,
+        "clocks": t["clocks"],
         "gpu_launches": (sum(1 + (2 * -(-ly["BH"] // qk_group(ly)) if args.qk else 1) for ly in layers)
-                         + len(merges)) * args.steps,
+                         + len(t["merges"])) * args.steps,
     }
     if e2e is not None:
         line["e2e"] = e2e
     if cpu is not None:
         line["cpu_baseline"] = cpu
+        line["parity"] = parity
+    if args.all_configs and ws == 1 and args.layers <= 0:
+        del layers
+        torch.cuda.empty_cache()
+        line["configs"] = other_configs(fqvit, args, dev, ws, peak)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if ws > 1:
@@ -668,29 +770,38 @@ def bench_e2e(fqvit, layers, tokens_per_step, args, dev, ws):
                    "three streams (upload, compute, download), layers pipelined"}
 
 
-def cpu_baseline(cfg, args):
-    """The oracle, as it stands, on this host's cores: a bounded sample of layer 0
-    (grown toward --cpu-seconds of work), repeated until the budget is spent."""
+def cpu_baseline(cfg, layers, args):
+    """The oracle, as it stands, on this host's cores (OracleLeg): the time of all of layer 0 on all
+    cores and of a bounded part of it on one core, each scaled to the whole step, and the parity
+    verdict of the same outputs and of sampled rows and heads of every other layer."""
     import oracle
 
-    probe = OracleSample(cfg, heads=1, ln_rows=256, qk=args.qk)
-    _, spent = probe.run()
-    scale = max(1, int(args.cpu_seconds / max(spent, 1e-3)))
-    st = cfg.stages[0]
-    smp = OracleSample(cfg, heads=min(st.BH, scale), ln_rows=min(st.rows, 256 * scale), qk=args.qk)
-    ests, total = [], 0.0
-    while total < args.cpu_seconds or not ests:
-        est, spent = smp.run()
-        ests.append(est)
-        total += spent
-    est = statistics.mean(ests)
-    return {"value": round(cfg.first_tokens / est, 2), "unit": "tokens/s", "cores": oracle.num_threads(),
-            "kind": "oracle",
-            "sample": f"{smp.describe()}; {len(ests)} repetition(s), {total:.1f} s of CPU work"}
+    oracle.build()
+    leg = OracleLeg(cfg, layers, args)
+    ln_s, at_s = leg.layer0_all_cores()
+    ln1_s, at1_s = leg.layer0_one_core()
+    leg.other_layers()
+    ln_el, logits = step_elements(cfg)
+    ly = layers[0]
+    ln0, lg0 = ly["rows"] * ly["C"], ly["BH"] * ly["L"] * ly["L"]
+    step_all = ln_s * ln_el / ln0 + at_s * logits / lg0
+    step_one = ln1_s * ln_el / ln0 + at1_s * logits / lg0
+    cores = os.cpu_count() or 1
+    cpu = {"value": round(cfg.first_tokens / step_all, 2), "unit": "tokens/s", "cores": cores, "kind": "oracle",
+           "single_thread": {"value": round(cfg.first_tokens / step_one, 2), "unit": "tokens/s", "cores": 1},
+           "extrapolated_from": "layer 0",
+           "sample": (f"all of layer 0 ({ly['rows']} LayerNorm rows, {ly['BH']} attention heads"
+                      f"{', logits from Q and K' if args.qk else ''}) on {cores} cores, {ln_s + at_s:.2f} s, and "
+                      f"256 rows and 2 {'images' if ly['window'] else 'heads'} of it on one core, each scaled by "
+                      f"the step's LayerNorm elements and attention logits to the {cfg.layers}-layer step")}
+    return cpu, leg.verdict()
 
 
 def bench_reference(args):
-    """The reference arm: the CPU oracle, as it stands, on the host cores."""
+    """The reference arm: the CPU oracle, as it stands, on the host cores.  Each step is the oracle
+    on all of layer 0 of the config (the same sample as the GPU arm's cpu_baseline leg), on the
+    inputs the GPU arm generates; ms_per_step is that measured time, and the tokens/s of the whole
+    stack is extrapolated from it by LayerNorm elements and attention logits."""
     ws, rank, local = _dist_env()
     if rank != 0:
         return
@@ -698,32 +809,70 @@ def bench_reference(args):
     import oracle
 
     oracle.build()
-    smp = OracleSample(cfg, heads=4, ln_rows=2048, qk=args.qk)
-    for _ in range(args.warmup):
-        smp.run()
-    ests = []
+    cores = os.cpu_count() or 1
+    oracle.set_num_threads(cores)
+    layer = make_host_layer0(cfg, args)
+    leg = OracleLeg(cfg, [layer], args)
+
+    def one():
+        t0 = time.perf_counter()
+        leg._ln(layer, slice(None))
+        t1 = time.perf_counter()
+        leg._attn(layer, 0, layer["BH"])
+        return t1 - t0, time.perf_counter() - t1
+
+    for _ in range(min(args.warmup, 1)):
+        one()
+    times = []
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        ests.append(smp.run()[0])
+        times.append(one())
     wall = time.perf_counter() - t0
-    step = statistics.mean(ests)
-    value = cfg.first_tokens / step
-    sample = f"per step: {smp.describe()}"
+    ln_s = statistics.mean(a for a, _ in times)
+    at_s = statistics.mean(b for _, b in times)
+    ln_el, logits = step_elements(cfg)
+    ln0, lg0 = layer["rows"] * layer["C"], layer["BH"] * layer["L"] * layer["L"]
+    step_est = ln_s * ln_el / ln0 + at_s * logits / lg0
+    value = cfg.first_tokens / step_est
+    sample = (f"per step: all of layer 0 ({layer['rows']} LayerNorm rows, {layer['BH']} attention heads) on "
+              f"{cores} cores; tokens/s extrapolated by LayerNorm elements and attention logits to the "
+              f"{cfg.layers}-layer step ({step_est * 1e3:.1f} ms)")
     line = {
         "impl": "reference",
         "metric": metric_name(args),
         "value": round(value, 3), "unit": "tokens/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": round(step * 1e3, 3), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "int8", "data": "synthetic (seeded generator of the paper's layer shapes and statistics)",
+        "ms_per_step": round((ln_s + at_s) * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int8",
+        "data": "synthetic (seeded generator of the paper's layer shapes and statistics)",
         "config": {"workload": f"{cfg.name}: {cfg.note}, {cfg.layers} layers of PTF LayerNorm + "
                                f"{'Q K^T + ' if args.qk else ''}LIS attention",
                    "tokens_per_step_per_gpu": cfg.first_tokens, "layers": cfg.layers},
-        "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": oracle.num_threads(),
-                         "kind": "oracle", "sample": sample},
+        "extrapolated_from": "layer 0",
+        "step_extrapolated_ms": round(step_est * 1e3, 3),
+        "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": sample},
         "e2e": {"value": round(value, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         "wall_s": round(wall, 2),
     }
     print(json.dumps(line), flush=True)
+
+
+def make_host_layer0(cfg, args):
+    """Layer 0 of a config generated on the host: the GPU arm's shapes and statistics (its device
+    generator draws other values), calibrated and quantized by the oracle."""
+    import oracle
+
+    st = synth.layer_stage(cfg, 0)
+    d = synth.ln_inputs(cfg, 0)
+    s, zp, alpha, _ = oracle.calibrate_ptf(d["x_calib"].numpy(), K=cfg.K)
+    xq = oracle.ptf_quantize(d["x"].numpy(), s, zp, alpha)
+    a = synth.attn_inputs(cfg, 0, sigma=args.sigma)
+    return dict(qk=args.qk, q=a["q"], k=a["k"], s_q=a["s_q"], s_k=a["s_k"], zp_logit=a["zp_logit"],
+                xq=torch.from_numpy(xq), zp=int(zp), alpha=torch.from_numpy(alpha), gamma=d["gamma"], beta=d["beta"],
+                s_out=d["s_out"], zp_out=d["zp_out"], logits=a["logits"], s_logit=a["s_logit"], v=a["v"],
+                bias=a["bias"], heads=a["heads"], window=a["window"],
+                region=synth.layer_window_mask(cfg, 0), mask_value=synth.swin_mask_value(a["s_logit"]),
+                rows=st.rows, C=st.C, BH=st.BH, L=st.L, d=st.d, merge=None)
 
 
 def main():
@@ -737,7 +886,6 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
-    ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--traffic", default=None, help="JSON {kernel: dram bytes per launch} from an ncu capture")
     ap.add_argument("--layers", type=int, default=0, help="time only the first N layers (profiling cases)")
     ap.add_argument("--no-graph", action="store_true", help="launch the timed steps eagerly instead of as one CUDA graph")
@@ -745,6 +893,8 @@ def main():
                     help="attention from int8 Q, K, V (fqvit_qk_lis_attention) instead of int8 logits")
     ap.add_argument("--out8", action="store_true",
                     help="the attention output requantized to 8 bits (fqvit_lis_attention_q) instead of int32")
+    ap.add_argument("--no-configs", dest="all_configs", action="store_false",
+                    help="skip the timing of the other four configs (reported under configs)")
     ap.add_argument("--no-linear", dest="linear", action="store_false",
                     help="skip the separate timing of the block's MinMax Linear layers (fqvit_linear_q), "
                          "which runs after the timed step and is reported under kernels.linear")

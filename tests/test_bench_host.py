@@ -33,6 +33,36 @@ def test_reference_arm_prints_one_json_line():
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
     assert d["e2e"] == {"value": d["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
     assert d["config"]["workload"].startswith("deit_t")
+    # the measured step is layer 0; the stack's rate is extrapolated from it, and says so
+    assert d["extrapolated_from"] == "layer 0"
+    assert d["ms_per_step"] * d["steps"] / 1e3 <= d["wall_s"] + 0.05
+    assert d["step_extrapolated_ms"] >= d["ms_per_step"]
+
+
+class _Args:
+    qk = False
+    out8 = False
+    sigma = 1.0
+
+
+def test_oracle_leg_parity_verdict():
+    """The cpu_baseline leg's parity check: outputs equal to the oracle's read as bit-exact, one
+    planted wrong element as a mismatch (host tensors stand in for the GPU step's)."""
+    import oracle
+
+    oracle.build()
+    cfg = synth.CONFIGS["deit_t"]
+    ly = bench.make_host_layer0(cfg, _Args)
+    leg = bench.OracleLeg(cfg, [ly], _Args)
+    ly["yq"] = torch.from_numpy(leg._ln(ly, slice(None)))
+    ly["acc"] = torch.from_numpy(leg._attn(ly, 0, ly["BH"]))
+    leg.layer0_all_cores()
+    leg.other_layers()
+    assert leg.verdict().startswith("bit-exact"), leg.verdict()
+    ly["acc"][1, 5, 7] += 1
+    leg2 = bench.OracleLeg(cfg, [ly], _Args)
+    leg2.layer0_all_cores()
+    assert leg2.verdict().startswith("MISMATCH") and "attention" in leg2.verdict()
 
 
 def test_metric_names():
