@@ -99,12 +99,18 @@ FQVIT_API int fqvit_calibrate_ptf(const float *x, int64_t rows, int32_t C, int64
  * is owned by another allocator that gives out no extra buffer.  There is no
  * counterpart in the paper; it is an interface of this library.
  *   - No workspace argument: the kernels use a fixed 160 KiB array of device
- *     memory that the library reserves on every GPU that loads it, for as long
- *     as it stays loaded.  The call allocates nothing.
- *   - Limit: C * (K + 1) <= 16384 (e.g. C = 4096 at K = 3); larger problems
- *     return FQVIT_ERR_UNSUPPORTED -- use fqvit_calibrate_ptf with a workspace.
- *   - The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress); make that first call before any stream capture.
+ *     memory that belongs to the library, one per GPU, kept until the process
+ *     ends or the context is reset.  The call itself allocates nothing.
+ *   - The array is reserved when the library's code is loaded on a GPU.  With
+ *     CUDA's default lazy module loading that is the first call on that GPU
+ *     (its lookup of the array's address loads the code), so that first call
+ *     may take device memory: make it at start-up, before the memory budget is
+ *     fixed and before any stream capture (or set CUDA_MODULE_LOADING=EAGER).
+ *     Later calls take none.
+ *   - Limit, when sse_opt is NULL (the error sums are then kept in the array):
+ *     C * (K + 1) <= 16384 (e.g. C = 4096 at K = 3); larger problems return
+ *     FQVIT_ERR_UNSUPPORTED -- pass sse_opt, or use fqvit_calibrate_ptf with a
+ *     workspace.  With sse_opt any supported C and K fit.
  *   - All calls share the array, which keeps the last call's contents (no
  *     call needs it zeroed).  Calls whose kernels overlap on the GPU race on
  *     it: do not run two of them concurrently.

@@ -41,7 +41,8 @@ cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, size_t 
 int record_error(int code, const char *msg);
 
 // ---- PTF calibration / quantizer (ptf.cu) ---------------------------------
-size_t calibrate_workspace_bytes(int64_t rows, int C, int K);
+// Workspace of launch_calibrate; with sums == false the caller's sse buffer holds the error sums.
+size_t calibrate_workspace_bytes(int64_t rows, int C, int K, bool sums = true);
 
 // Eqs. 8-9 from the calibration range, shared by the device path and the host
 // combine of sharded calibration: s0 = (mx - mn) / 255 (a zero range counts
@@ -160,7 +161,7 @@ bool qk_logits_supported(const QkArgs &a);
 cudaError_t launch_qk_logits(const QkArgs &a, cudaStream_t st);
 cudaError_t read_clear_qk_status(int *status);
 
-// tensor-core (tcgen05) fused path for rows of 65 .. 640 keys (lis_tc.cu); rows of 128 .. 384 keys
+// tensor-core (tcgen05) fused path for rows of 65 .. 592 keys (lis_tc.cu); rows of 128 .. 384 keys
 // take tiles packed across heads
 bool lis_attention_tc_eligible(const LisArgs &a, const AttnVArgs &b);
 cudaError_t launch_lis_attention_tc(const LisArgs &a, const AttnVArgs &b, cudaStream_t st);

@@ -210,10 +210,10 @@ int minmax_blocks(int64_t rows)
 
 }  // namespace
 
-size_t calibrate_workspace_bytes(int64_t rows, int C, int K)
+size_t calibrate_workspace_bytes(int64_t rows, int C, int K, bool sums)
 {
     (void)rows;
-    return (size_t)kWsHeader + sizeof(float2) * kMaxPartials + sizeof(double) * (size_t)C * (K + 1);
+    return (size_t)kWsHeader + sizeof(float2) * kMaxPartials + (sums ? sizeof(double) * (size_t)C * (K + 1) : 0);
 }
 
 cudaError_t launch_calibrate(const float *x, int64_t rows, int C, int64_t ld_x, int K, float *s,

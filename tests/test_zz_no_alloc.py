@@ -31,12 +31,14 @@ def _ptr(t):
     return ctypes.c_void_p(t.data_ptr()) if t is not None else None
 
 
-def _noalloc(lib, x, K):
+def _noalloc(lib, x, K, with_sse=True):
+    """The call with (or, with_sse=False, without) a caller buffer for the error sums; without one
+    the sums are kept in the library's array and only s, zp and alpha come back."""
     rows, C = x.shape
     s = torch.empty(1, dtype=torch.float32, device=x.device)
     zp = torch.empty(1, dtype=torch.int32, device=x.device)
     alpha = torch.empty(C, dtype=torch.uint8, device=x.device)
-    sse = torch.empty(C, K + 1, dtype=torch.float64, device=x.device)
+    sse = torch.empty(C, K + 1, dtype=torch.float64, device=x.device) if with_sse else None
     stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
     rc = lib.fqvit_calibrate_ptf_noalloc(_ptr(x), rows, C, x.stride(0), 8, K, _ptr(s), _ptr(zp), _ptr(alpha),
                                          _ptr(sse), stream)
@@ -72,6 +74,47 @@ def test_noalloc_matches_workspace_calibration_twice(lib):
         torch.cuda.synchronize()
         for a, b in zip(again, ref):
             assert torch.equal(a, b)
+
+
+def test_noalloc_sums_in_the_library_array(lib):
+    """Without a caller sse buffer the error sums live in the fixed array: its largest use (C = 4096
+    at K = 3, 16384 sums), then a smaller problem right after it, then the largest again; s, zp and
+    alpha bit for bit as with a workspace.  After the first call no call takes device memory."""
+    cases = [(_channels(5, 2000, 4096), 3), (_channels(6, 700, 192), 5), (_channels(7, 1500, 4096), 3)]
+    refs = [_with_workspace(x, K) for x, K in cases]
+    outs = [(torch.empty(1, dtype=torch.float32, device=x.device), torch.empty(1, dtype=torch.int32, device=x.device),
+             torch.empty(x.shape[1], dtype=torch.uint8, device=x.device)) for x, _ in cases]
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+
+    def call(i):
+        x, K = cases[i]
+        s, zp, alpha = outs[i]
+        rc = lib.fqvit_calibrate_ptf_noalloc(_ptr(x), x.shape[0], x.shape[1], x.stride(0), 8, K, _ptr(s), _ptr(zp),
+                                             _ptr(alpha), None, stream)
+        assert rc == 0, lib.fqvit_last_error().decode()
+
+    call(1)  # the first call may load the library's code (and so reserve its array)
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for i in range(len(cases)):
+        call(i)
+        torch.cuda.synchronize()
+        assert torch.cuda.mem_get_info()[0] == free0  # nothing allocated by the call
+        rs, rzp, ralpha, _ = refs[i]
+        s, zp, alpha = outs[i]
+        assert torch.equal(s.view(torch.int32), rs.view(torch.int32))
+        assert torch.equal(zp, rzp) and torch.equal(alpha, ralpha)
+
+
+def test_noalloc_with_caller_sums_takes_any_size(lib):
+    """With the caller's sse buffer the array holds only the small min/max part, so C (K + 1) may
+    exceed 16384."""
+    x = _channels(8, 300, 8192)
+    got = _noalloc(lib, x, 3)
+    ref = _with_workspace(x, 3)
+    torch.cuda.synchronize()
+    for a, b in zip(got, ref):
+        assert torch.equal(a, b)
 
 
 def test_noalloc_rejects_problems_beyond_its_scratch(lib):
