@@ -73,6 +73,12 @@ FQVIT_API int fqvit_selftest_bounded_wait(void *stream);
 /* Bytes of device workspace fqvit_calibrate_ptf needs (a few KB). */
 FQVIT_API size_t fqvit_calibrate_workspace_size(int64_t rows, int32_t C, int32_t K);
 
+/* The same size under the name of the planned interface: the workspace does not depend on the
+ * number of calibration rows (the min / max pass keeps at most 1024 block partials), so
+ * fqvit_workspace_size(C, K) == fqvit_calibrate_workspace_size(rows, C, K) for every rows >= 1.
+ * 0 for C < 1 or K outside 0..7. */
+FQVIT_API size_t fqvit_workspace_size(int32_t C, int32_t K);
+
 /*
  * Layer-wise scale s and zero point zp (Eqs. 8-9) and per-channel factors
  * alpha_c in {0..K} (Eq. 10) from a calibration batch x [rows, C] fp32.

@@ -95,6 +95,8 @@ size_t fqvit_calibrate_workspace_size(int64_t rows, int32_t C, int32_t K)
     return fqvit::calibrate_workspace_bytes(rows, C, K);
 }
 
+size_t fqvit_workspace_size(int32_t C, int32_t K) { return fqvit_calibrate_workspace_size(1, C, K); }
+
 int fqvit_calibrate_ptf(const float *x, int64_t rows, int32_t C, int64_t ld_x, int32_t bits,
                         int32_t K, float *s, int32_t *zp, uint8_t *alpha, double *sse_opt,
                         void *workspace, size_t ws_bytes, void *stream)

@@ -44,7 +44,8 @@ class BlockDesc(ctypes.Structure):
 
 
 EXPORTS = (
-    "fqvit_version", "fqvit_last_error", "fqvit_calibrate_workspace_size", "fqvit_calibrate_ptf",
+    "fqvit_version", "fqvit_last_error", "fqvit_calibrate_workspace_size", "fqvit_workspace_size",
+    "fqvit_calibrate_ptf",
     "fqvit_ptf_quantize", "fqvit_ptf_layernorm", "fqvit_lis_softmax", "fqvit_lis_attn_v",
     "fqvit_lis_attention", "fqvit_lis_attention_q", "fqvit_block_int", "fqvit_sync_status",
     "fqvit_calibrate_ptf_noalloc",
@@ -74,6 +75,7 @@ def load(path: str | Path | None = None):
         "fqvit_version": ([], ctypes.c_int),
         "fqvit_last_error": ([], ctypes.c_char_p),
         "fqvit_calibrate_workspace_size": ([i64, i32, i32], sz),
+        "fqvit_workspace_size": ([i32, i32], sz),
         "fqvit_calibrate_ptf": ([P, i64, i32, i64, i32, i32, P, P, P, P, P, sz, P], ctypes.c_int),
         "fqvit_ptf_quantize": ([P, i64, i32, i64, f32, i32, P, P, i64, P], ctypes.c_int),
         "fqvit_ptf_layernorm": ([P, i64, i32, i64, i32, P, P, P, f32, i32, P, i64, P, P, P], ctypes.c_int),

@@ -42,6 +42,15 @@ def test_version(lib):
     assert lib.fqvit_version() >= 1
 
 
+def test_workspace_size_alias(lib):
+    # the planned interface's fqvit_workspace_size(C, K) is the calibration workspace, which does
+    # not depend on the number of rows
+    for C, K in ((192, 3), (1024, 3), (4096, 7), (1, 0)):
+        w = lib.fqvit_workspace_size(C, K)
+        assert w > 0 and all(w == lib.fqvit_calibrate_workspace_size(rows, C, K) for rows in (1, 577, 10 ** 6))
+    assert lib.fqvit_workspace_size(0, 3) == 0 and lib.fqvit_workspace_size(64, 8) == 0
+
+
 def _err(lib):
     return lib.fqvit_last_error().decode()
 
