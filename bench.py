@@ -147,6 +147,8 @@ def recorded_traffic(config, kernel):
         return None
     h = hashlib.sha256()
     for src in rec["sources"]:
+        if not os.path.exists(os.path.join(ROOT, src)):
+            return None  # a source of the captured kernel is gone: the record is stale
         with open(os.path.join(ROOT, src), "rb") as f:
             h.update(f.read())
     return rec["dram_bytes_per_launch"] if h.hexdigest()[:16] == rec["source_sha"] else None

@@ -57,6 +57,17 @@ int sm_count()
     return cached[dev];
 }
 
+cudaError_t check_smem_fits(const void *kernel, size_t dynamic)
+{
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, kernel);
+    if (e != cudaSuccess) return e;
+    int dev = 0, optin = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess) return e;
+    return fa.sharedSizeBytes + dynamic <= (size_t)optin ? cudaSuccess : cudaErrorInvalidConfiguration;
+}
+
 int record_error(int code, const char *msg)
 {
     if (code == FQVIT_OK) return ok();

@@ -10,6 +10,11 @@ namespace fqvit {
 // Number of SMs of the current device (cached per device).
 int sm_count();
 
+// Launch check of a kernel's shared memory: the compiled static size (as the runtime reports it,
+// not an estimate) plus `dynamic` bytes within the device's opt-in limit per block.  Returns
+// cudaErrorInvalidConfiguration when they do not fit, or the runtime's error.
+cudaError_t check_smem_fits(const void *kernel, size_t dynamic);
+
 // Programmatic dependent launch.  The step's kernels are launched with programmatic stream
 // serialization: the next kernel's CTAs may start (and run their set-up: barriers, tensor
 // memory, tables computed from arguments) while the previous kernel's last CTAs finish.  Every

@@ -366,7 +366,9 @@ template <bool ACC>
 cudaError_t linear_launch(const LinParams &p, const CUtensorMap &tx, const CUtensorMap &tw, size_t smem, int grid,
                           cudaStream_t st)
 {
-    cudaError_t e = cudaFuncSetAttribute(linear_tc_kernel<ACC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = check_smem_fits((const void *)linear_tc_kernel<ACC>, smem);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(linear_tc_kernel<ACC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     return launch_pdl(linear_tc_kernel<ACC>, dim3(grid), dim3(LTHREADS), smem, st, p, tx, tw);
 }

@@ -922,8 +922,10 @@ bool use_pack(int L) { return L >= TM && L <= kPackMaxBlocks * TKB; }
 template <int NKB, bool SMALL_E, bool PACK>
 cudaError_t tc_launch(const TcParams &p, size_t smem, int grid, cudaStream_t st)
 {
-    cudaError_t e = cudaFuncSetAttribute(lis_attn_tc_kernel<NKB, SMALL_E, PACK>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = check_smem_fits((const void *)lis_attn_tc_kernel<NKB, SMALL_E, PACK>, smem);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(lis_attn_tc_kernel<NKB, SMALL_E, PACK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
     if (e != cudaSuccess) return e;
     return launch_pdl(lis_attn_tc_kernel<NKB, SMALL_E, PACK>, dim3(grid), dim3(TTHREADS), smem, st, p);
 }

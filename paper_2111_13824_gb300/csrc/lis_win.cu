@@ -522,8 +522,11 @@ bool small_iexp_w(const IexpC &c) { return ((double)c.q_b * c.q_b + c.q_c) * 327
 template <int D, bool BIAS, bool SMALL_E, int NQ, bool MASK>
 cudaError_t win_launch_q(const WinParams &p, size_t smem, int grid, cudaStream_t st)
 {
-    cudaError_t e = cudaFuncSetAttribute(lis_attn_win_kernel<D, BIAS, SMALL_E, NQ, MASK>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    // the static arrays as compiled for this instantiation, not the estimate the group count used
+    cudaError_t e = check_smem_fits((const void *)lis_attn_win_kernel<D, BIAS, SMALL_E, NQ, MASK>, smem);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(lis_attn_win_kernel<D, BIAS, SMALL_E, NQ, MASK>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     return launch_pdl(lis_attn_win_kernel<D, BIAS, SMALL_E, NQ, MASK>, dim3(grid), dim3(128 * p.ng), smem, st, p);
 }

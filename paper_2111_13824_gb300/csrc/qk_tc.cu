@@ -377,8 +377,9 @@ constexpr size_t kQkStaticSmem = sizeof(QkShared) + 64;
 template <bool FOLD, bool BULK>
 cudaError_t qk_launch(const QkParams &p, const CUtensorMap &tm, size_t smem, int grid, cudaStream_t st)
 {
-    cudaError_t e = cudaFuncSetAttribute(qk_logits_tc_kernel<FOLD, BULK>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = check_smem_fits((const void *)qk_logits_tc_kernel<FOLD, BULK>, smem);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(qk_logits_tc_kernel<FOLD, BULK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     return launch_pdl(qk_logits_tc_kernel<FOLD, BULK>, dim3(grid), dim3(QTHREADS), smem, st, p, tm);
 }
