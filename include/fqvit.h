@@ -54,6 +54,8 @@ FQVIT_API const char *fqvit_last_error(void);
  * two seconds, drains what it issued and returns) since the last call,
  * FQVIT_ERR_INVALID_ARG if fqvit_linear_q met a per-channel weight scale that
  * is not positive and finite (device data the host does not see),
+ * FQVIT_ERR_UNSUPPORTED if a kernel found its shared-memory layout different
+ * from the one the host computed and returned without writing its output,
  * FQVIT_ERR_CUDA if the stream reports an error, else FQVIT_OK.  The word is
  * cleared.  Not part of the paper; a diagnostic of this implementation. */
 FQVIT_API int fqvit_sync_status(void *stream);

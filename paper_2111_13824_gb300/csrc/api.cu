@@ -93,6 +93,10 @@ int fqvit_sync_status(void *stream)
     if (status == 0 || (status == FQVIT_ERR_INVALID_ARG && lst == FQVIT_ERR_TIMEOUT)) status = lst;
     if (status == FQVIT_ERR_TIMEOUT)
         return fail(FQVIT_ERR_TIMEOUT, "a kernel abandoned a bounded wait (results of that launch are invalid)");
+    if (status == FQVIT_ERR_UNSUPPORTED)
+        return fail(FQVIT_ERR_UNSUPPORTED,
+                    "a kernel found its shared-memory layout different from the host's (that launch wrote no "
+                    "output)");
     if (status == FQVIT_ERR_INVALID_ARG)
         return fail(FQVIT_ERR_INVALID_ARG,
                     "a Linear layer met a weight scale s_w[n] that is not positive and finite, or a multiplier "

@@ -99,6 +99,8 @@ struct LnArgs {
     int64_t *m2;
 };
 cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st);
+// Reads and clears the LayerNorm kernels' status word (5: a bounded wait gave up).
+cudaError_t read_clear_ln_status(int *status);
 
 // ---- Log-Int-Softmax and BitShift attention (lis.cu) -----------------------
 struct LisArgs {

@@ -993,7 +993,11 @@ cudaError_t read_clear_device_status(int *status, cudaStream_t st)
     if (*status == 0) *status = wst;
     int qst = 0;
     e = read_clear_qk_status(&qst);
+    if (e != cudaSuccess) return e;
     if (*status == 0) *status = qst;
+    int lnst = 0;
+    e = read_clear_ln_status(&lnst);
+    if (*status == 0) *status = lnst;
     return e;
 }
 

@@ -156,6 +156,21 @@ def test_layernorm_edge_rows():
     _assert_ln((xq, 255, alpha, gamma, beta, 5.0, 255))
 
 
+@pytest.mark.parametrize("zp", [0, 128, 255])
+def test_layernorm_extreme_values(zp):
+    """Bytes 0 and 255 only with alpha = 3 on every channel: |Xh| = 2040 at its largest, the bound of
+    the exact squares of the fp32 statistics path; rows of C = 1024 and 4096."""
+    rng = np.random.default_rng(zp)
+    for C in (1024, 4096):
+        rows = 67
+        xq = (rng.integers(0, 2, size=(rows, C)) * 255).astype(np.uint8)
+        xq[0, :] = 255 - zp if zp in (0, 255) else 255
+        alpha = np.full(C, 3, np.uint8)
+        gamma = (1 + 0.1 * rng.normal(size=C)).astype(np.float32)
+        beta = (0.1 * rng.normal(size=C)).astype(np.float32)
+        _assert_ln((xq, zp, alpha, gamma, beta, 0.02, 128))
+
+
 def test_layernorm_synthetic_configs():
     for name in ("deit_s", "vit_b", "swin_s"):
         cfg = synth.CONFIGS[name]
