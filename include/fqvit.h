@@ -432,6 +432,34 @@ FQVIT_API int fqvit_linear_q(const uint8_t *x, int64_t M, int32_t K, int64_t ld_
                              void *workspace, size_t workspace_bytes, void *stream);
 
 /* ------------------------------------------------------------------ */
+/* Head split and merge around the attention core (Fig. 4 dataflow)   */
+/* ------------------------------------------------------------------ */
+
+/*
+ * The QKV Linear's token-major output to head-major Q, K and V codes for
+ * fqvit_qk_logits and the attention calls: qkv [B*L][ld_qkv] uint8 (device),
+ * part p (0 Q, 1 K, 2 V) in columns p*H*d .. p*H*d + H*d - 1, head h at
+ * + h*d; q, k, v [B*H][L][ld_head] int8 (device, caller-owned), row
+ * (b*H + h)*L + i = the code of token b*L + i minus 128 (the signed form
+ * those calls take; the zero point moves by -128 with it).  Bytes past d of
+ * an output row are not written.  Supported: d a multiple of 16, ld_qkv and
+ * ld_head multiples of 16 with 16-byte aligned bases.  Errors: INVALID_ARG
+ * (NULL, shapes, strides, alignment), UNSUPPORTED (d).
+ */
+FQVIT_API int fqvit_split_qkv(const uint8_t *qkv, int64_t B, int32_t L, int32_t H, int32_t d, int64_t ld_qkv,
+                              int8_t *q, int8_t *k, int8_t *v, int64_t ld_head, void *stream);
+
+/*
+ * The attention output's head-major rows back to token rows for the
+ * projection Linear: heads [B*H][L][ld_head] uint8 (device; the 8-bit output
+ * of fqvit_lis_attention_q) -> out [B*L][ld_out] uint8 (device,
+ * caller-owned), head h in columns h*d .. h*d + d - 1 (codes unchanged).
+ * Supported and errors as fqvit_split_qkv.
+ */
+FQVIT_API int fqvit_merge_heads(const uint8_t *heads, int64_t B, int32_t L, int32_t H, int32_t d,
+                                int64_t ld_head, uint8_t *out, int64_t ld_out, void *stream);
+
+/* ------------------------------------------------------------------ */
 /* One layer: norm1 LayerNorm and the attention core (Fig. 4 dataflow) */
 /* ------------------------------------------------------------------ */
 

@@ -602,6 +602,43 @@ int fqvit_linear_q(const uint8_t *x, int64_t M, int32_t K, int64_t ld_x, int32_t
     return cuda_status(fqvit::launch_linear(a, as_stream(stream)), who);
 }
 
+static int heads_check(const char *who, int64_t B, int32_t H, int32_t L, int32_t d, int64_t ld_src,
+                       int64_t min_src, const void *src, int64_t ld_dst, int64_t min_dst)
+{
+    if (!src) return fail(FQVIT_ERR_INVALID_ARG, "%s: NULL pointer", who);
+    if (B < 1 || H < 1 || L < 1 || d < 1 || ld_src < min_src || ld_dst < min_dst)
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: bad shape B=%lld H=%d L=%d d=%d", who, (long long)B, H, L, d);
+    if (d % 16) return fail(FQVIT_ERR_UNSUPPORTED, "%s: d=%d (a multiple of 16)", who, d);
+    if (ld_src % 16 || ld_dst % 16 || !aligned(src, 16))
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: misaligned pointer or row stride", who);
+    return FQVIT_OK;
+}
+
+int fqvit_split_qkv(const uint8_t *qkv, int64_t B, int32_t L, int32_t H, int32_t d, int64_t ld_qkv, int8_t *q,
+                    int8_t *k, int8_t *v, int64_t ld_head, void *stream)
+{
+    const char *who = "split_qkv";
+    int rc = heads_check(who, B, H, L, d, ld_qkv, 3 * (int64_t)H * d, qkv, ld_head, d);
+    if (rc) return rc;
+    if (!q || !k || !v) return fail(FQVIT_ERR_INVALID_ARG, "%s: NULL pointer", who);
+    if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16))
+        return fail(FQVIT_ERR_INVALID_ARG, "%s: misaligned pointer or row stride", who);
+    fqvit::HeadsArgs a{qkv, nullptr, q, k, v, nullptr, B, H, L, d, ld_qkv, ld_head};
+    return cuda_status(fqvit::launch_split_qkv(a, as_stream(stream)), who);
+}
+
+int fqvit_merge_heads(const uint8_t *heads, int64_t B, int32_t L, int32_t H, int32_t d, int64_t ld_head,
+                      uint8_t *out, int64_t ld_out, void *stream)
+{
+    const char *who = "merge_heads";
+    int rc = heads_check(who, B, H, L, d, ld_head, d, heads, ld_out, (int64_t)H * d);
+    if (rc) return rc;
+    if (!out) return fail(FQVIT_ERR_INVALID_ARG, "%s: NULL pointer", who);
+    if (!aligned(out, 16)) return fail(FQVIT_ERR_INVALID_ARG, "%s: misaligned pointer or row stride", who);
+    fqvit::HeadsArgs a{nullptr, heads, nullptr, nullptr, nullptr, out, B, H, L, d, ld_head, ld_out};
+    return cuda_status(fqvit::launch_merge_heads(a, as_stream(stream)), who);
+}
+
 int fqvit_block_int(const fqvit_block_desc *b, void *stream)
 {
     if (!b) return fail(FQVIT_ERR_INVALID_ARG, "block_int: NULL descriptor");

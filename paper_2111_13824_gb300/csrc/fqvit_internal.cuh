@@ -99,6 +99,19 @@ struct LnArgs {
     int64_t *m2;
 };
 cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st);
+
+// ---- head split and merge of a block (heads.cu) ------------------------------
+struct HeadsArgs {
+    const uint8_t *src;      // split: the QKV Linear's output [B L][ld_src]
+    const uint8_t *src_u8;   // merge: attention output [B H][L][ld_src]
+    int8_t *q, *k, *v;       // split: [B H][L][ld_dst]
+    uint8_t *dst_u8;         // merge: [B L][ld_dst]
+    int64_t B;
+    int H, L, d;
+    int64_t ld_src, ld_dst;
+};
+cudaError_t launch_split_qkv(const HeadsArgs &a, cudaStream_t st);
+cudaError_t launch_merge_heads(const HeadsArgs &a, cudaStream_t st);
 // Reads and clears the LayerNorm kernels' status word (5: a bounded wait gave up).
 cudaError_t read_clear_ln_status(int *status);
 

@@ -53,6 +53,7 @@ EXPORTS = (
     "fqvit_lis_softmax_masked", "fqvit_lis_attention_masked", "fqvit_lis_attention_masked_q",
     "fqvit_qk_logits", "fqvit_qk_workspace_size", "fqvit_qk_lis_attention",
     "fqvit_linear_pack_weight", "fqvit_linear_workspace_size", "fqvit_linear_q",
+    "fqvit_split_qkv", "fqvit_merge_heads",
     "fqvit_selftest_bounded_wait",
 )
 
@@ -100,6 +101,8 @@ def load(path: str | Path | None = None):
         "fqvit_linear_q": ([P, i64, i32, i64, i32, f32, P, i32, P, P, f32, i32, P, i64, P, i64, P, sz, P],
                            ctypes.c_int),
         "fqvit_block_int": ([P, P], ctypes.c_int),
+        "fqvit_split_qkv": ([P, i64, i32, i32, i32, i64, P, P, P, i64, P], ctypes.c_int),
+        "fqvit_merge_heads": ([P, i64, i32, i32, i32, i64, P, i64, P], ctypes.c_int),
         "fqvit_sync_status": ([P], ctypes.c_int),
         "fqvit_calibrate_ptf_noalloc": ([P, i64, i32, i64, i32, i32, P, P, P, P, P], ctypes.c_int),
         "fqvit_calibrate_minmax": ([P, i64, i32, i64, P, P, sz, P], ctypes.c_int),
@@ -454,6 +457,26 @@ def linear_q(x: torch.Tensor, zp_x: int, s_x: float, w_h: torch.Tensor, s_w: tor
                                  float(s_y), int(zp_y), _p(out), _ld(out), _p(acc),
                                  _ld(acc) if acc is not None else 0, _p(workspace), workspace.numel(),
                                  _stream(stream)))
+    return out
+
+
+def split_qkv(qkv: torch.Tensor, B: int, L: int, H: int, d: int, ld_head: int | None = None, stream=None):
+    """The QKV Linear's uint8 output [B*L, >= 3 H d] -> int8 q, k, v [B*H, L, d] (codes minus 128)
+    (fqvit_split_qkv); ld_head pads the head rows (then the views are [B*H, L, ld_head][..., :d])."""
+    ld = d if ld_head is None else ld_head
+    outs = [torch.empty(B * H, L, ld, dtype=torch.int8, device=qkv.device) for _ in range(3)]
+    _check(load().fqvit_split_qkv(_p(qkv), int(B), int(L), int(H), int(d), _ld(qkv), _p(outs[0]), _p(outs[1]),
+                                  _p(outs[2]), ld, _stream(stream)))
+    return tuple(o[..., :d] for o in outs)
+
+
+def merge_heads(heads: torch.Tensor, B: int, L: int, H: int, out: torch.Tensor | None = None, stream=None):
+    """Head-major uint8 rows [B*H, L, d] -> token rows [B*L, H d] (fqvit_merge_heads)."""
+    d = heads.shape[-1]
+    if out is None:
+        out = torch.empty(B * L, H * d, dtype=torch.uint8, device=heads.device)
+    _check(load().fqvit_merge_heads(_p(heads), int(B), int(L), int(H), int(d), heads.stride(-2), _p(out), _ld(out),
+                                    _stream(stream)))
     return out
 
 
