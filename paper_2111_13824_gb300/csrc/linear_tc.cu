@@ -241,7 +241,13 @@ __global__ void __launch_bounds__(LTHREADS, 1)
         bool ok = true;
         for (int64_t t = t_begin; t < t_end && ok; ++t) {
             const int mt = (int)(t / p.ntiles), nt = (int)(t - (int64_t)mt * p.ntiles);
-            int sum[128];
+            // A chunk's sum v is an exact integer with |v| <= 2^22, so v + 1.5 2^23 is exact and its
+            // bit pattern is 0x4B400000 + v: the patterns are summed as integers (packed fp32 adds,
+            // no conversion instruction) and the bias of the chunks removed at the end (mod 2^32;
+            // the accumulator fits int32).
+            uint32_t sumb[128];
+#pragma unroll
+            for (int i = 0; i < 128; ++i) sumb[i] = 0u;
             for (int c = 0; c < nch; ++c, ++gc) {
                 const uint32_t b = gc & 1;
                 if (!mbar_wait_warp(&sh.cfull[b], (gc >> 1) & 1, abort_flag)) {
@@ -250,14 +256,21 @@ __global__ void __launch_bounds__(LTHREADS, 1)
                 }
                 tc_fence_after();
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {  // 16 columns at a time (registers: sum holds 128)
-                    uint32_t v[16];
-                    tmem_ld16(tl + b * LN + 16 * j, v);
+                for (int j = 0; j < 4; ++j) {  // 32 columns per wait (registers: sumb holds 128)
+                    uint32_t v[32];
+                    tmem_ld16(tl + b * LN + 32 * j, *reinterpret_cast<uint32_t(*)[16]>(v));
+                    tmem_ld16(tl + b * LN + 32 * j + 16, *reinterpret_cast<uint32_t(*)[16]>(v + 16));
                     tmem_wait_ld();
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const int a = __float2int_rn(__uint_as_float(v[i]));  // an exact integer
-                        sum[16 * j + i] = c == 0 ? a : sum[16 * j + i] + a;
+                    for (int i = 0; i < 32; i += 2) {
+                        uint32_t p0, p1;
+                        asm("{ .reg .b64 ra, rm, rd;\n\t"
+                            "mov.b64 ra, {%2, %3};\n\tmov.b64 rm, {%4, %4};\n\t"
+                            "add.rn.f32x2 rd, ra, rm;\n\tmov.b64 {%0, %1}, rd; }"
+                            : "=r"(p0), "=r"(p1)
+                            : "r"(v[i]), "r"(v[i + 1]), "r"(0x4B400000u));
+                        sumb[32 * j + i] += p0;
+                        sumb[32 * j + i + 1] += p1;
                     }
                 }
                 tc_fence_before();
@@ -265,6 +278,9 @@ __global__ void __launch_bounds__(LTHREADS, 1)
                 if (lane == 0) mbar_arrive(&sh.cempty[b]);
             }
             if (!ok) break;
+            int sum[128];
+#pragma unroll
+            for (int i = 0; i < 128; ++i) sum[i] = (int)(sumb[i] - (uint32_t)nch * 0x4B400000u);
             const int64_t row = (int64_t)mt * LM + 32 * q + lane;
             const int col0 = nt * LN + 128 * h;
 #pragma unroll
