@@ -34,6 +34,7 @@
 #include "tc_common.cuh"
 
 #include <cstring>
+#include <type_traits>
 #include <cuda.h>
 #include <cuda_fp16.h>
 #include <cudaTypedefs.h>
@@ -76,6 +77,7 @@ struct LinShared {
     uint64_t full[LST], empty[LST], cfull[2], cempty[2], fin;
     uint32_t tmem;
     int abort_flag;
+    int wide;  // some channel has a shift below 11: the 64-bit requantization
 };
 
 __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int x, int y, uint64_t *bar)
@@ -112,8 +114,29 @@ __device__ __forceinline__ int2 channel_constants(const LinParams &p, int n, boo
     return make_int2(mult | (shift << 24), p.bias ? p.bias[n] : 0);
 }
 
+// mult acc + 2^(shift-1) as a 64-bit product-sum, then its bits shift .. shift + 31: with
+// shift >= 11 (mult < 2^8 then, |acc| < 2^31) the quotient fits 32 bits, and R + zp_y for the
+// saturating pack (before the clip)
+__device__ __forceinline__ int y_pre(int acc, uint32_t chx, int zp_y)
+{
+    const int mult = (int)(chx & 0xFFFFFFu);
+    const uint32_t sh = chx >> 24;
+    const unsigned long long rnd = (1u << sh) >> 1;
+    const long long num = (long long)mult * acc + (long long)rnd;
+    return (int)__funnelshift_r((uint32_t)num, (uint32_t)((unsigned long long)num >> 32), sh) + zp_y;
+}
+
+// two values clipped to 0 .. 255, packed as bytes 0, 1 (c, shifted up 16 bits, above them)
+__device__ __forceinline__ uint32_t pack_sat_u8(int b0, int b1, uint32_t c)
+{
+    uint32_t d;
+    asm("cvt.pack.sat.u8.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(b1), "r"(b0), "r"(c));
+    return d;
+}
+
 // y code of one accumulator (the bias added): (mult acc + 2^(shift-1)) >> shift, + zp_y, clipped
-__device__ __forceinline__ uint32_t y_code(int acc, int2 ch, int zp_y)
+// (out of line: the rare channels with a shift below 11; it keeps the registers of the 32-bit loop)
+__device__ __noinline__ uint32_t y_code(int acc, int2 ch, int zp_y)
 {
     const int mult = ch.x & 0xFFFFFF, shift = ch.x >> 24;
     const long long num = (long long)mult * acc + (long long)((1u << shift) >> 1);
@@ -152,9 +175,15 @@ __global__ void __launch_bounds__(LTHREADS, 1)
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     pdl_wait();  // the set-up above touched no global memory
-    bool bad = false;
-    for (int n = tid; n < p.N; n += LTHREADS) CH[n] = channel_constants(p, n, bad);
+    bool bad = false, wide = false;
+    if (tid == 0) sh.wide = 0;
+    __syncthreads();
+    for (int n = tid; n < p.N; n += LTHREADS) {
+        CH[n] = channel_constants(p, n, bad);
+        wide |= (CH[n].x >> 24) < 11;
+    }
     if (bad) atomicExch(&g_status, 1);
+    if (wide) atomicExch(&sh.wide, 1);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -283,31 +312,43 @@ __global__ void __launch_bounds__(LTHREADS, 1)
             for (int i = 0; i < 128; ++i) sum[i] = (int)(sumb[i] - (uint32_t)nch * 0x4B400000u);
             const int64_t row = (int64_t)mt * LM + 32 * q + lane;
             const int col0 = nt * LN + 128 * h;
+            // the output bytes of a tile row, 16 columns at a time; WIDE: some channel's shift is below
+            // 11 (64-bit requantization), else 32-bit (one loop or the other for the whole tile)
+            auto store_row = [&](auto wide_tag) {
+                constexpr bool WIDE = decltype(wide_tag)::value;
 #pragma unroll
-            for (int g = 0; g < 8; ++g) {
-                const int col = col0 + 16 * g;
-                if (col >= p.N) break;  // N is a multiple of 16: whole groups
-                int a[16];
-                uint32_t w[4];
+                for (int g = 0; g < 8; ++g) {
+                    const int col = col0 + 16 * g;
+                    if (col >= p.N) break;  // N is a multiple of 16: whole groups
+                    int a[16];
+                    uint32_t w[4];
 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const int2 ch = CH[col + i];
-                    a[i] = sum[16 * g + i] + ch.y;
-                    const uint32_t yc = y_code(a[i], ch, p.zp_y);
-                    if ((i & 3) == 0)
-                        w[i >> 2] = yc;
-                    else
-                        w[i >> 2] |= yc << (8 * (i & 3));
-                }
-                if (row < p.M) {
-                    *reinterpret_cast<uint4 *>(p.y + row * p.ld_y + col) = make_uint4(w[0], w[1], w[2], w[3]);
-                    if (ACC) {
-                        int4 *dst = reinterpret_cast<int4 *>(p.acc + row * p.ld_acc + col);
+                    for (int k = 0; k < 4; ++k) {
+                        int r[4];
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) dst[i] = make_int4(a[4 * i], a[4 * i + 1], a[4 * i + 2], a[4 * i + 3]);
+                        for (int u = 0; u < 4; ++u) {
+                            const int i = 4 * k + u;
+                            const int2 ch = CH[col + i];
+                            a[i] = sum[16 * g + i] + ch.y;
+                            r[u] = WIDE ? (int)y_code(a[i], ch, p.zp_y) : y_pre(a[i], (uint32_t)ch.x, p.zp_y);
+                        }
+                        w[k] = pack_sat_u8(r[0], r[1], pack_sat_u8(r[2], r[3], 0u));
+                    }
+                    if (row < p.M) {
+                        *reinterpret_cast<uint4 *>(p.y + row * p.ld_y + col) = make_uint4(w[0], w[1], w[2], w[3]);
+                        if (ACC) {
+                            int4 *dst = reinterpret_cast<int4 *>(p.acc + row * p.ld_acc + col);
+#pragma unroll
+                            for (int i = 0; i < 4; ++i)
+                                dst[i] = make_int4(a[4 * i], a[4 * i + 1], a[4 * i + 2], a[4 * i + 3]);
+                        }
                     }
                 }
-            }
+            };
+            if (sh.wide)  // block-uniform
+                store_row(std::true_type{});
+            else
+                store_row(std::false_type{});
         }
     }
     tc_fence_before();
