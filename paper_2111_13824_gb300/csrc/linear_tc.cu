@@ -21,9 +21,12 @@
 // 128-byte swizzle: per stage a box of 64 (K) x 128 rows of X and 64 x 256 rows
 // of W, four stages.
 //
-// Roles (320 threads): warps 0-7 are the epilogue (warp w reads tensor-memory
-// lanes 32 (w % 4) .. and columns 128 (w / 4) .. of a tile), warp 8 lane 0
-// issues the TMA loads, warp 9 lane 0 the MMAs (M = 128, N <= 256, K = 16).
+// Roles (576 threads): warps 0-15 are the epilogue (warp w reads tensor-memory
+// lanes 32 (w % 4) .. and columns 64 (w / 4) .. of a tile), warp 16 lane 0
+// issues the TMA loads, warp 17 lane 0 the MMAs (M = 128, N <= 256, K = 16).
+// The epilogue adds a chunk's exact fp32 sums as integers (a biased packed add,
+// no conversion instruction) and requantizes in 32-bit arithmetic when every
+// channel's shift is at least 11.
 // Tiles of 128 x 256 outputs; each CTA (one per SM) takes a contiguous range
 // of tiles, N-tiles fastest, so consecutive tiles share their X rows in L2.
 // Two accumulators of 256 tensor-memory columns: the MMAs of the next chunk
@@ -52,8 +55,9 @@ constexpr int LST = 4;                    // stages
 constexpr int LA_BYTES = LM * LK * 2;     // 16 KB
 constexpr int LB_BYTES = LN * LK * 2;     // 32 KB
 constexpr int LSTAGE = LA_BYTES + LB_BYTES;
-constexpr int LTHREADS = 320;
-constexpr int LEPI_WARPS = 8;
+constexpr int LEPI_WARPS = 16;               // epilogue warps: 4 per lane quarter, 64 columns each
+constexpr int LCOLS = LN * 4 / LEPI_WARPS;    // columns of a tile per epilogue thread
+constexpr int LTHREADS = 32 * (LEPI_WARPS + 2);
 constexpr int LMAXN = 4096;               // channels of the shared-memory table
 
 struct LinParams {
@@ -262,9 +266,9 @@ __global__ void __launch_bounds__(LTHREADS, 1)
         }
         __syncwarp();
     } else {
-        // ---- epilogue: warp w, lanes 32 (w % 4) .. (tile rows), columns 128 (w / 4) ..
+        // ---- epilogue: warp w, lanes 32 (w % 4) .. (tile rows), columns LCOLS (w / 4) ..
         const int q = warp & 3, h = warp >> 2;
-        const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(128 * h);
+        const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(LCOLS * h);
         const int nch = (p.ksteps + p.kc - 1) / p.kc;
         uint32_t gc = 0;
         bool ok = true;
@@ -274,9 +278,9 @@ __global__ void __launch_bounds__(LTHREADS, 1)
             // bit pattern is 0x4B400000 + v: the patterns are summed as integers (packed fp32 adds,
             // no conversion instruction) and the bias of the chunks removed at the end (mod 2^32;
             // the accumulator fits int32).
-            uint32_t sumb[128];
+            uint32_t sumb[LCOLS];
 #pragma unroll
-            for (int i = 0; i < 128; ++i) sumb[i] = 0u;
+            for (int i = 0; i < LCOLS; ++i) sumb[i] = 0u;
             for (int c = 0; c < nch; ++c, ++gc) {
                 const uint32_t b = gc & 1;
                 if (!mbar_wait_warp(&sh.cfull[b], (gc >> 1) & 1, abort_flag)) {
@@ -285,7 +289,7 @@ __global__ void __launch_bounds__(LTHREADS, 1)
                 }
                 tc_fence_after();
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {  // 32 columns per wait (registers: sumb holds 128)
+                for (int j = 0; j < LCOLS / 32; ++j) {  // 32 columns per wait
                     uint32_t v[32];
                     tmem_ld16(tl + b * LN + 32 * j, *reinterpret_cast<uint32_t(*)[16]>(v));
                     tmem_ld16(tl + b * LN + 32 * j + 16, *reinterpret_cast<uint32_t(*)[16]>(v + 16));
@@ -307,17 +311,17 @@ __global__ void __launch_bounds__(LTHREADS, 1)
                 if (lane == 0) mbar_arrive(&sh.cempty[b]);
             }
             if (!ok) break;
-            int sum[128];
+            int sum[LCOLS];
 #pragma unroll
-            for (int i = 0; i < 128; ++i) sum[i] = (int)(sumb[i] - (uint32_t)nch * 0x4B400000u);
+            for (int i = 0; i < LCOLS; ++i) sum[i] = (int)(sumb[i] - (uint32_t)nch * 0x4B400000u);
             const int64_t row = (int64_t)mt * LM + 32 * q + lane;
-            const int col0 = nt * LN + 128 * h;
+            const int col0 = nt * LN + LCOLS * h;
             // the output bytes of a tile row, 16 columns at a time; WIDE: some channel's shift is below
             // 11 (64-bit requantization), else 32-bit (one loop or the other for the whole tile)
             auto store_row = [&](auto wide_tag) {
                 constexpr bool WIDE = decltype(wide_tag)::value;
 #pragma unroll
-                for (int g = 0; g < 8; ++g) {
+                for (int g = 0; g < LCOLS / 16; ++g) {
                     const int col = col0 + 16 * g;
                     if (col >= p.N) break;  // N is a multiple of 16: whole groups
                     int a[16];
