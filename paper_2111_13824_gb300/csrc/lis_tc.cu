@@ -680,7 +680,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
                     for (int i = 0; i < 4; ++i) {
                         if (q + 1 + 4 * i <= 15 && lo[i] < 256) {
                             red_add_u32(kTabAbs + ((uint32_t)lo[i] << 8) + 4u * (uint32_t)lane, inc);
-                            atomicAdd(&GT[lane * GT_LD + (lo[i] >> 4)], inc);
+                            red_add_u32(sa(&GT[lane * GT_LD + (lo[i] >> 4)]), inc);
                         }
                     }
                 }

@@ -174,7 +174,11 @@ __device__ __forceinline__ RowSum split_2s(unsigned long long S)
 // warp-collective tcgen05 instructions)
 __device__ __forceinline__ bool mbar_wait_warp(uint64_t *b, uint32_t parity, volatile int *abort_flag)
 {
-    return __all_sync(0xFFFFFFFFu, mbar_wait(b, parity, abort_flag));
+    // a phase that has already completed costs one probe, not the out-of-line wait (whose call makes
+    // the caller save and restore its live registers)
+    bool ok = mbar_try(b, parity);
+    if (!ok) ok = mbar_wait(b, parity, abort_flag);
+    return __all_sync(0xFFFFFFFFu, ok);
 }
 
 __device__ __forceinline__ uint32_t lds32(uint32_t a)
