@@ -70,8 +70,8 @@ __device__ __forceinline__ bool mbar_try_for(uint64_t *b, uint32_t parity, uint3
 // Bounded wait: the thread sleeps in the barrier (woken when the phase completes) in slices of
 // at most 50 us; false on timeout or (honor_abort) when another role gave up.  (Sleeps growing
 // to 256 ns between slices were tried: no gain for long rows, 5-8 % slower for short ones.)
-static __device__ __noinline__ bool mbar_wait(uint64_t *b, uint32_t parity, volatile int *abort_flag,
-                                       bool honor_abort = true)
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t *b, uint32_t parity, volatile int *abort_flag,
+                                            bool honor_abort)
 {
     if (mbar_try(b, parity)) return true;
     const uint64_t t0 = gtimer();
@@ -85,6 +85,14 @@ static __device__ __noinline__ bool mbar_wait(uint64_t *b, uint32_t parity, vola
         }
         __nanosleep(64);
     }
+}
+
+// A completed phase costs one inline probe; the out-of-line wait (whose call makes the caller save and
+// restore its live registers) runs only when the phase is still open.
+__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity, volatile int *abort_flag,
+                                          bool honor_abort = true)
+{
+    return mbar_try(b, parity) || mbar_wait_slow(b, parity, abort_flag, honor_abort);
 }
 
 __device__ __forceinline__ void prefetch_l2(const void *src, uint32_t bytes)
@@ -174,11 +182,7 @@ __device__ __forceinline__ RowSum split_2s(unsigned long long S)
 // warp-collective tcgen05 instructions)
 __device__ __forceinline__ bool mbar_wait_warp(uint64_t *b, uint32_t parity, volatile int *abort_flag)
 {
-    // a phase that has already completed costs one probe, not the out-of-line wait (whose call makes
-    // the caller save and restore its live registers)
-    bool ok = mbar_try(b, parity);
-    if (!ok) ok = mbar_wait(b, parity, abort_flag);
-    return __all_sync(0xFFFFFFFFu, ok);
+    return __all_sync(0xFFFFFFFFu, mbar_wait(b, parity, abort_flag));
 }
 
 __device__ __forceinline__ uint32_t lds32(uint32_t a)
