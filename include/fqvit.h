@@ -396,8 +396,9 @@ FQVIT_API int fqvit_qk_lis_attention(const int8_t *q, int64_t ld_q, int32_t zp_q
 FQVIT_API int fqvit_linear_pack_weight(const int8_t *w, int32_t N, int32_t K, int64_t ld_w, uint16_t *w_h,
                                        void *stream);
 
-/* Bytes of workspace fqvit_linear_q needs: the fp16 copy of the activations,
- * M x K x 2.  0 for a bad shape. */
+/* Bytes of workspace fqvit_linear_q needs: the fp16 copy of the activations
+ * (M x K x 2, rounded up to 256) and 4096 int32 per-channel weight sums.
+ * 0 for a bad shape. */
 FQVIT_API size_t fqvit_linear_workspace_size(int64_t M, int32_t K);
 
 /*

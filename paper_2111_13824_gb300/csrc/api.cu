@@ -558,7 +558,7 @@ int fqvit_selftest_bounded_wait(void *stream)
 size_t fqvit_linear_workspace_size(int64_t M, int32_t K)
 {
     if (M < 1 || K < 1) return 0;
-    return (size_t)M * (size_t)K * 2;
+    return fqvit::linear_workspace_bytes(M, K);
 }
 
 int fqvit_linear_pack_weight(const int8_t *w, int32_t N, int32_t K, int64_t ld_w, uint16_t *w_h, void *stream)

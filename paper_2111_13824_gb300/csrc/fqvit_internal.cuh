@@ -212,6 +212,8 @@ struct LinearArgs {
 };
 bool linear_supported(const LinearArgs &a);
 cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st);
+// Workspace of launch_linear: the fp16 copy of x (M K 2 bytes, rounded up to 256) and 4096 int32 weight sums.
+size_t linear_workspace_bytes(int64_t M, int K);
 cudaError_t launch_linear_pack_weight(const int8_t *w, int N, int K, int64_t ld_w, uint16_t *w_h, cudaStream_t st);
 cudaError_t read_clear_linear_status(int *status);
 // one CTA whose wait on an mbarrier that nothing completes gives up (the bounded wait's timeout)

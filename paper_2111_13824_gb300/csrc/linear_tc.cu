@@ -7,17 +7,18 @@
 // with N1_n, N2_n the dyadic form of M_n = s_x s_w[n] / s_y (the output stage of
 // the supplement's LayerNorm; N1_n <= 0 is a product by N2_n 2^min(-N1_n, 10)).
 //
-// Exactness.  x - zp_x lies in -255 .. 255 and w in -128 .. 127, both exact in
-// fp16, every product exact in fp32.  A sum of such integers is exact in fp32
-// while its partial sums stay within 2^24; the reduction runs in chunks of kc
-// steps of 64 with 64 kc max|x - zp_x| 128 <= 2^22 (kc = 2 for zp_x at 0 or
-// 255, 4 for zp_x = 128), the scale at which the attention's BitShift product
-// (sums near 2^22 with unit terms) is exact on these tensor cores.  Each chunk
-// is accumulated afresh in tensor memory and added in int32 by the epilogue.
+// Exactness.  The product runs on x - 128 (in -128 .. 127 whatever zp_x; the
+// term (128 - zp_x) sum_k w[n][k] joins the bias) and w in -128 .. 127, both
+// exact in fp16, every product exact in fp32.  A sum of such integers is exact
+// in fp32 while its partial sums stay within 2^24; the reduction runs in chunks
+// of 4 steps of 64 (64 4 128 128 = 2^22), the scale at which the attention's
+// BitShift product (sums near 2^22 with unit terms) is exact on these tensor
+// cores.  Each chunk is accumulated afresh in tensor memory and added as an
+// integer by the epilogue.
 //
 // Layout.  The weights are converted once to fp16 [N][K] (fqvit_linear_pack_weight);
-// the activations per call to fp16 (x - zp_x) [M][K] in a workspace by an
-// elementwise kernel.  Both reach shared memory by TMA tensor loads with the
+// per call a small kernel sums each channel's weights and an elementwise kernel
+// writes the activations as fp16 (x - 128) [M][K], both into the workspace.  Both reach shared memory by TMA tensor loads with the
 // 128-byte swizzle: per stage a box of 64 (K) x 128 rows of X and 64 x 256 rows
 // of W, four stages.
 //
@@ -69,6 +70,8 @@ struct LinParams {
     float s_x, s_y;
     const float *s_w;
     const int32_t *bias;
+    const int32_t *wsum;  // sum_k w[n][k], for the bias term of the shifted activations
+    int zcorr;            // 128 - zp_x
     uint8_t *y;
     int64_t ld_y;
     int32_t *acc;
@@ -115,7 +118,8 @@ __device__ __forceinline__ int2 channel_constants(const LinParams &p, int n, boo
     } else {
         bad = true;
     }
-    return make_int2(mult | (shift << 24), p.bias ? p.bias[n] : 0);
+    // the product runs on x - 128: sum_k (x - zp_x) w = sum_k (x - 128) w + (128 - zp_x) sum_k w
+    return make_int2(mult | (shift << 24), (p.bias ? p.bias[n] : 0) + p.zcorr * p.wsum[n]);
 }
 
 // mult acc + 2^(shift-1) as a 64-bit product-sum, then its bits shift .. shift + 31: with
@@ -476,9 +480,44 @@ cudaError_t launch_linear_pack_weight(const int8_t *w, int N, int K, int64_t ld_
     return launch_bytes_to_half(reinterpret_cast<const uint8_t *>(w), N, K, ld_w, 0x80808080u, 128, w_h, st);
 }
 
+// sum_k w[n][k] of the packed fp16 weights: a warp per channel; |sum| <= 2^21, exact in fp32
+__global__ void __launch_bounds__(256) weight_sum_kernel(const uint16_t *w_h, int N, int K, int32_t *wsum)
+{
+    pdl_release();
+    pdl_wait();
+    const int n = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+    if (n >= N) return;
+    const uint4 *row = reinterpret_cast<const uint4 *>(w_h + (size_t)n * K);  // K a multiple of 8
+    float s = 0.0f;
+    for (int c = lane; c < K / 8; c += 32) {
+        const uint4 v = row[c];
+        const __half2 *h = reinterpret_cast<const __half2 *>(&v);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = __half22float2(h[i]);
+            s += f.x + f.y;
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) wsum[n] = __float2int_rn(s);
+}
+
+size_t linear_workspace_bytes(int64_t M, int K)
+{
+    return ((size_t)M * (size_t)K * 2 + 255) / 256 * 256 + (size_t)LMAXN * sizeof(int32_t);
+}
+
 cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st)
 {
-    cudaError_t e = launch_bytes_to_half(a.x, a.M, a.K, a.ld_x, 0u, a.zp_x, a.xh, st);
+    // The activations enter the product as x - 128 (|x - 128| <= 128 whatever zp_x, so a chunk holds
+    // 4 K-steps); (128 - zp_x) sum_k w joins the bias.
+    int32_t *wsum = reinterpret_cast<int32_t *>(reinterpret_cast<unsigned char *>(a.xh) +
+                                                ((size_t)a.M * (size_t)a.K * 2 + 255) / 256 * 256);
+    cudaError_t e = launch_pdl(weight_sum_kernel, dim3((unsigned)((a.N + 7) / 8)), dim3(256), 0, st, a.w_h, a.N, a.K,
+                               wsum);
+    if (e != cudaSuccess) return e;
+    e = launch_bytes_to_half(a.x, a.M, a.K, a.ld_x, 0u, 128, a.xh, st);
     if (e != cudaSuccess) return e;
     CUtensorMap tx, tw;
     memset(&tx, 0, sizeof(tx));
@@ -490,8 +529,9 @@ cudaError_t launch_linear(const LinearArgs &a, cudaStream_t st)
     p.N = a.N;
     p.K = a.K;
     p.ksteps = (a.K + LK - 1) / LK;
-    const int maxabs = a.zp_x > 255 - a.zp_x ? a.zp_x : 255 - a.zp_x;  // 128 .. 255
-    p.kc = 512 / maxabs;  // 64 kc maxabs 128 <= 2^22
+    p.kc = 4;  // 64 kc 128 128 <= 2^22 (|x - 128| <= 128, |w| <= 128)
+    p.wsum = wsum;
+    p.zcorr = 128 - a.zp_x;
     p.zp_y = a.zp_y;
     p.s_x = a.s_x;
     p.s_y = a.s_y;
