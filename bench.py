@@ -16,6 +16,9 @@ timed steps run as one CUDA graph holding only the kernels, which are
 launched with programmatic dependent launch (a kernel's set-up overlaps the
 previous kernel's tail); the per-kernel times come from a second graph of up to
 three steps with timing events around each kernel (--no-graph: eager launches).
+Event nodes between kernels serialise them and add their own gaps, so each kernel
+kind is also timed alone: its launches of those steps back to back between one
+pair of events (`back_to_back`, the launches overlapping as in the step).
 
 Prints ONE JSON line (rank 0).
 
@@ -463,7 +466,24 @@ def time_config(fqvit, cfg, layers, args, steps, warmup, dev, ws, sample_clocks=
                 mark("attn", k, 1)
                 k += 1
 
-    graph = ev_graph = None
+    # each kernel kind alone, its launches of ev_steps steps back to back between one pair of events
+    # (programmatic dependent launch overlaps each launch's set-up with the previous one's tail, as in
+    # the step; no event between two launches)
+    grp = {k: (torch.cuda.Event(**ev_kw), torch.cuda.Event(**ev_kw)) for k in ("ln", "attn")}
+
+    def enqueue_groups():
+        grp["ln"][0].record()
+        for _ in range(ev_steps):
+            for ly in layers:
+                layernorm(fqvit, ly)
+        grp["ln"][1].record()
+        grp["attn"][0].record()
+        for _ in range(ev_steps):
+            for ly in layers:
+                attention(fqvit, ly, args.out8)
+        grp["attn"][1].record()
+
+    graph = ev_graph = grp_graph = None
     if use_graph:
         try:
             graph = torch.cuda.CUDAGraph()
@@ -472,13 +492,17 @@ def time_config(fqvit, cfg, layers, args, steps, warmup, dev, ws, sample_clocks=
             ev_graph = torch.cuda.CUDAGraph()
             with torch.cuda.graph(ev_graph):
                 enqueue_steps(ev_steps, True)
+            grp_graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(grp_graph):
+                enqueue_groups()
             graph.replay()  # upload and one untimed pass
             torch.cuda.synchronize()
         except Exception as exc:  # noqa: BLE001 - any capture failure falls back to eager launches
             print(f"bench: CUDA graph unavailable ({type(exc).__name__}: {exc}); eager launches", file=sys.stderr)
-            graph = ev_graph = None
+            graph = ev_graph = grp_graph = None
             torch.cuda.synchronize()
             new_events(dict(enable_timing=True))
+            grp = {k: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for k in grp}
     clocks = ClockSampler(torch.cuda.current_device()) if sample_clocks else None
     if ws > 1:
         torch.distributed.barrier()
@@ -507,7 +531,14 @@ def time_config(fqvit, cfg, layers, args, steps, warmup, dev, ws, sample_clocks=
     else:
         enqueue_steps(ev_steps, True)
     torch.cuda.synchronize()
+    if grp_graph is not None:
+        grp_graph.replay()
+    else:
+        enqueue_groups()
+    torch.cuda.synchronize()
     fqvit.sync_status()
+    n_launch = ev_steps * len(layers)
+    grp_ms = {k: grp[k][0].elapsed_time(grp[k][1]) / n_launch for k in grp}
     attn_ms = [a.elapsed_time(b) for a, b in ev["attn"]]
     ln_ms = [a.elapsed_time(b) for a, b in ev["ln"]]
     merge_ms = [a.elapsed_time(b) for a, b in ev["merge"]]
@@ -515,7 +546,7 @@ def time_config(fqvit, cfg, layers, args, steps, warmup, dev, ws, sample_clocks=
     lb = [ln_bytes(ly["rows"], ly["C"]) for ly in layers]
     mb = [ln_bytes(m["rows"], m["C"]) for m in merges]
     return dict(elapsed_ms=elapsed_ms, ms_per_step=elapsed_ms / steps, graph=graph is not None, clocks=clk,
-                ev_steps=ev_steps, attn_ms=attn_ms, ln_ms=ln_ms, merge_ms=merge_ms, ab=ab, lb=lb, mb=mb,
+                ev_steps=ev_steps, attn_ms=attn_ms, ln_ms=ln_ms, merge_ms=merge_ms, grp_ms=grp_ms, ab=ab, lb=lb, mb=mb,
                 merges=merges, step_bytes=sum(ab) + sum(lb) + sum(mb))
 
 
@@ -523,13 +554,21 @@ def kernel_stats(t, peak, ev_steps):
     """Per-kernel byte rates (algorithmic bytes over CUDA-event durations) of a time_config result."""
     attn_gbs = sum(t["ab"]) * ev_steps / (sum(t["attn_ms"]) / 1e3) / 1e9
     ln_gbs = sum(t["lb"]) * ev_steps / (sum(t["ln_ms"]) / 1e3) / 1e9
+    def b2b(kind, nbytes):
+        # the same launches back to back, one event pair around them (no event between kernels)
+        ms = t["grp_ms"][kind]
+        gbs = sum(nbytes) / len(nbytes) / (ms / 1e3) / 1e9
+        return {"ms_per_launch": round(ms, 5), "gbs": round(gbs, 1), "frac": round(gbs / peak, 4)}
+
     out = {
         "attention": {"gbs": round(attn_gbs, 1), "frac": round(attn_gbs / peak, 4),
                       "ms_per_launch": round(sum(t["attn_ms"]) / len(t["attn_ms"]), 5),
-                      "bytes_per_launch": round(sum(t["ab"]) / len(t["ab"]))},
+                      "bytes_per_launch": round(sum(t["ab"]) / len(t["ab"])),
+                      "back_to_back": b2b("attn", t["ab"])},
         "layernorm": {"gbs": round(ln_gbs, 1), "frac": round(ln_gbs / peak, 4),
                       "ms_per_launch": round(sum(t["ln_ms"]) / len(t["ln_ms"]), 5),
-                      "bytes_per_launch": round(sum(t["lb"]) / len(t["lb"]))},
+                      "bytes_per_launch": round(sum(t["lb"]) / len(t["lb"])),
+                      "back_to_back": b2b("ln", t["lb"])},
     }
     if t["merges"]:
         mg = sum(t["mb"]) * ev_steps / (sum(t["merge_ms"]) / 1e3) / 1e9
