@@ -393,9 +393,18 @@ __global__ void __launch_bounds__(stg::kStageThreads, 1) ln_stage_kernel(LnArgs 
         uint64_t *bar = &bars[warp][s];
         if (lane == 0) expect_tx(bar, (uint32_t)nv * (uint32_t)C);
         __syncwarp();
-        for (int k = lane; k < nv; k += 32) {
-            const int sg = k / R, j = k - sg * R;
-            bulk_load(ring + s * stage_bytes + sg * seg_stride + j * C, a.xq + (r0 + k) * a.ld_in, (uint32_t)C, bar);
+        if (a.ld_in == C) {  // packed rows: a segment's rows are one contiguous copy
+            for (int sg = lane; sg * R < nv; sg += 32) {
+                const int cnt = nv - sg * R < R ? nv - sg * R : R;
+                bulk_load(ring + s * stage_bytes + sg * seg_stride, a.xq + (r0 + (int64_t)sg * R) * C,
+                          (uint32_t)(cnt * C), bar);
+            }
+        } else {
+            for (int k = lane; k < nv; k += 32) {
+                const int sg = k / R, j = k - sg * R;
+                bulk_load(ring + s * stage_bytes + sg * seg_stride + j * C, a.xq + (r0 + k) * a.ld_in, (uint32_t)C,
+                          bar);
+            }
         }
     };
 
