@@ -287,7 +287,28 @@ __device__ __forceinline__ StageConsts stage_consts(unsigned char *smem, int nch
     return k;
 }
 
-__device__ void stage_prologue(const LnArgs &a, const StageConsts &k, LnShared &sh)
+// the parameters of channels c0 and c0 + blockDim.x (loaded before the rows' bulk copies are issued,
+// so that they do not queue behind them)
+struct ChLoad {
+    float g0, b0, g1, b1;
+    int al0, al1;
+};
+
+__device__ __forceinline__ ChLoad ch_load(const LnArgs &a, int c0)
+{
+    const int c1 = c0 + blockDim.x;
+    const bool has0 = c0 < a.C, has1 = c1 < a.C;
+    ChLoad l;
+    l.g0 = has0 ? a.gamma[c0] : 1.0f;
+    l.b0 = has0 ? a.beta[c0] : 0.0f;
+    l.al0 = has0 ? a.alpha[c0] : 0;
+    l.g1 = has1 ? a.gamma[c1] : 1.0f;
+    l.b1 = has1 ? a.beta[c1] : 0.0f;
+    l.al1 = has1 ? a.alpha[c1] : 0;
+    return l;
+}
+
+__device__ void stage_prologue(const LnArgs &a, const StageConsts &k, LnShared &sh, const ChLoad &first)
 {
     if (threadIdx.x == 0) {
         sh.gsmax = 0.0f;
@@ -305,8 +326,9 @@ __device__ void stage_prologue(const LnArgs &a, const StageConsts &k, LnShared &
       // two channels per pass, their loads issued together
       const int c1 = c0 + blockDim.x;
       const bool has1 = c1 < a.C;
-      const float g0 = a.gamma[c0], b0 = a.beta[c0], g1 = has1 ? a.gamma[c1] : 1.0f, b1 = has1 ? a.beta[c1] : 0.0f;
-      const int al0 = a.alpha[c0], al1 = has1 ? a.alpha[c1] : 0;
+      const ChLoad l = c0 == (int)threadIdx.x ? first : ch_load(a, c0);
+      const float g0 = l.g0, b0 = l.b0, g1 = l.g1, b1 = l.b1;
+      const int al0 = l.al0, al1 = l.al1;
 #pragma unroll
       for (int u = 0; u < 2; ++u) {
         if (u == 1 && !has1) break;
@@ -408,9 +430,10 @@ __global__ void __launch_bounds__(stg::kStageThreads, 1) ln_stage_kernel(LnArgs 
         }
     };
 
-    issue(wg0, 0);  // the first two groups arrive while the channel constants are derived
-    issue(wg0 + wgs, 1);
-    stage_prologue(a, K, sh);
+    const ChLoad first = ch_load(a, threadIdx.x);
+    issue(wg0, 0);  // the first group arrives while the channel constants are derived
+    stage_prologue(a, K, sh, first);
+    issue(wg0 + wgs, 1);  // the second once the first groups of every SM have the memory system to themselves
     const bool fp_m2 = sh.amax <= 3;
     const int64_t zsum = (int64_t)a.zp_in * sh.sumw;
     const float2 zh = make_float2((float)a.zp_out + 0.5f, (float)a.zp_out + 0.5f);
