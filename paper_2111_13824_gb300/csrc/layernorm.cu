@@ -431,9 +431,9 @@ __global__ void __launch_bounds__(stg::kStageThreads, 1) ln_stage_kernel(LnArgs 
     };
 
     const ChLoad first = ch_load(a, threadIdx.x);
-    issue(wg0, 0);  // the first group arrives while the channel constants are derived
+    issue(wg0, 0);  // the first two groups arrive while the channel constants are derived
+    issue(wg0 + wgs, 1);
     stage_prologue(a, K, sh, first);
-    issue(wg0 + wgs, 1);  // the second once the first groups of every SM have the memory system to themselves
     const bool fp_m2 = sh.amax <= 3;
     const int64_t zsum = (int64_t)a.zp_in * sh.sumw;
     const float2 zh = make_float2((float)a.zp_out + 0.5f, (float)a.zp_out + 0.5f);
