@@ -417,8 +417,10 @@ FQVIT_API size_t fqvit_linear_workspace_size(int64_t M, int32_t K);
  * y [M][ld_y] uint8 (device, caller-owned); acc_opt [M][ld_acc] int32
  * (device, may be NULL) receives acc; workspace (device, caller-owned, at
  * least fqvit_linear_workspace_size(M, K) bytes, 16-byte aligned) is
- * overwritten.  Two launches on `stream` (the fp16 copy of x, then the
- * tensor-core product and its requantization).
+ * overwritten.  Three launches on `stream`: the per-channel weight sums, the
+ * fp16 copy of x - 128 (the product runs on x - 128 and adds
+ * (128 - zp_x) sum_k w[n][k] to the bias, the same integer), then the
+ * tensor-core product and its requantization.
  * Supported: K <= 16384 a multiple of 8, N <= 4096 a multiple of 16,
  * ld_x a multiple of 8 with an 8-byte aligned base, ld_y a multiple of 16 and
  * ld_acc of 4 with 16-byte aligned bases, zero points in 0..255.  Errors:
