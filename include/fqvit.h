@@ -358,9 +358,9 @@ FQVIT_API int fqvit_qk_logits(const int8_t *q, int64_t ld_q, int32_t zp_q, const
                               float s_logit, int32_t zp_logit, int8_t *logits, int64_t ld_logit, void *stream);
 
 /* Bytes of logits workspace fqvit_qk_lis_attention needs for groups of
- * group_heads heads (<= 0: the library's choice, at most 48 MiB of logits so
- * that a group's logits stay in the 129 MB L2 between its two kernels):
- * group x L x ld with ld = L rounded up to 16.  0 for a bad shape. */
+ * group_heads heads (<= 0: the library's choice, every head in one group up to
+ * 1 GiB of logits; a smaller group bounds the workspace at the cost of more
+ * launches): group x L x ld with ld = L rounded up to 16.  0 for a bad shape. */
 FQVIT_API size_t fqvit_qk_workspace_size(int64_t BH, int32_t L, int64_t group_heads);
 
 /*
