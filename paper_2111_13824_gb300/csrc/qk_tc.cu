@@ -18,15 +18,20 @@
 // memory (B operand: keys x 64, K-major, 128-byte swizzle, d padded to 64 with
 // zeros); per tile, the 128 query rows of Q likewise (A operand).  The keys go
 // through the tensor cores in chunks of 128 (M = 128, N <= 128, K = 64) into four
-// tensor-memory buffers, up to four chunks ahead of the epilogue; the 16 warps read a
-// chunk back (warp w: lanes 32 (w % 4) .., columns 32 (w / 4) ..), quantize it
-// and write the bytes into a shared-memory tile of the output; all threads then
-// copy the tile out with coalesced 16-byte stores (its rows are contiguous in
-// global memory).  A bulk copy of the tile drained at a fraction of the SM's
-// share of the write bandwidth and held up the next tile; per-thread stores of
-// each row's pieces scattered the writes.  Every wait is bounded: after two
-// seconds the kernel records a timeout status, drains what it issued and
-// returns.
+// tensor-memory buffers, up to four chunks ahead of the epilogue.  Roles:
+//   warps 0-15 (epilogue): convert the operands, then read each chunk back
+//     (warp w: lanes 32 (w % 4) .., columns 32 (w / 4) ..), quantize it and
+//     write the bytes into a staging buffer (or, for strides the tensor store
+//     cannot take, into a shared-memory tile of the output that all of them
+//     copy out with coalesced 16-byte stores);
+//   warp 16, lane 0: the bulk copies of the next tile's Q and head's K and the
+//     MMAs (a tcgen05.mma holds its issuing thread about 200 cycles, so it does
+//     nothing else);
+//   warp 17, lane 0: the tensor stores of the staging buffers.
+// They meet only on mbarriers (chunk computed / read, staging written / read,
+// operands converted), so no warp waits at a block barrier for another's MMA
+// issue.  Every wait is bounded: after two seconds the kernel records a timeout
+// status, drains what it issued and returns.
 #include "fqvit_internal.cuh"
 #include "tc_common.cuh"
 
@@ -46,7 +51,13 @@ constexpr int QM = 128;          // query rows per tile (MMA M)
 constexpr int QNC = 128;         // keys per chunk (MMA N of a full chunk)
 constexpr int QNBUF = 4;         // tensor-memory buffers of a chunk (all 512 columns)
 constexpr int QKD = 64;          // the MMA's reduction: d padded to 64
-constexpr int QTHREADS = 512;
+constexpr int QTHREADS = 512;    // epilogue threads (16 warps)
+constexpr int QEPI_WARPS = QTHREADS / 32;
+constexpr int QMMA_WARP = QEPI_WARPS;      // warp 16, lane 0: operand copies and MMAs
+constexpr int QALL = QTHREADS + 64;        // + warp 17, lane 0: tensor stores
+// Register bound of the launch: 18 warps put five on two of the four schedulers, whose register files
+// (16384 each) then allow 96 per thread, the bound a block of 640 threads gets.
+constexpr int QBOUND = 640;
 constexpr int QMAXL = 640;       // keys of the longest row
 constexpr int QROW = QKD * 2;    // bytes of an fp16 operand row
 constexpr int QNST = 3;          // BULK: staging buffers of a chunk's output (128 x 128 bytes each)
@@ -67,10 +78,14 @@ struct QkParams {
 };
 
 struct QkShared {
-    uint64_t sfull[QNBUF], fin, qload, kload;
+    uint64_t sfull[QNBUF];   // the chunk in tensor-memory buffer b is computed (MMA commit)
+    uint64_t sempty[QNBUF];  // every epilogue warp has read buffer b
+    uint64_t stfull[QNST];   // every epilogue warp has written staging buffer s (BULK)
+    uint64_t stfree[QNST];   // the tensor store of staging buffer s has read it (BULK)
+    uint64_t opsready;       // the tile's Q (and a new head's K) are in the operand layout
+    uint64_t fin, qload, kload;
     uint32_t tmem;
     int abort_flag;
-    int stop;
 };
 
 __device__ __forceinline__ uint32_t pack_sat_s8(int hi, int lo, uint32_t c)
@@ -123,7 +138,7 @@ __device__ __forceinline__ int logit_of(uint32_t acc_bits, const QkParams &p, ui
 // one chunk overlaps the work on the next.  Else each thread loads its codes from global
 // memory as it converts them, and the tile's output is copied out from a shared-memory tile.
 template <bool FOLD, bool BULK>
-__global__ void __launch_bounds__(QTHREADS, 1)
+__global__ void __launch_bounds__(QBOUND, 1)
     qk_logits_tc_kernel(const __grid_constant__ QkParams p, const __grid_constant__ CUtensorMap tmap)
 {
     extern __shared__ unsigned char dsm_raw[];
@@ -137,15 +152,21 @@ __global__ void __launch_bounds__(QTHREADS, 1)
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile int *abort_flag = &sh.abort_flag;
-    volatile int *stop = &sh.stop;
     pdl_release();
     if (tid == 0) {
-        for (int b = 0; b < QNBUF; ++b) mbar_init(&sh.sfull[b], 1);
+        for (int b = 0; b < QNBUF; ++b) {
+            mbar_init(&sh.sfull[b], 1);
+            mbar_init(&sh.sempty[b], QEPI_WARPS);
+        }
+        for (int s = 0; s < QNST; ++s) {
+            mbar_init(&sh.stfull[s], QEPI_WARPS);
+            mbar_init(&sh.stfree[s], 1);
+        }
+        mbar_init(&sh.opsready, QEPI_WARPS);
         mbar_init(&sh.fin, 1);
         mbar_init(&sh.qload, 1);
         mbar_init(&sh.kload, 1);
         sh.abort_flag = 0;
-        sh.stop = 0;
     }
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(&sh.tmem)),
@@ -156,7 +177,7 @@ __global__ void __launch_bounds__(QTHREADS, 1)
     const int L16 = (L + 15) & ~15;                     // keys that go through the MMAs
     const int nch = (L + QNC - 1) / QNC;
     // bytes of each output row past the MMA'd keys (up to ld) stay zero for the whole launch
-    for (int x = tid; !BULK && x < QM * (int)(p.ld - L16); x += QTHREADS) {
+    for (int x = tid; !BULK && x < QM * (int)(p.ld - L16); x += QALL) {
         const int r = x / (int)(p.ld - L16), j = x - r * (int)(p.ld - L16);
         OS[(size_t)r * p.ld + L16 + j] = 0;
     }
@@ -169,195 +190,224 @@ __global__ void __launch_bounds__(QTHREADS, 1)
     const int64_t ntiles = p.BH * tpb;
     const int64_t t_begin = (int64_t)blockIdx.x * ntiles / gridDim.x;
     const int64_t t_end = (int64_t)(blockIdx.x + 1) * ntiles / gridDim.x;
-    // instruction descriptor: D f32, A/B f16 K-major, M = 128, N = n
-    auto idesc = [](int n) -> uint32_t { return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(QM >> 4) << 24); };
-    const __half2 zq2 = __half2half2(__int2half_rn(p.zp_q)), zk2 = __half2half2(__int2half_rn(p.zp_k));
-    // the requantization's constants in registers (an integer multiply-add takes one constant-bank operand)
-    uint32_t rn2 = (uint32_t)p.n2, rc1 = p.c1;
-    int rn1 = p.n1;
-    asm volatile("" : "+r"(rn2), "+r"(rc1), "+r"(rn1));
-
-    // BULK: the copies of a tile's Q rows and of a head's K rows
-    auto copy_q = [&](int64_t tt) {
-        const int bq = (int)(tt / tpb), rq = (int)(tt - (int64_t)bq * tpb) * QM;
-        const uint32_t bytes = (uint32_t)(min(QM, L - rq) * p.ld_q);
-        mbar_expect_tx(&sh.qload, bytes);
-        bulk_g2s(QST, p.q + ((size_t)bq * L + rq) * p.ld_q, bytes, &sh.qload);
-    };
-    auto copy_k = [&](int bk) {
-        const uint32_t bytes = (uint32_t)(L * p.ld_k);
-        mbar_expect_tx(&sh.kload, bytes);
-        bulk_g2s(KST, p.k + (size_t)bk * L * p.ld_k, bytes, &sh.kload);
-    };
-    // BULK: phases waited for and copies issued (thread 0) on the two copy barriers; a copy is
-    // issued only after the previous one on its barrier was waited for, so at most one is in flight
-    uint32_t qph = 0, kph = 0, qiss = 0, kiss = 0;
     pdl_wait();  // the set-up above touched no global memory
-    if (BULK && tid == 0 && t_begin < t_end) {
-        copy_q(t_begin);
-        copy_k((int)(t_begin / tpb));
-        qiss = kiss = 1;
-    }
 
-    // chunks are numbered across the CTA's tiles: chunk gc uses buffer gc % QNBUF, whose barrier
-    // then completes its phase gc / QNBUF
-    uint32_t g0 = 0;  // number of the tile's first chunk
-    uint32_t issued = 0;       // MMA commits issued (thread 0)
-    int cur_bh = -1;
-    for (int64_t t = t_begin; t < t_end; ++t) {
-        const int bh = (int)(t / tpb);
-        const int r0 = (int)(t - (int64_t)bh * tpb) * QM;
-        // ---- operands: K of a new head, the tile's Q rows (8 values = 16 bytes of fp16 per item)
-        bool cbad = false;
-        if (bh != cur_bh) {
-            if (BULK) {
-                cbad = !mbar_wait_warp(&sh.kload, kph & 1, abort_flag);
-                ++kph;
-            }
-            for (int x = tid; x < L16 * 8 && !cbad; x += QTHREADS) {
-                const int key = x >> 3, c = x & 7;
-                uint4 h = make_uint4(0, 0, 0, 0);
-                if (key < L && 8 * c < d) {
-                    const uint2 w = BULK ? *reinterpret_cast<const uint2 *>(KST + key * p.ld_k + 8 * c)
-                                         : __ldg(reinterpret_cast<const uint2 *>(p.k + ((size_t)bh * L + key) * p.ld_k + 8 * c));
-                    h = codes_to_h8(w, zk2);
-                }
-                *reinterpret_cast<uint4 *>(KS + key * QROW + ((c ^ (key & 7)) << 4)) = h;
-            }
-            cur_bh = bh;
-        }
-        if (BULK && !cbad) {
-            cbad = !mbar_wait_warp(&sh.qload, qph & 1, abort_flag);
-            ++qph;
-        }
-        for (int x = tid; x < QM * 8 && !cbad; x += QTHREADS) {
-            const int r = x >> 3, c = x & 7;
-            uint4 h = make_uint4(0, 0, 0, 0);
-            if (r0 + r < L && 8 * c < d) {
-                const uint2 w = BULK ? *reinterpret_cast<const uint2 *>(QST + r * p.ld_q + 8 * c)
-                                     : __ldg(reinterpret_cast<const uint2 *>(p.q + ((size_t)bh * L + r0 + r) * p.ld_q + 8 * c));
-                h = codes_to_h8(w, zq2);
-            }
-            *reinterpret_cast<uint4 *>(QS + r * QROW + ((c ^ (r & 7)) << 4)) = h;
-        }
-        if (cbad) *stop = 1;
-        fence_async_smem();  // the operands are read by the MMAs
-        tc_fence_before();
-        __syncthreads();
-        tc_fence_after();
-        if (*stop) break;
-        // ---- the staging buffers are converted: the next tile's Q (and the next head's K) may land
-        if (BULK && tid == 0 && t + 1 < t_end) {
-            copy_q(t + 1);
-            ++qiss;
-            if ((int)((t + 1) / tpb) != bh) {
-                copy_k((int)((t + 1) / tpb));
-                ++kiss;
-            }
-        }
-        // ---- the first chunks (up to one per buffer)
-        auto issue = [&](int c) {
-            const int n = min(QNC, L16 - c * QNC);
-            const uint32_t a0 = sa(QS), b0 = sa(KS) + (uint32_t)(c * QNC * QROW);
-#pragma unroll
-            for (int s = 0; s < QKD / 16; ++s)
-                mma_f16_ss(tmem + (uint32_t)(((g0 + c) % QNBUF) * QNC), smem_desc(a0 + 32 * s, 16, 1024),
-                           smem_desc(b0 + 32 * s, 16, 1024), idesc(n), s != 0);
-            mma_commit(&sh.sfull[(g0 + c) % QNBUF]);
-            ++issued;
-        };
-        if (tid == 0)
-            for (int c = 0; c < nch && c < QNBUF; ++c) issue(c);
-        // ---- chunks: read back, quantize, into the output tile
+    if (warp < QEPI_WARPS) {
+        // ---------------- epilogue warps: operands in, accumulators out
+        const __half2 zq2 = __half2half2(__int2half_rn(p.zp_q)), zk2 = __half2half2(__int2half_rn(p.zp_k));
+        // the requantization's constants in registers (an integer multiply-add takes one constant-bank operand)
+        uint32_t rn2 = (uint32_t)p.n2, rc1 = p.c1;
+        int rn1 = p.n1;
+        asm volatile("" : "+r"(rn2), "+r"(rc1), "+r"(rn1));
         const int qr = 32 * (warp & 3) + lane;  // tile row of this thread
         const int g = warp >> 2;                // 32-column group of a chunk
-        bool bad = false;
-        for (int c = 0; c < nch; ++c) {
-            const uint32_t b = (g0 + c) % QNBUF;
-            if (!mbar_wait_warp(&sh.sfull[b], ((g0 + c) / QNBUF) & 1, abort_flag)) {
-                bad = true;
-                *stop = 1;
-            }
-            tc_fence_after();
-            const int col0 = c * QNC + 32 * g;  // first key of this warp's 32 columns
-            // BULK: this chunk's staging buffer, 16-byte unit u of tile row qr at u ^ (qr % 8)
-            unsigned char *srow = OS + (size_t)((g0 + c) % QNST) * QST_BYTES + qr * QNC;
-            if (BULK && !bad && col0 >= L16 && col0 < p.ld) {  // bytes past the keys, inside the row
-                *reinterpret_cast<uint4 *>(srow + (((2 * g) ^ (qr & 7)) << 4)) = make_uint4(0, 0, 0, 0);
-                *reinterpret_cast<uint4 *>(srow + (((2 * g + 1) ^ (qr & 7)) << 4)) = make_uint4(0, 0, 0, 0);
-            }
-            if (!bad && col0 < L16) {
-                uint32_t v[32];
-                tmem_ld32(tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(b * QNC + 32 * g), v);
-                tmem_wait_ld();
-                uint32_t w[8];
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int l0 = logit_of<FOLD>(v[4 * i], p, rn2, rc1, rn1);
-                    const int l1 = logit_of<FOLD>(v[4 * i + 1], p, rn2, rc1, rn1);
-                    const int l2 = logit_of<FOLD>(v[4 * i + 2], p, rn2, rc1, rn1);
-                    const int l3 = logit_of<FOLD>(v[4 * i + 3], p, rn2, rc1, rn1);
-                    w[i] = pack_sat_s8(l1, l0, pack_sat_s8(l3, l2, 0u));
+        uint32_t qph = 0, kph = 0;              // BULK: phases of the copy barriers waited for
+        uint32_t gc = 0;                        // chunks are numbered across the CTA's tiles
+        int cur_bh = -1;
+        for (int64_t t = t_begin; t < t_end; ++t) {
+            const int bh = (int)(t / tpb);
+            const int r0 = (int)(t - (int64_t)bh * tpb) * QM;
+            // ---- operands: K of a new head, the tile's Q rows (8 values = 16 bytes of fp16 per item).
+            //      The MMAs of the previous tile, which read them, have completed: its last chunk was
+            //      waited for below.
+            bool bad = false;
+            if (bh != cur_bh) {
+                if (BULK) {
+                    bad = !mbar_wait_warp(&sh.kload, kph & 1, abort_flag);
+                    ++kph;
                 }
-                if (col0 + 32 > L) {  // keys at or past L: zero bytes (the last chunk only)
+                for (int x = tid; x < L16 * 8 && !bad; x += QTHREADS) {
+                    const int key = x >> 3, c = x & 7;
+                    uint4 h = make_uint4(0, 0, 0, 0);
+                    if (key < L && 8 * c < d) {
+                        const uint2 w = BULK ? *reinterpret_cast<const uint2 *>(KST + key * p.ld_k + 8 * c)
+                                             : __ldg(reinterpret_cast<const uint2 *>(p.k + ((size_t)bh * L + key) * p.ld_k + 8 * c));
+                        h = codes_to_h8(w, zk2);
+                    }
+                    *reinterpret_cast<uint4 *>(KS + key * QROW + ((c ^ (key & 7)) << 4)) = h;
+                }
+                cur_bh = bh;
+            }
+            if (BULK && !bad) {
+                bad = !mbar_wait_warp(&sh.qload, qph & 1, abort_flag);
+                ++qph;
+            }
+            for (int x = tid; x < QM * 8 && !bad; x += QTHREADS) {
+                const int r = x >> 3, c = x & 7;
+                uint4 h = make_uint4(0, 0, 0, 0);
+                if (r0 + r < L && 8 * c < d) {
+                    const uint2 w = BULK ? *reinterpret_cast<const uint2 *>(QST + r * p.ld_q + 8 * c)
+                                         : __ldg(reinterpret_cast<const uint2 *>(p.q + ((size_t)bh * L + r0 + r) * p.ld_q + 8 * c));
+                    h = codes_to_h8(w, zq2);
+                }
+                *reinterpret_cast<uint4 *>(QS + r * QROW + ((c ^ (r & 7)) << 4)) = h;
+            }
+            fence_async_smem();  // the operands are read by the MMAs (and the staging areas refilled)
+            tc_fence_before();
+            __syncwarp();
+            if (!bad && lane == 0) mbar_arrive(&sh.opsready);
+            // ---- chunks: read back, quantize, into the output staging (or tile)
+            for (int c = 0; c < nch && !bad; ++c, ++gc) {
+                const uint32_t b = gc % QNBUF, s = gc % QNST;
+                bad = !mbar_wait_warp(&sh.sfull[b], (gc / QNBUF) & 1, abort_flag);
+                // BULK: the store of chunk gc - QNST has read this staging buffer
+                if (BULK && !bad && gc >= (uint32_t)QNST)
+                    bad = !mbar_wait_warp(&sh.stfree[s], ((gc - QNST) / QNST) & 1, abort_flag);
+                if (bad) break;
+                tc_fence_after();
+                const int col0 = c * QNC + 32 * g;  // first key of this warp's 32 columns
+                // BULK: this chunk's staging buffer, 16-byte unit u of tile row qr at u ^ (qr % 8)
+                unsigned char *srow = OS + (size_t)s * QST_BYTES + qr * QNC;
+                if (BULK && col0 >= L16 && col0 < p.ld) {  // bytes past the keys, inside the row
+                    *reinterpret_cast<uint4 *>(srow + (((2 * g) ^ (qr & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+                    *reinterpret_cast<uint4 *>(srow + (((2 * g + 1) ^ (qr & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+                }
+                if (col0 < L16) {
+                    uint32_t v[32];
+                    tmem_ld32(tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(b * QNC + 32 * g), v);
+                    tmem_wait_ld();
+                    uint32_t w[8];
 #pragma unroll
                     for (int i = 0; i < 8; ++i) {
-                        const int k0 = col0 + 4 * i;
-                        if (k0 + 4 > L) w[i] &= k0 >= L ? 0u : (0xFFFFFFFFu >> (32 - 8 * (L - k0)));
+                        const int l0 = logit_of<FOLD>(v[4 * i], p, rn2, rc1, rn1);
+                        const int l1 = logit_of<FOLD>(v[4 * i + 1], p, rn2, rc1, rn1);
+                        const int l2 = logit_of<FOLD>(v[4 * i + 2], p, rn2, rc1, rn1);
+                        const int l3 = logit_of<FOLD>(v[4 * i + 3], p, rn2, rc1, rn1);
+                        w[i] = pack_sat_s8(l1, l0, pack_sat_s8(l3, l2, 0u));
+                    }
+                    if (col0 + 32 > L) {  // keys at or past L: zero bytes (the last chunk only)
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const int k0 = col0 + 4 * i;
+                            if (k0 + 4 > L) w[i] &= k0 >= L ? 0u : (0xFFFFFFFFu >> (32 - 8 * (L - k0)));
+                        }
+                    }
+                    if (BULK) {  // units past L16 hold zeros (w is masked past L) or lie past ld (clipped)
+                        *reinterpret_cast<uint4 *>(srow + (((2 * g) ^ (qr & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+                        *reinterpret_cast<uint4 *>(srow + (((2 * g + 1) ^ (qr & 7)) << 4)) =
+                            col0 + 16 < L16 ? make_uint4(w[4], w[5], w[6], w[7]) : make_uint4(0, 0, 0, 0);
+                    } else {
+                        unsigned char *dst = OS + (size_t)qr * p.ld + col0;
+                        *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+                        if (col0 + 16 < L16) *reinterpret_cast<uint4 *>(dst + 16) = make_uint4(w[4], w[5], w[6], w[7]);
                     }
                 }
-                if (BULK) {  // units past L16 hold zeros (w is masked past L) or lie past ld (clipped)
-                    *reinterpret_cast<uint4 *>(srow + (((2 * g) ^ (qr & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
-                    *reinterpret_cast<uint4 *>(srow + (((2 * g + 1) ^ (qr & 7)) << 4)) =
-                        col0 + 16 < L16 ? make_uint4(w[4], w[5], w[6], w[7]) : make_uint4(0, 0, 0, 0);
-                } else {
-                    unsigned char *dst = OS + (size_t)qr * p.ld + col0;
-                    *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
-                    if (col0 + 16 < L16) *reinterpret_cast<uint4 *>(dst + 16) = make_uint4(w[4], w[5], w[6], w[7]);
+                if (BULK) fence_async_smem();  // the staging bytes are read by the tensor store
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) {
+                    mbar_arrive(&sh.sempty[b]);  // this warp's part of buffer b is read
+                    if (BULK) mbar_arrive(&sh.stfull[s]);
                 }
             }
-            if (BULK) {
-                fence_async_smem();  // the staging bytes are read by the tensor store
-                // the store of chunk gc - 2 has read its buffer, which chunk gc + 1 writes next
-                if (tid == 0) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+            // ---- (without BULK) the tile's rows to global memory (contiguous there): 16 bytes per
+            //      thread and step, each warp's stores one contiguous 512-byte run.  Every epilogue
+            //      thread reaches this barrier, which also tells each of them whether any gave up; the
+            //      next tile's chunks are computed only after every epilogue warp has arrived on
+            //      opsready again, so after these copies.
+            if (!BULK) {
+                uint32_t any_bad;
+                asm volatile(
+                    "{ .reg .pred pb, pa; setp.ne.u32 pb, %1, 0; bar.red.or.pred pa, 1, %2, pb; selp.u32 %0, 1, 0, pa; }"
+                    : "=r"(any_bad)
+                    : "r"((uint32_t)bad), "n"(QTHREADS)
+                    : "memory");
+                if (any_bad) break;
+                const int64_t bytes = (int64_t)min(QM, L - r0) * p.ld;
+                int8_t *gdst = p.out + ((size_t)bh * L + r0) * p.ld;
+                for (int64_t x = 16 * (int64_t)tid; x < bytes; x += 16 * QTHREADS)
+                    *reinterpret_cast<uint4 *>(gdst + x) = *reinterpret_cast<const uint4 *>(OS + x);
+            } else if (bad) {
+                break;
             }
-            tc_fence_before();
-            __syncthreads();  // buffer b is read: chunk c + QNBUF may overwrite it
-            tc_fence_after();
-            if (*stop) break;
-            if (BULK && tid == 0) {  // chunk c of the tile: columns c 128 .., rows r0 .., head bh
+        }
+    } else if (warp == QMMA_WARP) {
+        // ---------------- warp 16, lane 0: the operand copies (BULK) and the MMAs
+        if (lane == 0) {
+            // instruction descriptor: D f32, A/B f16 K-major, M = 128, N = n
+            auto idesc = [](int n) -> uint32_t {
+                return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(QM >> 4) << 24);
+            };
+            auto copy_q = [&](int64_t tt) {
+                const int bq = (int)(tt / tpb), rq = (int)(tt - (int64_t)bq * tpb) * QM;
+                const uint32_t bytes = (uint32_t)(min(QM, L - rq) * p.ld_q);
+                mbar_expect_tx(&sh.qload, bytes);
+                bulk_g2s(QST, p.q + ((size_t)bq * L + rq) * p.ld_q, bytes, &sh.qload);
+            };
+            auto copy_k = [&](int bk) {
+                const uint32_t bytes = (uint32_t)(L * p.ld_k);
+                mbar_expect_tx(&sh.kload, bytes);
+                bulk_g2s(KST, p.k + (size_t)bk * L * p.ld_k, bytes, &sh.kload);
+            };
+            // a copy is issued only once the operands it replaces were converted (opsready), so at
+            // most one is in flight on each barrier
+            uint32_t qiss = 0, kiss = 0, issued = 0, gc = 0;
+            if (BULK && t_begin < t_end) {
+                copy_q(t_begin);
+                copy_k((int)(t_begin / tpb));
+                qiss = kiss = 1;
+            }
+            bool ok = true;
+            for (int64_t t = t_begin; t < t_end && ok; ++t) {
+                ok = mbar_wait(&sh.opsready, (uint32_t)(t - t_begin) & 1, abort_flag);
+                if (!ok) break;
+                tc_fence_after();
+                if (BULK && t + 1 < t_end) {  // the staging areas were converted: the next tile's operands
+                    copy_q(t + 1);
+                    ++qiss;
+                    if ((int)((t + 1) / tpb) != (int)(t / tpb)) {
+                        copy_k((int)((t + 1) / tpb));
+                        ++kiss;
+                    }
+                }
+                for (int c = 0; c < nch; ++c, ++gc) {
+                    const uint32_t b = gc % QNBUF;
+                    // the epilogue warps have read buffer b's previous chunk
+                    if (gc >= (uint32_t)QNBUF && !mbar_wait(&sh.sempty[b], ((gc - QNBUF) / QNBUF) & 1, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const int n = min(QNC, L16 - c * QNC);
+                    const uint32_t a0 = sa(QS), b0 = sa(KS) + (uint32_t)(c * QNC * QROW);
+#pragma unroll
+                    for (int s = 0; s < QKD / 16; ++s)
+                        mma_f16_ss(tmem + b * QNC, smem_desc(a0 + 32 * s, 16, 1024), smem_desc(b0 + 32 * s, 16, 1024),
+                                   idesc(n), s != 0);
+                    mma_commit(&sh.sfull[b]);
+                    ++issued;
+                }
+            }
+            // every copy and every MMA issued has completed before shared and tensor memory are released
+            if (BULK && qiss > 0) mbar_wait(&sh.qload, (qiss - 1) & 1, abort_flag, false);
+            if (BULK && kiss > 0) mbar_wait(&sh.kload, (kiss - 1) & 1, abort_flag, false);
+            if (issued > 0) {
+                mma_commit(&sh.fin);
+                mbar_wait(&sh.fin, 0, abort_flag, false);
+            }
+        }
+    } else if (BULK && lane == 0) {
+        // ---------------- warp 17, lane 0: the tensor stores of the chunks' staging buffers
+        uint32_t gc = 0;
+        bool ok = true;
+        for (int64_t t = t_begin; t < t_end && ok; ++t) {
+            const int bh = (int)(t / tpb);
+            const int r0 = (int)(t - (int64_t)bh * tpb) * QM;
+            for (int c = 0; c < nch; ++c, ++gc) {
+                const uint32_t s = gc % QNST;
+                ok = mbar_wait(&sh.stfull[s], (gc / QNST) & 1, abort_flag);
+                if (!ok) break;
+                // chunk c of the tile: columns c 128 .., rows r0 .., head bh
                 asm volatile(
                     "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(&tmap),
-                    "r"(c * QNC), "r"(r0), "r"(bh), "r"(sa(OS + (size_t)((g0 + c) % QNST) * QST_BYTES))
+                    "r"(c * QNC), "r"(r0), "r"(bh), "r"(sa(OS + (size_t)s * QST_BYTES))
                     : "memory");
                 asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+                asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");  // the buffer has been read
+                mbar_arrive(&sh.stfree[s]);
             }
-            if (tid == 0 && c + QNBUF < nch) issue(c + QNBUF);
         }
-        if (*stop) break;
-        g0 += (uint32_t)nch;
-        // ---- (without BULK) the tile's rows to global memory (contiguous there): 16 bytes per
-        //      thread and step, each warp's stores one contiguous 512-byte run; the next tile's
-        //      epilogue writes the tile again only after its first barrier
-        if (!BULK) {
-            __syncthreads();
-            const int64_t bytes = (int64_t)min(QM, L - r0) * p.ld;
-            int8_t *gdst = p.out + ((size_t)bh * L + r0) * p.ld;
-            for (int64_t x = 16 * (int64_t)tid; x < bytes; x += 16 * QTHREADS)
-                *reinterpret_cast<uint4 *>(gdst + x) = *reinterpret_cast<const uint4 *>(OS + x);
-        }
-    }
-    // every store and every MMA issued has completed before shared and tensor memory are released
-    if (tid == 0) {
-        if (BULK) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");  // the tensor stores
-        if (BULK) {  // a copy issued ahead and never waited for (the loop stopped early)
-            if (qph < qiss) mbar_wait(&sh.qload, qph & 1, abort_flag, false);
-            if (kph < kiss) mbar_wait(&sh.kload, kph & 1, abort_flag, false);
-        }
-        if (issued > 0) {
-            mma_commit(&sh.fin);
-            mbar_wait(&sh.fin, 0, abort_flag, false);
-        }
+        asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");  // every store has completed
     }
     tc_fence_before();
     __syncthreads();
@@ -381,7 +431,7 @@ cudaError_t qk_launch(const QkParams &p, const CUtensorMap &tm, size_t smem, int
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(qk_logits_tc_kernel<FOLD, BULK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(qk_logits_tc_kernel<FOLD, BULK>, dim3(grid), dim3(QTHREADS), smem, st, p, tm);
+    return launch_pdl(qk_logits_tc_kernel<FOLD, BULK>, dim3(grid), dim3(QALL), smem, st, p, tm);
 }
 
 // The logits as a 3-d tensor [BH][L][ld] of bytes for the tensor stores: boxes of 128 x 128 x 1,
