@@ -112,6 +112,24 @@ __device__ __forceinline__ uint4 codes_to_h8(uint2 w, __half2 z)
 //   FOLD: (N2 P + 2^(N1-1) + zp_l 2^N1) >> N1 in 32 bits (the host checked that it fits)
 //   else: the 64-bit formula, N1 of any sign
 // (n2, c1, n1: the launch's constants, held in registers by the caller)
+// Two accumulators plus 1.5 2^23 in one packed fp32 add (each sum exact: |P| < 2^22): the bit
+// patterns 0x4B400000 + P of the FOLD form below
+__device__ __forceinline__ void add_magic2(uint32_t a, uint32_t b, uint32_t &x, uint32_t &y)
+{
+    asm("{ .reg .b64 ra, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\t"
+        "add.rn.f32x2 rd, ra, %4;\n\t"
+        "mov.b64 {%0, %1}, rd; }"
+        : "=r"(x), "=r"(y)
+        : "r"(a), "r"(b), "l"(0x4B4000004B400000ull));
+}
+
+// The logit of an accumulator already in the form 0x4B400000 + P (FOLD): one multiply-add and a shift
+__device__ __forceinline__ int logit_of_biased(uint32_t x, uint32_t n2, uint32_t c1, int n1)
+{
+    return (int)(x * n2 + c1) >> n1;
+}
+
 template <bool FOLD>
 __device__ __forceinline__ int logit_of(uint32_t acc_bits, const QkParams &p, uint32_t n2, uint32_t c1, int n1)
 {
@@ -269,10 +287,21 @@ __global__ void __launch_bounds__(QBOUND, 1)
                     uint32_t w[8];
 #pragma unroll
                     for (int i = 0; i < 8; ++i) {
-                        const int l0 = logit_of<FOLD>(v[4 * i], p, rn2, rc1, rn1);
-                        const int l1 = logit_of<FOLD>(v[4 * i + 1], p, rn2, rc1, rn1);
-                        const int l2 = logit_of<FOLD>(v[4 * i + 2], p, rn2, rc1, rn1);
-                        const int l3 = logit_of<FOLD>(v[4 * i + 3], p, rn2, rc1, rn1);
+                        int l0, l1, l2, l3;
+                        if (FOLD) {  // the magic additions two at a time
+                            uint32_t x0, x1, x2, x3;
+                            add_magic2(v[4 * i], v[4 * i + 1], x0, x1);
+                            add_magic2(v[4 * i + 2], v[4 * i + 3], x2, x3);
+                            l0 = logit_of_biased(x0, rn2, rc1, rn1);
+                            l1 = logit_of_biased(x1, rn2, rc1, rn1);
+                            l2 = logit_of_biased(x2, rn2, rc1, rn1);
+                            l3 = logit_of_biased(x3, rn2, rc1, rn1);
+                        } else {
+                            l0 = logit_of<FOLD>(v[4 * i], p, rn2, rc1, rn1);
+                            l1 = logit_of<FOLD>(v[4 * i + 1], p, rn2, rc1, rn1);
+                            l2 = logit_of<FOLD>(v[4 * i + 2], p, rn2, rc1, rn1);
+                            l3 = logit_of<FOLD>(v[4 * i + 3], p, rn2, rc1, rn1);
+                        }
                         w[i] = pack_sat_s8(l1, l0, pack_sat_s8(l3, l2, 0u));
                     }
                     if (col0 + 32 > L) {  // keys at or past L: zero bytes (the last chunk only)
