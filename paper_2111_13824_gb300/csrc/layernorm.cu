@@ -706,6 +706,22 @@ cudaError_t stage_launch(const LnArgs &a, cudaStream_t st)
     return launch_pdl(ln_stage_kernel<S, R>, dim3(sh.grid), dim3(32 * sh.warps), sh.smem, st, a, sh.seg_stride);
 }
 
+// Rows per segment: the most (4, 2, 1) whose warp groups still give at least half of the grid's
+// warps one group each.  Fewer rows per segment amortize the channel constants and the row terms
+// over fewer rows; too few groups leave warps idle.  Measured at full size (µs per launch, R = 4 /
+// 2 / 1): DeiT-S (C = 384, 12608 rows) 9.7 / 6.7 / 9.6, ViT-B (C = 768, 12608 rows) 11.2 / 13.2 /
+// 13.9, Swin-S (mean over its stages) 10.9 / 8.2 / 10.2.
+template <int S>
+cudaError_t stage_rows(const LnArgs &a, cudaStream_t st)
+{
+    const int64_t half = (int64_t)sm_count() * stg::kMaxWarps / 2;
+    const int64_t spw = 32 / S;
+    auto groups = [&](int64_t R) { return (a.rows + spw * R - 1) / (spw * R); };
+    if (groups(4) >= half) return stage_launch<S, 4>(a, st);
+    if (groups(2) >= half) return stage_launch<S, 2>(a, st);
+    return stage_launch<S, 1>(a, st);
+}
+
 }  // namespace
 
 cudaError_t read_clear_ln_status(int *status)
@@ -723,9 +739,9 @@ cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st)
     if (staged) {
         cudaError_t e;
         switch (stage_segment(a.C / 16)) {
-        case 32: e = stage_launch<32, 4>(a, st); break;
-        case 16: e = stage_launch<16, 4>(a, st); break;
-        case 8: e = stage_launch<8, 4>(a, st); break;
+        case 32: e = stage_rows<32>(a, st); break;
+        case 16: e = stage_rows<16>(a, st); break;
+        case 8: e = stage_rows<8>(a, st); break;
         case 4: e = stage_launch<4, 4>(a, st); break;
         case 2: e = stage_launch<2, 2>(a, st); break;
         default: e = stage_launch<1, 1>(a, st); break;
