@@ -131,6 +131,14 @@ def test_layernorm_rows_per_warp(rows, C):
     _assert_ln(_ln_case(rows * 7 + C, rows, C))
 
 
+@pytest.mark.parametrize("rows,C", [(3001, 1024), (6007, 768), (10001, 384), (4000, 4096)])
+def test_layernorm_two_rows_per_segment(rows, C):
+    """Row counts between the thresholds of the rows-per-segment choice: on a 152-SM GPU these
+    take 2 rows per segment (the most that still gives half of the grid's warps a group), the
+    other counts of these tests 4 or 1."""
+    _assert_ln(_ln_case(rows + 3 * C, rows, C))
+
+
 def test_layernorm_strided_rows():
     _assert_ln(_ln_case(5, 200, 192), ld_in=208, ld_out=224)
     _assert_ln(_ln_case(6, 200, 192), ld_in=193, ld_out=195)
