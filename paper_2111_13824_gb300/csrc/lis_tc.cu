@@ -442,20 +442,28 @@ __global__ void __launch_bounds__(TTHREADS, 1) lis_attn_tc_kernel(TcParams p)
     }
     __syncthreads();
     {
+        // the 256 i-exp values once (the row-maximum exchange area is free until the first tile), then
+        // their 32 copies per table line
+        uint32_t *e_tmp = reinterpret_cast<uint32_t *>(red_max);
         const IexpC c = sh.c;
-        for (int i = tid; i < 256 * 32; i += blockDim.x)
-            sts_u32(kTabAbs + (uint32_t)(i >> 5) * 256u + LUT_BYTE + 4u * (i & 31), iexp_neg(i >> 5, c));
-        for (int d = tid; d < 256; d += blockDim.x) LUTF[d] = __uint2float_rn(iexp_neg(d, c));
+        for (int d = tid; d < 256; d += blockDim.x) {
+            const uint32_t e = iexp_neg(d, c);
+            e_tmp[d] = e;
+            LUTF[d] = __uint2float_rn(e);
+        }
         for (int i = tid; i < 128; i += blockDim.x) ONES[i] = 0x3C003C00u;
+        __syncthreads();
+        for (int i = tid; i < 256 * 32; i += blockDim.x)
+            sts_u32(kTabAbs + (uint32_t)(i >> 5) * 256u + LUT_BYTE + 4u * (i & 31), e_tmp[i >> 5]);
         for (int d = tid; d < 255; d += blockDim.x)
-            if (iexp_neg(d, c) < iexp_neg(d + 1, c)) sh.rising = 1;
+            if (e_tmp[d] < e_tmp[d + 1]) sh.rising = 1;
     }
     if (tid == 0) {
-        const int bkmax = (int)(__float_as_uint(__uint2float_rn(iexp_neg(0, sh.c)) * (1.0f + 0x1p-20f)) >> BK_SHIFT);
+        const int bkmax = (int)(__float_as_uint(LUTF[0] * (1.0f + 0x1p-20f)) >> BK_SHIFT);
         sh.bkmax = bkmax;
         sh.bk0 = bkmax - (BK_N - 1);
     }
-    __syncthreads();  // LUTF, rising, the bucket range
+    __syncthreads();  // the copies of the i-exp values read, rising, the bucket range
     if (!sh.rising) {
         // #{d : e(d) > x} by binary search (the values never rise with d)
         auto count_above = [&](float x) -> int {
